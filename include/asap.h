@@ -1,0 +1,221 @@
+/*
+ * asap.h -- C ABI of the GB300 implementation of ASAP's data-parallel hot
+ * path (Kadav & Kruus, "ASAP: Asynchronous Approximate Data-Parallel
+ * Computation", arXiv 1612.08608).
+ *
+ * One context holds N simulated workers on one GPU.  Worker i owns a
+ * parameter vector w_i (fp32) and a private data shard.  One round is the
+ * paper's Eq. A.1:
+ *
+ *     w_{t+1/2}^i = w_t^i - eta * grad f_i(w_t^i)          (local SGD step)
+ *     w_{t+1}^i   = sum_j P_t[i, j] * w_{t+1/2}^j          (stochastic reduce)
+ *
+ * where P_t is a doubly-stochastic mixing matrix with k+1 non-zeros per row
+ * (k in-neighbours plus the worker itself) from a sparse communication
+ * graph (Section 3, "stochastic reduce"; Appendix A, "Network requirement").
+ * NOTIFY-ACK (Section 4, "Fine-grained synchronization") is kept as
+ * per-worker round counters in device memory: worker i publishes
+ * ready[i] = t+1 after its step, a reduce reads worker j's half-step model
+ * only when ready[j] == t+1, and consumed[i] = t+1 acknowledges that every
+ * input of worker i's reduce has been read.  Parameters are double-buffered
+ * (W[t & 1] holds round t), so no reduce ever sees a torn or mixed-version
+ * input, whatever the schedule.
+ *
+ * Conventions for every entry point:
+ *  - The return value is an asap_status; no C++ exception crosses the ABI.
+ *  - Host pointers passed in are read during the call and never retained;
+ *    the caller keeps ownership.  Device memory is allocated and owned by the
+ *    context and released by asap_destroy.
+ *  - Calls marked "async" enqueue work on the context's stream and return;
+ *    they report launch errors at once.  Errors found on the device (a wait
+ *    that ran out, a stamp that did not match) are reported by the next
+ *    "syncing" call (asap_read_params, asap_read_metrics, asap_sync).
+ *  - asap_last_error(ctx) gives a one-line description of the last failure;
+ *    asap_last_error(NULL) gives the last failure of asap_create or of a
+ *    context-free helper on this thread.
+ *  - A context is not thread-safe; use one host thread per context.
+ */
+#ifndef ASAP_H
+#define ASAP_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct asap_ctx asap_ctx;
+
+typedef enum {
+  ASAP_OK = 0,
+  ASAP_ERR_ARG = 1,     /* invalid argument, size or call order             */
+  ASAP_ERR_CUDA = 2,    /* a CUDA runtime call or kernel launch failed       */
+  ASAP_ERR_OOM = 3,     /* device or pinned host allocation failed           */
+  ASAP_ERR_TIMEOUT = 4, /* a device-side NOTIFY/ACK wait ran out            */
+  ASAP_ERR_STATE = 5,   /* a round stamp did not match (protocol violation)  */
+  ASAP_ERR_GRAPH = 6    /* the requested graph cannot be built / is invalid  */
+} asap_status;
+
+/* Communication graphs (Section 3.1 and Fig. 2).  Row i of P lists i and its
+ * in-neighbours in ascending order; the default weights are 1/(k+1). */
+typedef enum {
+  ASAP_GRAPH_RING = 1,           /* chain closed into a ring: i <- i-1 (k = 1)        */
+  ASAP_GRAPH_ROOT = 2,           /* root expander: i <- i-1, i-isqrt(N) (k = 2, N>=4) */
+  ASAP_GRAPH_RANDOM_REGULAR = 3, /* seeded random k-regular digraph (see below)       */
+  ASAP_GRAPH_COMPLETE = 4,       /* all-reduce: every worker (k = N-1)                */
+  ASAP_GRAPH_EXPLICIT = 5,       /* user weights, see asap_set_mixing                 */
+  ASAP_GRAPH_IDENTITY = 6        /* no communication (k = 0)                          */
+} asap_graph_kind;
+
+typedef enum {
+  ASAP_LOSS_NONE = 0,     /* no local step: the context only mixes              */
+  ASAP_LOSS_HINGE = 1,    /* linear SVM, l = max(0, 1 - y m) (Section 5)         */
+  ASAP_LOSS_LOGISTIC = 2, /* l = ln(1 + exp(-y m))                              */
+  ASAP_LOSS_SOFTMAX = 3   /* dense softmax regression on bf16 features          */
+} asap_loss;
+
+typedef enum {
+  ASAP_SHARDS_DEVICE = 0, /* shards copied to HBM once at load time             */
+  ASAP_SHARDS_HOST = 1    /* shards kept in pinned host memory; each round's
+                             minibatch block is copied to the GPU as the round
+                             runs (overlapped with the previous round)         */
+} asap_residency;
+
+/* Create a context for N workers with d parameters each (d features; for
+ * softmax regression the model is C x d, see asap_set_model).  k is the
+ * number of in-neighbours besides the worker itself.  The default graph is
+ * IDENTITY for k = 0, RING for k = 1, COMPLETE for k = N-1 and
+ * RANDOM_REGULAR otherwise, built from graph_seed and fixed for all rounds.
+ * W_0 = 0 (Appendix A takes w_0 = 0).  Uses the current CUDA device.
+ * Limits: 1 <= N <= 1024, 1 <= d, 0 <= k <= N-1.  On failure *out = NULL. */
+asap_status asap_create(int N, int64_t d, uint64_t graph_seed, int k, asap_ctx** out);
+
+/* Choose the graph kind, and whether a new graph is drawn from
+ * (graph_seed, round) every round (Section 3.1: graphs should be "easy to
+ * generate", including re-configuration).  The kind must match k (RING: 1,
+ * ROOT: 2, COMPLETE: N-1, IDENTITY: 0).  RANDOM_REGULAR construction:
+ * SplitMix64 seeded with graph_seed ^ (0x9E3779B97F4A7C15 * (round+1));
+ * a uniform random Hamiltonian cycle (Fisher-Yates), then k-1 permutation
+ * layers drawn by Fisher-Yates with rejection (a node may not receive from
+ * itself or twice from the same node); at most 100,000 draws per layer,
+ * else ASAP_ERR_GRAPH.  Call before the first round that should use it. */
+asap_status asap_set_graph(asap_ctx* ctx, asap_graph_kind kind, int regenerate_every_round);
+
+/* Explicit mixing weights (kind EXPLICIT), fixed for all rounds.
+ * nbr: N*(k+1) int32, row-major, each row strictly ascending, ids in [0,N);
+ * wgt: N*(k+1) float, >= 0.  P must be doubly stochastic: every row sum and
+ * every column sum within 1e-6 of 1 (Appendix A), else ASAP_ERR_GRAPH.
+ * Rows may omit the worker itself.  Requires k+1 <= 32. */
+asap_status asap_set_mixing(asap_ctx* ctx, const int32_t* nbr, const float* wgt);
+
+/* The local objective f_i of Eq. A.1.  loss: ASAP_LOSS_*; num_classes: C for
+ * SOFTMAX (then each worker's model is C x d, class-major), 1 otherwise;
+ * batch: minibatch rows B per worker per round (round t uses rows
+ * [(t mod nb) B, (t mod nb) B + B), nb = floor(rows / B)); lr: eta (> 0);
+ * l2: coefficient of (l2/2) ||w||^2 in f_i (0 <= lr*l2 < 1).
+ * SOFTMAX requires d % 64 == 0, B % 128 == 0, C <= 1024.  Re-setting the
+ * model clears the shards and resets W to 0. */
+asap_status asap_set_model(asap_ctx* ctx, asap_loss loss, int num_classes, int batch, float lr, float l2);
+
+/* Stream for all device work of this context (a cudaStream_t, e.g.
+ * torch.cuda.current_stream().cuda_stream).  NULL selects the context's own
+ * non-blocking stream (the default). */
+asap_status asap_set_stream(asap_ctx* ctx, void* cuda_stream);
+
+/* Where the shards live.  Default DEVICE.  Called after loading, it moves
+ * the loaded shards (synchronous). */
+asap_status asap_set_shard_residency(asap_ctx* ctx, asap_residency residency);
+
+/* Bytes of the minibatch block that round `round` reads (all workers: the
+ * padded CSR rows, labels and the column-sorted copy).  With HOST residency
+ * this is what one round copies to the GPU.  Host only. */
+asap_status asap_shard_block_bytes(asap_ctx* ctx, int64_t round, uint64_t* bytes);
+
+/* Load one CSR shard per worker (hinge / logistic).  All pointers are host
+ * pointers, one per worker: rowptr[i] has n_rows[i]+1 int64 entries starting
+ * at 0; col[i] / val[i] have rowptr[i][n_rows[i]] entries; col ids in
+ * [0, d), distinct within a row; y[i] has n_rows[i] labels in {-1, +1}.
+ * Every worker needs n_rows[i] >= B.  The library builds, once, the batch
+ * layout the kernels read (rows padded to 4 entries; per batch a copy
+ * sorted by (column, row)).  Synchronous. */
+asap_status asap_load_shards(asap_ctx* ctx, const int64_t* const* rowptr, const int32_t* const* col,
+                             const float* const* val, const float* const* y, const int64_t* n_rows);
+
+/* Load one dense shard per worker (softmax): X[i] is n_rows[i] x d bf16
+ * (raw uint16 bits, row-major), y[i] n_rows[i] class ids in [0, C).
+ * Synchronous. */
+asap_status asap_load_dense_shards(asap_ctx* ctx, const uint16_t* const* X_bf16, const int32_t* const* y,
+                                   const int64_t* n_rows);
+
+/* Eq. A.1 first line for every worker, then NOTIFY (ready[i] = t+1).
+ * Async.  Between this call and asap_stochastic_reduce the current buffer
+ * holds w_{t+1/2} (divided by (1 - lr*l2) when l2 > 0). */
+asap_status asap_local_step(asap_ctx* ctx);
+
+/* Eq. A.1 second line for every worker: wait for the in-neighbours' NOTIFY,
+ * W[(t+1)&1] = P_t W[t&1], ACK (consumed[i] = t+1), record the round's
+ * metrics, advance t.  Without a preceding asap_local_step it mixes the
+ * current parameters (the reduce alone).  Async. */
+asap_status asap_stochastic_reduce(asap_ctx* ctx);
+
+/* T rounds of (asap_local_step; asap_stochastic_reduce).  Async. */
+asap_status asap_round(asap_ctx* ctx, int T);
+
+/* Wait for all queued work; report device-side errors.  Syncing. */
+asap_status asap_sync(asap_ctx* ctx);
+
+/* Copy the current parameters W_t (N rows of P = d or C*d floats, row-major,
+ * packed) to host_out; *round_out = t (may be NULL).  Syncing. */
+asap_status asap_read_params(asap_ctx* ctx, float* host_out, int64_t* round_out);
+
+/* Set W_t = host_in (N rows of P floats) and the round counter to `round`
+ * (resume from a checkpoint, or a custom W_0).  Synchronous. */
+asap_status asap_write_params(asap_ctx* ctx, const float* host_in, int64_t round);
+
+/* Per-round metrics of rounds [first_round, first_round + count): the mean
+ * over workers of the minibatch loss at the pre-step parameters (NaN for a
+ * reduce-only round) and the consensus error ||W_{t+1} - 1 wbar^T||_F.
+ * The last 65536 rounds are kept.  Either output pointer may be NULL.
+ * Syncing. */
+asap_status asap_read_metrics(asap_ctx* ctx, int64_t first_round, int64_t count, float* loss_out,
+                              float* consensus_out);
+
+/* Counters of the NOTIFY-ACK protocol since creation: reduces performed,
+ * in-neighbour inputs whose round stamp matched (Section 5.2 reports the
+ * share of such consistent reduces), and waits that ran out.  Syncing. */
+asap_status asap_read_counters(asap_ctx* ctx, uint64_t* reduces, uint64_t* consistent_inputs,
+                               uint64_t* timeouts);
+
+/* The graph used by round `round`: nbr_out N*(k+1) int32 and wgt_out
+ * N*(k+1) float (either may be NULL).  Host only. */
+asap_status asap_get_graph(asap_ctx* ctx, int64_t round, int32_t* nbr_out, float* wgt_out);
+
+/* Limit for every device-side NOTIFY/ACK wait, in nanoseconds (default
+ * 200 ms).  A wait that runs out sets ASAP_ERR_TIMEOUT and the kernel
+ * returns without writing the round's output. */
+asap_status asap_set_wait_limit_ns(asap_ctx* ctx, uint64_t ns);
+
+/* Fault injection for tests: the next asap_local_step does not publish
+ * NOTIFY for `worker` (a stalled worker), so every reduce that depends on it
+ * runs into its wait limit.  worker = -1 clears the injection. */
+asap_status asap_debug_skip_notify(asap_ctx* ctx, int worker);
+
+/* Number of this library's kernel launches since creation (host counter). */
+asap_status asap_kernel_launches(asap_ctx* ctx, uint64_t* launches);
+
+/* Context-free helper: build graph `kind` for (N, k, graph_seed, round) on
+ * the host, exactly as a context would.  nbr_out: N*(k+1) int32.  Needs no
+ * GPU. */
+asap_status asap_build_graph(asap_graph_kind kind, int N, int k, uint64_t graph_seed, int64_t round,
+                             int32_t* nbr_out);
+
+const char* asap_last_error(const asap_ctx* ctx);
+const char* asap_version(void);
+void asap_destroy(asap_ctx* ctx);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* ASAP_H */

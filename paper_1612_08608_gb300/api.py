@@ -1,0 +1,177 @@
+"""Python binding of the ASAP C ABI (include/asap.h): argument marshalling
+only.  Every step of a round runs in the CUDA kernels of libasap.so."""
+from __future__ import annotations
+
+import ctypes as C
+from typing import Optional, Sequence
+
+import numpy as np
+
+from ._lib import load_library
+
+STATUS = {0: "ASAP_OK", 1: "ASAP_ERR_ARG", 2: "ASAP_ERR_CUDA", 3: "ASAP_ERR_OOM",
+          4: "ASAP_ERR_TIMEOUT", 5: "ASAP_ERR_STATE", 6: "ASAP_ERR_GRAPH"}
+GRAPH = {"ring": 1, "root": 2, "random_regular": 3, "complete": 4, "explicit": 5, "identity": 6}
+LOSS = {"none": 0, "hinge": 1, "logistic": 2, "softmax": 3}
+RESIDENCY = {"device": 0, "host": 1}
+
+
+class AsapError(RuntimeError):
+    def __init__(self, status: int, message: str):
+        super().__init__("%s: %s" % (STATUS.get(status, status), message))
+        self.status = status
+        self.name = STATUS.get(status, str(status))
+
+
+def _check(lib, ctx, status: int):
+    if status != 0:
+        msg = lib.asap_last_error(ctx)
+        raise AsapError(status, msg.decode() if msg else "")
+
+
+def _ptr(a: np.ndarray) -> int:
+    return a.ctypes.data
+
+
+def _ptr_array(arrs):
+    return (C.c_void_p * len(arrs))(*[_ptr(a) for a in arrs])
+
+
+def build_graph(kind: str, N: int, k: int, graph_seed: int = 0, rnd: int = 0) -> np.ndarray:
+    """Host graph builder of the library (no GPU needed): [N, k+1] int32."""
+    lib = load_library()
+    out = np.empty((N, k + 1), dtype=np.int32)
+    _check(lib, None, lib.asap_build_graph(GRAPH[kind], N, k, graph_seed, rnd, _ptr(out)))
+    return out
+
+
+class Context:
+    """N simulated workers on the current CUDA device (see include/asap.h)."""
+
+    def __init__(self, N: int, d: int, graph_seed: int = 0, k: int = 0):
+        self._lib = load_library()
+        h = C.c_void_p()
+        _check(self._lib, None, self._lib.asap_create(N, d, graph_seed, k, C.byref(h)))
+        self._h = h
+        self.N, self.d, self.k = N, d, k
+        self.P = d
+        self._keep = []
+
+    # -- configuration -------------------------------------------------
+    def _c(self, status):
+        _check(self._lib, self._h, status)
+
+    def set_graph(self, kind: str, regenerate: bool = False):
+        self._c(self._lib.asap_set_graph(self._h, GRAPH[kind], int(regenerate)))
+
+    def set_mixing(self, nbr, wgt):
+        nbr = np.ascontiguousarray(nbr, dtype=np.int32)
+        wgt = np.ascontiguousarray(wgt, dtype=np.float32)
+        self._c(self._lib.asap_set_mixing(self._h, _ptr(nbr), _ptr(wgt)))
+
+    def set_model(self, loss: str, batch: int, lr: float, num_classes: int = 1, l2: float = 0.0):
+        self._c(self._lib.asap_set_model(self._h, LOSS[loss], num_classes, batch, lr, l2))
+        self.P = self.d * (num_classes if loss == "softmax" else 1)
+
+    def set_stream(self, stream):
+        """stream: a torch.cuda.Stream, an integer cudaStream_t, or None."""
+        handle = getattr(stream, "cuda_stream", stream)
+        self._c(self._lib.asap_set_stream(self._h, C.c_void_p(handle) if handle else None))
+
+    def set_shard_residency(self, where: str):
+        self._c(self._lib.asap_set_shard_residency(self._h, RESIDENCY[where]))
+
+    def shard_block_bytes(self, rnd: int) -> int:
+        v = C.c_uint64()
+        self._c(self._lib.asap_shard_block_bytes(self._h, rnd, C.byref(v)))
+        return v.value
+
+    def load_shards(self, shards=None, rowptr=None, col=None, val=None, y=None):
+        if shards is not None:
+            rowptr, col, val, y = shards.rowptr, shards.col, shards.val, shards.y
+        rp = [np.ascontiguousarray(a, dtype=np.int64) for a in rowptr]
+        cl = [np.ascontiguousarray(a, dtype=np.int32) for a in col]
+        vl = [np.ascontiguousarray(a, dtype=np.float32) for a in val]
+        yl = [np.ascontiguousarray(a, dtype=np.float32) for a in y]
+        n = np.array([a.shape[0] - 1 for a in rp], dtype=np.int64)
+        self._c(self._lib.asap_load_shards(self._h, _ptr_array(rp), _ptr_array(cl), _ptr_array(vl),
+                                           _ptr_array(yl), _ptr(n)))
+
+    def load_dense_shards(self, shards=None, X=None, y=None):
+        if shards is not None:
+            X, y = shards.X, shards.y
+        xl = [np.ascontiguousarray(a, dtype=np.uint16) for a in X]
+        yl = [np.ascontiguousarray(a, dtype=np.int32) for a in y]
+        n = np.array([a.shape[0] for a in xl], dtype=np.int64)
+        self._c(self._lib.asap_load_dense_shards(self._h, _ptr_array(xl), _ptr_array(yl), _ptr(n)))
+
+    # -- the round -----------------------------------------------------
+    def local_step(self):
+        self._c(self._lib.asap_local_step(self._h))
+
+    def stochastic_reduce(self):
+        self._c(self._lib.asap_stochastic_reduce(self._h))
+
+    def round(self, T: int = 1):
+        self._c(self._lib.asap_round(self._h, T))
+
+    def sync(self):
+        self._c(self._lib.asap_sync(self._h))
+
+    # -- state ---------------------------------------------------------
+    def read_params(self, out: Optional[np.ndarray] = None):
+        if out is None:
+            out = np.empty((self.N, self.P), dtype=np.float32)
+        r = C.c_int64()
+        self._c(self._lib.asap_read_params(self._h, _ptr(out), C.byref(r)))
+        return out, r.value
+
+    def write_params(self, W: np.ndarray, rnd: int = 0):
+        W = np.ascontiguousarray(W, dtype=np.float32)
+        assert W.shape == (self.N, self.P)
+        self._c(self._lib.asap_write_params(self._h, _ptr(W), rnd))
+
+    def read_metrics(self, first: int, count: int):
+        loss = np.empty(count, dtype=np.float32)
+        cons = np.empty(count, dtype=np.float32)
+        self._c(self._lib.asap_read_metrics(self._h, first, count, _ptr(loss), _ptr(cons)))
+        return loss, cons
+
+    def read_counters(self):
+        a, b, c = C.c_uint64(), C.c_uint64(), C.c_uint64()
+        self._c(self._lib.asap_read_counters(self._h, C.byref(a), C.byref(b), C.byref(c)))
+        return {"reduces": a.value, "consistent_inputs": b.value, "timeouts": c.value}
+
+    def get_graph(self, rnd: int = 0):
+        nbr = np.empty((self.N, self.k + 1), dtype=np.int32)
+        wgt = np.empty((self.N, self.k + 1), dtype=np.float32)
+        self._c(self._lib.asap_get_graph(self._h, rnd, _ptr(nbr), _ptr(wgt)))
+        return nbr, wgt
+
+    def set_wait_limit_ns(self, ns: int):
+        self._c(self._lib.asap_set_wait_limit_ns(self._h, ns))
+
+    def debug_skip_notify(self, worker: int):
+        self._c(self._lib.asap_debug_skip_notify(self._h, worker))
+
+    def kernel_launches(self) -> int:
+        v = C.c_uint64()
+        self._c(self._lib.asap_kernel_launches(self._h, C.byref(v)))
+        return v.value
+
+    def close(self):
+        if getattr(self, "_h", None):
+            self._lib.asap_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        self.close()

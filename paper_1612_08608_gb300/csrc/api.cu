@@ -1,0 +1,969 @@
+// Host runtime behind include/asap.h: context and device memory, graph
+// schedule, shard layout (index builder), launch sequencing of one ASAP
+// round (Eq. A.1), NOTIFY-ACK state and error reporting.
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <memory>
+#include <string>
+#include <thread>
+#include <vector>
+
+#include "asap_internal.h"
+
+namespace asap {
+int margin_ctas_for(int B);
+int update_ctas_for(int max_nnz);
+cudaError_t mix_occupancy(bool complete, int kp1, bool shadow, size_t smem, int* blocks);
+}  // namespace asap
+
+using namespace asap;
+
+namespace {
+
+thread_local std::string g_last_error;
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn get_encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  }
+  return fn;
+}
+
+inline size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+}  // namespace
+
+struct asap_ctx {
+  int dev = 0, sm_count = 0;
+  int N = 0;
+  int64_t d = 0;
+  uint64_t seed = 0;
+  int k = 0;
+  asap_graph_kind kind = ASAP_GRAPH_IDENTITY;
+  bool regen = false;
+  bool have_explicit = false;
+  std::vector<int32_t> ex_nbr;
+  std::vector<float> ex_wgt;
+  int tab_kp1 = 1;          // neighbours per row in the device tables (0 for COMPLETE)
+  int64_t graph_round_in_slot0 = -2;
+
+  asap_loss loss = ASAP_LOSS_NONE;
+  int C = 1, B = 0;
+  float lr = 0.f, l2 = 0.f;
+  int64_t P = 0, ld = 0;
+
+  float* W[2] = {nullptr, nullptr};
+  uint16_t* Wbf[2] = {nullptr, nullptr};
+  unsigned* ready = nullptr;
+  unsigned* consumed = nullptr;
+  unsigned* stamp = nullptr;     // [2][N]
+  unsigned* ticket = nullptr;    // [N]
+  DevState* st = nullptr;
+  float* m_loss = nullptr;
+  float* m_cons = nullptr;
+  float* r_scr = nullptr;
+  float* loss_part = nullptr;
+  double* cons_part = nullptr;
+  int cons_cap = 0;
+  int32_t* d_nbr = nullptr;
+  float* d_wgt = nullptr;
+  int32_t* h_nbr = nullptr;
+  float* h_wgt = nullptr;
+  cudaEvent_t slot_ev[kGraphRing];
+  bool slot_used[kGraphRing];
+
+  // sparse shards
+  asap_residency residency = ASAP_SHARDS_DEVICE;
+  unsigned char* pool = nullptr;  // device or pinned host
+  bool pool_pinned = false;
+  size_t pool_bytes = 0;
+  std::vector<size_t> block_off, block_bytes;
+  int nb = 0;
+  BatchDesc* d_desc = nullptr;
+  unsigned char* staging[2] = {nullptr, nullptr};
+  size_t staging_bytes = 0;
+  int64_t staged_round[2] = {-1, -1};
+  bool free_recorded[2] = {false, false};
+  cudaEvent_t staged_ev[2], free_ev[2];
+  int margin_ctas = 0, update_ctas = 0;
+  int max_nnz = 0;
+
+  cudaStream_t stream = nullptr, own_stream = nullptr, copy_stream = nullptr;
+
+  CUtensorMap tmap[2];
+  int S = 0, rows_pad = 0, box_rows = 0, n_boxes = 0, stages = 0;
+  long long n_slabs = 0;
+  int mix_grid = 0;
+  size_t mix_smem = 0;
+  int configured_key = -1;
+
+  int64_t round = 0;
+  int64_t graph_ready_round = -1;   // round whose tables are staged in graph_nbr/graph_wgt
+  const int* graph_nbr = nullptr;
+  const float* graph_wgt = nullptr;
+  bool step_pending = false;
+  int skip_notify = -1;
+  unsigned long long wait_ns = 200000000ull;
+  uint64_t launches = 0;
+  std::string err;
+};
+
+namespace {
+
+asap_status fail(asap_ctx* c, asap_status s, const std::string& msg) {
+  if (c) c->err = msg;
+  g_last_error = msg;
+  return s;
+}
+
+asap_status cuda_fail(asap_ctx* c, cudaError_t e, const char* what) {
+  std::string m = std::string(what) + ": " + cudaGetErrorString(e);
+  return fail(c, e == cudaErrorMemoryAllocation ? ASAP_ERR_OOM : ASAP_ERR_CUDA, m);
+}
+
+#define CU(call, what)                                   \
+  do {                                                   \
+    cudaError_t e_ = (call);                             \
+    if (e_ != cudaSuccess) return cuda_fail(c, e_, what); \
+  } while (0)
+
+template <typename T>
+void dfree(T*& p) {
+  if (p) cudaFree(p);
+  p = nullptr;
+}
+
+void free_shards(asap_ctx* c) {
+  if (c->pool) {
+    if (c->pool_pinned)
+      cudaFreeHost(c->pool);
+    else
+      cudaFree(c->pool);
+  }
+  c->pool = nullptr;
+  c->pool_bytes = 0;
+  dfree(c->d_desc);
+  dfree(c->staging[0]);
+  dfree(c->staging[1]);
+  c->block_off.clear();
+  c->block_bytes.clear();
+  c->nb = 0;
+  c->staged_round[0] = c->staged_round[1] = -1;
+  c->free_recorded[0] = c->free_recorded[1] = false;
+}
+
+// Host copy of the graph of round `rnd`: nbr/wgt with c->k + 1 entries per row.
+asap_status graph_host(asap_ctx* c, int64_t rnd, int32_t* nbr, float* wgt) {
+  const int kp1 = c->k + 1;
+  if (c->kind == ASAP_GRAPH_EXPLICIT) {
+    std::copy(c->ex_nbr.begin(), c->ex_nbr.end(), nbr);
+    if (wgt) std::copy(c->ex_wgt.begin(), c->ex_wgt.end(), wgt);
+    return ASAP_OK;
+  }
+  const char* why = "";
+  asap_status s = build_graph_host(c->kind, c->N, c->k, c->seed, c->regen ? rnd : 0, nbr, &why);
+  if (s != ASAP_OK) return fail(c, s, why);
+  if (wgt) std::fill(wgt, wgt + static_cast<size_t>(c->N) * kp1, 1.0f / static_cast<float>(kp1));
+  return ASAP_OK;
+}
+
+bool is_complete_kernel(const asap_ctx* c) { return c->kind == ASAP_GRAPH_COMPLETE; }
+
+asap_status setup_mix(asap_ctx* c) {
+  const int N = c->N;
+  c->n_boxes = (N + 255) / 256;
+  c->box_rows = (N + c->n_boxes - 1) / c->n_boxes;
+  c->rows_pad = c->n_boxes * c->box_rows;
+  int S = 256;
+  while (S > 8 && static_cast<size_t>(c->rows_pad) * S * 4 > 32768) S >>= 1;
+  int maxS = 8;
+  while (static_cast<int64_t>(maxS) * 2 <= c->ld && maxS < 256) maxS <<= 1;
+  c->S = std::min(S, maxS);
+  const size_t slab = align_up(static_cast<size_t>(c->rows_pad) * c->S * 4, 1024);
+  c->stages = static_cast<int>(std::max<size_t>(2, std::min<size_t>(8, 131072 / slab)));
+  c->n_slabs = (c->ld + c->S - 1) / c->S;
+  c->tab_kp1 = is_complete_kernel(c) ? 0 : c->k + 1;
+  c->mix_smem = mix_smem_bytes(N, c->tab_kp1, c->S, c->rows_pad, c->stages);
+  c->configured_key = -1;
+  EncodeTiledFn enc = get_encode_fn();
+  if (!enc) return fail(c, ASAP_ERR_CUDA, "cuTensorMapEncodeTiled is not available from the driver");
+  for (int b = 0; b < 2; ++b) {
+    cuuint64_t dims[2] = {static_cast<cuuint64_t>(c->ld), static_cast<cuuint64_t>(N)};
+    cuuint64_t strides[1] = {static_cast<cuuint64_t>(c->ld) * 4};
+    cuuint32_t box[2] = {static_cast<cuuint32_t>(c->S), static_cast<cuuint32_t>(c->box_rows)};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = enc(&c->tmap[b], CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, c->W[b], dims, strides, box, estr,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return fail(c, ASAP_ERR_CUDA, "cuTensorMapEncodeTiled failed for the parameter buffer");
+  }
+  return ASAP_OK;
+}
+
+asap_status configure_mix_launch(asap_ctx* c) {
+  const bool complete = is_complete_kernel(c);
+  const bool shadow = c->Wbf[0] != nullptr;
+  const int key = (complete ? 1 : 0) | (shadow ? 2 : 0) | (c->tab_kp1 << 2) | (static_cast<int>(c->mix_smem) << 8);
+  if (key == c->configured_key) return ASAP_OK;
+  CU(mix_configure(complete, c->tab_kp1, shadow, c->mix_smem), "configuring the reduce kernel");
+  int blocks = 0;
+  CU(mix_occupancy(complete, c->tab_kp1, shadow, c->mix_smem, &blocks), "occupancy of the reduce kernel");
+  if (blocks < 1) return fail(c, ASAP_ERR_ARG, "reduce kernel does not fit on an SM for this N");
+  c->mix_grid = static_cast<int>(std::min<long long>(c->n_slabs, static_cast<long long>(c->sm_count) * blocks));
+  if (c->mix_grid > c->cons_cap) return fail(c, ASAP_ERR_ARG, "internal: reduce grid exceeds its scratch");
+  c->configured_key = key;
+  return ASAP_OK;
+}
+
+asap_status reset_protocol(asap_ctx* c, int64_t rnd) {
+  std::vector<unsigned> v(c->N, static_cast<unsigned>(rnd));
+  CU(cudaMemcpy(c->ready, v.data(), 4 * c->N, cudaMemcpyHostToDevice), "resetting NOTIFY flags");
+  CU(cudaMemcpy(c->consumed, v.data(), 4 * c->N, cudaMemcpyHostToDevice), "resetting ACK flags");
+  CU(cudaMemcpy(c->stamp + (rnd & 1) * c->N, v.data(), 4 * c->N, cudaMemcpyHostToDevice), "resetting stamps");
+  CU(cudaMemset(c->ticket, 0, 4 * c->N), "resetting tickets");
+  c->round = rnd;
+  c->step_pending = false;
+  c->graph_ready_round = -1;
+  return ASAP_OK;
+}
+
+asap_status alloc_params(asap_ctx* c) {
+  CU(cudaStreamSynchronize(c->stream), "synchronising before re-allocation");
+  for (int b = 0; b < 2; ++b) {
+    dfree(c->W[b]);
+    dfree(c->Wbf[b]);
+  }
+  c->ld = static_cast<int64_t>(align_up(static_cast<size_t>(c->P), 64));
+  const size_t bytes = static_cast<size_t>(c->N) * c->ld * 4;
+  for (int b = 0; b < 2; ++b) {
+    CU(cudaMalloc(&c->W[b], bytes), "allocating the parameter buffers");
+    CU(cudaMemset(c->W[b], 0, bytes), "zeroing the parameter buffers");
+    if (c->loss == ASAP_LOSS_SOFTMAX) {
+      CU(cudaMalloc(&c->Wbf[b], bytes / 2), "allocating the bf16 parameter copy");
+      CU(cudaMemset(c->Wbf[b], 0, bytes / 2), "zeroing the bf16 parameter copy");
+    }
+  }
+  asap_status s = setup_mix(c);
+  if (s != ASAP_OK) return s;
+  return reset_protocol(c, 0);
+}
+
+asap_status upload_fixed_graph(asap_ctx* c) {
+  c->graph_round_in_slot0 = -2;
+  c->graph_ready_round = -1;
+  if (c->tab_kp1 == 0 || c->regen) return ASAP_OK;
+  const size_t n = static_cast<size_t>(c->N) * c->tab_kp1;
+  std::vector<int32_t> nbr(n);
+  std::vector<float> wgt(n);
+  asap_status s = graph_host(c, 0, nbr.data(), wgt.data());
+  if (s != ASAP_OK) return s;
+  CU(cudaStreamSynchronize(c->stream), "synchronising before a graph upload");
+  CU(cudaMemcpy(c->d_nbr, nbr.data(), n * 4, cudaMemcpyHostToDevice), "uploading the graph");
+  CU(cudaMemcpy(c->d_wgt, wgt.data(), n * 4, cudaMemcpyHostToDevice), "uploading the graph weights");
+  c->graph_round_in_slot0 = 0;
+  return ASAP_OK;
+}
+
+// Device tables for round `rnd` (regenerated graphs go through a ring of
+// pinned host slots and device slots; a slot is rewritten only after its
+// previous upload has completed).
+asap_status graph_tables(asap_ctx* c, int64_t rnd, const int** nbr, const float** wgt) {
+  *nbr = nullptr;
+  *wgt = nullptr;
+  if (c->tab_kp1 == 0) return ASAP_OK;
+  const size_t n = static_cast<size_t>(c->N) * c->tab_kp1;
+  if (!c->regen) {
+    *nbr = c->d_nbr;
+    *wgt = c->d_wgt;
+    return ASAP_OK;
+  }
+  const int slot = static_cast<int>(rnd % kGraphRing);
+  if (c->slot_used[slot]) CU(cudaEventSynchronize(c->slot_ev[slot]), "waiting for a graph slot");
+  int32_t* hn = c->h_nbr + slot * n;
+  float* hw = c->h_wgt + slot * n;
+  asap_status s = graph_host(c, rnd, hn, hw);
+  if (s != ASAP_OK) return s;
+  CU(cudaMemcpyAsync(c->d_nbr + slot * n, hn, n * 4, cudaMemcpyHostToDevice, c->stream), "graph upload");
+  CU(cudaMemcpyAsync(c->d_wgt + slot * n, hw, n * 4, cudaMemcpyHostToDevice, c->stream), "graph upload");
+  CU(cudaEventRecord(c->slot_ev[slot], c->stream), "graph upload event");
+  c->slot_used[slot] = true;
+  *nbr = c->d_nbr + slot * n;
+  *wgt = c->d_wgt + slot * n;
+  return ASAP_OK;
+}
+
+// Stage the graph of round r (no-op when it is already staged).
+asap_status prepare_graph(asap_ctx* c, int64_t r) {
+  if (c->graph_ready_round == r) return ASAP_OK;
+  asap_status s = graph_tables(c, r, &c->graph_nbr, &c->graph_wgt);
+  if (s != ASAP_OK) return s;
+  c->graph_ready_round = r;
+  return ASAP_OK;
+}
+
+asap_status check_device_error(asap_ctx* c) {
+  DevState h;
+  CU(cudaMemcpy(&h, c->st, sizeof(DevState), cudaMemcpyDeviceToHost), "reading device state");
+  if (h.err_code == 0) return ASAP_OK;
+  const unsigned zero = 0;
+  CU(cudaMemcpy(&c->st->err_code, &zero, 4, cudaMemcpyHostToDevice), "clearing device error");
+  char buf[200];
+  if (h.err_code == ASAP_ERR_TIMEOUT)
+    snprintf(buf, sizeof buf, "device: NOTIFY/ACK wait ran out (worker %u, round %u); parameters are undefined "
+             "until asap_write_params", h.err_worker, h.err_round);
+  else if (h.err_code == ASAP_ERR_STATE)
+    snprintf(buf, sizeof buf, "device: round stamp mismatch (worker %u, round %u)", h.err_worker, h.err_round);
+  else
+    snprintf(buf, sizeof buf, "device: error %u (worker %u, round %u)", h.err_code, h.err_worker, h.err_round);
+  return fail(c, static_cast<asap_status>(h.err_code), buf);
+}
+
+asap_status sync_all(asap_ctx* c) {
+  CU(cudaStreamSynchronize(c->stream), "synchronising the context stream");
+  if (c->copy_stream) CU(cudaStreamSynchronize(c->copy_stream), "synchronising the copy stream");
+  return check_device_error(c);
+}
+
+// Make round r's batch block available on the device (host residency).
+asap_status stage_block(asap_ctx* c, int64_t r) {
+  const int slot = static_cast<int>(r & 1);
+  if (c->staged_round[slot] == r) return ASAP_OK;
+  const int t = static_cast<int>(r % c->nb);
+  if (c->free_recorded[slot]) CU(cudaStreamWaitEvent(c->copy_stream, c->free_ev[slot], 0), "staging wait");
+  CU(cudaMemcpyAsync(c->staging[slot], c->pool + c->block_off[t], c->block_bytes[t], cudaMemcpyHostToDevice,
+                     c->copy_stream),
+     "copying a minibatch block to the device");
+  CU(cudaEventRecord(c->staged_ev[slot], c->copy_stream), "staging event");
+  c->staged_round[slot] = r;
+  return ASAP_OK;
+}
+
+}  // namespace
+
+// ---------------------------------------------------------------------------
+extern "C" {
+
+const char* asap_version(void) { return "asap-gb300 0.1 (sm_103a)"; }
+
+const char* asap_last_error(const asap_ctx* c) { return c ? c->err.c_str() : g_last_error.c_str(); }
+
+asap_status asap_build_graph(asap_graph_kind kind, int N, int k, uint64_t graph_seed, int64_t round,
+                             int32_t* nbr_out) {
+  if (!nbr_out || N < 1 || N > kMaxWorkers) return fail(nullptr, ASAP_ERR_ARG, "bad arguments to asap_build_graph");
+  const char* why = "";
+  asap_status s = build_graph_host(kind, N, k, graph_seed, round, nbr_out, &why);
+  if (s != ASAP_OK) return fail(nullptr, s, why);
+  return ASAP_OK;
+}
+
+asap_status asap_create(int N, int64_t d, uint64_t graph_seed, int k, asap_ctx** out) {
+  if (!out) return fail(nullptr, ASAP_ERR_ARG, "out is NULL");
+  *out = nullptr;
+  if (N < 1 || N > kMaxWorkers || d < 1 || k < 0 || k > N - 1)
+    return fail(nullptr, ASAP_ERR_ARG, "need 1 <= N <= 1024, d >= 1, 0 <= k <= N-1");
+  std::unique_ptr<asap_ctx> holder(new asap_ctx());
+  asap_ctx* c = holder.get();
+  c->N = N;
+  c->d = d;
+  c->seed = graph_seed;
+  c->k = k;
+  c->kind = (k == 0) ? ASAP_GRAPH_IDENTITY
+            : (k == N - 1) ? ASAP_GRAPH_COMPLETE
+            : (k == 1) ? ASAP_GRAPH_RING
+                       : ASAP_GRAPH_RANDOM_REGULAR;
+  if (c->kind == ASAP_GRAPH_RANDOM_REGULAR && k + 1 > kMaxKp1Sparse)
+    return fail(nullptr, ASAP_ERR_ARG, "k+1 > 32 is supported only for the complete graph");
+  c->P = d;
+  CU(cudaGetDevice(&c->dev), "cudaGetDevice");
+  CU(cudaDeviceGetAttribute(&c->sm_count, cudaDevAttrMultiProcessorCount, c->dev), "querying SM count");
+  CU(cudaStreamCreateWithFlags(&c->own_stream, cudaStreamNonBlocking), "creating a stream");
+  CU(cudaStreamCreateWithFlags(&c->copy_stream, cudaStreamNonBlocking), "creating a copy stream");
+  c->stream = c->own_stream;
+  for (int i = 0; i < kGraphRing; ++i) {
+    CU(cudaEventCreateWithFlags(&c->slot_ev[i], cudaEventDisableTiming), "creating events");
+    c->slot_used[i] = false;
+  }
+  for (int b = 0; b < 2; ++b) {
+    CU(cudaEventCreateWithFlags(&c->staged_ev[b], cudaEventDisableTiming), "creating events");
+    CU(cudaEventCreateWithFlags(&c->free_ev[b], cudaEventDisableTiming), "creating events");
+  }
+  CU(cudaMalloc(&c->ready, 4 * N), "allocating flags");
+  CU(cudaMalloc(&c->consumed, 4 * N), "allocating flags");
+  CU(cudaMalloc(&c->stamp, 8 * N), "allocating stamps");
+  CU(cudaMemset(c->stamp, 0, 8 * N), "zeroing stamps");
+  CU(cudaMalloc(&c->ticket, 4 * N), "allocating tickets");
+  CU(cudaMalloc(&c->st, sizeof(DevState)), "allocating device state");
+  CU(cudaMemset(c->st, 0, sizeof(DevState)), "zeroing device state");
+  CU(cudaMalloc(&c->m_loss, 4 * kMetricsCap), "allocating metrics");
+  CU(cudaMalloc(&c->m_cons, 4 * kMetricsCap), "allocating metrics");
+  CU(cudaMemset(c->m_loss, 0xff, 4 * kMetricsCap), "clearing metrics");
+  CU(cudaMemset(c->m_cons, 0xff, 4 * kMetricsCap), "clearing metrics");
+  c->cons_cap = c->sm_count * 32;
+  CU(cudaMalloc(&c->cons_part, 8 * static_cast<size_t>(c->cons_cap)), "allocating reduce scratch");
+  const int kp1_tab = std::min(k + 1, kMaxKp1Sparse);
+  const size_t ring = static_cast<size_t>(kGraphRing) * N * kp1_tab;
+  CU(cudaMalloc(&c->d_nbr, ring * 4), "allocating graph slots");
+  CU(cudaMalloc(&c->d_wgt, ring * 4), "allocating graph slots");
+  CU(cudaHostAlloc(&c->h_nbr, ring * 4, cudaHostAllocDefault), "allocating pinned graph slots");
+  CU(cudaHostAlloc(&c->h_wgt, ring * 4, cudaHostAllocDefault), "allocating pinned graph slots");
+  asap_status s = alloc_params(c);
+  if (s != ASAP_OK) {
+    g_last_error = c->err;
+    asap_destroy(holder.release());
+    return s;
+  }
+  s = upload_fixed_graph(c);
+  if (s != ASAP_OK) {
+    g_last_error = c->err;
+    asap_destroy(holder.release());
+    return s;
+  }
+  *out = holder.release();
+  return ASAP_OK;
+}
+
+void asap_destroy(asap_ctx* c) {
+  if (!c) return;
+  if (c->stream) cudaStreamSynchronize(c->stream);
+  if (c->copy_stream) cudaStreamSynchronize(c->copy_stream);
+  free_shards(c);
+  for (int b = 0; b < 2; ++b) {
+    dfree(c->W[b]);
+    dfree(c->Wbf[b]);
+  }
+  dfree(c->ready);
+  dfree(c->consumed);
+  dfree(c->stamp);
+  dfree(c->ticket);
+  dfree(c->st);
+  dfree(c->m_loss);
+  dfree(c->m_cons);
+  dfree(c->r_scr);
+  dfree(c->loss_part);
+  dfree(c->cons_part);
+  dfree(c->d_nbr);
+  dfree(c->d_wgt);
+  if (c->h_nbr) cudaFreeHost(c->h_nbr);
+  if (c->h_wgt) cudaFreeHost(c->h_wgt);
+  for (int i = 0; i < kGraphRing; ++i)
+    if (c->slot_ev[i]) cudaEventDestroy(c->slot_ev[i]);
+  for (int b = 0; b < 2; ++b) {
+    if (c->staged_ev[b]) cudaEventDestroy(c->staged_ev[b]);
+    if (c->free_ev[b]) cudaEventDestroy(c->free_ev[b]);
+  }
+  if (c->own_stream) cudaStreamDestroy(c->own_stream);
+  if (c->copy_stream) cudaStreamDestroy(c->copy_stream);
+  delete c;
+}
+
+asap_status asap_set_graph(asap_ctx* c, asap_graph_kind kind, int regenerate_every_round) {
+  if (!c) return fail(nullptr, ASAP_ERR_ARG, "ctx is NULL");
+  if (kind == ASAP_GRAPH_EXPLICIT && !c->have_explicit)
+    return fail(c, ASAP_ERR_ARG, "EXPLICIT needs asap_set_mixing");
+  if (kind == ASAP_GRAPH_EXPLICIT && regenerate_every_round)
+    return fail(c, ASAP_ERR_ARG, "an explicit graph cannot be regenerated");
+  if (kind != ASAP_GRAPH_EXPLICIT) {
+    std::vector<int32_t> probe(static_cast<size_t>(c->N) * (c->k + 1));
+    const char* why = "";
+    asap_status s = build_graph_host(kind, c->N, c->k, c->seed, 0, probe.data(), &why);
+    if (s != ASAP_OK) return fail(c, s, why);
+    if (kind != ASAP_GRAPH_COMPLETE && c->k + 1 > kMaxKp1Sparse)
+      return fail(c, ASAP_ERR_ARG, "k+1 > 32 is supported only for the complete graph");
+  }
+  asap_status s0 = asap_sync(c);
+  if (s0 != ASAP_OK) return s0;
+  c->kind = kind;
+  c->regen = regenerate_every_round != 0 && kind == ASAP_GRAPH_RANDOM_REGULAR;
+  asap_status s = setup_mix(c);
+  if (s != ASAP_OK) return s;
+  return upload_fixed_graph(c);
+}
+
+asap_status asap_set_mixing(asap_ctx* c, const int32_t* nbr, const float* wgt) {
+  if (!c || !nbr || !wgt) return fail(c, ASAP_ERR_ARG, "NULL argument");
+  const int N = c->N, kp1 = c->k + 1;
+  if (kp1 > kMaxKp1Sparse) return fail(c, ASAP_ERR_ARG, "explicit mixing supports k+1 <= 32");
+  std::vector<double> colsum(N, 0.0);
+  for (int i = 0; i < N; ++i) {
+    double rs = 0.0;
+    for (int m = 0; m < kp1; ++m) {
+      const int j = nbr[i * kp1 + m];
+      const float w = wgt[i * kp1 + m];
+      if (j < 0 || j >= N) return fail(c, ASAP_ERR_GRAPH, "neighbour id out of range");
+      if (m > 0 && j <= nbr[i * kp1 + m - 1]) return fail(c, ASAP_ERR_GRAPH, "rows must be strictly ascending");
+      if (!(w >= 0.f) || !std::isfinite(w)) return fail(c, ASAP_ERR_GRAPH, "weights must be finite and >= 0");
+      rs += w;
+      colsum[j] += w;
+    }
+    if (std::fabs(rs - 1.0) > 1e-6) return fail(c, ASAP_ERR_GRAPH, "a row of P does not sum to 1");
+  }
+  for (int j = 0; j < N; ++j)
+    if (std::fabs(colsum[j] - 1.0) > 1e-6)
+      return fail(c, ASAP_ERR_GRAPH, "a column of P does not sum to 1 (P must be doubly stochastic)");
+  asap_status s0 = asap_sync(c);
+  if (s0 != ASAP_OK) return s0;
+  c->ex_nbr.assign(nbr, nbr + static_cast<size_t>(N) * kp1);
+  c->ex_wgt.assign(wgt, wgt + static_cast<size_t>(N) * kp1);
+  c->have_explicit = true;
+  c->kind = ASAP_GRAPH_EXPLICIT;
+  c->regen = false;
+  asap_status s = setup_mix(c);
+  if (s != ASAP_OK) return s;
+  return upload_fixed_graph(c);
+}
+
+asap_status asap_set_model(asap_ctx* c, asap_loss loss, int num_classes, int batch, float lr, float l2) {
+  if (!c) return fail(nullptr, ASAP_ERR_ARG, "ctx is NULL");
+  if (loss != ASAP_LOSS_NONE && loss != ASAP_LOSS_HINGE && loss != ASAP_LOSS_LOGISTIC && loss != ASAP_LOSS_SOFTMAX)
+    return fail(c, ASAP_ERR_ARG, "unknown loss");
+  if (loss != ASAP_LOSS_NONE && (batch < 1 || batch > 65535 || !(lr > 0.f) || !(l2 >= 0.f) || !(lr * l2 < 1.f)))
+    return fail(c, ASAP_ERR_ARG, "need 1 <= batch <= 65535, lr > 0, l2 >= 0, lr*l2 < 1");
+  if (loss == ASAP_LOSS_SOFTMAX)
+    return fail(c, ASAP_ERR_ARG, "softmax regression needs the dense kernels, not built in this version");
+  if (loss != ASAP_LOSS_SOFTMAX && num_classes != 1) return fail(c, ASAP_ERR_ARG, "num_classes must be 1");
+  asap_status s0 = asap_sync(c);
+  if (s0 != ASAP_OK) return s0;
+  free_shards(c);
+  c->loss = loss;
+  c->C = num_classes;
+  c->B = batch;
+  c->lr = lr;
+  c->l2 = l2;
+  c->P = c->d;
+  asap_status s = alloc_params(c);
+  if (s != ASAP_OK) return s;
+  s = upload_fixed_graph(c);
+  if (s != ASAP_OK) return s;
+  dfree(c->r_scr);
+  dfree(c->loss_part);
+  if (loss != ASAP_LOSS_NONE) {
+    c->margin_ctas = margin_ctas_for(batch);
+    CU(cudaMalloc(&c->r_scr, 4 * static_cast<size_t>(c->N) * batch), "allocating step scratch");
+    CU(cudaMalloc(&c->loss_part, 4 * static_cast<size_t>(c->N) * c->margin_ctas), "allocating step scratch");
+  }
+  return ASAP_OK;
+}
+
+asap_status asap_set_stream(asap_ctx* c, void* s) {
+  if (!c) return fail(nullptr, ASAP_ERR_ARG, "ctx is NULL");
+  cudaStream_t ns = s ? static_cast<cudaStream_t>(s) : c->own_stream;
+  if (ns != c->stream) {
+    CU(cudaStreamSynchronize(c->stream), "synchronising the old stream");
+    c->stream = ns;
+  }
+  return ASAP_OK;
+}
+
+asap_status asap_set_shard_residency(asap_ctx* c, asap_residency r) {
+  if (!c) return fail(nullptr, ASAP_ERR_ARG, "ctx is NULL");
+  if (r != ASAP_SHARDS_DEVICE && r != ASAP_SHARDS_HOST) return fail(c, ASAP_ERR_ARG, "unknown residency");
+  if (r == c->residency) return ASAP_OK;
+  if (c->nb) {
+    // Move the loaded shards; the layout is the same in both places.
+    asap_status s0 = sync_all(c);
+    if (s0 != ASAP_OK) return s0;
+    unsigned char* np = nullptr;
+    if (r == ASAP_SHARDS_DEVICE) {
+      CU(cudaMalloc(&np, c->pool_bytes), "allocating device shard memory");
+      CU(cudaMemcpy(np, c->pool, c->pool_bytes, cudaMemcpyHostToDevice), "moving shards to the device");
+      cudaFreeHost(c->pool);
+      dfree(c->staging[0]);
+      dfree(c->staging[1]);
+    } else {
+      CU(cudaHostAlloc(&np, c->pool_bytes, cudaHostAllocDefault), "allocating pinned shard memory");
+      CU(cudaMemcpy(np, c->pool, c->pool_bytes, cudaMemcpyDeviceToHost), "moving shards to the host");
+      cudaFree(c->pool);
+      size_t mb = 0;
+      for (size_t b : c->block_bytes) mb = std::max(mb, b);
+      c->staging_bytes = mb;
+      for (int b = 0; b < 2; ++b) CU(cudaMalloc(&c->staging[b], mb), "allocating staging buffers");
+    }
+    c->pool = np;
+    c->pool_pinned = (r == ASAP_SHARDS_HOST);
+    c->staged_round[0] = c->staged_round[1] = -1;
+    c->free_recorded[0] = c->free_recorded[1] = false;
+  }
+  c->residency = r;
+  return ASAP_OK;
+}
+
+asap_status asap_shard_block_bytes(asap_ctx* c, int64_t round, uint64_t* bytes) {
+  if (!c || !bytes || round < 0) return fail(c, ASAP_ERR_ARG, "bad argument");
+  if (!c->nb) return fail(c, ASAP_ERR_ARG, "no shards loaded");
+  *bytes = c->block_bytes[static_cast<size_t>(round % c->nb)];
+  return ASAP_OK;
+}
+
+asap_status asap_load_shards(asap_ctx* c, const int64_t* const* rowptr, const int32_t* const* col,
+                             const float* const* val, const float* const* y, const int64_t* n_rows) {
+  if (!c || !rowptr || !col || !val || !y || !n_rows) return fail(c, ASAP_ERR_ARG, "NULL argument");
+  if (c->loss != ASAP_LOSS_HINGE && c->loss != ASAP_LOSS_LOGISTIC)
+    return fail(c, ASAP_ERR_ARG, "set a hinge or logistic model before loading CSR shards");
+  const int N = c->N, B = c->B;
+  int nb = -1;
+  for (int i = 0; i < N; ++i) {
+    if (!rowptr[i] || !col[i] || !val[i] || !y[i]) return fail(c, ASAP_ERR_ARG, "NULL shard pointer");
+    if (n_rows[i] < B) return fail(c, ASAP_ERR_ARG, "a shard has fewer rows than one minibatch");
+    const int64_t nbi = n_rows[i] / B;
+    if (nb >= 0 && nbi != nb) return fail(c, ASAP_ERR_ARG, "all shards must hold the same number of minibatches");
+    nb = static_cast<int>(std::min<int64_t>(nbi, 1 << 30));
+    if (rowptr[i][0] != 0) return fail(c, ASAP_ERR_ARG, "rowptr must start at 0");
+  }
+  asap_status s0 = asap_sync(c);
+  if (s0 != ASAP_OK) return s0;
+  free_shards(c);
+
+  // Pass 1: sizes.  Segment (t, i) = rp | y | col | val | ccol | cval | crow.
+  std::vector<BatchDesc> desc(static_cast<size_t>(nb) * N);
+  c->block_off.assign(nb, 0);
+  c->block_bytes.assign(nb, 0);
+  size_t total = 0, max_block = 0;
+  int max_nnz = 0;
+  for (int t = 0; t < nb; ++t) {
+    size_t off = 0;
+    for (int i = 0; i < N; ++i) {
+      const int64_t* rp = rowptr[i];
+      const int64_t r0 = static_cast<int64_t>(t) * B;
+      int64_t nnz = 0, nnz_pad = 0;
+      for (int b = 0; b < B; ++b) {
+        const int64_t len = rp[r0 + b + 1] - rp[r0 + b];
+        if (len < 0) return fail(c, ASAP_ERR_ARG, "rowptr must be non-decreasing");
+        nnz += len;
+        nnz_pad += (len + 3) / 4 * 4;
+      }
+      if (nnz_pad > (1ll << 30)) return fail(c, ASAP_ERR_ARG, "a minibatch holds more than 2^30 entries");
+      BatchDesc& dd = desc[static_cast<size_t>(t) * N + i];
+      dd.rp = static_cast<int64_t>(off);
+      off = align_up(off + 4 * static_cast<size_t>(B + 1), 16);
+      dd.y = static_cast<int64_t>(off);
+      off = align_up(off + 4 * static_cast<size_t>(B), 16);
+      dd.col = static_cast<int64_t>(off);
+      off += 4 * static_cast<size_t>(nnz_pad);
+      dd.val = static_cast<int64_t>(off);
+      off += 4 * static_cast<size_t>(nnz_pad);
+      dd.ccol = static_cast<int64_t>(off);
+      off = align_up(off + 4 * static_cast<size_t>(nnz), 16);
+      dd.cval = static_cast<int64_t>(off);
+      off = align_up(off + 4 * static_cast<size_t>(nnz), 16);
+      dd.crow = static_cast<int64_t>(off);
+      off = align_up(off + 2 * static_cast<size_t>(nnz), 16);
+      dd.nnz_pad = static_cast<int32_t>(nnz_pad);
+      dd.nnz = static_cast<int32_t>(nnz);
+      max_nnz = std::max<int>(max_nnz, static_cast<int>(nnz));
+    }
+    off = align_up(off, 256);
+    c->block_off[t] = total;
+    c->block_bytes[t] = off;
+    total += off;
+    max_block = std::max(max_block, off);
+  }
+
+  // Host image of the pool: pinned when it stays on the host.
+  unsigned char* host = nullptr;
+  std::vector<unsigned char> pageable;
+  if (c->residency == ASAP_SHARDS_HOST) {
+    CU(cudaHostAlloc(&host, total, cudaHostAllocDefault), "allocating pinned shard memory");
+    c->pool = host;
+    c->pool_pinned = true;
+  } else {
+    pageable.resize(total);
+    host = pageable.data();
+  }
+
+  // Pass 2: fill, in parallel over (t, i) segments.
+  const int64_t d = c->d;
+  std::vector<int> bad(static_cast<size_t>(nb) * N, 0);
+  auto fill = [&](size_t seg) {
+    const int t = static_cast<int>(seg / N), i = static_cast<int>(seg % N);
+    const BatchDesc& dd = desc[seg];
+    unsigned char* base = host + c->block_off[t];
+    int32_t* rp_o = reinterpret_cast<int32_t*>(base + dd.rp);
+    float* y_o = reinterpret_cast<float*>(base + dd.y);
+    int32_t* col_o = reinterpret_cast<int32_t*>(base + dd.col);
+    float* val_o = reinterpret_cast<float*>(base + dd.val);
+    int32_t* ccol_o = reinterpret_cast<int32_t*>(base + dd.ccol);
+    float* cval_o = reinterpret_cast<float*>(base + dd.cval);
+    uint16_t* crow_o = reinterpret_cast<uint16_t*>(base + dd.crow);
+    const int64_t* rp = rowptr[i];
+    const int64_t r0 = static_cast<int64_t>(t) * B;
+    std::vector<uint64_t> keys;
+    keys.reserve(dd.nnz);
+    std::vector<uint16_t> row_of;
+    row_of.reserve(dd.nnz);
+    std::vector<float> vals;
+    vals.reserve(dd.nnz);
+    int32_t q = 0;
+    for (int b = 0; b < B; ++b) {
+      rp_o[b] = q;
+      y_o[b] = y[i][r0 + b];
+      const int64_t a0 = rp[r0 + b], a1 = rp[r0 + b + 1];
+      for (int64_t e = a0; e < a1; ++e) {
+        const int32_t cc = col[i][e];
+        if (cc < 0 || cc >= d) bad[seg] = 1;
+        col_o[q] = cc;
+        val_o[q] = val[i][e];
+        keys.push_back((static_cast<uint64_t>(static_cast<uint32_t>(cc)) << 32) | keys.size());
+        row_of.push_back(static_cast<uint16_t>(b));
+        vals.push_back(val[i][e]);
+        ++q;
+      }
+      while (q & 3) {   // pad the row to a multiple of 4 entries
+        col_o[q] = 0;
+        val_o[q] = 0.f;
+        ++q;
+      }
+    }
+    rp_o[B] = q;
+    std::sort(keys.begin(), keys.end());   // by column, then by position (= by row)
+    for (size_t e = 0; e < keys.size(); ++e) {
+      const uint32_t pos = static_cast<uint32_t>(keys[e] & 0xffffffffu);
+      ccol_o[e] = static_cast<int32_t>(keys[e] >> 32);
+      cval_o[e] = vals[pos];
+      crow_o[e] = row_of[pos];
+    }
+  };
+  {
+    const size_t nseg = desc.size();
+    const unsigned nthr = std::max(1u, std::min(32u, std::thread::hardware_concurrency()));
+    std::vector<std::thread> pool;
+    for (unsigned w = 0; w < nthr; ++w)
+      pool.emplace_back([&, w]() {
+        for (size_t s = w; s < nseg; s += nthr) fill(s);
+      });
+    for (auto& th : pool) th.join();
+  }
+  for (int v : bad)
+    if (v) {
+      free_shards(c);
+      return fail(c, ASAP_ERR_ARG, "column id out of range [0, d)");
+    }
+
+  if (c->residency == ASAP_SHARDS_DEVICE) {
+    CU(cudaMalloc(&c->pool, total), "allocating device shard memory");
+    c->pool_pinned = false;
+    CU(cudaMemcpy(c->pool, host, total, cudaMemcpyHostToDevice), "copying shards to the device");
+  } else {
+    c->staging_bytes = max_block;
+    for (int b = 0; b < 2; ++b) CU(cudaMalloc(&c->staging[b], max_block), "allocating staging buffers");
+  }
+  c->pool_bytes = total;
+  CU(cudaMalloc(&c->d_desc, desc.size() * sizeof(BatchDesc)), "allocating batch descriptors");
+  CU(cudaMemcpy(c->d_desc, desc.data(), desc.size() * sizeof(BatchDesc), cudaMemcpyHostToDevice),
+     "copying batch descriptors");
+  c->nb = nb;
+  c->max_nnz = max_nnz;
+  c->update_ctas = update_ctas_for(max_nnz);
+  return ASAP_OK;
+}
+
+asap_status asap_load_dense_shards(asap_ctx* c, const uint16_t* const*, const int32_t* const*, const int64_t*) {
+  return fail(c, ASAP_ERR_ARG, "dense shards need the softmax kernels, not built in this version");
+}
+
+asap_status asap_local_step(asap_ctx* c) {
+  if (!c) return fail(nullptr, ASAP_ERR_ARG, "ctx is NULL");
+  if (c->loss == ASAP_LOSS_NONE) return fail(c, ASAP_ERR_ARG, "no model set (asap_set_model)");
+  if (!c->nb) return fail(c, ASAP_ERR_ARG, "no shards loaded");
+  if (c->step_pending) return fail(c, ASAP_ERR_ARG, "local step already taken this round; reduce first");
+  const int64_t r = c->round;
+  const int t = static_cast<int>(r % c->nb);
+  const unsigned char* block;
+  if (c->residency == ASAP_SHARDS_HOST) {
+    asap_status s = stage_block(c, r);
+    if (s != ASAP_OK) return s;
+    CU(cudaStreamWaitEvent(c->stream, c->staged_ev[r & 1], 0), "waiting for the staged block");
+    block = c->staging[r & 1];
+  } else {
+    block = c->pool + c->block_off[t];
+  }
+  SparseStepArgs a;
+  a.block = block;
+  a.desc = c->d_desc + static_cast<size_t>(t) * c->N;
+  a.W = c->W[r & 1];
+  a.ld = c->ld;
+  a.r = c->r_scr;
+  a.loss_part = c->loss_part;
+  a.ready = c->ready;
+  a.worker_ticket = c->ticket;
+  a.B = c->B;
+  a.scale = c->lr / (static_cast<float>(c->B) * (1.0f - c->lr * c->l2));
+  a.round = static_cast<unsigned>(r);
+  a.skip_worker = c->skip_notify;
+  c->skip_notify = -1;
+  asap_status sg = prepare_graph(c, r);   // upload a regenerated graph ahead of the reduce
+  if (sg != ASAP_OK) return sg;
+  CU(launch_sparse_step(a, c->N, c->loss, c->margin_ctas, c->update_ctas, c->stream), "launching the local step");
+  c->launches += 2;
+  c->step_pending = true;
+  if (c->residency == ASAP_SHARDS_HOST) {
+    CU(cudaEventRecord(c->free_ev[r & 1], c->stream), "staging event");
+    c->free_recorded[r & 1] = true;
+    asap_status s = stage_block(c, r + 1);   // prefetch the next round's block
+    if (s != ASAP_OK) return s;
+  }
+  return ASAP_OK;
+}
+
+asap_status asap_stochastic_reduce(asap_ctx* c) {
+  if (!c) return fail(nullptr, ASAP_ERR_ARG, "ctx is NULL");
+  const int64_t r = c->round;
+  asap_status s = configure_mix_launch(c);
+  if (s != ASAP_OK) return s;
+  s = prepare_graph(c, r);
+  if (s != ASAP_OK) return s;
+  const int* nbr = c->graph_nbr;
+  const float* wgt = c->graph_wgt;
+  c->graph_ready_round = -1;
+  MixArgs a;
+  a.out = c->W[(r + 1) & 1];
+  a.shadow = c->Wbf[(r + 1) & 1];
+  a.ld = c->ld;
+  a.N = c->N;
+  a.kp1 = c->tab_kp1;
+  a.nbr = nbr;
+  a.wgt = wgt;
+  a.wscale = c->step_pending ? (1.0f - c->lr * c->l2) : 1.0f;
+  a.S = c->S;
+  a.rows_pad = c->rows_pad;
+  a.box_rows = c->box_rows;
+  a.n_boxes = c->n_boxes;
+  a.stages = c->stages;
+  a.n_slabs = c->n_slabs;
+  a.cons_part = c->cons_part;
+  a.loss_part = c->loss_part;
+  a.n_loss_part = c->step_pending ? c->N * c->margin_ctas : 0;
+  a.loss_norm = c->B > 0 ? 1.0f / (static_cast<float>(c->N) * static_cast<float>(c->B)) : 0.f;
+  a.have_loss = c->step_pending ? 1 : 0;
+  a.metrics_loss = c->m_loss;
+  a.metrics_cons = c->m_cons;
+  a.ready = c->ready;
+  a.consumed = c->consumed;
+  a.stamp_next = c->stamp + ((r + 1) & 1) * c->N;
+  a.st = c->st;
+  a.round = static_cast<unsigned>(r);
+  a.expect_notify = c->step_pending ? 1 : 0;
+  a.wait_ns = c->wait_ns;
+  CU(launch_mix(c->tmap[r & 1], a, is_complete_kernel(c), c->mix_grid, c->mix_smem, c->stream),
+     "launching the stochastic reduce");
+  c->launches += 1;
+  c->round = r + 1;
+  c->step_pending = false;
+  return ASAP_OK;
+}
+
+asap_status asap_round(asap_ctx* c, int T) {
+  if (!c) return fail(nullptr, ASAP_ERR_ARG, "ctx is NULL");
+  if (T < 0) return fail(c, ASAP_ERR_ARG, "T must be >= 0");
+  for (int t = 0; t < T; ++t) {
+    if (c->loss != ASAP_LOSS_NONE) {
+      asap_status s = asap_local_step(c);
+      if (s != ASAP_OK) return s;
+    }
+    asap_status s = asap_stochastic_reduce(c);
+    if (s != ASAP_OK) return s;
+  }
+  return ASAP_OK;
+}
+
+asap_status asap_sync(asap_ctx* c) {
+  if (!c) return fail(nullptr, ASAP_ERR_ARG, "ctx is NULL");
+  return sync_all(c);
+}
+
+asap_status asap_read_params(asap_ctx* c, float* host_out, int64_t* round_out) {
+  if (!c || !host_out) return fail(c, ASAP_ERR_ARG, "NULL argument");
+  asap_status s = sync_all(c);
+  if (s != ASAP_OK) return s;
+  CU(cudaMemcpy2D(host_out, c->P * 4, c->W[c->round & 1], c->ld * 4, c->P * 4, c->N, cudaMemcpyDeviceToHost),
+     "reading parameters");
+  if (round_out) *round_out = c->round;
+  return ASAP_OK;
+}
+
+asap_status asap_write_params(asap_ctx* c, const float* host_in, int64_t round) {
+  if (!c || !host_in || round < 0) return fail(c, ASAP_ERR_ARG, "bad argument");
+  asap_status s = sync_all(c);
+  if (s != ASAP_OK) return s;
+  float* dst = c->W[round & 1];
+  CU(cudaMemcpy2D(dst, c->ld * 4, host_in, c->P * 4, c->P * 4, c->N, cudaMemcpyHostToDevice), "writing parameters");
+  if (c->Wbf[round & 1]) {
+    CU(launch_cast_bf16(dst, c->Wbf[round & 1], static_cast<int64_t>(c->N) * c->ld, c->stream), "bf16 copy");
+    c->launches += 1;
+    CU(cudaStreamSynchronize(c->stream), "bf16 copy");
+  }
+  return reset_protocol(c, round);
+}
+
+asap_status asap_read_metrics(asap_ctx* c, int64_t first, int64_t count, float* loss_out, float* cons_out) {
+  if (!c || first < 0 || count < 0) return fail(c, ASAP_ERR_ARG, "bad argument");
+  if (first + count > c->round || first < c->round - kMetricsCap)
+    return fail(c, ASAP_ERR_ARG, "rounds outside the kept metrics window");
+  asap_status s = sync_all(c);
+  if (s != ASAP_OK) return s;
+  for (int64_t r = first; r < first + count;) {
+    const int64_t slot = r % kMetricsCap;
+    const int64_t n = std::min<int64_t>(first + count - r, kMetricsCap - slot);
+    if (loss_out) CU(cudaMemcpy(loss_out + (r - first), c->m_loss + slot, 4 * n, cudaMemcpyDeviceToHost), "metrics");
+    if (cons_out) CU(cudaMemcpy(cons_out + (r - first), c->m_cons + slot, 4 * n, cudaMemcpyDeviceToHost), "metrics");
+    r += n;
+  }
+  return ASAP_OK;
+}
+
+asap_status asap_read_counters(asap_ctx* c, uint64_t* reduces, uint64_t* consistent, uint64_t* timeouts) {
+  if (!c) return fail(nullptr, ASAP_ERR_ARG, "ctx is NULL");
+  CU(cudaStreamSynchronize(c->stream), "synchronising");
+  DevState h;
+  CU(cudaMemcpy(&h, c->st, sizeof h, cudaMemcpyDeviceToHost), "reading counters");
+  if (reduces) *reduces = h.reduces;
+  if (consistent) *consistent = h.consistent_inputs;
+  if (timeouts) *timeouts = h.timeouts;
+  return ASAP_OK;
+}
+
+asap_status asap_get_graph(asap_ctx* c, int64_t round, int32_t* nbr_out, float* wgt_out) {
+  if (!c || round < 0) return fail(c, ASAP_ERR_ARG, "bad argument");
+  const size_t n = static_cast<size_t>(c->N) * (c->k + 1);
+  std::vector<int32_t> nbr(n);
+  std::vector<float> wgt(n);
+  asap_status s = graph_host(c, round, nbr.data(), wgt.data());
+  if (s != ASAP_OK) return s;
+  if (nbr_out) std::copy(nbr.begin(), nbr.end(), nbr_out);
+  if (wgt_out) std::copy(wgt.begin(), wgt.end(), wgt_out);
+  return ASAP_OK;
+}
+
+asap_status asap_set_wait_limit_ns(asap_ctx* c, uint64_t ns) {
+  if (!c || ns == 0) return fail(c, ASAP_ERR_ARG, "bad argument");
+  c->wait_ns = ns;
+  return ASAP_OK;
+}
+
+asap_status asap_debug_skip_notify(asap_ctx* c, int worker) {
+  if (!c || worker < -1 || worker >= c->N) return fail(c, ASAP_ERR_ARG, "bad worker");
+  c->skip_notify = worker;
+  return ASAP_OK;
+}
+
+asap_status asap_kernel_launches(asap_ctx* c, uint64_t* launches) {
+  if (!c || !launches) return fail(c, ASAP_ERR_ARG, "NULL argument");
+  *launches = c->launches;
+  return ASAP_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,108 @@
+// Internal declarations shared by the host runtime and the kernels of the
+// ASAP library.  Nothing here is part of the public ABI (include/asap.h).
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <cstdint>
+#include <string>
+#include <vector>
+
+#include "asap.h"
+
+namespace asap {
+
+constexpr int kMaxWorkers = 1024;
+constexpr int kMaxKp1Sparse = 32;     // neighbours per row for the sparse reduce
+constexpr int kMetricsCap = 65536;    // rounds of metrics kept on the device
+constexpr int kGraphRing = 64;        // device slots for per-round graphs
+constexpr int kThreads = 256;         // block size of every kernel here
+
+// Device-side protocol and error state (one per context).
+struct DevState {
+  unsigned int err_code;     // first asap_status raised on the device (0 = none)
+  unsigned int err_worker;
+  unsigned int err_round;
+  unsigned int mix_ticket;   // CTAs of the current reduce that have finished
+  unsigned long long reduces;
+  unsigned long long consistent_inputs;
+  unsigned long long timeouts;
+};
+
+// Where one worker's minibatch lives inside a batch block (byte offsets from
+// the block start).  Rows are padded to multiples of 4 entries (16 B) with
+// col = 0, val = 0 so that the margin kernel can use 128-bit loads.
+struct BatchDesc {
+  int64_t rp;     // int32 [B+1]: padded row starts, in entries
+  int64_t y;      // float [B]
+  int64_t col;    // int32 [nnz_pad]
+  int64_t val;    // float [nnz_pad]
+  int64_t ccol;   // int32 [nnz]: entries sorted by (column, row)
+  int64_t cval;   // float [nnz]
+  int64_t crow;   // uint16 [nnz]: row within the batch
+  int32_t nnz_pad;
+  int32_t nnz;
+};
+
+// Arguments of the sparse local step (margin kernel, then update kernel).
+struct SparseStepArgs {
+  const unsigned char* block;  // batch block of this round
+  const BatchDesc* desc;       // [N] descriptors of this round's batch
+  float* W;                    // current parameter buffer, rows of ld floats
+  int64_t ld;
+  float* r;                    // scratch [N][B]: d loss / d margin
+  float* loss_part;            // scratch [N][margin CTAs per worker]
+  unsigned int* ready;         // NOTIFY flags [N]
+  unsigned int* worker_ticket; // [N] finished update CTAs of this round
+  int B;
+  float scale;                 // eta / (B (1 - eta l2))
+  unsigned int round;
+  int skip_worker;             // fault injection: do not NOTIFY this worker
+};
+
+// Arguments of the stochastic reduce.
+struct MixArgs {
+  float* out;                  // next parameter buffer
+  uint16_t* shadow;            // bf16 copy of `out` (softmax) or nullptr
+  int64_t ld;                  // row stride of W (floats), multiple of 64
+  int N;
+  int kp1;                     // neighbours per row (sparse kind)
+  const int* nbr;              // [N][kp1]
+  const float* wgt;            // [N][kp1]
+  float wscale;                // (1 - eta l2) after a local step, else 1
+  int S;                       // slab width (columns)
+  int rows_pad;                // smem rows per slab (box_rows * n_boxes)
+  int box_rows;
+  int n_boxes;
+  int stages;
+  long long n_slabs;
+  double* cons_part;           // scratch [gridDim.x]
+  const float* loss_part;      // [n_loss_part] from the margin kernel
+  int n_loss_part;
+  float loss_norm;             // 1 / (N B)
+  int have_loss;
+  float* metrics_loss;         // ring of kMetricsCap
+  float* metrics_cons;
+  unsigned int* ready;
+  unsigned int* consumed;
+  unsigned int* stamp_next;    // [N] stamp of the buffer being written
+  DevState* st;
+  unsigned int round;
+  int expect_notify;
+  unsigned long long wait_ns;
+};
+
+asap_status build_graph_host(asap_graph_kind kind, int N, int k, uint64_t seed, int64_t round,
+                             int32_t* nbr, const char** why);
+
+// Launchers (kernels_*.cu).  Each returns the cudaError_t of the launch.
+cudaError_t launch_sparse_step(const SparseStepArgs& a, int N, int loss, int margin_ctas, int update_ctas,
+                               cudaStream_t s);
+cudaError_t launch_mix(const CUtensorMap& tmap, const MixArgs& a, bool complete, int grid, size_t smem,
+                       cudaStream_t s);
+size_t mix_smem_bytes(int N, int kp1, int S, int rows_pad, int stages);
+cudaError_t mix_configure(bool complete, int kp1, bool shadow, size_t smem);
+cudaError_t launch_cast_bf16(const float* src, uint16_t* dst, int64_t n, cudaStream_t s);
+
+}  // namespace asap

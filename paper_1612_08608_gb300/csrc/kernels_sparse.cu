@@ -1,0 +1,208 @@
+// Local minibatch SGD step for sparse linear models (Eq. A.1, first line):
+//   m_b = x_b . w_i                                  (margin kernel)
+//   r_b = d loss(y_b, m_b) / d m_b                   (hinge or logistic)
+//   w_i[c] -= eta/B * sum_{b : c in x_b} r_b x_{b,c} (update kernel)
+// followed by NOTIFY: the last update CTA of worker i publishes
+// ready[i] = t+1 with release semantics (Section 4, NOTIFY-ACK).
+//
+// Margin kernel: one warp per row, 128-bit loads of column ids and values
+// (rows are padded to 4 entries), gathers of w[col], a fixed butterfly sum.
+// Update kernel: entries of the minibatch sorted by (column, row) are cut
+// into 32-entry chunks, one warp per chunk; a segmented warp scan sums each
+// column's run, and the warp that holds the first entry of a column owns
+// that column: it finishes runs that cross into later chunks itself.  No
+// global atomics touch W and every sum has a fixed order, so the result
+// does not depend on the schedule.
+#include <cuda_runtime.h>
+
+#include <climits>
+#include <cstdint>
+
+#include "asap_internal.h"
+
+namespace asap {
+
+namespace {
+
+constexpr unsigned kFull = 0xffffffffu;
+constexpr int kMarginRowsPerCta = 32;     // 8 warps x 4 rows
+constexpr int kUpdateChunksPerCta = 32;   // 8 warps x 4 chunks of 32 entries
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(kFull, v, o);
+  return v;
+}
+
+__device__ __forceinline__ int4 ld_stream_i4(const int4* p) {
+  int4 v;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.s32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "l"(p));
+  return v;
+}
+
+__device__ __forceinline__ float4 ld_stream_f4(const float4* p) {
+  float4 v;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.f32 {%0,%1,%2,%3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "l"(p));
+  return v;
+}
+
+__device__ __forceinline__ void st_release_u32(unsigned int* p, unsigned int v) {
+  asm volatile("st.release.gpu.global.u32 [%0], %1;" :: "l"(p), "r"(v) : "memory");
+}
+
+// loss(y, m) and r = d loss / d m.
+template <int LOSS>
+__device__ __forceinline__ void loss_and_r(float y, float m, float& l, float& r) {
+  const float z = y * m;
+  if (LOSS == ASAP_LOSS_HINGE) {
+    l = fmaxf(0.f, 1.f - z);
+    r = (z < 1.f) ? -y : 0.f;                 // strict: the corner z = 1 takes r = 0
+  } else {
+    // ln(1 + e^{-z}) = max(-z, 0) + ln(1 + e^{-|z|});  sigmoid(-z) = 1 / (1 + e^{z})
+    l = fmaxf(-z, 0.f) + log1pf(expf(-fabsf(z)));
+    r = -y / (1.f + expf(z));
+  }
+}
+
+template <int LOSS>
+__global__ void __launch_bounds__(kThreads) k_margin_loss(SparseStepArgs a) {
+  const int i = blockIdx.y;
+  const BatchDesc dsc = a.desc[i];
+  const int* rp = reinterpret_cast<const int*>(a.block + dsc.rp);
+  const float* y = reinterpret_cast<const float*>(a.block + dsc.y);
+  const int4* col4 = reinterpret_cast<const int4*>(a.block + dsc.col);
+  const float4* val4 = reinterpret_cast<const float4*>(a.block + dsc.val);
+  const float* w = a.W + static_cast<int64_t>(i) * a.ld;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int row_end = min(a.B, static_cast<int>(blockIdx.x + 1) * kMarginRowsPerCta);
+  float lsum = 0.f;
+  for (int b = blockIdx.x * kMarginRowsPerCta + warp; b < row_end; b += kThreads / 32) {
+    const int q0 = rp[b] >> 2, q1 = rp[b + 1] >> 2;
+    float acc = 0.f;
+    for (int q = q0 + lane; q < q1; q += 32) {
+      const int4 c = ld_stream_i4(col4 + q);
+      const float4 v = ld_stream_f4(val4 + q);
+      acc = fmaf(v.x, __ldg(w + c.x), acc);
+      acc = fmaf(v.y, __ldg(w + c.y), acc);
+      acc = fmaf(v.z, __ldg(w + c.z), acc);
+      acc = fmaf(v.w, __ldg(w + c.w), acc);
+    }
+    const float m = warp_sum(acc);
+    if (lane == 0) {
+      float l, r;
+      loss_and_r<LOSS>(y[b], m, l, r);
+      a.r[static_cast<int64_t>(i) * a.B + b] = r;
+      lsum += l;
+    }
+  }
+  __shared__ float part[kThreads / 32];
+  if (lane == 0) part[warp] = lsum;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float s = 0.f;
+#pragma unroll
+    for (int k = 0; k < kThreads / 32; ++k) s += part[k];
+    a.loss_part[static_cast<int64_t>(i) * gridDim.x + blockIdx.x] = s;
+  }
+}
+
+__global__ void __launch_bounds__(kThreads) k_segment_update(SparseStepArgs a) {
+  const int i = blockIdx.y;
+  const BatchDesc dsc = a.desc[i];
+  const int nnz = dsc.nnz;
+  const int* ccol = reinterpret_cast<const int*>(a.block + dsc.ccol);
+  const float* cval = reinterpret_cast<const float*>(a.block + dsc.cval);
+  const uint16_t* crow = reinterpret_cast<const uint16_t*>(a.block + dsc.crow);
+  const float* r = a.r + static_cast<int64_t>(i) * a.B;
+  float* w = a.W + static_cast<int64_t>(i) * a.ld;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const unsigned le_mask = (lane == 31) ? kFull : ((2u << lane) - 1u);
+
+  const int n_chunks = (nnz + 31) >> 5;
+  for (int first = blockIdx.x * kUpdateChunksPerCta; first < n_chunks; first += gridDim.x * kUpdateChunksPerCta)
+  for (int j = warp; j < kUpdateChunksPerCta; j += kThreads / 32) {
+    const int chunk = first + j;
+    if (chunk >= n_chunks) break;                  // warp-uniform
+    const int e = chunk * 32 + lane;
+    const bool valid = e < nnz;
+    const int c = valid ? ccol[e] : -1;
+    int cprev = __shfl_up_sync(kFull, c, 1);
+    if (lane == 0) cprev = (e > 0) ? ccol[e - 1] : -2;
+    const bool head = valid && (c != cprev);
+    float p = valid ? r[crow[e]] * cval[e] : 0.f;
+    const unsigned heads = __ballot_sync(kFull, head);
+    const unsigned hl = heads & le_mask;
+    const int start = hl ? (31 - __clz(hl)) : -1;   // first lane of this lane's run, -1: began earlier
+    const int s_eff = start < 0 ? 0 : start;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const float v = __shfl_up_sync(kFull, p, off);
+      if (lane - off >= s_eff) p += v;
+    }
+    const bool next_head = __shfl_down_sync(kFull, head, 1);
+    const bool next_valid = __shfl_down_sync(kFull, valid, 1);
+    // Runs that end inside the chunk: the tail lane writes if the run began here.
+    if (valid && lane < 31 && (next_head || !next_valid) && start >= 0) {
+      w[c] = fmaf(-a.scale, p, w[c]);
+    }
+    // The run through lane 31.
+    const int c31 = __shfl_sync(kFull, c, 31);
+    const int start31 = __shfl_sync(kFull, start, 31);
+    const float p31 = __shfl_sync(kFull, p, 31);
+    if (c31 >= 0 && start31 >= 0) {
+      const int e31 = chunk * 32 + 31;
+      bool cont = (e31 + 1 < nnz) && (ccol[e31 + 1] == c31);
+      float acc = p31;
+      int base = e31 + 1;
+      while (cont) {
+        const int e2 = base + lane;
+        const bool in_run = (e2 < nnz) && (ccol[e2] == c31);
+        const float q = in_run ? r[crow[e2]] * cval[e2] : 0.f;
+        acc += warp_sum(q);
+        const unsigned run = __ballot_sync(kFull, in_run);
+        cont = (run == kFull) && (base + 32 < nnz) && (ccol[base + 32] == c31);
+        base += 32;
+      }
+      if (lane == 0) w[c31] = fmaf(-a.scale, acc, w[c31]);
+    }
+  }
+
+  // NOTIFY: the last CTA of worker i publishes ready[i] = round + 1 after
+  // every CTA's writes to w_i are visible device-wide.
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    const unsigned int done = atomicAdd(&a.worker_ticket[i], 1u);
+    if (done == gridDim.x - 1) {
+      a.worker_ticket[i] = 0u;
+      __threadfence();
+      if (i != a.skip_worker) st_release_u32(&a.ready[i], a.round + 1u);
+    }
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_sparse_step(const SparseStepArgs& a, int N, int loss, int margin_ctas, int update_ctas,
+                               cudaStream_t s) {
+  const dim3 g1(margin_ctas, N), g2(update_ctas, N);
+  if (loss == ASAP_LOSS_HINGE)
+    k_margin_loss<ASAP_LOSS_HINGE><<<g1, kThreads, 0, s>>>(a);
+  else
+    k_margin_loss<ASAP_LOSS_LOGISTIC><<<g1, kThreads, 0, s>>>(a);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  k_segment_update<<<g2, kThreads, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
+int margin_ctas_for(int B) { return (B + kMarginRowsPerCta - 1) / kMarginRowsPerCta; }
+int update_ctas_for(int max_nnz) {
+  const int chunks = (max_nnz + 31) / 32;
+  const int c = (chunks + kUpdateChunksPerCta - 1) / kUpdateChunksPerCta;
+  return c < 1 ? 1 : c;
+}
+
+}  // namespace asap

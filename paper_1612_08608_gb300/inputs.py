@@ -108,6 +108,15 @@ def _row_scores(rowptr: np.ndarray, col: np.ndarray, val: np.ndarray, wstar: np.
     return np.bincount(row_of, weights=val.astype(np.float64) * wstar[col], minlength=n)
 
 
+def _per_worker(fn, N):
+    """fn(i) for every worker, on a thread pool (each worker has its own
+    streams, so the result does not depend on the pool)."""
+    import os
+    from concurrent.futures import ThreadPoolExecutor
+    with ThreadPoolExecutor(max_workers=max(1, min(N, os.cpu_count() or 1, 16))) as ex:
+        return list(ex.map(fn, range(N)))
+
+
 def _distinct_columns(rng: np.random.Generator, lengths: np.ndarray, sample) -> tuple:
     """Draw ``lengths[r]`` distinct column ids for every row r with ``sample(m)``
     (which returns m iid ids); duplicates inside a row are redrawn until none
@@ -169,7 +178,8 @@ def sparse_hinge_svm(seed: int = 0, N: int = 16, d: int = 47236, rows: int = 200
     wstar = _rng(seed, _TEACHER).standard_normal(d)
     mu = np.log(mean_nnz) - 0.5 * sigma * sigma
     out = SparseShards(d=d)
-    for i in range(N):
+
+    def one(i):
         lengths = np.rint(_rng(seed, _ROWLEN, i).lognormal(mu, sigma, rows)).astype(np.int64)
         lengths = np.clip(lengths, lo, min(hi, d))
         crng = _rng(seed, _COLS, i)
@@ -182,10 +192,14 @@ def sparse_hinge_svm(seed: int = 0, N: int = 16, d: int = 47236, rows: int = 200
         row_of = np.repeat(np.arange(rows), lengths)
         norms = np.sqrt(np.bincount(row_of, weights=raw * raw, minlength=rows))
         val = (raw / norms[row_of]).astype(np.float32)
+        return rowptr, col, val, _labels_from_teacher(_row_scores(rowptr, col, val, wstar), flip,
+                                                      _rng(seed, _FLIPS, i))
+
+    for rowptr, col, val, y in _per_worker(one, N):
         out.rowptr.append(rowptr)
         out.col.append(col)
         out.val.append(val)
-        out.y.append(_labels_from_teacher(_row_scores(rowptr, col, val, wstar), flip, _rng(seed, _FLIPS, i)))
+        out.y.append(y)
     return out
 
 
@@ -197,7 +211,8 @@ def sparse_logistic_hashed(seed: int = 0, N: int = 64, d: int = 1 << 20, rows: i
     """Exactly ``nnz`` distinct uniform column ids per row, N(0,1) values."""
     wstar = _rng(seed, _TEACHER).standard_normal(d)
     out = SparseShards(d=d)
-    for i in range(N):
+
+    def one(i):
         crng = _rng(seed, _COLS, i)
         col = crng.integers(0, d, size=(rows, nnz), dtype=np.int32)
         col.sort(axis=1)
@@ -211,10 +226,13 @@ def sparse_logistic_hashed(seed: int = 0, N: int = 64, d: int = 1 << 20, rows: i
         val = _rng(seed, _VALS, i).standard_normal(rows * nnz, dtype=np.float32)
         rowptr = np.arange(0, rows * nnz + 1, nnz, dtype=np.int64)
         scores = (val.astype(np.float64) * wstar[col]).reshape(rows, nnz).sum(axis=1)
+        return rowptr, col, val, _labels_from_teacher(scores, flip, _rng(seed, _FLIPS, i))
+
+    for rowptr, col, val, y in _per_worker(one, N):
         out.rowptr.append(rowptr)
         out.col.append(col)
         out.val.append(val)
-        out.y.append(_labels_from_teacher(scores, flip, _rng(seed, _FLIPS, i)))
+        out.y.append(y)
     return out
 
 

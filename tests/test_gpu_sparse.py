@@ -1,0 +1,153 @@
+"""GPU parity of the sparse ASAP round (hinge / logistic SGD step, then the
+stochastic reduce) against the CPU oracle, through the C ABI.
+
+Protocol: each round is checked on its own, the oracle restarting from the
+GPU's W_t (fp32 parameters within 1e-5 normwise relative error per worker);
+the free-running loss trajectory must stay within 1e-4 absolute."""
+import numpy as np
+import pytest
+
+from oracle import graphs, reduce, rounds
+from paper_1612_08608_gb300 import inputs
+from parity import rel_err_rows, sparse_round_matching
+
+pytestmark = pytest.mark.gpu
+
+TOL = 1e-5
+
+
+def _ctx(N, d, k, seed, kind, regen, loss, B, lr, shards, explicit=None, residency="device", l2=0.0):
+    from paper_1612_08608_gb300 import Context
+    ctx = Context(N, d, graph_seed=seed, k=k)
+    ctx.set_model(loss, batch=B, lr=lr, l2=l2)
+    if explicit is not None:
+        ctx.set_mixing(*explicit)
+    else:
+        ctx.set_graph(kind, regenerate=regen)
+    ctx.set_shard_residency(residency)
+    ctx.load_shards(shards)
+    return ctx
+
+
+def _run_parity(ctx, shards, T, B, loss, lr, sched, l2=0.0, check_graph=True):
+    losses_gpu = []
+    W_t, _ = ctx.read_params()
+    for t in range(T):
+        nbr, wgt = sched(t)
+        if check_graph:
+            g_nbr, _ = ctx.get_graph(t)
+            assert np.array_equal(g_nbr, nbr)
+        ctx.round(1)
+        W_n, rnd = ctx.read_params()
+        assert rnd == t + 1
+        err, lref, cref = sparse_round_matching(W_t.astype(np.float64), W_n, shards, t, B, loss, lr, nbr, wgt,
+                                                TOL, l2=l2)
+        assert err <= TOL, (t, err)
+        lg, cg = ctx.read_metrics(t, 1)
+        assert abs(lg[0] - lref) <= 1e-5 * max(1.0, abs(lref)), (t, lg[0], lref)
+        assert abs(cg[0] - cref) <= 1e-4 * cref + 1e-6 * np.abs(W_n).max() * np.sqrt(W_n.size), (t, cg[0], cref)
+        losses_gpu.append(lg[0])
+        W_t = W_n
+    return np.array(losses_gpu)
+
+
+def test_tiny_dense_logistic_ring_half_quarter():
+    sh = inputs.tiny_dense_logistic(seed=0)
+    N, B, lr, T = 4, 32, 0.1, 10
+    nbr = np.array([[0, 1, 3], [0, 1, 2], [1, 2, 3], [0, 2, 3]], np.int32)
+    wgt = np.array([[0.5, 0.25, 0.25], [0.25, 0.5, 0.25], [0.25, 0.5, 0.25], [0.25, 0.25, 0.5]], np.float32)
+    sched = rounds.graph_schedule("explicit", N, 2, explicit=(nbr, wgt.astype(np.float64)))
+    ctx = _ctx(N, sh.d, 2, 0, None, False, "logistic", B, lr, sh, explicit=(nbr, wgt))
+    lg = _run_parity(ctx, sh, T, B, "logistic", lr, sched, check_graph=False)
+    _, lref, _ = rounds.run_sparse(sh, T, B, "logistic", lr, sched)
+    assert np.abs(lg - lref).max() <= 1e-4
+    c = ctx.read_counters()
+    assert c["reduces"] == N * T and c["consistent_inputs"] == N * 3 * T and c["timeouts"] == 0
+    assert ctx.kernel_launches() == 3 * T
+
+
+@pytest.mark.parametrize("loss", ["hinge", "logistic"])
+@pytest.mark.parametrize("residency", ["device", "host"])
+def test_ragged_edge_cases(loss, residency):
+    # Empty rows, rows of up to 300 entries, a column in every row (runs much
+    # longer than one 32-entry chunk), d not a multiple of 64, B not a
+    # multiple of 32, a graph regenerated every round.
+    N, d, B, lr, T = 6, 1000, 70, 0.5, 6
+    rng = np.random.default_rng(5)
+    lengths = [np.where(rng.random(4 * B) < 0.1, 0, rng.integers(1, 300, 4 * B)) for _ in range(N)]
+    sh = inputs.sparse_custom(seed=11, N=N, d=d, rows=4 * B, lengths=lengths, hot_col=17)
+    sched = rounds.graph_schedule("random_regular", N, 2, graph_seed=9, regenerate=True)
+    ctx = _ctx(N, d, 2, 9, "random_regular", True, loss, B, lr, sh, residency=residency)
+    _run_parity(ctx, sh, T, B, loss, lr, sched)
+
+
+def test_l2_regularised_logistic():
+    N, d, B, lr, l2, T = 5, 300, 40, 0.3, 0.1, 5
+    sh = inputs.sparse_custom(seed=4, N=N, d=d, rows=3 * B, max_len=30)
+    sched = rounds.graph_schedule("ring", N, 1)
+    ctx = _ctx(N, d, 1, 0, "ring", False, "logistic", B, lr, sh, l2=l2)
+    _run_parity(ctx, sh, T, B, "logistic", lr, sched, l2=l2)
+
+
+def test_single_worker_and_complete_graph():
+    sh = inputs.sparse_custom(seed=6, N=1, d=200, rows=64, max_len=20)
+    ctx = _ctx(1, 200, 0, 0, "identity", False, "hinge", 16, 0.2, sh)
+    _run_parity(ctx, sh, 5, 16, "hinge", 0.2, rounds.graph_schedule("identity", 1, 0))
+    sh = inputs.sparse_custom(seed=7, N=8, d=500, rows=64, max_len=20)
+    ctx = _ctx(8, 500, 7, 0, "complete", False, "logistic", 16, 0.2, sh)
+    _run_parity(ctx, sh, 4, 16, "logistic", 0.2, rounds.graph_schedule("complete", 8, 7))
+    W, _ = ctx.read_params()
+    assert np.abs(W - W[0]).max() <= 1e-6 * np.abs(W).max()
+
+
+def test_sparse_hinge_svm_full_size():
+    # RCV1-shaped: N=16, d=47,236, lognormal rows (mean 75), Zipf(1.1)
+    # columns, hinge loss, B=256, k=2 random regular graph, 50 rounds.
+    N, d, B, lr, T = 16, 47236, 256, 0.1, 50
+    sh = inputs.sparse_hinge_svm(seed=0, N=N, rows=20000)
+    sched = rounds.graph_schedule("random_regular", N, 2, graph_seed=0)
+    ctx = _ctx(N, d, 2, 0, "random_regular", False, "hinge", B, lr, sh)
+    lg = _run_parity(ctx, sh, T, B, "hinge", lr, sched)
+    _, lref, _ = rounds.run_sparse(sh, T, B, "hinge", lr, sched)
+    assert np.abs(lg - lref).max() <= 1e-4, np.abs(lg - lref).max()
+
+
+def test_sparse_logistic_hashed_full_shapes():
+    # N=64, d=2^20, 100 uniform columns per row, B=512, k=4 expander drawn
+    # anew every round; 4 minibatches per shard keep the data small.
+    N, d, B, lr, T = 64, 1 << 20, 512, 0.1, 5
+    sh = inputs.sparse_logistic_hashed(seed=0, N=N, rows=4 * B)
+    sched = rounds.graph_schedule("random_regular", N, 4, graph_seed=0, regenerate=True)
+    ctx = _ctx(N, d, 4, 0, "random_regular", True, "logistic", B, lr, sh)
+    _run_parity(ctx, sh, T, B, "logistic", lr, sched)
+
+
+def test_notify_timeout_is_reported_and_recoverable():
+    from paper_1612_08608_gb300 import AsapError
+    sh = inputs.sparse_custom(seed=3, N=4, d=100, rows=64, max_len=10)
+    ctx = _ctx(4, 100, 1, 0, "ring", False, "logistic", 16, 0.1, sh)
+    ctx.round(1)
+    W1, _ = ctx.read_params()
+    ctx.set_wait_limit_ns(20_000_000)         # 20 ms
+    ctx.debug_skip_notify(2)                  # worker 2 never publishes NOTIFY
+    ctx.round(1)
+    with pytest.raises(AsapError) as ei:
+        ctx.sync()
+    assert ei.value.name == "ASAP_ERR_TIMEOUT"
+    assert ctx.read_counters()["timeouts"] >= 1
+    # Resume from the last good parameters: the protocol state is reset.
+    ctx.write_params(W1, 1)
+    ctx.round(2)
+    W3, rnd = ctx.read_params()
+    assert rnd == 3 and np.isfinite(W3).all()
+
+
+def test_two_runs_bit_identical():
+    sh = inputs.sparse_custom(seed=8, N=8, d=3000, rows=256, max_len=60, hot_col=3)
+    outs = []
+    for _ in range(2):
+        ctx = _ctx(8, 3000, 2, 5, "random_regular", True, "hinge", 64, 0.3, sh)
+        ctx.round(8)
+        outs.append(ctx.read_params()[0])
+        ctx.close()
+    assert np.array_equal(outs[0], outs[1])

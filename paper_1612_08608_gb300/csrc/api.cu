@@ -187,7 +187,9 @@ bool is_complete_kernel(const asap_ctx* c) { return c->kind == ASAP_GRAPH_COMPLE
 asap_status setup_mix(asap_ctx* c) {
   const int N = c->N;
   c->n_boxes = (N + 255) / 256;
-  c->box_rows = (N + c->n_boxes - 1) / c->n_boxes;
+  // Rows per TMA box, a multiple of 4 so that every box starts 128-byte
+  // aligned in shared memory (S >= 8 floats per row).
+  c->box_rows = ((N + c->n_boxes - 1) / c->n_boxes + 3) / 4 * 4;
   c->rows_pad = c->n_boxes * c->box_rows;
   int S = 256;
   while (S > 8 && static_cast<size_t>(c->rows_pad) * S * 4 > 32768) S >>= 1;

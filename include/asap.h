@@ -210,6 +210,33 @@ asap_status asap_kernel_launches(asap_ctx* ctx, uint64_t* launches);
 asap_status asap_build_graph(asap_graph_kind kind, int N, int k, uint64_t graph_seed, int64_t round,
                              int32_t* nbr_out);
 
+/* Stochastic reduce W_out = P W_in with its consensus error, for callers
+ * that cannot allocate device memory (a host framework that owns all of
+ * HBM through its own pool, or a latency-critical loop where cudaMalloc /
+ * cudaFree may synchronise the device).  The paper has no counterpart: it
+ * is the reduce of asap_stochastic_reduce without a context.
+ * All pointers are device pointers owned by the caller: W_in, W_out
+ * N rows of `ld` floats (row stride ld, ld >= d, ld % 4 == 0, 16-byte
+ * aligned, not aliased; columns [d, ld) are mixed too); nbr / wgt N*kp1
+ * int32 / float (row i = the ids in [0, N) and weights of worker i's
+ * inputs, summed in the given order; ids outside [0, N) are clamped into
+ * range, never read out of bounds); consensus_out one float, set to
+ * ||W_out - 1 wbar^T||_F with wbar the column mean of W_in.  Limits:
+ * 1 <= N <= 256, 1 <= kp1 <= 32, and ld within the built-in scratch (32768
+ * column slabs: ld <= 8,388,608 for N <= 16, ld <= 524,288 for N = 256);
+ * larger sizes return ASAP_ERR_ARG without touching the GPU.
+ * It calls no cudaMalloc, cudaFree or other allocating routine: its scratch
+ * (about 256 KB) is a file-scope device array that every GPU loading this
+ * library holds until the process exits.  The first call on each device
+ * looks up that array's device address (cudaGetSymbolAddress) with the
+ * device current, so make that first call before any stream capture.  Every
+ * call shares the array and clears what must start at zero; calls that
+ * overlap on the GPU (other streams, other threads) race on it and must be
+ * serialised by the caller.  Async on cuda_stream (NULL: legacy default
+ * stream); no device-side error is reported. */
+asap_status asap_mix_noalloc(const float* W_in, float* W_out, int N, int64_t d, int64_t ld, const int32_t* nbr,
+                             const float* wgt, int kp1, float* consensus_out, void* cuda_stream);
+
 const char* asap_last_error(const asap_ctx* ctx);
 const char* asap_version(void);
 void asap_destroy(asap_ctx* ctx);

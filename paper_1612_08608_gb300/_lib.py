@@ -37,6 +37,7 @@ SIGNATURES = {
     "asap_debug_skip_notify": (C.c_int, [_P, C.c_int]),
     "asap_kernel_launches": (C.c_int, [_P, C.POINTER(C.c_uint64)]),
     "asap_build_graph": (C.c_int, [C.c_int, C.c_int, C.c_int, C.c_uint64, C.c_int64, _P]),
+    "asap_mix_noalloc": (C.c_int, [_P, _P, C.c_int, C.c_int64, C.c_int64, _P, _P, C.c_int, _P, _P]),
     "asap_last_error": (C.c_char_p, [_P]),
     "asap_version": (C.c_char_p, []),
     "asap_destroy": (None, [_P]),

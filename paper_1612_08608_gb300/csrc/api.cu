@@ -48,6 +48,11 @@ inline size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 
 }  // namespace
 
+namespace asap {
+// Records a failure message for asap_last_error(NULL) on this thread.
+void set_thread_error(const char* msg) { g_last_error = msg; }
+}  // namespace asap
+
 struct asap_ctx {
   int dev = 0, sm_count = 0;
   int N = 0;

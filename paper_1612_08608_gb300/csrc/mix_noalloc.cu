@@ -1,0 +1,239 @@
+// asap_mix_noalloc: the stochastic reduce with its consensus error, for
+// callers that must not allocate device memory.
+//
+// Some callers cannot call cudaMalloc: a host framework that reserves
+// (nearly) all of HBM for its own pool and tracks every byte, where an
+// untracked cudaMalloc fails or breaks its budget; or a latency-critical
+// loop, where cudaMalloc / cudaFree may synchronise the device and take an
+// unbounded time.  The context API allocates its scratch at creation, so it
+// does not suit them.  This entry point takes only caller-owned inputs and
+// outputs.  Its one piece of scratch (a ticket counter and per-slab partial
+// sums of the consensus error) is the file-scope array below, which every
+// GPU that loads this library holds until the process exits.
+//
+// Compared with the context's reduce kernel it uses plain vectorised loads
+// instead of a TMA pipeline, no NOTIFY-ACK flags and at most 256 workers;
+// the arithmetic (weights applied in row order, column means from the
+// input, fp64 partial sums) is the same.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstdint>
+#include <mutex>
+
+#include "asap_internal.h"
+
+namespace asap {
+void set_thread_error(const char* msg);
+}
+
+namespace {
+
+using namespace asap;
+
+constexpr int kNoAllocMaxN = 256;
+constexpr int kNoAllocMaxSlabs = 32768;               // consensus partials: one per column slab
+constexpr int kNoAllocTicketBytes = 256;
+constexpr size_t kNoAllocScratchBytes = kNoAllocTicketBytes + 8u * kNoAllocMaxSlabs;   // 262,400 bytes
+constexpr int kNoAllocMaxDevices = 64;
+
+// [0, 4): ticket counter; [256, 256 + 8 * kNoAllocMaxSlabs): double partials.
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
+
+struct NoAllocArgs {
+  const float* in;
+  float* out;
+  int64_t ld;
+  int N;
+  int kp1;
+  const int* nbr;
+  const float* wgt;
+  int S;           // slab width (columns), a power of two >= 4
+  long long n_slabs;
+  float* consensus_out;
+  unsigned int* ticket;
+  double* partial;
+};
+
+__device__ __forceinline__ double block_sum(double v, double* red) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  __syncthreads();
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = v;
+  __syncthreads();
+  double t = 0.0;
+  if (threadIdx.x == 0)
+    for (int w = 0; w < kThreads / 32; ++w) t += red[w];
+  return t;
+}
+
+__global__ void __launch_bounds__(kThreads) k_mix_noalloc(const NoAllocArgs a) {
+  extern __shared__ __align__(16) unsigned char smem[];
+  const int S = a.S, nq = S >> 2;
+  const int lq = __ffs(nq) - 1;
+  float4* slab = reinterpret_cast<float4*>(smem);                       // [N][nq]
+  float4* mean = slab + static_cast<size_t>(a.N) * nq;                  // [nq]
+  float4* red4 = mean + nq;                                             // [kThreads]
+  double* red = reinterpret_cast<double*>(red4 + kThreads);             // [kThreads / 32]
+  int* flag = reinterpret_cast<int*>(red + kThreads / 32);
+  const int tid = threadIdx.x;
+  const int G = kThreads >> lq;
+  const int q_m = tid & (nq - 1), g_m = tid >> lq;
+  const float inv_n = 1.0f / static_cast<float>(a.N);
+
+  for (long long s = blockIdx.x; s < a.n_slabs; s += gridDim.x) {
+    const long long c0 = s * S;
+    for (int idx = tid; idx < (a.N << lq); idx += kThreads) {
+      const int i = idx >> lq, q = idx & (nq - 1);
+      const long long c = c0 + 4 * q;
+      slab[idx] = (c < a.ld) ? *reinterpret_cast<const float4*>(a.in + static_cast<int64_t>(i) * a.ld + c)
+                             : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+    __syncthreads();
+    float4 part = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int j = g_m; j < a.N; j += G) {
+      const float4 x = slab[j * nq + q_m];
+      part.x += x.x; part.y += x.y; part.z += x.z; part.w += x.w;
+    }
+    red4[tid] = part;
+    __syncthreads();
+    for (int h = G >> 1; h >= 1; h >>= 1) {
+      if (g_m < h) {
+        const float4 o = red4[tid + (h << lq)];
+        float4 t = red4[tid];
+        t.x += o.x; t.y += o.y; t.z += o.z; t.w += o.w;
+        red4[tid] = t;
+      }
+      __syncthreads();
+    }
+    if (tid < nq) {
+      const float4 t = red4[tid];
+      mean[tid] = make_float4(t.x * inv_n, t.y * inv_n, t.z * inv_n, t.w * inv_n);
+    }
+    __syncthreads();
+    float cacc = 0.f;
+    for (int idx = tid; idx < (a.N << lq); idx += kThreads) {
+      const int i = idx >> lq, q = idx & (nq - 1);
+      const int* nb = a.nbr + i * a.kp1;
+      const float* wt = a.wgt + i * a.kp1;
+      // Ids outside [0, N) are clamped so that a bad table cannot read
+      // outside the slab; the caller must pass valid ids.
+      const float w0 = __ldg(wt);
+      const float4 x0 = slab[min(max(__ldg(nb), 0), a.N - 1) * nq + q];
+      float4 acc = make_float4(w0 * x0.x, w0 * x0.y, w0 * x0.z, w0 * x0.w);
+      for (int m = 1; m < a.kp1; ++m) {
+        const float w = __ldg(wt + m);
+        const float4 x = slab[min(max(__ldg(nb + m), 0), a.N - 1) * nq + q];
+        acc.x = fmaf(w, x.x, acc.x);
+        acc.y = fmaf(w, x.y, acc.y);
+        acc.z = fmaf(w, x.z, acc.z);
+        acc.w = fmaf(w, x.w, acc.w);
+      }
+      const float4 mu = mean[q];
+      const float dx = acc.x - mu.x, dy = acc.y - mu.y, dz = acc.z - mu.z, dw = acc.w - mu.w;
+      cacc = fmaf(dx, dx, fmaf(dy, dy, fmaf(dz, dz, fmaf(dw, dw, cacc))));
+      const long long c = c0 + 4 * q;
+      if (c < a.ld) *reinterpret_cast<float4*>(a.out + static_cast<int64_t>(i) * a.ld + c) = acc;
+    }
+    const double ps = block_sum(static_cast<double>(cacc), red);
+    if (tid == 0) a.partial[s] = ps;
+    __syncthreads();   // the slab buffer is reused by the next slab
+  }
+
+  // The last CTA sums the per-slab partials in slab order.
+  __threadfence();
+  __syncthreads();
+  if (tid == 0) flag[0] = (atomicAdd(a.ticket, 1u) == gridDim.x - 1) ? 1 : 0;
+  __syncthreads();
+  if (!flag[0]) return;
+  __threadfence();
+  double v = 0.0;
+  for (long long s = tid; s < a.n_slabs; s += kThreads) v += __ldcg(a.partial + s);
+  const double total = block_sum(v, red);
+  if (tid == 0) {
+    a.consensus_out[0] = static_cast<float>(sqrt(total));
+    *a.ticket = 0u;
+  }
+}
+
+struct DeviceSlot {
+  void* scratch = nullptr;
+  int sm_count = 0;
+};
+
+std::mutex g_noalloc_mu;
+DeviceSlot g_noalloc_dev[kNoAllocMaxDevices];
+
+asap_status reject(asap_status s, const char* msg) {
+  set_thread_error(msg);
+  return s;
+}
+
+}  // namespace
+
+extern "C" asap_status asap_mix_noalloc(const float* W_in, float* W_out, int N, int64_t d, int64_t ld,
+                                        const int32_t* nbr, const float* wgt, int kp1, float* consensus_out,
+                                        void* cuda_stream) {
+  if (!W_in || !W_out || !nbr || !wgt || !consensus_out)
+    return reject(ASAP_ERR_ARG, "asap_mix_noalloc: NULL pointer");
+  if (W_in == W_out) return reject(ASAP_ERR_ARG, "asap_mix_noalloc: W_in and W_out must not alias");
+  if (N < 1 || N > kNoAllocMaxN) return reject(ASAP_ERR_ARG, "asap_mix_noalloc: need 1 <= N <= 256");
+  if (kp1 < 1 || kp1 > kMaxKp1Sparse) return reject(ASAP_ERR_ARG, "asap_mix_noalloc: need 1 <= k+1 <= 32");
+  if (d < 1 || ld < d || ld % 4 != 0)
+    return reject(ASAP_ERR_ARG, "asap_mix_noalloc: need d >= 1, ld >= d and ld a multiple of 4");
+  if ((reinterpret_cast<uintptr_t>(W_in) | reinterpret_cast<uintptr_t>(W_out)) & 15u)
+    return reject(ASAP_ERR_ARG, "asap_mix_noalloc: W_in and W_out must be 16-byte aligned");
+  int S = 256;
+  while (S > 4 && static_cast<size_t>(N) * S * 4 > 16384) S >>= 1;
+  const long long n_slabs = (ld + S - 1) / S;
+  if (n_slabs > kNoAllocMaxSlabs)
+    return reject(ASAP_ERR_ARG, "asap_mix_noalloc: ld too large for the built-in scratch "
+                                "(at most 32768 slabs of 256 columns for N <= 16, 16 columns for N = 256)");
+
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kNoAllocMaxDevices)
+    return reject(ASAP_ERR_CUDA, "asap_mix_noalloc: no usable current device");
+  DeviceSlot slot;
+  {
+    std::lock_guard<std::mutex> lock(g_noalloc_mu);
+    DeviceSlot& ds = g_noalloc_dev[dev];
+    if (!ds.scratch) {
+      // First call on this device: resolve the device address of the
+      // file-scope scratch (the host-side name is only a stand-in).
+      void* p = nullptr;
+      if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p)
+        return reject(ASAP_ERR_CUDA, "asap_mix_noalloc: cudaGetSymbolAddress failed for the scratch array");
+      int sms = 0;
+      if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms < 1)
+        return reject(ASAP_ERR_CUDA, "asap_mix_noalloc: cannot query the SM count");
+      ds.scratch = p;
+      ds.sm_count = sms;
+    }
+    slot = ds;
+  }
+  cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
+  unsigned char* base = static_cast<unsigned char*>(slot.scratch);
+  NoAllocArgs a;
+  a.in = W_in;
+  a.out = W_out;
+  a.ld = ld;
+  a.N = N;
+  a.kp1 = kp1;
+  a.nbr = nbr;
+  a.wgt = wgt;
+  a.S = S;
+  a.n_slabs = n_slabs;
+  a.consensus_out = consensus_out;
+  a.ticket = reinterpret_cast<unsigned int*>(base);
+  a.partial = reinterpret_cast<double*>(base + kNoAllocTicketBytes);
+  // The ticket must start at zero; the array keeps whatever the last call left.
+  if (cudaMemsetAsync(a.ticket, 0, sizeof(unsigned int), s) != cudaSuccess)
+    return reject(ASAP_ERR_CUDA, "asap_mix_noalloc: clearing the ticket failed");
+  const int nq = S / 4;
+  const size_t smem = 16 * (static_cast<size_t>(N) * nq + nq + kThreads) + 8 * (kThreads / 32) + 16;
+  const int grid = static_cast<int>(std::min<long long>(n_slabs, 4LL * slot.sm_count));
+  k_mix_noalloc<<<grid, kThreads, smem, s>>>(a);
+  if (cudaGetLastError() != cudaSuccess) return reject(ASAP_ERR_CUDA, "asap_mix_noalloc: launch failed");
+  return ASAP_OK;
+}

@@ -108,6 +108,16 @@ struct asap_ctx {
   int margin_ctas = 0, update_ctas = 0;
   int max_nnz = 0;
 
+  // dense softmax shards and scratch
+  uint16_t* X = nullptr;     // [N][nb*B][d] bf16
+  uint16_t* XT = nullptr;    // [N][nb][d][B] bf16
+  int32_t* Yd = nullptr;     // [N][nb*B]
+  uint16_t* RT = nullptr;    // [N][Cq*256][B] bf16
+  int Cq = 0;
+  int n_loss_part = 0;
+  CUtensorMap tmX, tmXT, tmR, tmWbf[2];
+  bool dense_configured = false;
+
   cudaStream_t stream = nullptr, own_stream = nullptr, copy_stream = nullptr;
 
   CUtensorMap tmap[2];
@@ -163,6 +173,9 @@ void free_shards(asap_ctx* c) {
   c->pool = nullptr;
   c->pool_bytes = 0;
   dfree(c->d_desc);
+  dfree(c->X);
+  dfree(c->XT);
+  dfree(c->Yd);
   dfree(c->staging[0]);
   dfree(c->staging[1]);
   c->block_off.clear();
@@ -222,6 +235,33 @@ asap_status setup_mix(asap_ctx* c) {
   return ASAP_OK;
 }
 
+// bf16 tiled map with 128-byte swizzle (64-element inner box), for the
+// tensor-core operands.
+asap_status bf16_map(asap_ctx* c, CUtensorMap* m, void* base, int rank, const cuuint64_t* dims,
+                     const cuuint64_t* strides_bytes, const cuuint32_t* box) {
+  EncodeTiledFn enc = get_encode_fn();
+  if (!enc) return fail(c, ASAP_ERR_CUDA, "cuTensorMapEncodeTiled is not available from the driver");
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank, base, dims, strides_bytes, box, estr,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return fail(c, ASAP_ERR_CUDA, "cuTensorMapEncodeTiled failed for a bf16 operand");
+  return ASAP_OK;
+}
+
+// Maps of the two bf16 parameter copies: [N][C][d], box 64 x 256 x 1.
+asap_status setup_dense_param_maps(asap_ctx* c) {
+  for (int b = 0; b < 2; ++b) {
+    cuuint64_t dims[3] = {static_cast<cuuint64_t>(c->d), static_cast<cuuint64_t>(c->C),
+                          static_cast<cuuint64_t>(c->N)};
+    cuuint64_t str[2] = {static_cast<cuuint64_t>(c->d) * 2, static_cast<cuuint64_t>(c->ld) * 2};
+    cuuint32_t box[3] = {64, 256, 1};
+    asap_status s = bf16_map(c, &c->tmWbf[b], c->Wbf[b], 3, dims, str, box);
+    if (s != ASAP_OK) return s;
+  }
+  return ASAP_OK;
+}
+
 asap_status configure_mix_launch(asap_ctx* c) {
   const bool complete = is_complete_kernel(c);
   const bool shadow = c->Wbf[0] != nullptr;
@@ -267,6 +307,10 @@ asap_status alloc_params(asap_ctx* c) {
   }
   asap_status s = setup_mix(c);
   if (s != ASAP_OK) return s;
+  if (c->loss == ASAP_LOSS_SOFTMAX) {
+    s = setup_dense_param_maps(c);
+    if (s != ASAP_OK) return s;
+  }
   return reset_protocol(c, 0);
 }
 
@@ -462,6 +506,7 @@ void asap_destroy(asap_ctx* c) {
   dfree(c->m_cons);
   dfree(c->r_scr);
   dfree(c->loss_part);
+  dfree(c->RT);
   dfree(c->cons_part);
   dfree(c->d_nbr);
   dfree(c->d_wgt);
@@ -540,8 +585,10 @@ asap_status asap_set_model(asap_ctx* c, asap_loss loss, int num_classes, int bat
     return fail(c, ASAP_ERR_ARG, "unknown loss");
   if (loss != ASAP_LOSS_NONE && (batch < 1 || batch > 65535 || !(lr > 0.f) || !(l2 >= 0.f) || !(lr * l2 < 1.f)))
     return fail(c, ASAP_ERR_ARG, "need 1 <= batch <= 65535, lr > 0, l2 >= 0, lr*l2 < 1");
-  if (loss == ASAP_LOSS_SOFTMAX)
-    return fail(c, ASAP_ERR_ARG, "softmax regression needs the dense kernels, not built in this version");
+  if (loss == ASAP_LOSS_SOFTMAX &&
+      (num_classes < 2 || num_classes > 1024 || c->d % 256 != 0 || batch % 128 != 0 ||
+       static_cast<int64_t>(c->N) * ((num_classes + 255) / 256) * 256 > (1ll << 31) / batch))
+    return fail(c, ASAP_ERR_ARG, "softmax needs 2 <= C <= 1024, d % 256 == 0 and B % 128 == 0");
   if (loss != ASAP_LOSS_SOFTMAX && num_classes != 1) return fail(c, ASAP_ERR_ARG, "num_classes must be 1");
   asap_status s0 = asap_sync(c);
   if (s0 != ASAP_OK) return s0;
@@ -551,18 +598,37 @@ asap_status asap_set_model(asap_ctx* c, asap_loss loss, int num_classes, int bat
   c->B = batch;
   c->lr = lr;
   c->l2 = l2;
-  c->P = c->d;
+  c->P = (loss == ASAP_LOSS_SOFTMAX) ? c->d * num_classes : c->d;
   asap_status s = alloc_params(c);
   if (s != ASAP_OK) return s;
   s = upload_fixed_graph(c);
   if (s != ASAP_OK) return s;
   dfree(c->r_scr);
   dfree(c->loss_part);
-  if (loss != ASAP_LOSS_NONE) {
+  dfree(c->RT);
+  c->n_loss_part = 0;
+  if (loss == ASAP_LOSS_HINGE || loss == ASAP_LOSS_LOGISTIC) {
     c->margin_ctas = margin_ctas_for(batch);
+    c->n_loss_part = c->N * c->margin_ctas;
     CU(cudaMalloc(&c->r_scr, 4 * static_cast<size_t>(c->N) * batch), "allocating step scratch");
-    CU(cudaMalloc(&c->loss_part, 4 * static_cast<size_t>(c->N) * c->margin_ctas), "allocating step scratch");
+  } else if (loss == ASAP_LOSS_SOFTMAX) {
+    c->Cq = (num_classes + 255) / 256;
+    c->n_loss_part = c->N * (batch / 128) * c->Cq;
+    const size_t rt = static_cast<size_t>(c->N) * c->Cq * 256 * batch;
+    CU(cudaMalloc(&c->RT, 2 * rt), "allocating the softmax residual scratch");
+    CU(cudaMemset(c->RT, 0, 2 * rt), "zeroing the softmax residual scratch");
+    cuuint64_t dims[2] = {static_cast<cuuint64_t>(batch), static_cast<cuuint64_t>(c->N) * c->Cq * 256};
+    cuuint64_t str[1] = {static_cast<cuuint64_t>(batch) * 2};
+    cuuint32_t box[2] = {64, 128};
+    s = bf16_map(c, &c->tmR, c->RT, 2, dims, str, box);
+    if (s != ASAP_OK) return s;
+    if (!c->dense_configured) {
+      CU(dense_configure(), "configuring the tensor-core kernels");
+      c->dense_configured = true;
+    }
   }
+  if (c->n_loss_part > 0)
+    CU(cudaMalloc(&c->loss_part, 4 * static_cast<size_t>(c->n_loss_part)), "allocating step scratch");
   return ASAP_OK;
 }
 
@@ -778,8 +844,71 @@ asap_status asap_load_shards(asap_ctx* c, const int64_t* const* rowptr, const in
   return ASAP_OK;
 }
 
-asap_status asap_load_dense_shards(asap_ctx* c, const uint16_t* const*, const int32_t* const*, const int64_t*) {
-  return fail(c, ASAP_ERR_ARG, "dense shards need the softmax kernels, not built in this version");
+asap_status asap_load_dense_shards(asap_ctx* c, const uint16_t* const* X, const int32_t* const* y,
+                                   const int64_t* n_rows) {
+  if (!c || !X || !y || !n_rows) return fail(c, ASAP_ERR_ARG, "NULL argument");
+  if (c->loss != ASAP_LOSS_SOFTMAX) return fail(c, ASAP_ERR_ARG, "set a softmax model before loading dense shards");
+  if (c->residency != ASAP_SHARDS_DEVICE) return fail(c, ASAP_ERR_ARG, "dense shards are device-resident only");
+  const int N = c->N, B = c->B;
+  const int64_t d = c->d;
+  int64_t nb = -1;
+  for (int i = 0; i < N; ++i) {
+    if (!X[i] || !y[i]) return fail(c, ASAP_ERR_ARG, "NULL shard pointer");
+    if (n_rows[i] < B) return fail(c, ASAP_ERR_ARG, "a shard has fewer rows than one minibatch");
+    if (nb >= 0 && n_rows[i] / B != nb)
+      return fail(c, ASAP_ERR_ARG, "all shards must hold the same number of minibatches");
+    nb = n_rows[i] / B;
+    for (int64_t r = 0; r < nb * B; ++r)
+      if (y[i][r] < 0 || y[i][r] >= c->C) return fail(c, ASAP_ERR_ARG, "class id out of range [0, C)");
+  }
+  if (static_cast<int64_t>(N) * nb * B > (1ll << 31) || static_cast<int64_t>(N) * nb * d > (1ll << 31))
+    return fail(c, ASAP_ERR_ARG, "dense shards too large for 32-bit tile coordinates");
+  asap_status s0 = asap_sync(c);
+  if (s0 != ASAP_OK) return s0;
+  free_shards(c);
+  const size_t rows = static_cast<size_t>(nb) * B;
+  const size_t xe = static_cast<size_t>(N) * rows * d;
+  CU(cudaMalloc(&c->X, 2 * xe), "allocating dense features");
+  CU(cudaMalloc(&c->XT, 2 * xe), "allocating transposed dense features");
+  CU(cudaMalloc(&c->Yd, 4 * static_cast<size_t>(N) * rows), "allocating labels");
+  std::vector<uint16_t> tr(rows * d);
+  for (int i = 0; i < N; ++i) {
+    CU(cudaMemcpy(c->X + static_cast<size_t>(i) * rows * d, X[i], 2 * rows * d, cudaMemcpyHostToDevice),
+       "copying dense features");
+    CU(cudaMemcpy(c->Yd + static_cast<size_t>(i) * rows, y[i], 4 * rows, cudaMemcpyHostToDevice), "copying labels");
+    // Per minibatch, the features transposed to [d][B] (the K-major operand
+    // of the gradient GEMM, whose reduction runs over the batch).
+    const unsigned nthr = std::max(1u, std::min(16u, std::thread::hardware_concurrency()));
+    std::vector<std::thread> pool;
+    for (unsigned w = 0; w < nthr; ++w)
+      pool.emplace_back([&, w]() {
+        for (int64_t t = w; t < nb; t += nthr) {
+          const uint16_t* src = X[i] + static_cast<size_t>(t) * B * d;
+          uint16_t* dst = tr.data() + static_cast<size_t>(t) * d * B;
+          for (int b = 0; b < B; ++b)
+            for (int64_t k = 0; k < d; ++k) dst[k * B + b] = src[static_cast<size_t>(b) * d + k];
+        }
+      });
+    for (auto& th : pool) th.join();
+    CU(cudaMemcpy(c->XT + static_cast<size_t>(i) * rows * d, tr.data(), 2 * rows * d, cudaMemcpyHostToDevice),
+       "copying transposed features");
+  }
+  {
+    cuuint64_t dims[2] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(N) * rows};
+    cuuint64_t str[1] = {static_cast<cuuint64_t>(d) * 2};
+    cuuint32_t box[2] = {64, 128};
+    asap_status s = bf16_map(c, &c->tmX, c->X, 2, dims, str, box);
+    if (s != ASAP_OK) return s;
+  }
+  {
+    cuuint64_t dims[2] = {static_cast<cuuint64_t>(B), static_cast<cuuint64_t>(N) * nb * d};
+    cuuint64_t str[1] = {static_cast<cuuint64_t>(B) * 2};
+    cuuint32_t box[2] = {64, 256};
+    asap_status s = bf16_map(c, &c->tmXT, c->XT, 2, dims, str, box);
+    if (s != ASAP_OK) return s;
+  }
+  c->nb = static_cast<int>(nb);
+  return ASAP_OK;
 }
 
 asap_status asap_local_step(asap_ctx* c) {
@@ -789,6 +918,45 @@ asap_status asap_local_step(asap_ctx* c) {
   if (c->step_pending) return fail(c, ASAP_ERR_ARG, "local step already taken this round; reduce first");
   const int64_t r = c->round;
   const int t = static_cast<int>(r % c->nb);
+  if (c->loss == ASAP_LOSS_SOFTMAX) {
+    asap_status sg = prepare_graph(c, r);
+    if (sg != ASAP_OK) return sg;
+    DenseFwdArgs f;
+    f.C = c->C;
+    f.Cq = c->Cq;
+    f.d = static_cast<int>(c->d);
+    f.B = c->B;
+    f.nb = c->nb;
+    f.t = t;
+    f.y = c->Yd;
+    f.RT = c->RT;
+    f.loss_part = c->loss_part;
+    f.inv_B = 1.0f / static_cast<float>(c->B);
+    f.st = c->st;
+    f.round = static_cast<unsigned>(r);
+    DenseGradArgs g;
+    g.C = c->C;
+    g.Cq = c->Cq;
+    g.d = static_cast<int>(c->d);
+    g.B = c->B;
+    g.nb = c->nb;
+    g.t = t;
+    g.W = c->W[r & 1];
+    g.ld = c->ld;
+    g.lr = c->lr;
+    g.decay = 1.0f - c->lr * c->l2;
+    g.ready = c->ready;
+    g.worker_ticket = c->ticket;
+    g.skip_worker = c->skip_notify;
+    g.st = c->st;
+    g.round = static_cast<unsigned>(r);
+    c->skip_notify = -1;
+    CU(launch_dense_step(c->tmX, c->tmWbf[r & 1], c->tmR, c->tmXT, f, g, c->N, c->stream),
+       "launching the dense local step");
+    c->launches += 2;
+    c->step_pending = true;
+    return ASAP_OK;
+  }
   const unsigned char* block;
   if (c->residency == ASAP_SHARDS_HOST) {
     asap_status s = stage_block(c, r);
@@ -844,7 +1012,7 @@ asap_status asap_stochastic_reduce(asap_ctx* c) {
   a.kp1 = c->tab_kp1;
   a.nbr = nbr;
   a.wgt = wgt;
-  a.wscale = c->step_pending ? (1.0f - c->lr * c->l2) : 1.0f;
+  a.wscale = (c->step_pending && c->loss != ASAP_LOSS_SOFTMAX) ? (1.0f - c->lr * c->l2) : 1.0f;
   a.S = c->S;
   a.rows_pad = c->rows_pad;
   a.box_rows = c->box_rows;
@@ -853,7 +1021,7 @@ asap_status asap_stochastic_reduce(asap_ctx* c) {
   a.n_slabs = c->n_slabs;
   a.cons_part = c->cons_part;
   a.loss_part = c->loss_part;
-  a.n_loss_part = c->step_pending ? c->N * c->margin_ctas : 0;
+  a.n_loss_part = c->step_pending ? c->n_loss_part : 0;
   a.loss_norm = c->B > 0 ? 1.0f / (static_cast<float>(c->N) * static_cast<float>(c->B)) : 0.f;
   a.have_loss = c->step_pending ? 1 : 0;
   a.metrics_loss = c->m_loss;

@@ -93,6 +93,30 @@ struct MixArgs {
   unsigned long long wait_ns;
 };
 
+// Arguments of the dense softmax-regression step (kernels_dense.cu).
+struct DenseFwdArgs {
+  int C, Cq, d, B, nb, t;      // Cq = ceil(C / 256) CTAs per cluster
+  const int* y;                // [N][nb*B] class ids
+  uint16_t* RT;                // [N][Cq*256][B] bf16: R^T
+  float* loss_part;            // [N][B/128][Cq]
+  float inv_B;
+  DevState* st;
+  unsigned int round;
+};
+
+struct DenseGradArgs {
+  int C, Cq, d, B, nb, t;
+  float* W;                    // fp32 master [N][ld], worker row = C x d class-major
+  int64_t ld;
+  float lr;
+  float decay;                 // 1 - lr * l2
+  unsigned int* ready;
+  unsigned int* worker_ticket;
+  int skip_worker;
+  DevState* st;
+  unsigned int round;
+};
+
 asap_status build_graph_host(asap_graph_kind kind, int N, int k, uint64_t seed, int64_t round,
                              int32_t* nbr, const char** why);
 
@@ -103,6 +127,11 @@ cudaError_t launch_mix(const CUtensorMap& tmap, const MixArgs& a, bool complete,
                        cudaStream_t s);
 size_t mix_smem_bytes(int N, int kp1, int S, int rows_pad, int stages);
 cudaError_t mix_configure(bool complete, int kp1, bool shadow, size_t smem);
+size_t dense_smem_bytes();
+cudaError_t dense_configure();
+cudaError_t launch_dense_step(const CUtensorMap& tmX, const CUtensorMap& tmW, const CUtensorMap& tmR,
+                              const CUtensorMap& tmXT, const DenseFwdArgs& f, const DenseGradArgs& g, int N,
+                              cudaStream_t s);
 cudaError_t launch_cast_bf16(const float* src, uint16_t* dst, int64_t n, cudaStream_t s);
 
 }  // namespace asap

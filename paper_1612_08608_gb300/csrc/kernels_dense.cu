@@ -1,0 +1,478 @@
+// Local SGD step of dense softmax regression on bf16 features (the dense
+// variant of Eq. A.1, first line), on the 5th-generation tensor cores.
+//
+//   forward  Z = X_b W^T           X_b [B x d] bf16, W [C x d] (bf16 copy of the fp32 master)
+//            R = (softmax(Z) - onehot(y)) / B   -> bf16, stored transposed R^T [C x B]
+//   gradient G = R^T X_b           [C x d], fp32 accumulate
+//            W_half = (1 - eta l2) W - eta G    (fp32 master, in place), then NOTIFY
+//
+// Both GEMMs: one CTA per 128 x 256 output tile, 4 warps.  Warp 0 lane 0
+// issues TMA loads (128-byte swizzled, K-major tiles of 64 bf16) into a ring
+// of stages guarded by full/empty mbarriers; warp 1 lane 0 issues
+// tcgen05.mma (M=128, N=256, K=16, bf16 x bf16 -> fp32 in TMEM) and commits
+// each stage back to its empty barrier; all four warps then read the
+// accumulator out of TMEM (warp w owns TMEM lanes 32w..32w+31, i.e. rows).
+//
+// Softmax needs all C logits of a row, more than one CTA's 256 TMEM
+// columns: the forward kernel runs as a cluster of ceil(C/256) CTAs along
+// the classes, and the CTAs exchange per-row maxima and exp-sums through
+// distributed shared memory.
+//
+// Every wait is time-limited; a wait that runs out records an error in the
+// context's device state, and the CTA still passes every barrier and frees
+// its TMEM before returning.
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include <cstdint>
+
+#include "asap_internal.h"
+
+namespace asap {
+
+namespace {
+
+constexpr int kDenseThreads = 128;
+constexpr int kTileM = 128;
+constexpr int kTileN = 256;
+constexpr int kTileK = 64;                  // one 128-byte swizzle row of bf16
+constexpr int kStages = 2;
+constexpr uint32_t kABytes = kTileM * kTileK * 2;   // 16 KB
+constexpr uint32_t kBBytes = kTileN * kTileK * 2;   // 32 KB
+constexpr uint32_t kTmemCols = 256;
+constexpr unsigned long long kWaitNs = 2000000000ull;
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ unsigned long long now_ns() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" :: "r"(smem_u32(bar)), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" :: "r"(smem_u32(bar)), "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
+      : "=r"(ok) : "r"(smem_u32(bar)), "r"(parity) : "memory");
+  return ok != 0;
+}
+
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const unsigned long long t0 = now_ns();
+  for (;;) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (now_ns() - t0 > kWaitNs) return false;
+  }
+}
+
+__device__ __forceinline__ void tma_2d(void* dst, const CUtensorMap* m, uint64_t* bar, int x, int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];"
+      :: "r"(smem_u32(dst)), "l"(reinterpret_cast<uint64_t>(m)), "r"(x), "r"(y), "r"(smem_u32(bar)) : "memory");
+}
+
+__device__ __forceinline__ void tma_3d(void* dst, const CUtensorMap* m, uint64_t* bar, int x, int y, int z) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], [%5];"
+      :: "r"(smem_u32(dst)), "l"(reinterpret_cast<uint64_t>(m)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar))
+      : "memory");
+}
+
+// --- tcgen05 -----------------------------------------------------------
+__device__ __forceinline__ void tmem_alloc(uint32_t* slot, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" :: "r"(smem_u32(slot)),
+               "r"(ncols) : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" :: "r"(taddr), "r"(ncols) : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+// D[tmem] (+)= A[smem] * B[smem]^T, kind::f16 (bf16 inputs, fp32 accumulator).
+__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                          uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n"
+      :: "r"(d_tmem), "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate) : "memory");
+}
+
+// Arrive on `bar` once every tcgen05.mma issued so far by this thread is done.
+__device__ __forceinline__ void umma_commit(uint64_t* bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" :: "r"(smem_u32(bar))
+               : "memory");
+}
+
+// 32 consecutive fp32 accumulator columns of this thread's TMEM lane.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
+}
+
+// Shared-memory matrix descriptor: K-major tile, rows of 128 bytes, 128-byte
+// swizzle (the layout TMA writes with CU_TENSOR_MAP_SWIZZLE_128B), 8-row
+// groups 1024 bytes apart.
+__device__ __forceinline__ uint64_t smem_desc_sw128(const void* p) {
+  const uint32_t a = smem_u32(p);
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((a & 0x3FFFFu) >> 4);     // start address
+  d |= static_cast<uint64_t>(1) << 16;                  // leading byte offset (unused for this layout)
+  d |= static_cast<uint64_t>(1024 >> 4) << 32;          // stride byte offset: 8 rows x 128 B
+  d |= static_cast<uint64_t>(1) << 46;                  // descriptor version for tcgen05
+  d |= static_cast<uint64_t>(2) << 61;                  // 128-byte swizzle
+  return d;
+}
+
+// Instruction descriptor: bf16 A and B (K-major), fp32 D, M x N.
+__host__ __device__ constexpr uint32_t idesc_bf16(int M, int N) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | (static_cast<uint32_t>(N >> 3) << 17) |
+         (static_cast<uint32_t>(M >> 4) << 24);
+}
+
+__device__ __forceinline__ void record_error(DevState* st, unsigned code, unsigned worker, unsigned round) {
+  if (atomicCAS(&st->err_code, 0u, code) == 0u) {
+    st->err_worker = worker;
+    st->err_round = round;
+  }
+}
+
+// --- cluster helpers ----------------------------------------------------
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\nbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ uint32_t cluster_size() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_nctarank;" : "=r"(r));
+  return r;
+}
+
+__device__ __forceinline__ float ld_dsmem_f32(const float* local, uint32_t rank) {
+  uint32_t remote;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(local)), "r"(rank));
+  float v;
+  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(remote) : "memory");
+  return v;
+}
+
+struct GemmSmem {
+  unsigned char* a;     // kStages x kABytes
+  unsigned char* b;     // kStages x kBBytes
+  uint64_t* full;
+  uint64_t* empty;
+  uint64_t* accum;
+  uint32_t* tmem_slot;
+  float* row_a;         // [128]
+  float* row_b;         // [128]
+  float* red;           // [4]
+  int* fail;
+};
+
+__device__ __forceinline__ GemmSmem carve(unsigned char* raw) {
+  GemmSmem s;
+  uintptr_t p = (reinterpret_cast<uintptr_t>(raw) + 1023) & ~static_cast<uintptr_t>(1023);
+  s.a = reinterpret_cast<unsigned char*>(p);
+  p += kStages * kABytes;
+  s.b = reinterpret_cast<unsigned char*>(p);
+  p += kStages * kBBytes;
+  s.full = reinterpret_cast<uint64_t*>(p);
+  s.empty = s.full + kStages;
+  s.accum = s.empty + kStages;
+  p += 8 * (2 * kStages + 1);
+  s.tmem_slot = reinterpret_cast<uint32_t*>(p);
+  p += 16;
+  s.row_a = reinterpret_cast<float*>(p);
+  p += 4 * kTileM;
+  s.row_b = reinterpret_cast<float*>(p);
+  p += 4 * kTileM;
+  s.red = reinterpret_cast<float*>(p);
+  p += 16;
+  s.fail = reinterpret_cast<int*>(p);
+  return s;
+}
+
+// The producer / MMA part shared by both GEMMs.  A tiles come from tmA at
+// (k, a_row), B tiles from tmB at (k, b_row[, b_z]) (3-D when b_is_3d).
+__device__ void gemm_mainloop(const GemmSmem& sm, const CUtensorMap* tmA, const CUtensorMap* tmB, bool b_is_3d,
+                              int a_row, int b_row, int b_z, int k_tiles, uint32_t tmem, DevState* st,
+                              unsigned worker, unsigned round) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (warp == 0) {
+    if (lane == 0) {
+      for (int kt = 0; kt < k_tiles; ++kt) {
+        const int s = kt % kStages;
+        if (kt >= kStages && !mbar_wait(sm.empty + s, ((kt / kStages) - 1) & 1)) {
+          record_error(st, ASAP_ERR_CUDA, worker, round);
+          atomicOr(sm.fail, 1);
+          break;
+        }
+        mbar_expect_tx(sm.full + s, kABytes + kBBytes);
+        tma_2d(sm.a + s * kABytes, tmA, sm.full + s, kt * kTileK, a_row);
+        if (b_is_3d)
+          tma_3d(sm.b + s * kBBytes, tmB, sm.full + s, kt * kTileK, b_row, b_z);
+        else
+          tma_2d(sm.b + s * kBBytes, tmB, sm.full + s, kt * kTileK, b_row);
+      }
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    if (lane == 0) {
+      constexpr uint32_t idesc = idesc_bf16(kTileM, kTileN);
+      bool ok = true;
+      for (int kt = 0; kt < k_tiles; ++kt) {
+        const int s = kt % kStages;
+        if (!mbar_wait(sm.full + s, (kt / kStages) & 1)) {
+          record_error(st, ASAP_ERR_CUDA, worker, round);
+          atomicOr(sm.fail, 1);
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+#pragma unroll
+        for (int kk = 0; kk < kTileK / 16; ++kk) {
+          const uint64_t ad = smem_desc_sw128(sm.a + s * kABytes + kk * 32);
+          const uint64_t bd = smem_desc_sw128(sm.b + s * kBBytes + kk * 32);
+          umma_bf16(tmem, ad, bd, idesc, (kt | kk) != 0 ? 1u : 0u);
+        }
+        umma_commit(sm.empty + s);
+      }
+      if (ok) umma_commit(sm.accum);
+    }
+    __syncwarp();
+  }
+}
+
+__device__ __forceinline__ void setup(const GemmSmem& sm) {
+  const int warp = threadIdx.x >> 5;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(sm.full + s, 1);
+      mbar_init(sm.empty + s, 1);
+    }
+    mbar_init(sm.accum, 1);
+    *sm.fail = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) tmem_alloc(sm.tmem_slot, kTmemCols);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+}
+
+__device__ __forceinline__ void teardown(const GemmSmem& sm, uint32_t tmem) {
+  tc_fence_before();
+  __syncthreads();
+  if ((threadIdx.x >> 5) == 1) tmem_dealloc(tmem, kTmemCols);
+}
+
+// ----------------------------------------------------------------------------
+// Forward: logits, softmax across the cluster, R^T, loss partials.
+// grid (Cq, B/128, N), cluster (Cq, 1, 1); CTA rank q owns classes [256q, 256q+256).
+__global__ void __launch_bounds__(kDenseThreads, 1)
+    k_dense_fwd(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmW, DenseFwdArgs a) {
+  extern __shared__ unsigned char smem_raw[];
+  const GemmSmem sm = carve(smem_raw);
+  const int q = blockIdx.x, mt = blockIdx.y, i = blockIdx.z;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  setup(sm);
+  const uint32_t tmem = *sm.tmem_slot;
+
+  const int row0 = (i * a.nb + a.t) * a.B + mt * kTileM;        // row of X
+  gemm_mainloop(sm, &tmX, &tmW, true, row0, q * kTileN, i, a.d / kTileK, tmem, a.st, i, a.round);
+
+  // ---- epilogue: thread = batch row ----
+  const bool ok = __all_sync(0xffffffffu, mbar_wait(sm.accum, 0));
+  if (!ok) {
+    record_error(a.st, ASAP_ERR_CUDA, i, a.round);
+    atomicOr(sm.fail, 1);
+  }
+  __syncwarp();
+  tc_fence_after();
+  const uint32_t trow = tmem + (static_cast<uint32_t>(warp * 32) << 16);
+  const int b = mt * kTileM + threadIdx.x;                       // row within the batch
+  const int yb = a.y[(i * a.nb + a.t) * a.B + b];
+  const int c0 = q * kTileN;
+  float v[32];
+  float m = -INFINITY;
+  if (ok) {
+    for (int ch = 0; ch < kTileN / 32; ++ch) {
+      tmem_ld32(trow + ch * 32, v);
+#pragma unroll
+      for (int j = 0; j < 32; ++j)
+        if (c0 + ch * 32 + j < a.C) m = fmaxf(m, v[j]);
+    }
+  }
+  sm.row_a[threadIdx.x] = m;
+  cluster_sync();
+  const uint32_t nr = cluster_size();
+  float gmax = -INFINITY;
+  for (uint32_t r = 0; r < nr; ++r) gmax = fmaxf(gmax, ld_dsmem_f32(sm.row_a + threadIdx.x, r));
+  float s = 0.f, zy = 0.f;
+  if (ok) {
+    for (int ch = 0; ch < kTileN / 32; ++ch) {
+      tmem_ld32(trow + ch * 32, v);
+#pragma unroll
+      for (int j = 0; j < 32; ++j) {
+        const int c = c0 + ch * 32 + j;
+        if (c < a.C) s += __expf(v[j] - gmax);
+        if (c == yb) zy = v[j];
+      }
+    }
+  }
+  sm.row_b[threadIdx.x] = s;
+  cluster_sync();
+  float S = 0.f;
+  for (uint32_t r = 0; r < nr; ++r) S += ld_dsmem_f32(sm.row_b + threadIdx.x, r);
+  const float invS = 1.0f / S;
+  if (ok) {
+    __nv_bfloat16* rt = reinterpret_cast<__nv_bfloat16*>(a.RT) +
+                        (static_cast<int64_t>(i) * a.Cq * kTileN + c0) * a.B + b;
+    for (int ch = 0; ch < kTileN / 32; ++ch) {
+      tmem_ld32(trow + ch * 32, v);
+#pragma unroll
+      for (int j = 0; j < 32; ++j) {
+        const int c = c0 + ch * 32 + j;
+        float r = 0.f;
+        if (c < a.C) r = (__expf(v[j] - gmax) * invS - (c == yb ? 1.f : 0.f)) * a.inv_B;
+        rt[static_cast<int64_t>(ch * 32 + j) * a.B] = __float2bfloat16_rn(r);
+      }
+    }
+  }
+  // loss of the rows whose label falls in this CTA's classes
+  float l = (ok && yb >= c0 && yb < c0 + kTileN) ? (gmax + __logf(S) - zy) : 0.f;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
+  if (lane == 0) sm.red[warp] = l;
+  cluster_sync();   // no CTA leaves while its row maxima / sums may still be read
+  if (threadIdx.x == 0)
+    a.loss_part[(static_cast<int64_t>(i) * gridDim.y + mt) * gridDim.x + q] =
+        sm.red[0] + sm.red[1] + sm.red[2] + sm.red[3];
+  teardown(sm, tmem);
+}
+
+// ----------------------------------------------------------------------------
+// Gradient and update: G tile [128 classes x 256 features] = R^T X_b, then
+// W = (1 - eta l2) W - eta G on the fp32 master; the last CTA of a worker
+// publishes NOTIFY.  grid (d/256, ceil(C/128), N).
+__global__ void __launch_bounds__(kDenseThreads, 1)
+    k_dense_grad(const __grid_constant__ CUtensorMap tmR, const __grid_constant__ CUtensorMap tmXT, DenseGradArgs a) {
+  extern __shared__ unsigned char smem_raw[];
+  const GemmSmem sm = carve(smem_raw);
+  const int nt = blockIdx.x, mt = blockIdx.y, i = blockIdx.z;
+  const int warp = threadIdx.x >> 5;
+  setup(sm);
+  const uint32_t tmem = *sm.tmem_slot;
+
+  const int a_row = i * a.Cq * kTileN + mt * kTileM;             // row of R^T
+  const int b_row = (i * a.nb + a.t) * a.d + nt * kTileN;        // row of X^T
+  gemm_mainloop(sm, &tmR, &tmXT, false, a_row, b_row, 0, a.B / kTileK, tmem, a.st, i, a.round);
+
+  const bool ok = __all_sync(0xffffffffu, mbar_wait(sm.accum, 0));
+  if (!ok) {
+    record_error(a.st, ASAP_ERR_CUDA, i, a.round);
+    atomicOr(sm.fail, 1);
+  }
+  __syncwarp();
+  tc_fence_after();
+  const uint32_t trow = tmem + (static_cast<uint32_t>(warp * 32) << 16);
+  const int c = mt * kTileM + threadIdx.x;                       // class row
+  float g[32];
+  float* w = a.W + static_cast<int64_t>(i) * a.ld + static_cast<int64_t>(c) * a.d + nt * kTileN;
+  for (int ch = 0; ch < kTileN / 32; ++ch) {
+    if (ok) tmem_ld32(trow + ch * 32, g);
+    if (ok && c < a.C) {
+      float4* w4 = reinterpret_cast<float4*>(w + ch * 32);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        float4 x = w4[j];
+        x.x = fmaf(-a.lr, g[4 * j + 0], a.decay * x.x);
+        x.y = fmaf(-a.lr, g[4 * j + 1], a.decay * x.y);
+        x.z = fmaf(-a.lr, g[4 * j + 2], a.decay * x.z);
+        x.w = fmaf(-a.lr, g[4 * j + 3], a.decay * x.w);
+        w4[j] = x;
+      }
+    }
+  }
+  teardown(sm, tmem);
+  // NOTIFY once every tile of worker i is written.
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    const unsigned total = gridDim.x * gridDim.y;
+    const unsigned done = atomicAdd(&a.worker_ticket[i], 1u);
+    if (done == total - 1) {
+      a.worker_ticket[i] = 0u;
+      __threadfence();
+      if (i != a.skip_worker) asm volatile("st.release.gpu.global.u32 [%0], %1;" :: "l"(a.ready + i),
+                                           "r"(a.round + 1u) : "memory");
+    }
+  }
+}
+
+}  // namespace
+
+size_t dense_smem_bytes() {
+  return 1024 + kStages * (kABytes + kBBytes) + 8 * (2 * kStages + 1) + 16 + 8 * kTileM + 16 + 16;
+}
+
+cudaError_t dense_configure() {
+  const int smem = static_cast<int>(dense_smem_bytes());
+  cudaError_t e = cudaFuncSetAttribute(k_dense_fwd, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  if (e != cudaSuccess) return e;
+  e = cudaFuncSetAttribute(k_dense_fwd, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(k_dense_grad, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+}
+
+cudaError_t launch_dense_step(const CUtensorMap& tmX, const CUtensorMap& tmW, const CUtensorMap& tmR,
+                              const CUtensorMap& tmXT, const DenseFwdArgs& f, const DenseGradArgs& g, int N,
+                              cudaStream_t s) {
+  const size_t smem = dense_smem_bytes();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(f.Cq, f.B / kTileM, N);
+  cfg.blockDim = dim3(kDenseThreads, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = f.Cq;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cudaError_t e = cudaLaunchKernelEx(&cfg, k_dense_fwd, tmX, tmW, f);
+  if (e != cudaSuccess) return e;
+  const dim3 g2(g.d / kTileN, (g.C + kTileM - 1) / kTileM, N);
+  k_dense_grad<<<g2, kDenseThreads, smem, s>>>(tmR, tmXT, g);
+  return cudaGetLastError();
+}
+
+}  // namespace asap

@@ -1,0 +1,54 @@
+"""GPU parity of the dense softmax-regression round (tcgen05 bf16 GEMMs with
+fp32 accumulation, softmax across a cluster, fp32 master update, then the
+stochastic reduce writing the next round's bf16 copy) against the oracle,
+which mirrors the bf16 rounding points.  Tolerance: 1e-3 normwise relative
+error per worker per round (bf16-input GEMM path), loss within 1e-4."""
+import numpy as np
+import pytest
+
+from oracle import rounds
+from paper_1612_08608_gb300 import inputs
+from parity import rel_err_rows
+
+pytestmark = pytest.mark.gpu
+
+TOL = 1e-3
+
+
+def _run(N, d, C, B, lr, k, kind, T, seed=0, l2=0.0):
+    from paper_1612_08608_gb300 import Context
+    sh = inputs.dense_softmax(seed=seed, N=N, d=d, C=C, rows=T * B)
+    ctx = Context(N, d, graph_seed=seed, k=k)
+    ctx.set_model("softmax", batch=B, lr=lr, num_classes=C, l2=l2)
+    ctx.set_graph(kind)
+    ctx.load_dense_shards(sh)
+    sched = rounds.graph_schedule(kind, N, k, graph_seed=seed)
+    W_t, _ = ctx.read_params()
+    assert W_t.shape == (N, C * d) and not W_t.any()
+    for t in range(T):
+        ctx.round(1)
+        W_n, rnd = ctx.read_params()
+        assert rnd == t + 1
+        nbr, wgt = sched(t)
+        ref, lref, cref = rounds.softmax_round(W_t, sh, t, B, lr, nbr, wgt, l2=l2)
+        err = rel_err_rows(W_n, ref)
+        assert err <= TOL, (t, err)
+        lg, cg = ctx.read_metrics(t, 1)
+        assert abs(lg[0] - lref) <= 1e-4 * max(1.0, abs(lref)), (t, lg[0], lref)
+        assert abs(cg[0] - cref) <= 2e-3 * cref + 1e-7, (t, cg[0], cref)
+        W_t = W_n
+    return ctx
+
+
+def test_dense_small_one_cluster_cta():
+    _run(N=4, d=256, C=10, B=128, lr=0.5, k=1, kind="ring", T=3)
+
+
+def test_dense_ragged_classes_two_cluster_ctas_l2():
+    _run(N=6, d=512, C=300, B=256, lr=0.3, k=2, kind="random_regular", T=3, seed=2, l2=0.01)
+
+
+def test_dense_softmax_full_size():
+    # N=32 workers, d=2048 bf16 features, C=1000 classes, B=512, root graph.
+    ctx = _run(N=32, d=2048, C=1000, B=512, lr=0.1, k=2, kind="root", T=3)
+    assert ctx.read_counters()["timeouts"] == 0

@@ -38,8 +38,19 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 METRIC = "worker-samples/s per SGD+reduce round; stochastic-reduce HBM GB/s vs peak"
-WORKLOAD = dict(name="sparse_logistic_hashed", N=64, d=1 << 20, rows=50000, nnz=100, B=512, lr=0.1, k=4,
-                loss="logistic", graph="random_regular", regenerate=True, graph_seed=0)
+WORKLOADS = {
+    # hashed sparse logistic regression (the default, HBM-scale)
+    "sparse_logistic_hashed": dict(name="sparse_logistic_hashed", N=64, d=1 << 20, rows=50000, nnz=100, B=512,
+                                   lr=0.1, k=4, loss="logistic", graph="random_regular", regenerate=True,
+                                   graph_seed=0),
+    # RCV1-shaped hinge SVM (L2-resident)
+    "sparse_hinge_svm": dict(name="sparse_hinge_svm", N=16, d=47236, rows=20000, B=256, lr=0.1, k=2,
+                             loss="hinge", graph="random_regular", regenerate=False, graph_seed=0),
+    # dense softmax regression on bf16 features (tensor cores)
+    "dense_softmax": dict(name="dense_softmax", N=32, d=2048, C=1000, rows=25600, B=512, lr=0.1, k=2,
+                          loss="softmax", graph="root", regenerate=False, graph_seed=0),
+}
+WORKLOAD = WORKLOADS["sparse_logistic_hashed"]
 PROFILE = os.path.join(ROOT, "profiles", "stochastic_reduce_sparse_logistic_hashed.txt")
 MIX_SOURCE = os.path.join(ROOT, "paper_1612_08608_gb300", "csrc", "kernels_mix.cu")
 
@@ -51,6 +62,7 @@ def parse():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", default="asap", choices=["asap", "reference"])
     ap.add_argument("--rows", type=int, default=None, help="rows per worker (default: the workload's)")
+    ap.add_argument("--workload", default="sparse_logistic_hashed", choices=sorted(WORKLOADS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     return ap.parse_args()
@@ -142,8 +154,50 @@ class ClockSampler:
 
 def make_shards(rows, seed):
     from paper_1612_08608_gb300 import inputs
-    return inputs.sparse_logistic_hashed(seed=seed, N=WORKLOAD["N"], d=WORKLOAD["d"], rows=rows,
-                                         nnz=WORKLOAD["nnz"])
+    w = WORKLOAD
+    if w["name"] == "sparse_logistic_hashed":
+        return inputs.sparse_logistic_hashed(seed=seed, N=w["N"], d=w["d"], rows=rows, nnz=w["nnz"])
+    if w["name"] == "sparse_hinge_svm":
+        return inputs.sparse_hinge_svm(seed=seed, N=w["N"], d=w["d"], rows=rows)
+    return inputs.dense_softmax(seed=seed, N=w["N"], d=w["d"], C=w["C"], rows=rows)
+
+
+def kernel_work(sh):
+    """Algorithmic work of one launch of each kernel kind: (unit, amount, bound).
+    Sparse byte counts use the mean minibatch over a sample of batches."""
+    import numpy as np
+    w = WORKLOAD
+    N, B, d = w["N"], w["B"], w["d"]
+    ld = (d * w.get("C", 1) + 63) // 64 * 64
+    out = {}
+    if w["loss"] == "softmax":
+        C = w["C"]
+        out["dense_fwd"] = ("TFLOP/s", 2.0 * N * B * C * d, "tensor")
+        out["dense_grad"] = ("TFLOP/s", 2.0 * N * C * d * B, "tensor")
+        out["reduce"] = ("GB/s", 10.0 * N * ld, "hbm")     # fp32 read + write, bf16 copy write
+        return out
+    rng = np.random.default_rng(0)
+    nnz = pad = touched = 0.0
+    samples = 16
+    for _ in range(samples):
+        i = int(rng.integers(N))
+        t = int(rng.integers(sh.n_rows(i) // B))
+        rp = sh.rowptr[i][t * B:(t + 1) * B + 1]
+        lens = np.diff(rp)
+        nnz += lens.sum()
+        pad += ((lens + 3) // 4 * 4).sum()
+        touched += np.unique(sh.col[i][rp[0]:rp[-1]]).shape[0]
+    nnz, pad, touched = nnz * N / samples, pad * N / samples, touched * N / samples
+    out["margin"] = ("GB/s", 8.0 * pad + 4.0 * nnz + 8.0 * N * B, "hbm")
+    out["update"] = ("GB/s", 10.0 * nnz + 8.0 * touched + 4.0 * N * B, "hbm")
+    out["reduce"] = ("GB/s", 8.0 * N * ld, "hbm")
+    return out
+
+
+def _sched():
+    from oracle import rounds
+    w = WORKLOAD
+    return rounds.graph_schedule(w["graph"], w["N"], w["k"], w["graph_seed"], w["regenerate"])
 
 
 def oracle_round_sample(sh, W, t, workers):
@@ -151,44 +205,59 @@ def oracle_round_sample(sh, W, t, workers):
     row of each listed worker (neighbours' half-steps taken from W when not
     in the sample).  Returns the worker-samples processed."""
     import numpy as np
-    from oracle import rounds, sgd
-    sched = rounds.graph_schedule(WORKLOAD["graph"], WORKLOAD["N"], WORKLOAD["k"], WORKLOAD["graph_seed"],
-                                  WORKLOAD["regenerate"])
-    nbr, wgt = sched(t)
+    from oracle import sgd
+    w = WORKLOAD
+    nbr, wgt = _sched()(t)
     H = {}
     for i in workers:
-        H[i], _, _ = sgd.sparse_worker_step(W[i], sh.rowptr[i], sh.col[i], sh.val[i], sh.y[i], t, WORKLOAD["B"],
-                                            WORKLOAD["loss"], WORKLOAD["lr"])
+        if w["loss"] == "softmax":
+            Wm = W[i].astype(np.float32).reshape(w["C"], w["d"])
+            H[i] = sgd.softmax_worker_step(Wm, sh.X[i], sh.y[i], t, w["B"], w["lr"])[0].reshape(-1)
+        else:
+            H[i], _, _ = sgd.sparse_worker_step(W[i], sh.rowptr[i], sh.col[i], sh.val[i], sh.y[i], t, w["B"],
+                                                w["loss"], w["lr"])
     for i in workers:
         acc = np.zeros(W.shape[1])
         for m in range(nbr.shape[1]):
             j = int(nbr[i, m])
             acc += wgt[i, m] * (H[j] if j in H else W[j])
-    return len(workers) * WORKLOAD["B"]
+    return len(workers) * w["B"]
 
 
 def cpu_baseline(sh):
-    """One full round of the oracle (rounds.sparse_round) as it stands."""
+    """One full round of the oracle as it stands."""
     import numpy as np
     from oracle import rounds
-    sched = rounds.graph_schedule(WORKLOAD["graph"], WORKLOAD["N"], WORKLOAD["k"], WORKLOAD["graph_seed"],
-                                  WORKLOAD["regenerate"])
-    W = np.zeros((WORKLOAD["N"], WORKLOAD["d"]))
-    nbr, wgt = sched(0)
+    w = WORKLOAD
+    P = w["d"] * w.get("C", 1)
+    W = np.zeros((w["N"], P))
+    nbr, wgt = _sched()(0)
     t0 = time.perf_counter()
-    rounds.sparse_round(W, sh, 0, WORKLOAD["B"], WORKLOAD["loss"], WORKLOAD["lr"], nbr, wgt)
+    if w["loss"] == "softmax":
+        rounds.softmax_round(W.astype(np.float32), sh, 0, w["B"], w["lr"], nbr, wgt)
+    else:
+        rounds.sparse_round(W, sh, 0, w["B"], w["loss"], w["lr"], nbr, wgt)
     dt = time.perf_counter() - t0
-    return {"value": WORKLOAD["N"] * WORKLOAD["B"] / dt, "unit": "worker-samples/s", "cores": 1,
-            "kind": "oracle", "sample": "one full round (64 workers' SGD steps, the reduce and both metrics), "
-                                        "numpy fp64, single thread; %.1f s" % dt}
+    return {"value": w["N"] * w["B"] / dt, "unit": "worker-samples/s", "cores": 1,
+            "kind": "oracle", "sample": "one full round (%d workers' SGD steps, the reduce and both metrics), "
+                                        "numpy fp64%s; %.1f s" % (w["N"], ", BLAS matmuls" if w["loss"] == "softmax"
+                                                                   else ", single thread", dt)}
 
 
 def config(rows):
-    return {"workload": WORKLOAD["name"], "N_workers": WORKLOAD["N"], "d": WORKLOAD["d"], "B": WORKLOAD["B"],
-            "rows_per_worker": rows, "nnz_per_row": WORKLOAD["nnz"], "loss": WORKLOAD["loss"],
-            "graph": "random_regular k=4, regenerated every round", "lr": WORKLOAD["lr"],
-            "l2_flush": "none: inputs larger than L2 (W 2 x 256 MiB, shards > 5 GB)",
-            "parallelism": "independent replicas, one per GPU"}
+    w = WORKLOAD
+    c = {"workload": w["name"], "N_workers": w["N"], "d": w["d"], "B": w["B"], "rows_per_worker": rows,
+         "loss": w["loss"], "lr": w["lr"],
+         "graph": "%s k=%d%s" % (w["graph"], w["k"], ", regenerated every round" if w["regenerate"] else ""),
+         "parallelism": "independent replicas, one per GPU"}
+    if "nnz" in w:
+        c["nnz_per_row"] = w["nnz"]
+    if "C" in w:
+        c["classes"] = w["C"]
+    c["l2_flush"] = {"sparse_logistic_hashed": "none: inputs larger than L2 (W 2 x 256 MiB, shards > 5 GB)",
+                     "dense_softmax": "none: inputs larger than L2 (fp32 W 2 x 262 MB, features 6.7 GB)",
+                     "sparse_hinge_svm": "none: the whole working set (~25 MB) stays in L2 by design"}[w["name"]]
+    return c
 
 
 def dist_env():
@@ -205,7 +274,7 @@ def run_reference(args):
         return
     rows = args.rows or WORKLOAD["rows"]
     sh = make_shards(rows, seed=0)
-    W = np.zeros((WORKLOAD["N"], WORKLOAD["d"]))
+    W = np.zeros((WORKLOAD["N"], WORKLOAD["d"] * WORKLOAD.get("C", 1)))
     t0 = time.perf_counter()
     oracle_round_sample(sh, W, 0, [0])
     t_one = time.perf_counter() - t0
@@ -222,13 +291,25 @@ def run_reference(args):
     value = units / dt
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "worker-samples/s", "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt / args.steps * 1e3,
-            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic (seeded)",
             "config": config(rows),
             "cpu_baseline": {"value": value, "unit": "worker-samples/s", "cores": 1, "kind": "oracle",
-                             "sample": "per step: %d of 64 workers' SGD step and reduce row (numpy fp64, one "
-                                       "thread)" % per_step},
+                             "sample": "per step: %d of %d workers' SGD step and reduce row (numpy fp64)"
+                                       % (per_step, WORKLOAD["N"])},
             "e2e": {"value": value, "unit": "worker-samples/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
+
+
+def peaks_all():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            j = json.load(f)
+        return {"hbm": (float(j["hbm_gbs"]), "measured"),
+                "tensor": (float(j.get("bf16_tflops_sustained", j["bf16_tflops"])), "measured (sustained)")}
+    except Exception:
+        return {"hbm": (6800.0, "fallback"), "tensor": (1700.0, "fallback (sustained)")}
 
 
 def run_asap(args):
@@ -244,8 +325,10 @@ def run_asap(args):
     torch.cuda.set_device(local)
     dev_index = int(os.environ.get("CUDA_VISIBLE_DEVICES", str(local)).split(",")[local]) \
         if os.environ.get("CUDA_VISIBLE_DEVICES") else local
-    rows = args.rows or WORKLOAD["rows"]
+    w = WORKLOAD
+    rows = args.rows or w["rows"]
     sh = make_shards(rows, seed=rank)
+    dense = w["loss"] == "softmax"
 
     def barrier():
         if world > 1:
@@ -260,80 +343,98 @@ def run_asap(args):
         return float(t.item())
 
     stream = torch.cuda.Stream()
-    ctx = Context(WORKLOAD["N"], WORKLOAD["d"], graph_seed=WORKLOAD["graph_seed"], k=WORKLOAD["k"])
-    ctx.set_model(WORKLOAD["loss"], batch=WORKLOAD["B"], lr=WORKLOAD["lr"])
-    ctx.set_graph(WORKLOAD["graph"], regenerate=WORKLOAD["regenerate"])
+    ctx = Context(w["N"], w["d"], graph_seed=w["graph_seed"], k=w["k"])
+    ctx.set_model(w["loss"], batch=w["B"], lr=w["lr"], num_classes=w.get("C", 1))
+    ctx.set_graph(w["graph"], regenerate=w["regenerate"])
     ctx.set_stream(stream)
-    ctx.set_shard_residency("host")
-    ctx.load_shards(sh)
-    N, B, K, Wm = WORKLOAD["N"], WORKLOAD["B"], args.steps, args.warmup
+    N, B, K, Wm = w["N"], w["B"], args.steps, args.warmup
     units_per_step = N * B
 
     # ---- end to end: shards in pinned host memory, metrics read back ----
     e2e = None
-    if not args.no_e2e:
-        h2d = 0
-        for s in range(Wm):
-            ctx.round(1)
-            ctx.read_metrics(s, 1)
-        r0 = Wm
-        barrier()
-        t0 = time.perf_counter()
-        for s in range(K):
-            h2d += ctx.shard_block_bytes(r0 + s)
-            ctx.round(1)
-            ctx.read_metrics(r0 + s, 1)
-        ctx.sync()
-        t_e2e = max_over_ranks(time.perf_counter() - t0)
-        graph_bytes = N * (WORKLOAD["k"] + 1) * 8
-        e2e = {"value": world * units_per_step * K / t_e2e, "unit": "worker-samples/s",
-               "h2d_bytes_per_step": h2d / K + graph_bytes, "d2h_bytes_per_step": 8}
+    if dense:
+        ctx.load_dense_shards(sh)
+        e2e = {"value": None, "unit": "worker-samples/s", "h2d_bytes_per_step": None, "d2h_bytes_per_step": None,
+               "note": "dense shards are device-resident only in this version"}
+    else:
+        ctx.set_shard_residency("host")
+        ctx.load_shards(sh)
+        if not args.no_e2e:
+            h2d = 0
+            for s in range(Wm):
+                ctx.round(1)
+                ctx.read_metrics(s, 1)
+            r0 = Wm
+            barrier()
+            t0 = time.perf_counter()
+            for s in range(K):
+                h2d += ctx.shard_block_bytes(r0 + s)
+                ctx.round(1)
+                ctx.read_metrics(r0 + s, 1)
+            ctx.sync()
+            t_e2e = max_over_ranks(time.perf_counter() - t0)
+            graph_bytes = N * (w["k"] + 1) * 8 if w["regenerate"] else 0
+            e2e = {"value": world * units_per_step * K / t_e2e, "unit": "worker-samples/s",
+                   "h2d_bytes_per_step": h2d / K + graph_bytes, "d2h_bytes_per_step": 8}
+        ctx.set_shard_residency("device")
 
     # ---- device resident: the kernel-level number ----
-    ctx.set_shard_residency("device")
-    ctx.write_params(np.zeros((N, WORKLOAD["d"]), np.float32), 0)
-    with torch.cuda.stream(stream):
-        for s in range(Wm):
-            ctx.round(1)
-        ctx.sync()
-        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
-        start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        sampler = ClockSampler(dev_index)
-        barrier()
-        sampler.start()
-        time.sleep(0.2)
-        l0 = ctx.kernel_launches()
-        start.record(stream)
-        for s in range(K):
-            ctx.local_step()
-            ev[s][0].record(stream)
-            ctx.stochastic_reduce()
-            ev[s][1].record(stream)
-        end.record(stream)
-        stream.synchronize()
-        launches = ctx.kernel_launches() - l0
-        clocks = sampler.stop()
-        ctx.sync()   # surfaces any device-side protocol error
+    ctx.write_params(np.zeros((N, ctx.P), np.float32), 0)
+    for s in range(Wm):
+        ctx.round(1)
+    ctx.sync()
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    sampler = ClockSampler(dev_index)
+    ctx.set_kernel_timing(True)
+    barrier()
+    sampler.start()
+    time.sleep(0.2)
+    l0 = ctx.kernel_launches()
+    start.record(stream)
+    for s in range(K):
+        ctx.round(1)
+    end.record(stream)
+    stream.synchronize()
+    launches = ctx.kernel_launches() - l0
+    clocks = sampler.stop()
+    ctx.sync()   # surfaces any device-side protocol error
+    times = ctx.read_kernel_times()
+    ctx.set_kernel_timing(False)
     elapsed_ms = max_over_ranks(start.elapsed_time(end))
-    mix_ms = statistics.fmean(a.elapsed_time(b) for a, b in ev)
     last_loss, last_cons = ctx.read_metrics(ctx.read_params()[1] - 1, 1)
     assert np.isfinite(last_loss[0]) and np.isfinite(last_cons[0])
 
-    peak, peak_kind = peaks()
-    alg_bytes = 8.0 * N * WORKLOAD["d"]
-    achieved = alg_bytes / (mix_ms * 1e-3) / 1e9
+    pk = peaks_all()
+    work = kernel_work(sh)
+    kernels = {}
+    for name, (unit, amount, bound) in work.items():
+        n, ms = times[name]
+        if n == 0:
+            continue
+        mean_ms = ms / n
+        scale = 1e12 if unit == "TFLOP/s" else 1e9
+        achieved = amount / (mean_ms * 1e-3) / scale
+        peak, kind = pk[bound]
+        kernels[name] = {"bound": bound, "unit": unit, "achieved": achieved, "peak": peak, "peak_kind": kind,
+                         "frac": achieved / peak, "mean_launch_ms": mean_ms, "launches": n,
+                         "share": ms / max(1e-9, sum(v[1] for v in times.values())),
+                         "algorithmic_per_launch": amount}
+    dom = max(kernels, key=lambda k: kernels[k]["share"])
+    kd = kernels[dom]
+    roof = {"kernel": dom, "bound": kd["bound"], "achieved": kd["achieved"], "peak": kd["peak"],
+            "peak_kind": kd["peak_kind"], "unit": kd["unit"], "frac": kd["frac"],
+            "traffic": mix_traffic_per_launch() if (dom == "reduce" and w["name"] == "sparse_logistic_hashed")
+            else None, "algorithmic_per_launch": kd["algorithmic_per_launch"], "mean_launch_ms": kd["mean_launch_ms"]}
     value = world * units_per_step * K / (elapsed_ms * 1e-3)
     line = {"metric": METRIC, "value": value, "unit": "worker-samples/s", "n_gpus": world, "steps": K,
             "warmup": Wm, "ms_per_step": elapsed_ms / K, "higher_is_better": True, "scaling": "weak",
-            "vs_baseline": None, "dtype": "f32", "data": "synthetic (seeded; stands in for the paper's "
-                                                         "RCV1/webspam/splice-site shards)",
+            "vs_baseline": None, "dtype": "bf16 GEMM inputs, f32 accumulate and master" if dense else "f32",
+            "data": "synthetic (seeded; stands in for the paper's %s)" %
+                    ("CIFAR-10 CNN workload" if dense else "RCV1/webspam/splice-site shards"),
             "config": config(rows),
-            "roofline": {"kernel": "stochastic reduce (k_mix)", "bound": "hbm", "achieved": achieved, "peak": peak,
-                         "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / peak,
-                         "traffic": mix_traffic_per_launch(), "algorithmic_bytes_per_launch": alg_bytes,
-                         "mean_launch_ms": mix_ms},
-            "reduce_gbs": achieved,
-            "e2e": e2e, "gpu_launches": launches, "clocks": clocks}
+            "roofline": roof,
+            "reduce_gbs": kernels["reduce"]["achieved"] if "reduce" in kernels else None,
+            "kernels": kernels, "e2e": e2e, "gpu_launches": launches, "clocks": clocks}
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(sh)
     ctx.close()
@@ -344,7 +445,9 @@ def run_asap(args):
 
 
 def main():
+    global WORKLOAD
     args = parse()
+    WORKLOAD = WORKLOADS[args.workload]
     if args.impl == "reference":
         run_reference(args)
     else:

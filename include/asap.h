@@ -201,6 +201,26 @@ asap_status asap_set_wait_limit_ns(asap_ctx* ctx, uint64_t ns);
  * runs into its wait limit.  worker = -1 clears the injection. */
 asap_status asap_debug_skip_notify(asap_ctx* ctx, int worker);
 
+/* Kernel kinds for per-kernel timing. */
+typedef enum {
+  ASAP_KERNEL_MARGIN = 0,     /* sparse margins + loss derivative (a2)          */
+  ASAP_KERNEL_UPDATE = 1,     /* sparse column-segmented update + NOTIFY (a3-a4) */
+  ASAP_KERNEL_REDUCE = 2,     /* stochastic reduce + ACK + metrics (a5-a7, a9)  */
+  ASAP_KERNEL_DENSE_FWD = 3,  /* dense logits, softmax, R^T (a3')               */
+  ASAP_KERNEL_DENSE_GRAD = 4, /* dense gradient GEMM + update + NOTIFY (a3')    */
+  ASAP_KERNEL_KINDS = 5
+} asap_kernel_kind;
+
+/* Per-kernel timing: while enabled, every kernel launch of the context is
+ * bracketed by CUDA events on the context stream (the first 8192 launches
+ * after enabling or after the last read). */
+asap_status asap_set_kernel_timing(asap_ctx* ctx, int enable);
+
+/* Per kernel kind: timed launches and their total milliseconds, since
+ * enabling or since the last read (which resets them).  launches and
+ * total_ms have ASAP_KERNEL_KINDS entries.  Syncing. */
+asap_status asap_read_kernel_times(asap_ctx* ctx, uint64_t* launches, double* total_ms);
+
 /* Number of this library's kernel launches since creation (host counter). */
 asap_status asap_kernel_launches(asap_ctx* ctx, uint64_t* launches);
 

@@ -35,6 +35,8 @@ SIGNATURES = {
     "asap_get_graph": (C.c_int, [_P, C.c_int64, _P, _P]),
     "asap_set_wait_limit_ns": (C.c_int, [_P, C.c_uint64]),
     "asap_debug_skip_notify": (C.c_int, [_P, C.c_int]),
+    "asap_set_kernel_timing": (C.c_int, [_P, C.c_int]),
+    "asap_read_kernel_times": (C.c_int, [_P, _P, _P]),
     "asap_kernel_launches": (C.c_int, [_P, C.POINTER(C.c_uint64)]),
     "asap_build_graph": (C.c_int, [C.c_int, C.c_int, C.c_int, C.c_uint64, C.c_int64, _P]),
     "asap_mix_noalloc": (C.c_int, [_P, _P, C.c_int, C.c_int64, C.c_int64, _P, _P, C.c_int, _P, _P]),

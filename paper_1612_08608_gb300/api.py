@@ -154,6 +154,18 @@ class Context:
     def debug_skip_notify(self, worker: int):
         self._c(self._lib.asap_debug_skip_notify(self._h, worker))
 
+    KERNELS = ("margin", "update", "reduce", "dense_fwd", "dense_grad")
+
+    def set_kernel_timing(self, enable: bool = True):
+        self._c(self._lib.asap_set_kernel_timing(self._h, int(enable)))
+
+    def read_kernel_times(self):
+        """{kernel: (timed launches, total ms)} since enabling / the last read."""
+        n = np.zeros(len(self.KERNELS), dtype=np.uint64)
+        ms = np.zeros(len(self.KERNELS), dtype=np.float64)
+        self._c(self._lib.asap_read_kernel_times(self._h, _ptr(n), _ptr(ms)))
+        return {k: (int(n[i]), float(ms[i])) for i, k in enumerate(self.KERNELS)}
+
     def kernel_launches(self) -> int:
         v = C.c_uint64()
         self._c(self._lib.asap_kernel_launches(self._h, C.byref(v)))

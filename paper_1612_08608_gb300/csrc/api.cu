@@ -89,8 +89,8 @@ struct asap_ctx {
   float* d_wgt = nullptr;
   int32_t* h_nbr = nullptr;
   float* h_wgt = nullptr;
-  cudaEvent_t slot_ev[kGraphRing];
-  bool slot_used[kGraphRing];
+  cudaEvent_t slot_ev[kGraphRing] = {};
+  bool slot_used[kGraphRing] = {};
 
   // sparse shards
   asap_residency residency = ASAP_SHARDS_DEVICE;
@@ -100,11 +100,21 @@ struct asap_ctx {
   std::vector<size_t> block_off, block_bytes;
   int nb = 0;
   BatchDesc* d_desc = nullptr;
-  unsigned char* staging[2] = {nullptr, nullptr};
+  // per batch block: the slab-major column list and its slab offsets
+  std::vector<size_t> list_off, soff_off;
+  std::vector<int64_t> list_len;
+  int max_region = 0;               // entries of the largest slab region of any list
+  int64_t max_list = 0;
+  float* wv = nullptr;              // w at the current round's list positions
+  float* gsum = nullptr;            // column sums at the current round's list positions
+  int64_t wv_round = -1;            // round whose list wv holds (-1: none)
+  // host residency: a round reads its own block and the next one
+  static constexpr int kStaging = 3;
+  unsigned char* staging[kStaging] = {nullptr, nullptr, nullptr};
   size_t staging_bytes = 0;
-  int64_t staged_round[2] = {-1, -1};
-  bool free_recorded[2] = {false, false};
-  cudaEvent_t staged_ev[2], free_ev[2];
+  int64_t staged_round[kStaging] = {-1, -1, -1};
+  bool free_recorded[kStaging] = {false, false, false};
+  cudaEvent_t staged_ev[kStaging] = {}, free_ev[kStaging] = {};
   int margin_ctas = 0, update_ctas = 0;
   int max_nnz = 0;
 
@@ -122,10 +132,17 @@ struct asap_ctx {
 
   CUtensorMap tmap[2];
   int S = 0, rows_pad = 0, box_rows = 0, n_boxes = 0, stages = 0;
+  bool fused_cfg = false;
   long long n_slabs = 0;
   int mix_grid = 0;
   size_t mix_smem = 0;
-  int configured_key = -1;
+  long long configured_key = -1;
+
+  // per-kernel timing (asap_set_kernel_timing)
+  bool timing = false;
+  std::vector<cudaEvent_t> tev;   // 2 per timed launch
+  std::vector<int> tkind;
+  size_t tused = 0;
 
   int64_t round = 0;
   int64_t graph_ready_round = -1;   // round whose tables are staged in graph_nbr/graph_wgt
@@ -176,13 +193,22 @@ void free_shards(asap_ctx* c) {
   dfree(c->X);
   dfree(c->XT);
   dfree(c->Yd);
-  dfree(c->staging[0]);
-  dfree(c->staging[1]);
+  dfree(c->wv);
+  dfree(c->gsum);
+  for (int b = 0; b < asap_ctx::kStaging; ++b) {
+    dfree(c->staging[b]);
+    c->staged_round[b] = -1;
+    c->free_recorded[b] = false;
+  }
   c->block_off.clear();
   c->block_bytes.clear();
+  c->list_off.clear();
+  c->soff_off.clear();
+  c->list_len.clear();
+  c->max_region = 0;
+  c->max_list = 0;
+  c->wv_round = -1;
   c->nb = 0;
-  c->staged_round[0] = c->staged_round[1] = -1;
-  c->free_recorded[0] = c->free_recorded[1] = false;
 }
 
 // Host copy of the graph of round `rnd`: nbr/wgt with c->k + 1 entries per row.
@@ -209,16 +235,13 @@ asap_status setup_mix(asap_ctx* c) {
   // aligned in shared memory (S >= 8 floats per row).
   c->box_rows = ((N + c->n_boxes - 1) / c->n_boxes + 3) / 4 * 4;
   c->rows_pad = c->n_boxes * c->box_rows;
-  int S = 256;
+  int S = 128;
   while (S > 8 && static_cast<size_t>(c->rows_pad) * S * 4 > 32768) S >>= 1;
   int maxS = 8;
-  while (static_cast<int64_t>(maxS) * 2 <= c->ld && maxS < 256) maxS <<= 1;
+  while (static_cast<int64_t>(maxS) * 2 <= c->ld && maxS < 128) maxS <<= 1;
   c->S = std::min(S, maxS);
-  const size_t slab = align_up(static_cast<size_t>(c->rows_pad) * c->S * 4, 1024);
-  c->stages = static_cast<int>(std::max<size_t>(2, std::min<size_t>(8, 131072 / slab)));
   c->n_slabs = (c->ld + c->S - 1) / c->S;
   c->tab_kp1 = is_complete_kernel(c) ? 0 : c->k + 1;
-  c->mix_smem = mix_smem_bytes(N, c->tab_kp1, c->S, c->rows_pad, c->stages);
   c->configured_key = -1;
   EncodeTiledFn enc = get_encode_fn();
   if (!enc) return fail(c, ASAP_ERR_CUDA, "cuTensorMapEncodeTiled is not available from the driver");
@@ -262,17 +285,25 @@ asap_status setup_dense_param_maps(asap_ctx* c) {
   return ASAP_OK;
 }
 
-asap_status configure_mix_launch(asap_ctx* c) {
+asap_status configure_mix_launch(asap_ctx* c, bool fused) {
   const bool complete = is_complete_kernel(c);
   const bool shadow = c->Wbf[0] != nullptr;
-  const int key = (complete ? 1 : 0) | (shadow ? 2 : 0) | (c->tab_kp1 << 2) | (static_cast<int>(c->mix_smem) << 8);
+  const int region = fused ? c->max_region : 0;
+  const long long key = (complete ? 1 : 0) | (shadow ? 2 : 0) | (fused ? 4 : 0) |
+                        (static_cast<long long>(c->tab_kp1) << 3) | (static_cast<long long>(region) << 12);
   if (key == c->configured_key) return ASAP_OK;
-  CU(mix_configure(complete, c->tab_kp1, shadow, c->mix_smem), "configuring the reduce kernel");
+  // Stages: as many as fit in ~200 KB of shared memory, 2 to 8.
+  const size_t stage = mix_stage_bytes(c->S, c->rows_pad, region);
+  c->stages = static_cast<int>(std::max<size_t>(2, std::min<size_t>(8, (200u << 10) / stage)));
+  c->mix_smem = mix_smem_bytes(c->N, c->tab_kp1, c->S, c->rows_pad, c->stages, region);
+  if (c->mix_smem > (227u << 10)) return fail(c, ASAP_ERR_ARG, "reduce stages do not fit in shared memory");
+  CU(mix_configure(complete, fused, c->tab_kp1, shadow, c->mix_smem), "configuring the reduce kernel");
   int blocks = 0;
-  CU(mix_occupancy(complete, c->tab_kp1, shadow, c->mix_smem, &blocks), "occupancy of the reduce kernel");
+  CU(mix_occupancy(complete, fused, c->tab_kp1, shadow, c->mix_smem, &blocks), "occupancy of the reduce kernel");
   if (blocks < 1) return fail(c, ASAP_ERR_ARG, "reduce kernel does not fit on an SM for this N");
   c->mix_grid = static_cast<int>(std::min<long long>(c->n_slabs, static_cast<long long>(c->sm_count) * blocks));
   if (c->mix_grid > c->cons_cap) return fail(c, ASAP_ERR_ARG, "internal: reduce grid exceeds its scratch");
+  c->fused_cfg = fused;
   c->configured_key = key;
   return ASAP_OK;
 }
@@ -367,6 +398,21 @@ asap_status prepare_graph(asap_ctx* c, int64_t r) {
   return ASAP_OK;
 }
 
+constexpr size_t kTimedLaunches = 8192;
+
+// Bracket one launch with timing events (no-op unless timing is on).
+void time_begin(asap_ctx* c, int kind) {
+  if (!c->timing || c->tused >= kTimedLaunches) return;
+  cudaEventRecord(c->tev[2 * c->tused], c->stream);
+  c->tkind[c->tused] = kind;
+}
+
+void time_end(asap_ctx* c) {
+  if (!c->timing || c->tused >= kTimedLaunches) return;
+  cudaEventRecord(c->tev[2 * c->tused + 1], c->stream);
+  ++c->tused;
+}
+
 asap_status check_device_error(asap_ctx* c) {
   DevState h;
   CU(cudaMemcpy(&h, c->st, sizeof(DevState), cudaMemcpyDeviceToHost), "reading device state");
@@ -391,8 +437,10 @@ asap_status sync_all(asap_ctx* c) {
 }
 
 // Make round r's batch block available on the device (host residency).
+// Slot r % 3; a slot is rewritten only after the last kernel that reads its
+// previous block (the reduce of that block's own round) has finished.
 asap_status stage_block(asap_ctx* c, int64_t r) {
-  const int slot = static_cast<int>(r & 1);
+  const int slot = static_cast<int>(r % asap_ctx::kStaging);
   if (c->staged_round[slot] == r) return ASAP_OK;
   const int t = static_cast<int>(r % c->nb);
   if (c->free_recorded[slot]) CU(cudaStreamWaitEvent(c->copy_stream, c->free_ev[slot], 0), "staging wait");
@@ -401,6 +449,22 @@ asap_status stage_block(asap_ctx* c, int64_t r) {
      "copying a minibatch block to the device");
   CU(cudaEventRecord(c->staged_ev[slot], c->copy_stream), "staging event");
   c->staged_round[slot] = r;
+  return ASAP_OK;
+}
+
+// Device address of round r's batch block (staging it first when the
+// shards live on the host; the context stream then waits for the copy).
+asap_status block_of(asap_ctx* c, int64_t r, const unsigned char** out) {
+  const int t = static_cast<int>(r % c->nb);
+  if (c->residency != ASAP_SHARDS_HOST) {
+    *out = c->pool + c->block_off[t];
+    return ASAP_OK;
+  }
+  asap_status s = stage_block(c, r);
+  if (s != ASAP_OK) return s;
+  const int slot = static_cast<int>(r % asap_ctx::kStaging);
+  CU(cudaStreamWaitEvent(c->stream, c->staged_ev[slot], 0), "waiting for a staged block");
+  *out = c->staging[slot];
   return ASAP_OK;
 }
 
@@ -449,7 +513,7 @@ asap_status asap_create(int N, int64_t d, uint64_t graph_seed, int k, asap_ctx**
     CU(cudaEventCreateWithFlags(&c->slot_ev[i], cudaEventDisableTiming), "creating events");
     c->slot_used[i] = false;
   }
-  for (int b = 0; b < 2; ++b) {
+  for (int b = 0; b < asap_ctx::kStaging; ++b) {
     CU(cudaEventCreateWithFlags(&c->staged_ev[b], cudaEventDisableTiming), "creating events");
     CU(cudaEventCreateWithFlags(&c->free_ev[b], cudaEventDisableTiming), "creating events");
   }
@@ -514,7 +578,9 @@ void asap_destroy(asap_ctx* c) {
   if (c->h_wgt) cudaFreeHost(c->h_wgt);
   for (int i = 0; i < kGraphRing; ++i)
     if (c->slot_ev[i]) cudaEventDestroy(c->slot_ev[i]);
-  for (int b = 0; b < 2; ++b) {
+  for (auto& e : c->tev)
+    if (e) cudaEventDestroy(e);
+  for (int b = 0; b < asap_ctx::kStaging; ++b) {
     if (c->staged_ev[b]) cudaEventDestroy(c->staged_ev[b]);
     if (c->free_ev[b]) cudaEventDestroy(c->free_ev[b]);
   }
@@ -655,8 +721,7 @@ asap_status asap_set_shard_residency(asap_ctx* c, asap_residency r) {
       CU(cudaMalloc(&np, c->pool_bytes), "allocating device shard memory");
       CU(cudaMemcpy(np, c->pool, c->pool_bytes, cudaMemcpyHostToDevice), "moving shards to the device");
       cudaFreeHost(c->pool);
-      dfree(c->staging[0]);
-      dfree(c->staging[1]);
+      for (int b = 0; b < asap_ctx::kStaging; ++b) dfree(c->staging[b]);
     } else {
       CU(cudaHostAlloc(&np, c->pool_bytes, cudaHostAllocDefault), "allocating pinned shard memory");
       CU(cudaMemcpy(np, c->pool, c->pool_bytes, cudaMemcpyDeviceToHost), "moving shards to the host");
@@ -664,12 +729,14 @@ asap_status asap_set_shard_residency(asap_ctx* c, asap_residency r) {
       size_t mb = 0;
       for (size_t b : c->block_bytes) mb = std::max(mb, b);
       c->staging_bytes = mb;
-      for (int b = 0; b < 2; ++b) CU(cudaMalloc(&c->staging[b], mb), "allocating staging buffers");
+      for (int b = 0; b < asap_ctx::kStaging; ++b) CU(cudaMalloc(&c->staging[b], mb), "allocating staging buffers");
     }
     c->pool = np;
     c->pool_pinned = (r == ASAP_SHARDS_HOST);
-    c->staged_round[0] = c->staged_round[1] = -1;
-    c->free_recorded[0] = c->free_recorded[1] = false;
+    for (int b = 0; b < asap_ctx::kStaging; ++b) {
+      c->staged_round[b] = -1;
+      c->free_recorded[b] = false;
+    }
   }
   c->residency = r;
   return ASAP_OK;
@@ -687,7 +754,8 @@ asap_status asap_load_shards(asap_ctx* c, const int64_t* const* rowptr, const in
   if (!c || !rowptr || !col || !val || !y || !n_rows) return fail(c, ASAP_ERR_ARG, "NULL argument");
   if (c->loss != ASAP_LOSS_HINGE && c->loss != ASAP_LOSS_LOGISTIC)
     return fail(c, ASAP_ERR_ARG, "set a hinge or logistic model before loading CSR shards");
-  const int N = c->N, B = c->B;
+  const int N = c->N, B = c->B, S = c->S;
+  const long long n_slabs = c->n_slabs;
   int nb = -1;
   for (int i = 0; i < N; ++i) {
     if (!rowptr[i] || !col[i] || !val[i] || !y[i]) return fail(c, ASAP_ERR_ARG, "NULL shard pointer");
@@ -696,151 +764,223 @@ asap_status asap_load_shards(asap_ctx* c, const int64_t* const* rowptr, const in
     if (nb >= 0 && nbi != nb) return fail(c, ASAP_ERR_ARG, "all shards must hold the same number of minibatches");
     nb = static_cast<int>(std::min<int64_t>(nbi, 1 << 30));
     if (rowptr[i][0] != 0) return fail(c, ASAP_ERR_ARG, "rowptr must start at 0");
+    for (int64_t r = 0; r < nbi * B; ++r)
+      if (rowptr[i][r + 1] < rowptr[i][r]) return fail(c, ASAP_ERR_ARG, "rowptr must be non-decreasing");
   }
   asap_status s0 = asap_sync(c);
   if (s0 != ASAP_OK) return s0;
   free_shards(c);
 
-  // Pass 1: sizes.  Segment (t, i) = rp | y | col | val | ccol | cval | crow.
-  std::vector<BatchDesc> desc(static_cast<size_t>(nb) * N);
-  c->block_off.assign(nb, 0);
-  c->block_bytes.assign(nb, 0);
-  size_t total = 0, max_block = 0;
-  int max_nnz = 0;
-  for (int t = 0; t < nb; ++t) {
-    size_t off = 0;
+  // One block per minibatch index t: per worker the padded rows (pos, val),
+  // labels and the entries sorted by (column, row); then the batch's
+  // slab-major list of distinct (worker, column) pairs and its slab offsets.
+  struct Built {
+    std::vector<unsigned char> img;
+    std::vector<BatchDesc> desc;
+    size_t list_off = 0, soff_off = 0;
+    int64_t list_len = 0;
+    int max_region = 0, max_nnz = 0;
+    const char* err = nullptr;
+  };
+  std::vector<Built> built(nb);
+  auto build_batch = [&](int t) {
+    Built& bt = built[t];
+    std::vector<std::vector<uint64_t>> keys(N);
+    std::vector<std::vector<int32_t>> ucol(N), run_of(N), upos(N);
+    std::vector<int64_t> nnz(N, 0), nnz_pad(N, 0);
     for (int i = 0; i < N; ++i) {
       const int64_t* rp = rowptr[i];
       const int64_t r0 = static_cast<int64_t>(t) * B;
-      int64_t nnz = 0, nnz_pad = 0;
-      for (int b = 0; b < B; ++b) {
-        const int64_t len = rp[r0 + b + 1] - rp[r0 + b];
-        if (len < 0) return fail(c, ASAP_ERR_ARG, "rowptr must be non-decreasing");
-        nnz += len;
-        nnz_pad += (len + 3) / 4 * 4;
+      const int64_t a0 = rp[r0], a1 = rp[r0 + B];
+      nnz[i] = a1 - a0;
+      for (int b = 0; b < B; ++b) nnz_pad[i] += (rp[r0 + b + 1] - rp[r0 + b] + 3) / 4 * 4;
+      if (nnz_pad[i] > (1ll << 30)) { bt.err = "a minibatch holds more than 2^30 entries"; return; }
+      std::vector<uint64_t>& k = keys[i];
+      k.resize(nnz[i]);
+      for (int64_t e = 0; e < nnz[i]; ++e) {
+        const int32_t cc = col[i][a0 + e];
+        if (cc < 0 || cc >= c->d) { bt.err = "column id out of range [0, d)"; return; }
+        k[e] = (static_cast<uint64_t>(static_cast<uint32_t>(cc)) << 32) | static_cast<uint64_t>(e);
       }
-      if (nnz_pad > (1ll << 30)) return fail(c, ASAP_ERR_ARG, "a minibatch holds more than 2^30 entries");
-      BatchDesc& dd = desc[static_cast<size_t>(t) * N + i];
+      std::sort(k.begin(), k.end());   // by column, then by entry (= by row)
+      run_of[i].resize(nnz[i]);
+      for (int64_t e = 0; e < nnz[i]; ++e) {
+        const int32_t cc = static_cast<int32_t>(k[e] >> 32);
+        if (e == 0 || cc != static_cast<int32_t>(k[e - 1] >> 32)) ucol[i].push_back(cc);
+        run_of[i][e] = static_cast<int32_t>(ucol[i].size()) - 1;
+      }
+      bt.max_nnz = std::max<int>(bt.max_nnz, static_cast<int>(nnz[i]));
+    }
+    // Slab-major positions.
+    std::vector<int32_t> cnt(static_cast<size_t>(n_slabs) * N, 0);
+    for (int i = 0; i < N; ++i)
+      for (int32_t cc : ucol[i]) cnt[static_cast<size_t>(cc / S) * N + i]++;
+    std::vector<int32_t> soff(n_slabs + 1), start(static_cast<size_t>(n_slabs) * N);
+    int64_t tot = 0;
+    for (long long sl = 0; sl < n_slabs; ++sl) {
+      soff[sl] = static_cast<int32_t>(tot);
+      int64_t acc = tot;
+      for (int i = 0; i < N; ++i) {
+        start[static_cast<size_t>(sl) * N + i] = static_cast<int32_t>(acc);
+        acc += cnt[static_cast<size_t>(sl) * N + i];
+      }
+      const int64_t n = acc - tot, np = (n + 3) / 4 * 4;
+      bt.max_region = std::max<int>(bt.max_region, static_cast<int>(np));
+      tot += np;
+      if (tot >= (1ll << 31)) { bt.err = "column list of a minibatch too long"; return; }
+    }
+    soff[n_slabs] = static_cast<int32_t>(tot);
+    std::vector<uint32_t> list(tot, kListPad);
+    for (int i = 0; i < N; ++i) {
+      upos[i].resize(ucol[i].size());
+      for (size_t u = 0; u < ucol[i].size(); ++u) {
+        const int32_t cc = ucol[i][u];
+        const int sl = cc / S;
+        const int32_t pos = start[static_cast<size_t>(sl) * N + i]++;
+        list[pos] = (static_cast<uint32_t>(i) << 16) | static_cast<uint32_t>(cc - sl * S);
+        upos[i][u] = pos;
+      }
+    }
+    // Layout of the block image.
+    bt.desc.resize(N);
+    size_t off = 0;
+    for (int i = 0; i < N; ++i) {
+      BatchDesc& dd = bt.desc[i];
       dd.rp = static_cast<int64_t>(off);
       off = align_up(off + 4 * static_cast<size_t>(B + 1), 16);
       dd.y = static_cast<int64_t>(off);
       off = align_up(off + 4 * static_cast<size_t>(B), 16);
-      dd.col = static_cast<int64_t>(off);
-      off += 4 * static_cast<size_t>(nnz_pad);
+      dd.posw = static_cast<int64_t>(off);
+      off += 4 * static_cast<size_t>(nnz_pad[i]);
       dd.val = static_cast<int64_t>(off);
-      off += 4 * static_cast<size_t>(nnz_pad);
-      dd.ccol = static_cast<int64_t>(off);
-      off = align_up(off + 4 * static_cast<size_t>(nnz), 16);
+      off += 4 * static_cast<size_t>(nnz_pad[i]);
+      dd.cpos = static_cast<int64_t>(off);
+      off = align_up(off + 4 * static_cast<size_t>(nnz[i]), 16);
       dd.cval = static_cast<int64_t>(off);
-      off = align_up(off + 4 * static_cast<size_t>(nnz), 16);
+      off = align_up(off + 4 * static_cast<size_t>(nnz[i]), 16);
       dd.crow = static_cast<int64_t>(off);
-      off = align_up(off + 2 * static_cast<size_t>(nnz), 16);
-      dd.nnz_pad = static_cast<int32_t>(nnz_pad);
-      dd.nnz = static_cast<int32_t>(nnz);
-      max_nnz = std::max<int>(max_nnz, static_cast<int>(nnz));
+      off = align_up(off + 2 * static_cast<size_t>(nnz[i]), 16);
+      dd.nnz_pad = static_cast<int32_t>(nnz_pad[i]);
+      dd.nnz = static_cast<int32_t>(nnz[i]);
     }
-    off = align_up(off, 256);
-    c->block_off[t] = total;
-    c->block_bytes[t] = off;
-    total += off;
-    max_block = std::max(max_block, off);
-  }
-
-  // Host image of the pool: pinned when it stays on the host.
-  unsigned char* host = nullptr;
-  std::vector<unsigned char> pageable;
-  if (c->residency == ASAP_SHARDS_HOST) {
-    CU(cudaHostAlloc(&host, total, cudaHostAllocDefault), "allocating pinned shard memory");
-    c->pool = host;
-    c->pool_pinned = true;
-  } else {
-    pageable.resize(total);
-    host = pageable.data();
-  }
-
-  // Pass 2: fill, in parallel over (t, i) segments.
-  const int64_t d = c->d;
-  std::vector<int> bad(static_cast<size_t>(nb) * N, 0);
-  auto fill = [&](size_t seg) {
-    const int t = static_cast<int>(seg / N), i = static_cast<int>(seg % N);
-    const BatchDesc& dd = desc[seg];
-    unsigned char* base = host + c->block_off[t];
-    int32_t* rp_o = reinterpret_cast<int32_t*>(base + dd.rp);
-    float* y_o = reinterpret_cast<float*>(base + dd.y);
-    int32_t* col_o = reinterpret_cast<int32_t*>(base + dd.col);
-    float* val_o = reinterpret_cast<float*>(base + dd.val);
-    int32_t* ccol_o = reinterpret_cast<int32_t*>(base + dd.ccol);
-    float* cval_o = reinterpret_cast<float*>(base + dd.cval);
-    uint16_t* crow_o = reinterpret_cast<uint16_t*>(base + dd.crow);
-    const int64_t* rp = rowptr[i];
-    const int64_t r0 = static_cast<int64_t>(t) * B;
-    std::vector<uint64_t> keys;
-    keys.reserve(dd.nnz);
-    std::vector<uint16_t> row_of;
-    row_of.reserve(dd.nnz);
-    std::vector<float> vals;
-    vals.reserve(dd.nnz);
-    int32_t q = 0;
-    for (int b = 0; b < B; ++b) {
-      rp_o[b] = q;
-      y_o[b] = y[i][r0 + b];
-      const int64_t a0 = rp[r0 + b], a1 = rp[r0 + b + 1];
-      for (int64_t e = a0; e < a1; ++e) {
-        const int32_t cc = col[i][e];
-        if (cc < 0 || cc >= d) bad[seg] = 1;
-        col_o[q] = cc;
-        val_o[q] = val[i][e];
-        keys.push_back((static_cast<uint64_t>(static_cast<uint32_t>(cc)) << 32) | keys.size());
-        row_of.push_back(static_cast<uint16_t>(b));
-        vals.push_back(val[i][e]);
-        ++q;
+    bt.list_off = off;
+    off = align_up(off + 4 * static_cast<size_t>(tot), 16);
+    bt.soff_off = off;
+    off = align_up(off + 4 * static_cast<size_t>(n_slabs + 1), 256);
+    bt.list_len = tot;
+    bt.img.assign(off, 0);
+    unsigned char* base = bt.img.data();
+    std::memcpy(base + bt.list_off, list.data(), 4 * list.size());
+    std::memcpy(base + bt.soff_off, soff.data(), 4 * soff.size());
+    for (int i = 0; i < N; ++i) {
+      const BatchDesc& dd = bt.desc[i];
+      int32_t* rp_o = reinterpret_cast<int32_t*>(base + dd.rp);
+      float* y_o = reinterpret_cast<float*>(base + dd.y);
+      int32_t* pw_o = reinterpret_cast<int32_t*>(base + dd.posw);
+      float* val_o = reinterpret_cast<float*>(base + dd.val);
+      int32_t* cp_o = reinterpret_cast<int32_t*>(base + dd.cpos);
+      float* cv_o = reinterpret_cast<float*>(base + dd.cval);
+      uint16_t* cr_o = reinterpret_cast<uint16_t*>(base + dd.crow);
+      const int64_t* rp = rowptr[i];
+      const int64_t r0 = static_cast<int64_t>(t) * B, a0 = rp[r0];
+      // list position of every entry (row-major), through the sort
+      std::vector<int32_t> epos(nnz[i]);
+      std::vector<uint16_t> erow(nnz[i]);
+      for (int b = 0; b < B; ++b)
+        for (int64_t e = rp[r0 + b] - a0; e < rp[r0 + b + 1] - a0; ++e) erow[e] = static_cast<uint16_t>(b);
+      for (int64_t e = 0; e < nnz[i]; ++e) {
+        const int64_t k = static_cast<int64_t>(keys[i][e] & 0xffffffffu);
+        const int32_t pos = upos[i][run_of[i][e]];
+        epos[k] = pos;
+        cp_o[e] = pos;
+        cv_o[e] = val[i][a0 + k];
+        cr_o[e] = erow[k];
       }
-      while (q & 3) {   // pad the row to a multiple of 4 entries
-        col_o[q] = 0;
-        val_o[q] = 0.f;
-        ++q;
+      int32_t q = 0;
+      for (int b = 0; b < B; ++b) {
+        rp_o[b] = q;
+        y_o[b] = y[i][r0 + b];
+        for (int64_t e = rp[r0 + b] - a0; e < rp[r0 + b + 1] - a0; ++e) {
+          pw_o[q] = epos[e];
+          val_o[q] = val[i][a0 + e];
+          ++q;
+        }
+        while (q & 3) {   // pad the row to a multiple of 4 entries (value 0)
+          pw_o[q] = 0;
+          val_o[q] = 0.f;
+          ++q;
+        }
       }
-    }
-    rp_o[B] = q;
-    std::sort(keys.begin(), keys.end());   // by column, then by position (= by row)
-    for (size_t e = 0; e < keys.size(); ++e) {
-      const uint32_t pos = static_cast<uint32_t>(keys[e] & 0xffffffffu);
-      ccol_o[e] = static_cast<int32_t>(keys[e] >> 32);
-      cval_o[e] = vals[pos];
-      crow_o[e] = row_of[pos];
+      rp_o[B] = q;
     }
   };
   {
-    const size_t nseg = desc.size();
     const unsigned nthr = std::max(1u, std::min(32u, std::thread::hardware_concurrency()));
     std::vector<std::thread> pool;
     for (unsigned w = 0; w < nthr; ++w)
       pool.emplace_back([&, w]() {
-        for (size_t s = w; s < nseg; s += nthr) fill(s);
+        for (int t = static_cast<int>(w); t < nb; t += static_cast<int>(nthr)) build_batch(t);
       });
     for (auto& th : pool) th.join();
   }
-  for (int v : bad)
-    if (v) {
-      free_shards(c);
-      return fail(c, ASAP_ERR_ARG, "column id out of range [0, d)");
+  size_t total = 0;
+  int max_nnz = 0, max_region = 0;
+  int64_t max_list = 0;
+  c->block_off.assign(nb, 0);
+  c->block_bytes.assign(nb, 0);
+  c->list_off.assign(nb, 0);
+  c->soff_off.assign(nb, 0);
+  c->list_len.assign(nb, 0);
+  std::vector<BatchDesc> desc(static_cast<size_t>(nb) * N);
+  for (int t = 0; t < nb; ++t) {
+    if (built[t].err) return fail(c, ASAP_ERR_ARG, built[t].err);
+    c->block_off[t] = total;
+    c->block_bytes[t] = built[t].img.size();
+    c->list_off[t] = built[t].list_off;
+    c->soff_off[t] = built[t].soff_off;
+    c->list_len[t] = built[t].list_len;
+    total += built[t].img.size();
+    max_nnz = std::max(max_nnz, built[t].max_nnz);
+    max_region = std::max(max_region, built[t].max_region);
+    max_list = std::max(max_list, built[t].list_len);
+    std::copy(built[t].desc.begin(), built[t].desc.end(), desc.begin() + static_cast<size_t>(t) * N);
+  }
+  if (c->residency == ASAP_SHARDS_HOST) {
+    CU(cudaHostAlloc(&c->pool, total, cudaHostAllocDefault), "allocating pinned shard memory");
+    c->pool_pinned = true;
+    size_t mb = 0;
+    for (int t = 0; t < nb; ++t) {
+      std::memcpy(c->pool + c->block_off[t], built[t].img.data(), built[t].img.size());
+      mb = std::max(mb, built[t].img.size());
+      std::vector<unsigned char>().swap(built[t].img);
     }
-
-  if (c->residency == ASAP_SHARDS_DEVICE) {
+    c->staging_bytes = mb;
+    for (int b = 0; b < asap_ctx::kStaging; ++b) CU(cudaMalloc(&c->staging[b], mb), "allocating staging buffers");
+  } else {
     CU(cudaMalloc(&c->pool, total), "allocating device shard memory");
     c->pool_pinned = false;
-    CU(cudaMemcpy(c->pool, host, total, cudaMemcpyHostToDevice), "copying shards to the device");
-  } else {
-    c->staging_bytes = max_block;
-    for (int b = 0; b < 2; ++b) CU(cudaMalloc(&c->staging[b], max_block), "allocating staging buffers");
+    for (int t = 0; t < nb; ++t) {
+      CU(cudaMemcpy(c->pool + c->block_off[t], built[t].img.data(), built[t].img.size(), cudaMemcpyHostToDevice),
+         "copying shards to the device");
+      std::vector<unsigned char>().swap(built[t].img);
+    }
   }
   c->pool_bytes = total;
   CU(cudaMalloc(&c->d_desc, desc.size() * sizeof(BatchDesc)), "allocating batch descriptors");
   CU(cudaMemcpy(c->d_desc, desc.data(), desc.size() * sizeof(BatchDesc), cudaMemcpyHostToDevice),
      "copying batch descriptors");
+  const size_t lb = 4 * static_cast<size_t>(std::max<int64_t>(max_list, 4));
+  CU(cudaMalloc(&c->wv, lb), "allocating the list value buffer");
+  CU(cudaMalloc(&c->gsum, lb), "allocating the column-sum buffer");
+  CU(cudaMemset(c->wv, 0, lb), "zeroing the list value buffer");
+  CU(cudaMemset(c->gsum, 0, lb), "zeroing the column-sum buffer");
   c->nb = nb;
   c->max_nnz = max_nnz;
+  c->max_region = max_region;
+  c->max_list = max_list;
+  c->wv_round = -1;
   c->update_ctas = update_ctas_for(max_nnz);
+  c->configured_key = -1;
   return ASAP_OK;
 }
 
@@ -951,60 +1091,68 @@ asap_status asap_local_step(asap_ctx* c) {
     g.st = c->st;
     g.round = static_cast<unsigned>(r);
     c->skip_notify = -1;
-    CU(launch_dense_step(c->tmX, c->tmWbf[r & 1], c->tmR, c->tmXT, f, g, c->N, c->stream),
-       "launching the dense local step");
+    time_begin(c, ASAP_KERNEL_DENSE_FWD);
+    CU(launch_dense_fwd(c->tmX, c->tmWbf[r & 1], f, c->N, c->stream), "launching the dense forward kernel");
+    time_end(c);
+    time_begin(c, ASAP_KERNEL_DENSE_GRAD);
+    CU(launch_dense_grad(c->tmR, c->tmXT, g, c->N, c->stream), "launching the dense gradient kernel");
+    time_end(c);
     c->launches += 2;
     c->step_pending = true;
     return ASAP_OK;
   }
-  const unsigned char* block;
-  if (c->residency == ASAP_SHARDS_HOST) {
-    asap_status s = stage_block(c, r);
-    if (s != ASAP_OK) return s;
-    CU(cudaStreamWaitEvent(c->stream, c->staged_ev[r & 1], 0), "waiting for the staged block");
-    block = c->staging[r & 1];
-  } else {
-    block = c->pool + c->block_off[t];
+  const unsigned char* block = nullptr;
+  asap_status sb = block_of(c, r, &block);
+  if (sb != ASAP_OK) return sb;
+  if (c->wv_round != r) {
+    // No exported w values for this round's columns (parameters came from
+    // the host): gather them once.
+    CU(launch_gather_wv(c->W[r & 1], c->ld, reinterpret_cast<const uint32_t*>(block + c->list_off[t]),
+                        reinterpret_cast<const int*>(block + c->soff_off[t]), c->n_slabs, c->S, c->wv, c->sm_count,
+                        c->stream),
+       "launching the gather kernel");
+    c->launches += 1;
+    c->wv_round = r;
   }
   SparseStepArgs a;
   a.block = block;
   a.desc = c->d_desc + static_cast<size_t>(t) * c->N;
-  a.W = c->W[r & 1];
-  a.ld = c->ld;
+  a.wv = c->wv;
+  a.gsum = c->gsum;
   a.r = c->r_scr;
   a.loss_part = c->loss_part;
   a.ready = c->ready;
   a.worker_ticket = c->ticket;
   a.B = c->B;
-  a.scale = c->lr / (static_cast<float>(c->B) * (1.0f - c->lr * c->l2));
   a.round = static_cast<unsigned>(r);
   a.skip_worker = c->skip_notify;
   c->skip_notify = -1;
   asap_status sg = prepare_graph(c, r);   // upload a regenerated graph ahead of the reduce
   if (sg != ASAP_OK) return sg;
-  CU(launch_sparse_step(a, c->N, c->loss, c->margin_ctas, c->update_ctas, c->stream), "launching the local step");
+  time_begin(c, ASAP_KERNEL_MARGIN);
+  CU(launch_margin(a, c->N, c->loss, c->margin_ctas, c->stream), "launching the margin kernel");
+  time_end(c);
+  time_begin(c, ASAP_KERNEL_UPDATE);
+  CU(launch_update(a, c->N, c->update_ctas, c->stream), "launching the update kernel");
+  time_end(c);
   c->launches += 2;
   c->step_pending = true;
-  if (c->residency == ASAP_SHARDS_HOST) {
-    CU(cudaEventRecord(c->free_ev[r & 1], c->stream), "staging event");
-    c->free_recorded[r & 1] = true;
-    asap_status s = stage_block(c, r + 1);   // prefetch the next round's block
-    if (s != ASAP_OK) return s;
-  }
   return ASAP_OK;
 }
 
 asap_status asap_stochastic_reduce(asap_ctx* c) {
   if (!c) return fail(nullptr, ASAP_ERR_ARG, "ctx is NULL");
   const int64_t r = c->round;
-  asap_status s = configure_mix_launch(c);
+  const bool sparse = c->loss == ASAP_LOSS_HINGE || c->loss == ASAP_LOSS_LOGISTIC;
+  const bool fused = c->step_pending && sparse;
+  asap_status s = configure_mix_launch(c, fused);
   if (s != ASAP_OK) return s;
   s = prepare_graph(c, r);
   if (s != ASAP_OK) return s;
   const int* nbr = c->graph_nbr;
   const float* wgt = c->graph_wgt;
   c->graph_ready_round = -1;
-  MixArgs a;
+  MixArgs a = {};
   a.out = c->W[(r + 1) & 1];
   a.shadow = c->Wbf[(r + 1) & 1];
   a.ld = c->ld;
@@ -1012,13 +1160,30 @@ asap_status asap_stochastic_reduce(asap_ctx* c) {
   a.kp1 = c->tab_kp1;
   a.nbr = nbr;
   a.wgt = wgt;
-  a.wscale = (c->step_pending && c->loss != ASAP_LOSS_SOFTMAX) ? (1.0f - c->lr * c->l2) : 1.0f;
+  a.wscale = (c->step_pending && sparse) ? (1.0f - c->lr * c->l2) : 1.0f;
   a.S = c->S;
   a.rows_pad = c->rows_pad;
   a.box_rows = c->box_rows;
   a.n_boxes = c->n_boxes;
   a.stages = c->stages;
   a.n_slabs = c->n_slabs;
+  if (fused) {
+    const unsigned char* bt = nullptr;
+    const unsigned char* bn = nullptr;
+    s = block_of(c, r, &bt);
+    if (s != ASAP_OK) return s;
+    s = block_of(c, r + 1, &bn);
+    if (s != ASAP_OK) return s;
+    const int t = static_cast<int>(r % c->nb), tn = static_cast<int>((r + 1) % c->nb);
+    a.upd_list = reinterpret_cast<const uint32_t*>(bt + c->list_off[t]);
+    a.upd_off = reinterpret_cast<const int*>(bt + c->soff_off[t]);
+    a.gsum = c->gsum;
+    a.upd_scale = c->lr / (static_cast<float>(c->B) * (1.0f - c->lr * c->l2));
+    a.exp_list = reinterpret_cast<const uint32_t*>(bn + c->list_off[tn]);
+    a.exp_off = reinterpret_cast<const int*>(bn + c->soff_off[tn]);
+    a.wv_out = c->wv;
+    a.max_region = c->max_region;
+  }
   a.cons_part = c->cons_part;
   a.loss_part = c->loss_part;
   a.n_loss_part = c->step_pending ? c->n_loss_part : 0;
@@ -1033,9 +1198,19 @@ asap_status asap_stochastic_reduce(asap_ctx* c) {
   a.round = static_cast<unsigned>(r);
   a.expect_notify = c->step_pending ? 1 : 0;
   a.wait_ns = c->wait_ns;
-  CU(launch_mix(c->tmap[r & 1], a, is_complete_kernel(c), c->mix_grid, c->mix_smem, c->stream),
+  time_begin(c, ASAP_KERNEL_REDUCE);
+  CU(launch_mix(c->tmap[r & 1], a, is_complete_kernel(c), fused, c->mix_grid, c->mix_smem, c->stream),
      "launching the stochastic reduce");
+  time_end(c);
   c->launches += 1;
+  c->wv_round = fused ? r + 1 : -1;
+  if (fused && c->residency == ASAP_SHARDS_HOST) {
+    const int slot = static_cast<int>(r % asap_ctx::kStaging);
+    CU(cudaEventRecord(c->free_ev[slot], c->stream), "staging event");   // block r is no longer read
+    c->free_recorded[slot] = true;
+    s = stage_block(c, r + 2);                                            // prefetch
+    if (s != ASAP_OK) return s;
+  }
   c->round = r + 1;
   c->step_pending = false;
   return ASAP_OK;
@@ -1081,6 +1256,7 @@ asap_status asap_write_params(asap_ctx* c, const float* host_in, int64_t round) 
     c->launches += 1;
     CU(cudaStreamSynchronize(c->stream), "bf16 copy");
   }
+  c->wv_round = -1;
   return reset_protocol(c, round);
 }
 
@@ -1132,6 +1308,36 @@ asap_status asap_set_wait_limit_ns(asap_ctx* c, uint64_t ns) {
 asap_status asap_debug_skip_notify(asap_ctx* c, int worker) {
   if (!c || worker < -1 || worker >= c->N) return fail(c, ASAP_ERR_ARG, "bad worker");
   c->skip_notify = worker;
+  return ASAP_OK;
+}
+
+asap_status asap_set_kernel_timing(asap_ctx* c, int enable) {
+  if (!c) return fail(nullptr, ASAP_ERR_ARG, "ctx is NULL");
+  CU(cudaStreamSynchronize(c->stream), "synchronising");
+  if (enable && c->tev.empty()) {
+    c->tev.resize(2 * kTimedLaunches);
+    c->tkind.resize(kTimedLaunches);
+    for (auto& e : c->tev) CU(cudaEventCreate(&e), "creating timing events");
+  }
+  c->timing = enable != 0;
+  c->tused = 0;
+  return ASAP_OK;
+}
+
+asap_status asap_read_kernel_times(asap_ctx* c, uint64_t* launches, double* total_ms) {
+  if (!c || !launches || !total_ms) return fail(c, ASAP_ERR_ARG, "NULL argument");
+  CU(cudaStreamSynchronize(c->stream), "synchronising");
+  for (int k = 0; k < ASAP_KERNEL_KINDS; ++k) {
+    launches[k] = 0;
+    total_ms[k] = 0.0;
+  }
+  for (size_t u = 0; u < c->tused; ++u) {
+    float ms = 0.f;
+    CU(cudaEventElapsedTime(&ms, c->tev[2 * u], c->tev[2 * u + 1]), "reading timing events");
+    launches[c->tkind[u]] += 1;
+    total_ms[c->tkind[u]] += ms;
+  }
+  c->tused = 0;
   return ASAP_OK;
 }
 

@@ -11,6 +11,12 @@
 
 #include "asap.h"
 
+#ifdef __CUDACC__
+#define ASAP_HD __host__ __device__
+#else
+#define ASAP_HD
+#endif
+
 namespace asap {
 
 constexpr int kMaxWorkers = 1024;
@@ -30,33 +36,36 @@ struct DevState {
   unsigned long long timeouts;
 };
 
+constexpr uint32_t kListPad = 0xffffffffu;   // padding entry of a column list
+
 // Where one worker's minibatch lives inside a batch block (byte offsets from
 // the block start).  Rows are padded to multiples of 4 entries (16 B) with
-// col = 0, val = 0 so that the margin kernel can use 128-bit loads.
+// pos = 0, val = 0 so that the margin kernel can use 128-bit loads.  `pos`
+// indexes the batch's slab-major column list (one entry per distinct
+// (worker, column) of the minibatch).
 struct BatchDesc {
   int64_t rp;     // int32 [B+1]: padded row starts, in entries
   int64_t y;      // float [B]
-  int64_t col;    // int32 [nnz_pad]
+  int64_t posw;   // int32 [nnz_pad]: list position of each entry's column
   int64_t val;    // float [nnz_pad]
-  int64_t ccol;   // int32 [nnz]: entries sorted by (column, row)
+  int64_t cpos;   // int32 [nnz]: entries sorted by (column, row): list position
   int64_t cval;   // float [nnz]
   int64_t crow;   // uint16 [nnz]: row within the batch
   int32_t nnz_pad;
   int32_t nnz;
 };
 
-// Arguments of the sparse local step (margin kernel, then update kernel).
+// Arguments of the sparse local step (margin kernel, then column sums).
 struct SparseStepArgs {
   const unsigned char* block;  // batch block of this round
   const BatchDesc* desc;       // [N] descriptors of this round's batch
-  float* W;                    // current parameter buffer, rows of ld floats
-  int64_t ld;
+  const float* wv;             // w values at the round's list positions
+  float* gsum;                 // column sums at the round's list positions
   float* r;                    // scratch [N][B]: d loss / d margin
   float* loss_part;            // scratch [N][margin CTAs per worker]
   unsigned int* ready;         // NOTIFY flags [N]
   unsigned int* worker_ticket; // [N] finished update CTAs of this round
   int B;
-  float scale;                 // eta / (B (1 - eta l2))
   unsigned int round;
   int skip_worker;             // fault injection: do not NOTIFY this worker
 };
@@ -77,8 +86,18 @@ struct MixArgs {
   int n_boxes;
   int stages;
   long long n_slabs;
+  // fused sparse update / export (FUSED kernels only)
+  const uint32_t* upd_list;    // this round's column list (slab-major)
+  const int* upd_off;          // [n_slabs + 1] slab regions of upd_list
+  const float* gsum;           // column sums at upd_list positions
+  float upd_scale;             // eta / (B (1 - eta l2))
+  const uint32_t* exp_list;    // next round's column list
+  const int* exp_off;          // [n_slabs + 1]
+  float* wv_out;               // w_{t+1} at exp_list positions
+  int max_region;              // entries: the largest slab region of any list
+  // metrics and protocol
   double* cons_part;           // scratch [gridDim.x]
-  const float* loss_part;      // [n_loss_part] from the margin kernel
+  const float* loss_part;      // [n_loss_part] from the local step
   int n_loss_part;
   float loss_norm;             // 1 / (N B)
   int have_loss;
@@ -121,16 +140,23 @@ asap_status build_graph_host(asap_graph_kind kind, int N, int k, uint64_t seed, 
                              int32_t* nbr, const char** why);
 
 // Launchers (kernels_*.cu).  Each returns the cudaError_t of the launch.
-cudaError_t launch_sparse_step(const SparseStepArgs& a, int N, int loss, int margin_ctas, int update_ctas,
-                               cudaStream_t s);
-cudaError_t launch_mix(const CUtensorMap& tmap, const MixArgs& a, bool complete, int grid, size_t smem,
+cudaError_t launch_margin(const SparseStepArgs& a, int N, int loss, int margin_ctas, cudaStream_t s);
+cudaError_t launch_update(const SparseStepArgs& a, int N, int update_ctas, cudaStream_t s);
+cudaError_t launch_gather_wv(const float* W, int64_t ld, const uint32_t* list, const int* slab_off, long long n_slabs,
+                             int S, float* wv, int sm_count, cudaStream_t s);
+constexpr int kMixComputeWarps = 8;
+constexpr int kMixThreads = (kMixComputeWarps + 1) * 32;   // + one TMA producer warp
+cudaError_t launch_mix(const CUtensorMap& tmap, const MixArgs& a, bool complete, bool fused, int grid, size_t smem,
                        cudaStream_t s);
-size_t mix_smem_bytes(int N, int kp1, int S, int rows_pad, int stages);
-cudaError_t mix_configure(bool complete, int kp1, bool shadow, size_t smem);
+ASAP_HD size_t mix_stage_bytes(int S, int rows_pad, int max_region);
+size_t mix_smem_bytes(int N, int kp1, int S, int rows_pad, int stages, int max_region);
+cudaError_t mix_configure(bool complete, bool fused, int kp1, bool shadow, size_t smem);
+cudaError_t mix_occupancy(bool complete, bool fused, int kp1, bool shadow, size_t smem, int* blocks);
 size_t dense_smem_bytes();
 cudaError_t dense_configure();
-cudaError_t launch_dense_step(const CUtensorMap& tmX, const CUtensorMap& tmW, const CUtensorMap& tmR,
-                              const CUtensorMap& tmXT, const DenseFwdArgs& f, const DenseGradArgs& g, int N,
+cudaError_t launch_dense_fwd(const CUtensorMap& tmX, const CUtensorMap& tmW, const DenseFwdArgs& f, int N,
+                             cudaStream_t s);
+cudaError_t launch_dense_grad(const CUtensorMap& tmR, const CUtensorMap& tmXT, const DenseGradArgs& g, int N,
                               cudaStream_t s);
 cudaError_t launch_cast_bf16(const float* src, uint16_t* dst, int64_t n, cudaStream_t s);
 

@@ -452,14 +452,12 @@ cudaError_t dense_configure() {
   return cudaFuncSetAttribute(k_dense_grad, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
 }
 
-cudaError_t launch_dense_step(const CUtensorMap& tmX, const CUtensorMap& tmW, const CUtensorMap& tmR,
-                              const CUtensorMap& tmXT, const DenseFwdArgs& f, const DenseGradArgs& g, int N,
-                              cudaStream_t s) {
-  const size_t smem = dense_smem_bytes();
+cudaError_t launch_dense_fwd(const CUtensorMap& tmX, const CUtensorMap& tmW, const DenseFwdArgs& f, int N,
+                             cudaStream_t s) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(f.Cq, f.B / kTileM, N);
   cfg.blockDim = dim3(kDenseThreads, 1, 1);
-  cfg.dynamicSmemBytes = smem;
+  cfg.dynamicSmemBytes = dense_smem_bytes();
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -468,10 +466,13 @@ cudaError_t launch_dense_step(const CUtensorMap& tmX, const CUtensorMap& tmW, co
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  cudaError_t e = cudaLaunchKernelEx(&cfg, k_dense_fwd, tmX, tmW, f);
-  if (e != cudaSuccess) return e;
+  return cudaLaunchKernelEx(&cfg, k_dense_fwd, tmX, tmW, f);
+}
+
+cudaError_t launch_dense_grad(const CUtensorMap& tmR, const CUtensorMap& tmXT, const DenseGradArgs& g, int N,
+                              cudaStream_t s) {
   const dim3 g2(g.d / kTileN, (g.C + kTileM - 1) / kTileM, N);
-  k_dense_grad<<<g2, kDenseThreads, smem, s>>>(tmR, tmXT, g);
+  k_dense_grad<<<g2, kDenseThreads, dense_smem_bytes(), s>>>(tmR, tmXT, g);
   return cudaGetLastError();
 }
 

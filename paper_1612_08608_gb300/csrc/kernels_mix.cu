@@ -1,29 +1,37 @@
 // Stochastic reduce (Eq. A.1, second line; Section 3):
-//   W_next[i, :] = sum_{m < k+1} wgt[i, m] * W[nbr[i, m], :]
+//   W_next[i, :] = sum_{m < k+1} wgt[i, m] * W_half[nbr[i, m], :]
 // plus, fused, the round's metrics (consensus error ||W_next - 1 wbar^T||_F
 // and the mean minibatch loss) and the NOTIFY-ACK bookkeeping of Section 4.
 //
-// Layout and data movement.  W is [N][ld] fp32 (ld a multiple of 64).  The
-// kernel is persistent: CTA b walks column slabs b, b + grid, ...  A slab is
-// S columns of *all* N rows; it is brought into shared memory by TMA 2-D
-// tiled loads (one box per 256 rows) into a ring of `stages` buffers guarded
-// by mbarriers, so every element of W is read from HBM exactly once however
-// many neighbours use it.  Each output row is then k+1 float4 shared-memory
-// reads per float4 written; outputs go straight from registers to HBM.
-// The complete graph (all-reduce, k = N-1, equal weights) needs only the
-// column mean, which the slab pass computes anyway: every row gets it.
+// Data movement.  W is [N][ld] fp32 (ld a multiple of 64).  The kernel is
+// persistent: CTA b walks column slabs b, b + grid, ...  A slab is S (<= 128)
+// columns of *all* N rows.  One producer warp brings slabs into a ring of
+// shared-memory stages with TMA 2-D tiled loads (one box per 256 rows), so
+// every element of W is read from HBM exactly once however many neighbours
+// use it; eight compute warps mix and write the outputs straight from
+// registers.  A stage goes back to the producer when all eight compute warps
+// have arrived on its "empty" mbarrier: no CTA-wide barrier in steady state.
 //
-// Consensus error: the column mean of W_next equals the column mean of W
-// scaled by the weight scale when P is doubly stochastic (Appendix A), so
-// the mean comes from the input slab and the squared deviations from the
-// output registers.  Partial sums per CTA are fp64; the last CTA to finish
-// (ticket) reduces them in a fixed order, so the metric is deterministic.
+// Sparse models (FUSED): the local step left, per distinct (worker, column)
+// of the minibatch, the column sum g of r_b x_b (kernels_sparse.cu).  The
+// producer also copies the slab's part of that list (and of the next
+// round's list) into the stage; the compute warps apply
+// w -= eta/B (1 - eta l2)^-1 g to the slab first -- so w_{t+1/2} exists only
+// in shared memory -- and after mixing they export w_{t+1} at the next
+// round's columns, which is all the next margin kernel reads.
 //
-// Protocol (Section 4, NOTIFY-ACK): before touching any input each CTA
-// waits, with a time limit, until ready[j] == round+1 for every worker j
-// (j's half-step model is complete) and consumed[j] >= round (the buffer
-// about to be overwritten was fully read by the previous reduce).  The last
-// CTA then ACKs: consumed[j] = round+1, stamp_next[j] = round+1.
+// Consensus error per column: with K the column's value in row 0 (a shift
+// against cancellation), sum_i (w_i - wbar)^2 = sum_i (w_i - K)^2 -
+// (sum_i (w_i - K))^2 / N.  Squares accumulate per thread in fp64; the
+// per-column sums are combined across warps by the producer warp when the
+// stage comes back.  The complete graph (all-reduce, equal weights) writes
+// the column mean to every row and adds nothing.
+//
+// Protocol (Section 4, NOTIFY-ACK): before touching any input each CTA waits,
+// with a time limit, until ready[j] == round+1 for every worker j and
+// consumed[j] >= round.  The last CTA to finish (ticket) reduces the metric
+// partials in a fixed order and ACKs: consumed[j] = round+1,
+// stamp_next[j] = round+1.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -40,6 +48,8 @@ namespace {
 
 constexpr unsigned kFull = 0xffffffffu;
 constexpr unsigned long long kTmaWaitNs = 2000000000ull;   // 2 s: a TMA load never takes this long
+constexpr int kCompute = kMixComputeWarps * 32;            // compute threads
+constexpr int kProducerWarp = kMixComputeWarps;
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -70,6 +80,10 @@ __device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
                : "memory");
 }
 
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" :: "r"(smem_u32(bar)) : "memory");
+}
+
 __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   uint32_t ok;
   asm volatile(
@@ -93,6 +107,13 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, u
       "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];"
       :: "r"(smem_u32(dst)), "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_u32(bar))
       : "memory");
+}
+
+// Untiled bulk copy global -> shared (16-byte aligned, size a multiple of 16).
+__device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+               :: "r"(smem_u32(dst)), "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(smem_u32(bar))
+               : "memory");
 }
 
 __device__ __forceinline__ void record_error(DevState* st, unsigned code, unsigned worker, unsigned round) {
@@ -130,6 +151,12 @@ __device__ __forceinline__ float4 f4_add(float4 a, float4 b) {
   return make_float4(a.x + b.x, a.y + b.y, a.z + b.z, a.w + b.w);
 }
 
+__device__ __forceinline__ float4 f4_shfl_xor(float4 v, int m) {
+  return make_float4(__shfl_xor_sync(kFull, v.x, m), __shfl_xor_sync(kFull, v.y, m), __shfl_xor_sync(kFull, v.z, m),
+                     __shfl_xor_sync(kFull, v.w, m));
+}
+
+// Sum over all threads of the block (kMixThreads); valid in thread 0.
 __device__ __forceinline__ double block_sum_f64(double v, double* scratch) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(kFull, v, o);
@@ -139,37 +166,52 @@ __device__ __forceinline__ double block_sum_f64(double v, double* scratch) {
   __syncthreads();
   double t = 0.0;
   if (threadIdx.x == 0)
-    for (int k = 0; k < kThreads / 32; ++k) t += scratch[k];
-  return t;   // valid in thread 0
+    for (int k = 0; k < kMixThreads / 32; ++k) t += scratch[k];
+  return t;
+}
+
+__device__ __forceinline__ void compute_bar() { asm volatile("bar.sync 1, %0;" :: "n"(kCompute) : "memory"); }
+
+// Barrier among the compute warps that also returns the OR of `v` over them.
+__device__ __forceinline__ bool compute_bar_or(bool v) {
+  uint32_t r;
+  asm volatile(
+      "{\n .reg .pred p, q;\n setp.ne.u32 p, %1, 0;\n bar.red.or.pred q, 1, %2, p;\n selp.u32 %0, 1, 0, q;\n}"
+      : "=r"(r) : "r"(static_cast<uint32_t>(v)), "n"(kCompute) : "memory");
+  return r != 0;
 }
 
 struct MixSmem {
-  float* slabs;
+  unsigned char* stage0;
+  size_t stage_bytes;
   uint64_t* full;
+  uint64_t* empty;
+  float4* part;      // [stages][warps][nq]: per-warp column sums (consensus / complete-graph mean)
+  int* info;         // [stages][4]: n_upd, n_exp, exp_base
   int* nbr;
   float* wgt;
-  float4* mean;
-  float4* red;
   double* dscratch;
-  int* flags;   // [0]: fail, [1]: last
+  int* flags;        // [0]: fail, [1]: last
 };
 
 __device__ __forceinline__ MixSmem carve(unsigned char* raw, const MixArgs& a, int kp1) {
   MixSmem m;
   uintptr_t base = (reinterpret_cast<uintptr_t>(raw) + 1023) & ~static_cast<uintptr_t>(1023);
-  const size_t slab_bytes = (static_cast<size_t>(a.rows_pad) * a.S * 4 + 1023) & ~static_cast<size_t>(1023);
-  m.slabs = reinterpret_cast<float*>(base);
-  base += slab_bytes * a.stages;
+  m.stage_bytes = mix_stage_bytes(a.S, a.rows_pad, a.max_region);
+  m.stage0 = reinterpret_cast<unsigned char*>(base);
+  base += m.stage_bytes * a.stages;
   m.full = reinterpret_cast<uint64_t*>(base);
   base += 8 * a.stages;
+  m.empty = reinterpret_cast<uint64_t*>(base);
+  base += 8 * a.stages;
   m.dscratch = reinterpret_cast<double*>(base);
-  base += 8 * (kThreads / 32);
+  base += (8 * (kMixThreads / 32) + 15) & ~15;
   m.flags = reinterpret_cast<int*>(base);
   base += 16;
-  m.mean = reinterpret_cast<float4*>(base);
-  base += 16 * (a.S / 4);
-  m.red = reinterpret_cast<float4*>(base);
-  base += 16 * kThreads;
+  m.info = reinterpret_cast<int*>(base);
+  base += 16 * a.stages;
+  m.part = reinterpret_cast<float4*>(base);   // 16-byte aligned: every region above is a multiple of 16
+  base += 16 * static_cast<size_t>(a.stages) * kMixComputeWarps * (a.S / 4);
   m.nbr = reinterpret_cast<int*>(base);
   base += 4 * static_cast<size_t>(a.N) * kp1;
   m.wgt = reinterpret_cast<float*>(base);
@@ -179,22 +221,23 @@ __device__ __forceinline__ MixSmem carve(unsigned char* raw, const MixArgs& a, i
 // KP1 > 0: sparse graph with KP1 neighbours per row (compile-time);
 // KP1 == 0: sparse graph, runtime a.kp1 (<= kMaxKp1Sparse);
 // KP1 < 0: complete graph with equal weights.
-template <int KP1, bool SHADOW>
-__global__ void __launch_bounds__(kThreads, 1) k_mix(const __grid_constant__ CUtensorMap tmap, const MixArgs a) {
+template <int KP1, bool SHADOW, bool FUSED>
+__global__ void __launch_bounds__(kMixThreads, 1) k_mix(const __grid_constant__ CUtensorMap tmap, const MixArgs a) {
   extern __shared__ unsigned char smem_raw[];
   const int kp1 = KP1 > 0 ? KP1 : (KP1 == 0 ? a.kp1 : 0);
   MixSmem sm = carve(smem_raw, a, kp1);
-  const int tid = threadIdx.x;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int S = a.S, nq = S >> 2;
-  const int lq = __ffs(nq) - 1;            // nq is a power of two
-  const int G = kThreads >> lq;            // row groups in the mean pass
-  const size_t slab_floats = ((static_cast<size_t>(a.rows_pad) * S * 4 + 1023) & ~static_cast<size_t>(1023)) / 4;
+  const int lq = __ffs(nq) - 1;              // nq is a power of two, <= 32
+  const size_t slab_floats = static_cast<size_t>(a.rows_pad) * S;
+  const size_t list_off = (slab_floats * 4 + 15) & ~static_cast<size_t>(15);
+  const size_t list_bytes = (static_cast<size_t>(a.max_region) * 4 + 15) & ~static_cast<size_t>(15);
 
   if (tid == 0) { sm.flags[0] = 0; sm.flags[1] = 0; }
   __syncthreads();
 
   // ---- NOTIFY / ACK checks (time-limited waits) ----
-  for (int j = tid; j < a.N; j += kThreads) {
+  for (int j = tid; j < a.N; j += kMixThreads) {
     unsigned e = 0;
     if (a.expect_notify) e = wait_flag(a.ready + j, a.round + 1u, true, a.wait_ns);
     if (!e) e = wait_flag(a.consumed + j, a.round, false, a.wait_ns);
@@ -207,115 +250,220 @@ __global__ void __launch_bounds__(kThreads, 1) k_mix(const __grid_constant__ CUt
   __syncthreads();
   bool failed = sm.flags[0] != 0;
 
-  double cons = 0.0;
+  double s2 = 0.0;     // compute threads: sum of (w - K)^2;  producer lanes: sum of S1^2 / N
   if (!failed) {
     if (KP1 >= 0) {
-      for (int idx = tid; idx < a.N * kp1; idx += kThreads) {
+      for (int idx = tid; idx < a.N * kp1; idx += kMixThreads) {
         sm.nbr[idx] = a.nbr[idx];
         sm.wgt[idx] = a.wgt[idx] * a.wscale;
       }
     }
     if (tid == 0) {
-      for (int s = 0; s < a.stages; ++s) mbar_init(sm.full + s, 1);
+      for (int s = 0; s < a.stages; ++s) {
+        mbar_init(sm.full + s, 1);
+        mbar_init(sm.empty + s, kMixComputeWarps);
+      }
       asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     __syncthreads();
 
     const long long stride = gridDim.x;
-    const uint32_t tx_bytes = static_cast<uint32_t>(a.n_boxes) * a.box_rows * S * 4u;
-    auto issue = [&](int stage, long long slab) {
-      mbar_expect_tx(sm.full + stage, tx_bytes);
-      float* dst = sm.slabs + stage * slab_floats;
-      for (int b = 0; b < a.n_boxes; ++b)
-        tma_load_2d(dst + static_cast<size_t>(b) * a.box_rows * S, &tmap, sm.full + stage,
-                    static_cast<int>(slab * S), b * a.box_rows);
-    };
-    if (tid == 0) {
-      for (int s = 0; s < a.stages; ++s) {
-        const long long slab = blockIdx.x + s * stride;
-        if (slab < a.n_slabs) issue(s, slab);
-      }
-    }
-
+    const long long n_my = (a.n_slabs - blockIdx.x + stride - 1) / stride;   // slabs of this CTA
     const float inv_n = 1.0f / static_cast<float>(a.N);
-    const int q_m = tid & (nq - 1), g_m = tid >> lq;
-    int it = 0;
-    for (long long slab = blockIdx.x; slab < a.n_slabs; slab += stride, ++it) {
-      const int stage = it % a.stages;
-      const uint32_t parity = static_cast<uint32_t>((it / a.stages) & 1);
-      const bool ok = mbar_wait_bounded(sm.full + stage, parity);
-      if (__syncthreads_or(!ok)) {
-        if (tid == 0) record_error(a.st, ASAP_ERR_CUDA, 0xffffffffu, a.round);
-        failed = true;
-        break;
-      }
-      const float4* x4 = reinterpret_cast<const float4*>(sm.slabs + stage * slab_floats);
-      const long long c0 = slab * S;
 
-      // Column sums over all N rows: strided partials, then a fixed tree.
-      float4 part = make_float4(0.f, 0.f, 0.f, 0.f);
-      for (int j = g_m; j < a.N; j += G) part = f4_add(part, x4[j * nq + q_m]);
-      sm.red[tid] = part;
-      __syncthreads();
-      for (int h = G >> 1; h >= 1; h >>= 1) {
-        if (g_m < h) sm.red[tid] = f4_add(sm.red[tid], sm.red[tid + (h << lq)]);
-        __syncthreads();
+    if (warp == kProducerWarp) {
+      // ================= producer warp =================
+      double term = 0.0;
+      for (long long it = 0; it < n_my + a.stages; ++it) {
+        if (it >= a.stages) {
+          const long long done = it - a.stages;
+          const int st = static_cast<int>(done % a.stages);
+          if (!mbar_wait_bounded(sm.empty + st, static_cast<uint32_t>((done / a.stages) & 1))) {
+            if (lane == 0) record_error(a.st, ASAP_ERR_CUDA, 0xfffffffeu, a.round);
+            failed = true;
+            break;
+          }
+          if (KP1 >= 0 && lane < nq) {
+            const float4* p = sm.part + static_cast<size_t>(st) * kMixComputeWarps * nq;
+            float4 t = p[lane];
+            for (int w = 1; w < kMixComputeWarps; ++w) t = f4_add(t, p[w * nq + lane]);
+            term += (static_cast<double>(t.x) * t.x + static_cast<double>(t.y) * t.y +
+                     static_cast<double>(t.z) * t.z + static_cast<double>(t.w) * t.w) / a.N;
+          }
+          __syncwarp();
+        }
+        if (it < n_my && lane == 0) {
+          const long long slab = blockIdx.x + it * stride;
+          const int st = static_cast<int>(it % a.stages);
+          unsigned char* base = sm.stage0 + st * sm.stage_bytes;
+          uint32_t bytes = static_cast<uint32_t>(a.n_boxes) * a.box_rows * S * 4u;
+          int n_upd = 0, n_exp = 0, x0 = 0, u0 = 0;
+          if (FUSED) {
+            u0 = a.upd_off[slab];
+            n_upd = a.upd_off[slab + 1] - u0;
+            x0 = a.exp_off[slab];
+            n_exp = a.exp_off[slab + 1] - x0;
+            bytes += 8u * n_upd + 4u * n_exp;
+          }
+          int* info = sm.info + 4 * st;
+          info[0] = n_upd;
+          info[1] = n_exp;
+          info[2] = x0;
+          mbar_expect_tx(sm.full + st, bytes);
+          for (int b = 0; b < a.n_boxes; ++b)
+            tma_load_2d(base + static_cast<size_t>(b) * a.box_rows * S * 4, &tmap, sm.full + st,
+                        static_cast<int>(slab * S), b * a.box_rows);
+          if (FUSED) {
+            if (n_upd > 0) {
+              bulk_load(base + list_off, a.upd_list + u0, 4u * n_upd, sm.full + st);
+              bulk_load(base + list_off + list_bytes, a.gsum + u0, 4u * n_upd, sm.full + st);
+            }
+            if (n_exp > 0) bulk_load(base + list_off + 2 * list_bytes, a.exp_list + x0, 4u * n_exp, sm.full + st);
+          }
+        }
+        __syncwarp();
       }
-      if (tid < nq) {
-        const float4 t = sm.red[tid];
-        const float sc = inv_n * a.wscale;
-        sm.mean[tid] = make_float4(t.x * sc, t.y * sc, t.z * sc, t.w * sc);
-      }
-      __syncthreads();
-
-      float cacc = 0.f;
-      for (int idx = tid; idx < (a.N << lq); idx += kThreads) {
-        const int i = idx >> lq, q = idx & (nq - 1);
-        const float4 mean = sm.mean[q];
-        float4 acc;
-        if (KP1 < 0) {
-          acc = mean;
+      s2 = -term;
+    } else {
+      // ================= compute warps =================
+      const int rows_w = (a.N - warp + kMixComputeWarps - 1) / kMixComputeWarps;   // rows i = warp + 8 r
+      const int pairs = rows_w << lq;
+      const int q_l = lane & (nq - 1);
+      for (long long it = 0; it < n_my; ++it) {
+        const long long slab = blockIdx.x + it * stride;
+        const int st = static_cast<int>(it % a.stages);
+        bool ok = mbar_wait_bounded(sm.full + st, static_cast<uint32_t>((it / a.stages) & 1));
+        unsigned char* base = sm.stage0 + st * sm.stage_bytes;
+        float* x = reinterpret_cast<float*>(base);
+        const float4* x4 = reinterpret_cast<const float4*>(base);
+        const int* info = sm.info + 4 * st;
+        float4* part = sm.part + (static_cast<size_t>(st) * kMixComputeWarps + warp) * nq;
+        const long long c0 = slab * S;
+        if (ok && FUSED) {
+          // w_half = w - eta/B g on the slab (distinct (worker, column) per entry).
+          const uint32_t* ul = reinterpret_cast<const uint32_t*>(base + list_off);
+          const float* ug = reinterpret_cast<const float*>(base + list_off + list_bytes);
+          const int n_upd = info[0];
+          for (int e = tid; e < n_upd; e += kCompute) {
+            const uint32_t code = ul[e];
+            if (code != kListPad) {
+              float* px = x + (code >> 16) * S + (code & 0xffffu);
+              *px = fmaf(-a.upd_scale, ug[e], *px);
+            }
+          }
+        }
+        if (FUSED && KP1 < 0) ok = !compute_bar_or(!ok);   // the update is visible to the column sums
+        if (ok && KP1 < 0) {
+          // Complete graph: per-warp column sums over its rows.
+          float4 cs = make_float4(0.f, 0.f, 0.f, 0.f);
+          for (int p = lane; p < pairs; p += 32) cs = f4_add(cs, x4[((warp + ((p >> lq) << 3)) << lq) + q_l]);
+          for (int o = nq; o < 32; o <<= 1) cs = f4_add(cs, f4_shfl_xor(cs, o));
+          if (lane < nq) part[lane] = cs;
+        }
+        if (FUSED || KP1 < 0) ok = !compute_bar_or(!ok);   // uniform decision; the update / sums are visible
+        if (!ok) {
+          if (lane == 0) record_error(a.st, ASAP_ERR_CUDA, 0xffffffffu, a.round);
+          failed = true;
+          break;
+        }
+        if constexpr (KP1 < 0) {
+          // Complete graph: column mean over all N rows, written to every row.
+          float4* p0 = sm.part + static_cast<size_t>(st) * kMixComputeWarps * nq;
+          float4 t = p0[q_l];
+          for (int w = 1; w < kMixComputeWarps; ++w) t = f4_add(t, p0[w * nq + q_l]);
+          const float sc = inv_n * a.wscale;
+          const float4 mean = make_float4(t.x * sc, t.y * sc, t.z * sc, t.w * sc);
+          for (int p = lane; p < pairs; p += 32) {
+            const int i = warp + ((p >> lq) << 3);
+            const long long c = c0 + 4 * q_l;
+            if (c < a.ld) {
+              *reinterpret_cast<float4*>(a.out + static_cast<int64_t>(i) * a.ld + c) = mean;
+              if (SHADOW) {
+                __nv_bfloat162 lo = __floats2bfloat162_rn(mean.x, mean.y);
+                __nv_bfloat162 hi = __floats2bfloat162_rn(mean.z, mean.w);
+                uint2 pk;
+                pk.x = *reinterpret_cast<uint32_t*>(&lo);
+                pk.y = *reinterpret_cast<uint32_t*>(&hi);
+                *reinterpret_cast<uint2*>(a.shadow + static_cast<int64_t>(i) * a.ld + c) = pk;
+              }
+            }
+          }
+          if (FUSED) {
+            // every lane needs the means of all columns: keep them in the partial slot of warp 0
+            compute_bar();
+            if (warp == 0 && lane < nq) p0[lane] = mean;   // p0 aliases warp 0's partials (read above)
+            compute_bar();
+            const uint32_t* xl = reinterpret_cast<const uint32_t*>(base + list_off + 2 * list_bytes);
+            const int n_exp = info[1], xbase = info[2];
+            const float* means = reinterpret_cast<const float*>(p0);
+            for (int e = tid; e < n_exp; e += kCompute) {
+              const uint32_t code = xl[e];
+              if (code != kListPad) a.wv_out[xbase + e] = means[code & 0xffffu];
+            }
+          }
         } else {
-          const int* nb = sm.nbr + i * kp1;
-          const float* wt = sm.wgt + i * kp1;
-          const float4 x0 = x4[nb[0] * nq + q];
-          acc = make_float4(wt[0] * x0.x, wt[0] * x0.y, wt[0] * x0.z, wt[0] * x0.w);
+          const float4 K = x4[q_l];        // shift: row 0 of the (updated) slab
+          float4 s1 = make_float4(0.f, 0.f, 0.f, 0.f);
+          float sq = 0.f;
+          for (int p = lane; p < pairs; p += 32) {
+            const int i = warp + ((p >> lq) << 3);
+            const int* nb = sm.nbr + i * kp1;
+            const float* wt = sm.wgt + i * kp1;
+            const float4 xa = x4[(nb[0] << lq) + q_l];
+            float4 acc = make_float4(wt[0] * xa.x, wt[0] * xa.y, wt[0] * xa.z, wt[0] * xa.w);
 #pragma unroll
-          for (int m = 1; m < (KP1 > 0 ? KP1 : kMaxKp1Sparse); ++m) {
-            if (KP1 == 0 && m >= kp1) break;
-            acc = f4_fma(wt[m], x4[nb[m] * nq + q], acc);
+            for (int m = 1; m < (KP1 > 0 ? KP1 : kMaxKp1Sparse); ++m) {
+              if (KP1 == 0 && m >= kp1) break;
+              acc = f4_fma(wt[m], x4[(nb[m] << lq) + q_l], acc);
+            }
+            const long long c = c0 + 4 * q_l;
+            if (c < a.ld) {
+              *reinterpret_cast<float4*>(a.out + static_cast<int64_t>(i) * a.ld + c) = acc;
+              if (SHADOW) {
+                __nv_bfloat162 lo = __floats2bfloat162_rn(acc.x, acc.y);
+                __nv_bfloat162 hi = __floats2bfloat162_rn(acc.z, acc.w);
+                uint2 pk;
+                pk.x = *reinterpret_cast<uint32_t*>(&lo);
+                pk.y = *reinterpret_cast<uint32_t*>(&hi);
+                *reinterpret_cast<uint2*>(a.shadow + static_cast<int64_t>(i) * a.ld + c) = pk;
+              }
+            }
+            const float dx = acc.x - K.x, dy = acc.y - K.y, dz = acc.z - K.z, dw = acc.w - K.w;
+            s1 = f4_add(s1, make_float4(dx, dy, dz, dw));
+            sq = fmaf(dx, dx, fmaf(dy, dy, fmaf(dz, dz, fmaf(dw, dw, sq))));
           }
-          const float dx = acc.x - mean.x, dy = acc.y - mean.y, dz = acc.z - mean.z, dw = acc.w - mean.w;
-          cacc = fmaf(dx, dx, fmaf(dy, dy, fmaf(dz, dz, fmaf(dw, dw, cacc))));
-        }
-        const long long c = c0 + 4 * q;
-        if (c < a.ld) {
-          *reinterpret_cast<float4*>(a.out + static_cast<int64_t>(i) * a.ld + c) = acc;
-          if (SHADOW) {
-            __nv_bfloat162 lo = __floats2bfloat162_rn(acc.x, acc.y);
-            __nv_bfloat162 hi = __floats2bfloat162_rn(acc.z, acc.w);
-            uint2 pk;
-            pk.x = *reinterpret_cast<uint32_t*>(&lo);
-            pk.y = *reinterpret_cast<uint32_t*>(&hi);
-            *reinterpret_cast<uint2*>(a.shadow + static_cast<int64_t>(i) * a.ld + c) = pk;
+          s2 += static_cast<double>(sq);
+          for (int o = nq; o < 32; o <<= 1) s1 = f4_add(s1, f4_shfl_xor(s1, o));
+          if (lane < nq) part[lane] = s1;
+          if (FUSED) {
+            // w_{t+1} at the next round's columns, recomputed with the same
+            // operations in the same order as the stored outputs.
+            const uint32_t* xl = reinterpret_cast<const uint32_t*>(base + list_off + 2 * list_bytes);
+            const int n_exp = info[1], xbase = info[2];
+            for (int e = tid; e < n_exp; e += kCompute) {
+              const uint32_t code = xl[e];
+              if (code == kListPad) continue;
+              const int i = static_cast<int>(code >> 16), cl = static_cast<int>(code & 0xffffu);
+              const int* nb = sm.nbr + i * kp1;
+              const float* wt = sm.wgt + i * kp1;
+              float v = wt[0] * x[nb[0] * S + cl];
+              for (int m = 1; m < kp1; ++m) v = fmaf(wt[m], x[nb[m] * S + cl], v);
+              a.wv_out[xbase + e] = v;
+            }
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");   // generic writes before the next TMA
           }
         }
-      }
-      cons += static_cast<double>(cacc);
-      __syncthreads();   // every thread is done with this stage and with mean/red
-      if (tid == 0) {
-        const long long nxt = slab + a.stages * stride;
-        if (nxt < a.n_slabs) issue(stage, nxt);
+        __syncwarp();
+        if (lane == 0) mbar_arrive(sm.empty + st);
       }
     }
   }
 
   // ---- per-CTA partial, ticket, and the last CTA's finalisation ----
-  const double csum = block_sum_f64(cons, sm.dscratch);
-  if (tid == 0) {
-    a.cons_part[blockIdx.x] = csum;
-    if (failed) atomicOr(&sm.flags[0], 1);
-  }
+  const double csum = block_sum_f64(s2, sm.dscratch);
+  if (failed) atomicOr(&sm.flags[0], 1);
+  __syncthreads();
+  if (tid == 0) a.cons_part[blockIdx.x] = csum;
   __threadfence();
   __syncthreads();
   if (tid == 0) {
@@ -329,15 +477,15 @@ __global__ void __launch_bounds__(kThreads, 1) k_mix(const __grid_constant__ CUt
   const unsigned ticket = atomicAdd(&a.st->mix_ticket, 0u);
   const bool any_fail = (ticket >> 16) != 0;
   double v = 0.0;
-  for (int b = tid; b < static_cast<int>(gridDim.x); b += kThreads) v += __ldcg(a.cons_part + b);
+  for (int b = tid; b < static_cast<int>(gridDim.x); b += kMixThreads) v += __ldcg(a.cons_part + b);
   const double ctot = block_sum_f64(v, sm.dscratch);
   double lv = 0.0;
   if (a.have_loss)
-    for (int b = tid; b < a.n_loss_part; b += kThreads) lv += static_cast<double>(__ldcg(a.loss_part + b));
+    for (int b = tid; b < a.n_loss_part; b += kMixThreads) lv += static_cast<double>(__ldcg(a.loss_part + b));
   const double ltot = block_sum_f64(lv, sm.dscratch);
   if (tid == 0) {
     const int slot = static_cast<int>(a.round % kMetricsCap);
-    a.metrics_cons[slot] = any_fail ? __int_as_float(0x7fc00000) : static_cast<float>(sqrt(ctot));
+    a.metrics_cons[slot] = any_fail ? __int_as_float(0x7fc00000) : static_cast<float>(sqrt(fmax(ctot, 0.0)));
     a.metrics_loss[slot] = (a.have_loss && !any_fail) ? static_cast<float>(ltot * a.loss_norm)
                                                       : __int_as_float(0x7fc00000);
     if (!any_fail) {
@@ -349,63 +497,52 @@ __global__ void __launch_bounds__(kThreads, 1) k_mix(const __grid_constant__ CUt
   }
   if (!any_fail) {
     __threadfence();
-    for (int j = tid; j < a.N; j += kThreads) {
+    for (int j = tid; j < a.N; j += kMixThreads) {
       a.stamp_next[j] = a.round + 1u;
       st_release_u32(a.consumed + j, a.round + 1u);
     }
   }
 }
 
-template <int KP1, bool SHADOW>
-cudaError_t set_attr(size_t smem) {
-  return cudaFuncSetAttribute(k_mix<KP1, SHADOW>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              static_cast<int>(smem));
-}
+template <int KP1, bool SHADOW, bool FUSED>
+struct MixKernel {
+  static cudaError_t attr(size_t smem) {
+    return cudaFuncSetAttribute(k_mix<KP1, SHADOW, FUSED>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                static_cast<int>(smem));
+  }
+  static cudaError_t occ(size_t smem, int* blocks) {
+    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks, k_mix<KP1, SHADOW, FUSED>, kMixThreads, smem);
+  }
+  static cudaError_t launch(const CUtensorMap& tmap, const MixArgs& a, int grid, size_t smem, cudaStream_t s) {
+    k_mix<KP1, SHADOW, FUSED><<<grid, kMixThreads, smem, s>>>(tmap, a);
+    return cudaGetLastError();
+  }
+};
 
-template <bool SHADOW>
-cudaError_t launch_t(const CUtensorMap& tmap, const MixArgs& a, bool complete, int grid, size_t smem,
-                     cudaStream_t s) {
-  if (complete) {
-    k_mix<-1, SHADOW><<<grid, kThreads, smem, s>>>(tmap, a);
-  } else {
-    switch (a.kp1) {
-      case 1: k_mix<1, SHADOW><<<grid, kThreads, smem, s>>>(tmap, a); break;
-      case 2: k_mix<2, SHADOW><<<grid, kThreads, smem, s>>>(tmap, a); break;
-      case 3: k_mix<3, SHADOW><<<grid, kThreads, smem, s>>>(tmap, a); break;
-      case 5: k_mix<5, SHADOW><<<grid, kThreads, smem, s>>>(tmap, a); break;
-      default: k_mix<0, SHADOW><<<grid, kThreads, smem, s>>>(tmap, a); break;
+// Dispatch over (complete / k+1, shadow, fused); Op is a functor template.
+template <template <int, bool, bool> class K, bool SHADOW, bool FUSED>
+struct ByKp1 {
+  template <typename F>
+  static cudaError_t go(bool complete, int kp1, F&& f) {
+    if (complete) return f(K<-1, SHADOW, FUSED>());
+    switch (kp1) {
+      case 1: return f(K<1, SHADOW, FUSED>());
+      case 2: return f(K<2, SHADOW, FUSED>());
+      case 3: return f(K<3, SHADOW, FUSED>());
+      case 5: return f(K<5, SHADOW, FUSED>());
+      default: return f(K<0, SHADOW, FUSED>());
     }
   }
-  return cudaGetLastError();
-}
+};
 
-template <bool SHADOW>
-cudaError_t configure_t(bool complete, int kp1, size_t smem) {
-  if (complete) return set_attr<-1, SHADOW>(smem);
-  switch (kp1) {
-    case 1: return set_attr<1, SHADOW>(smem);
-    case 2: return set_attr<2, SHADOW>(smem);
-    case 3: return set_attr<3, SHADOW>(smem);
-    case 5: return set_attr<5, SHADOW>(smem);
-    default: return set_attr<0, SHADOW>(smem);
+template <typename F>
+cudaError_t dispatch(bool complete, bool fused, int kp1, bool shadow, F&& f) {
+  if (shadow) {
+    if (fused) return cudaErrorInvalidValue;   // dense models never fuse a sparse update
+    return ByKp1<MixKernel, true, false>::go(complete, kp1, f);
   }
-}
-
-template <int KP1, bool SHADOW>
-cudaError_t occ_one(size_t smem, int* blocks) {
-  return cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks, k_mix<KP1, SHADOW>, kThreads, smem);
-}
-
-template <bool SHADOW>
-cudaError_t occupancy_t(bool complete, int kp1, size_t smem, int* blocks) {
-  if (complete) return occ_one<-1, SHADOW>(smem, blocks);
-  switch (kp1) {
-    case 1: return occ_one<1, SHADOW>(smem, blocks);
-    case 2: return occ_one<2, SHADOW>(smem, blocks);
-    case 3: return occ_one<3, SHADOW>(smem, blocks);
-    case 5: return occ_one<5, SHADOW>(smem, blocks);
-    default: return occ_one<0, SHADOW>(smem, blocks);
-  }
+  return fused ? ByKp1<MixKernel, false, true>::go(complete, kp1, f)
+               : ByKp1<MixKernel, false, false>::go(complete, kp1, f);
 }
 
 __global__ void k_cast_bf16(const float* __restrict__ src, uint16_t* __restrict__ dst, int64_t n) {
@@ -418,24 +555,29 @@ __global__ void k_cast_bf16(const float* __restrict__ src, uint16_t* __restrict_
 
 }  // namespace
 
-size_t mix_smem_bytes(int N, int kp1, int S, int rows_pad, int stages) {
-  const size_t slab_bytes = (static_cast<size_t>(rows_pad) * S * 4 + 1023) & ~static_cast<size_t>(1023);
-  return 1024 + slab_bytes * stages + 8 * stages + 8 * (kThreads / 32) + 16 + 16 * (S / 4) + 16 * kThreads +
-         8 * static_cast<size_t>(N) * kp1;
+ASAP_HD size_t mix_stage_bytes(int S, int rows_pad, int max_region) {
+  const size_t slab = (static_cast<size_t>(rows_pad) * S * 4 + 15) & ~static_cast<size_t>(15);
+  const size_t list = (static_cast<size_t>(max_region) * 4 + 15) & ~static_cast<size_t>(15);
+  return (slab + 3 * list + 1023) & ~static_cast<size_t>(1023);
 }
 
-cudaError_t mix_configure(bool complete, int kp1, bool shadow, size_t smem) {
-  return shadow ? configure_t<true>(complete, kp1, smem) : configure_t<false>(complete, kp1, smem);
+size_t mix_smem_bytes(int N, int kp1, int S, int rows_pad, int stages, int max_region) {
+  return 1024 + mix_stage_bytes(S, rows_pad, max_region) * stages + 16 * stages + ((8 * (kMixThreads / 32) + 15) & ~15) + 16 +
+         16 * stages + 16 * static_cast<size_t>(stages) * kMixComputeWarps * (S / 4) + 8 * static_cast<size_t>(N) * kp1;
 }
 
-cudaError_t mix_occupancy(bool complete, int kp1, bool shadow, size_t smem, int* blocks) {
-  return shadow ? occupancy_t<true>(complete, kp1, smem, blocks) : occupancy_t<false>(complete, kp1, smem, blocks);
+cudaError_t mix_configure(bool complete, bool fused, int kp1, bool shadow, size_t smem) {
+  return dispatch(complete, fused, kp1, shadow, [&](auto k) { return decltype(k)::attr(smem); });
 }
 
-cudaError_t launch_mix(const CUtensorMap& tmap, const MixArgs& a, bool complete, int grid, size_t smem,
+cudaError_t mix_occupancy(bool complete, bool fused, int kp1, bool shadow, size_t smem, int* blocks) {
+  return dispatch(complete, fused, kp1, shadow, [&](auto k) { return decltype(k)::occ(smem, blocks); });
+}
+
+cudaError_t launch_mix(const CUtensorMap& tmap, const MixArgs& a, bool complete, bool fused, int grid, size_t smem,
                        cudaStream_t s) {
-  return a.shadow ? launch_t<true>(tmap, a, complete, grid, smem, s)
-                  : launch_t<false>(tmap, a, complete, grid, smem, s);
+  return dispatch(complete, fused, a.kp1, a.shadow != nullptr,
+                  [&](auto k) { return decltype(k)::launch(tmap, a, grid, smem, s); });
 }
 
 cudaError_t launch_cast_bf16(const float* src, uint16_t* dst, int64_t n, cudaStream_t s) {

@@ -1,21 +1,29 @@
-// Local minibatch SGD step for sparse linear models (Eq. A.1, first line):
-//   m_b = x_b . w_i                                  (margin kernel)
-//   r_b = d loss(y_b, m_b) / d m_b                   (hinge or logistic)
-//   w_i[c] -= eta/B * sum_{b : c in x_b} r_b x_{b,c} (update kernel)
-// followed by NOTIFY: the last update CTA of worker i publishes
-// ready[i] = t+1 with release semantics (Section 4, NOTIFY-ACK).
+// Local minibatch SGD step for sparse linear models (Eq. A.1, first line).
 //
-// Margin kernel: one warp per row, 128-bit loads of column ids and values
-// (rows are padded to 4 entries), gathers of w[col], a fixed butterfly sum.
-// Update kernel: entries of the minibatch sorted by (column, row) are cut
-// into 32-entry chunks, one warp per chunk; a segmented warp scan sums each
-// column's run, and the warp that holds the first entry of a column owns
-// that column: it finishes runs that cross into later chunks itself.  No
-// global atomics touch W and every sum has a fixed order, so the result
-// does not depend on the schedule.
+// The step is split so that no kernel touches w at random addresses:
+//
+//   margin kernel   m_b = sum_e val_e * wv[pos_e]          (one warp per row)
+//                   r_b = d loss(y_b, m_b) / d m_b        (hinge or logistic)
+//   update kernel   g[p] = sum_{e : pos_e = p} r_{row_e} val_e   (column sums)
+//                   then NOTIFY ready[i] = t+1
+//
+// Each round's minibatch has, per worker, a list of the distinct columns it
+// touches.  The lists of all workers are laid out slab-major (by column slab
+// of the stochastic reduce, then worker, then column) and `pos` indexes that
+// list.  `wv[pos]` holds w_i[col] for the round's columns: the previous
+// round's reduce writes it while it holds the column slab in shared memory
+// (or, after parameters were written from the host, the gather kernel
+// below).  The reduce applies w_i[col] -= eta/B * g[pos] to the slab before
+// mixing it, so w_{t+1/2} never has to be written to HBM.
+//
+// Margin kernel: 128-bit loads of (pos, val), the L2-resident wv gathered,
+// a fixed butterfly sum.  Update kernel: entries sorted by (column, row) are
+// cut into 32-entry chunks, one warp per chunk; a segmented warp scan sums
+// each column's run and the warp holding a run's first entry owns it,
+// finishing runs that cross into later chunks itself.  No atomics on data,
+// every sum in a fixed order: the result does not depend on the schedule.
 #include <cuda_runtime.h>
 
-#include <climits>
 #include <cstdint>
 
 #include "asap_internal.h"
@@ -72,9 +80,9 @@ __global__ void __launch_bounds__(kThreads) k_margin_loss(SparseStepArgs a) {
   const BatchDesc dsc = a.desc[i];
   const int* rp = reinterpret_cast<const int*>(a.block + dsc.rp);
   const float* y = reinterpret_cast<const float*>(a.block + dsc.y);
-  const int4* col4 = reinterpret_cast<const int4*>(a.block + dsc.col);
+  const int4* pos4 = reinterpret_cast<const int4*>(a.block + dsc.posw);
   const float4* val4 = reinterpret_cast<const float4*>(a.block + dsc.val);
-  const float* w = a.W + static_cast<int64_t>(i) * a.ld;
+  const float* wv = a.wv;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int row_end = min(a.B, static_cast<int>(blockIdx.x + 1) * kMarginRowsPerCta);
   float lsum = 0.f;
@@ -82,12 +90,12 @@ __global__ void __launch_bounds__(kThreads) k_margin_loss(SparseStepArgs a) {
     const int q0 = rp[b] >> 2, q1 = rp[b + 1] >> 2;
     float acc = 0.f;
     for (int q = q0 + lane; q < q1; q += 32) {
-      const int4 c = ld_stream_i4(col4 + q);
+      const int4 p = ld_stream_i4(pos4 + q);
       const float4 v = ld_stream_f4(val4 + q);
-      acc = fmaf(v.x, __ldg(w + c.x), acc);
-      acc = fmaf(v.y, __ldg(w + c.y), acc);
-      acc = fmaf(v.z, __ldg(w + c.z), acc);
-      acc = fmaf(v.w, __ldg(w + c.w), acc);
+      acc = fmaf(v.x, __ldg(wv + p.x), acc);
+      acc = fmaf(v.y, __ldg(wv + p.y), acc);
+      acc = fmaf(v.z, __ldg(wv + p.z), acc);
+      acc = fmaf(v.w, __ldg(wv + p.w), acc);
     }
     const float m = warp_sum(acc);
     if (lane == 0) {
@@ -108,15 +116,15 @@ __global__ void __launch_bounds__(kThreads) k_margin_loss(SparseStepArgs a) {
   }
 }
 
-__global__ void __launch_bounds__(kThreads) k_segment_update(SparseStepArgs a) {
+__global__ void __launch_bounds__(kThreads) k_column_sums(SparseStepArgs a) {
   const int i = blockIdx.y;
   const BatchDesc dsc = a.desc[i];
   const int nnz = dsc.nnz;
-  const int* ccol = reinterpret_cast<const int*>(a.block + dsc.ccol);
+  const int* cpos = reinterpret_cast<const int*>(a.block + dsc.cpos);
   const float* cval = reinterpret_cast<const float*>(a.block + dsc.cval);
   const uint16_t* crow = reinterpret_cast<const uint16_t*>(a.block + dsc.crow);
   const float* r = a.r + static_cast<int64_t>(i) * a.B;
-  float* w = a.W + static_cast<int64_t>(i) * a.ld;
+  float* g = a.gsum;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const unsigned le_mask = (lane == 31) ? kFull : ((2u << lane) - 1u);
 
@@ -127,9 +135,9 @@ __global__ void __launch_bounds__(kThreads) k_segment_update(SparseStepArgs a) {
     if (chunk >= n_chunks) break;                  // warp-uniform
     const int e = chunk * 32 + lane;
     const bool valid = e < nnz;
-    const int c = valid ? ccol[e] : -1;
+    const int c = valid ? cpos[e] : -1;
     int cprev = __shfl_up_sync(kFull, c, 1);
-    if (lane == 0) cprev = (e > 0) ? ccol[e - 1] : -2;
+    if (lane == 0) cprev = (e > 0) ? cpos[e - 1] : -2;
     const bool head = valid && (c != cprev);
     float p = valid ? r[crow[e]] * cval[e] : 0.f;
     const unsigned heads = __ballot_sync(kFull, head);
@@ -144,33 +152,31 @@ __global__ void __launch_bounds__(kThreads) k_segment_update(SparseStepArgs a) {
     const bool next_head = __shfl_down_sync(kFull, head, 1);
     const bool next_valid = __shfl_down_sync(kFull, valid, 1);
     // Runs that end inside the chunk: the tail lane writes if the run began here.
-    if (valid && lane < 31 && (next_head || !next_valid) && start >= 0) {
-      w[c] = fmaf(-a.scale, p, w[c]);
-    }
+    if (valid && lane < 31 && (next_head || !next_valid) && start >= 0) g[c] = p;
     // The run through lane 31.
     const int c31 = __shfl_sync(kFull, c, 31);
     const int start31 = __shfl_sync(kFull, start, 31);
     const float p31 = __shfl_sync(kFull, p, 31);
     if (c31 >= 0 && start31 >= 0) {
       const int e31 = chunk * 32 + 31;
-      bool cont = (e31 + 1 < nnz) && (ccol[e31 + 1] == c31);
+      bool cont = (e31 + 1 < nnz) && (cpos[e31 + 1] == c31);
       float acc = p31;
       int base = e31 + 1;
       while (cont) {
         const int e2 = base + lane;
-        const bool in_run = (e2 < nnz) && (ccol[e2] == c31);
+        const bool in_run = (e2 < nnz) && (cpos[e2] == c31);
         const float q = in_run ? r[crow[e2]] * cval[e2] : 0.f;
         acc += warp_sum(q);
         const unsigned run = __ballot_sync(kFull, in_run);
-        cont = (run == kFull) && (base + 32 < nnz) && (ccol[base + 32] == c31);
+        cont = (run == kFull) && (base + 32 < nnz) && (cpos[base + 32] == c31);
         base += 32;
       }
-      if (lane == 0) w[c31] = fmaf(-a.scale, acc, w[c31]);
+      if (lane == 0) g[c31] = acc;
     }
   }
 
-  // NOTIFY: the last CTA of worker i publishes ready[i] = round + 1 after
-  // every CTA's writes to w_i are visible device-wide.
+  // NOTIFY: the last CTA of worker i publishes ready[i] = round + 1 once all
+  // of worker i's column sums are visible device-wide.
   __threadfence();
   __syncthreads();
   if (threadIdx.x == 0) {
@@ -183,18 +189,44 @@ __global__ void __launch_bounds__(kThreads) k_segment_update(SparseStepArgs a) {
   }
 }
 
+// wv[e] = W[i][s*S + cl] for every entry e of the round's column list
+// (parameters written from the host have no exported copy yet).
+__global__ void __launch_bounds__(kThreads) k_gather_wv(const float* __restrict__ W, int64_t ld,
+                                                       const uint32_t* __restrict__ list,
+                                                       const int* __restrict__ slab_off, long long n_slabs, int S,
+                                                       float* __restrict__ wv) {
+  for (long long s = blockIdx.x; s < n_slabs; s += gridDim.x) {
+    const int a0 = slab_off[s], a1 = slab_off[s + 1];
+    for (int e = a0 + threadIdx.x; e < a1; e += blockDim.x) {
+      const uint32_t code = list[e];
+      if (code == kListPad) continue;
+      const int i = static_cast<int>(code >> 16), cl = static_cast<int>(code & 0xffffu);
+      wv[e] = W[static_cast<int64_t>(i) * ld + s * S + cl];
+    }
+  }
+}
+
 }  // namespace
 
-cudaError_t launch_sparse_step(const SparseStepArgs& a, int N, int loss, int margin_ctas, int update_ctas,
-                               cudaStream_t s) {
-  const dim3 g1(margin_ctas, N), g2(update_ctas, N);
+cudaError_t launch_margin(const SparseStepArgs& a, int N, int loss, int margin_ctas, cudaStream_t s) {
+  const dim3 g1(margin_ctas, N);
   if (loss == ASAP_LOSS_HINGE)
     k_margin_loss<ASAP_LOSS_HINGE><<<g1, kThreads, 0, s>>>(a);
   else
     k_margin_loss<ASAP_LOSS_LOGISTIC><<<g1, kThreads, 0, s>>>(a);
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
-  k_segment_update<<<g2, kThreads, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_update(const SparseStepArgs& a, int N, int update_ctas, cudaStream_t s) {
+  const dim3 g2(update_ctas, N);
+  k_column_sums<<<g2, kThreads, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gather_wv(const float* W, int64_t ld, const uint32_t* list, const int* slab_off, long long n_slabs,
+                             int S, float* wv, int sm_count, cudaStream_t s) {
+  const int grid = static_cast<int>(n_slabs < 4LL * sm_count ? n_slabs : 4LL * sm_count);
+  k_gather_wv<<<grid > 0 ? grid : 1, kThreads, 0, s>>>(W, ld, list, slab_off, n_slabs, S, wv);
   return cudaGetLastError();
 }
 

@@ -63,7 +63,7 @@ def test_tiny_dense_logistic_ring_half_quarter():
     assert np.abs(lg - lref).max() <= 1e-4
     c = ctx.read_counters()
     assert c["reduces"] == N * T and c["consistent_inputs"] == N * 3 * T and c["timeouts"] == 0
-    assert ctx.kernel_launches() == 3 * T
+    assert ctx.kernel_launches() == 3 * T + 1     # one gather of w at the first round
 
 
 @pytest.mark.parametrize("loss", ["hinge", "logistic"])

@@ -148,6 +148,7 @@ struct asap_ctx {
   int64_t graph_ready_round = -1;   // round whose tables are staged in graph_nbr/graph_wgt
   const int* graph_nbr = nullptr;
   const float* graph_wgt = nullptr;
+  bool graph_uniform = false;       // every weight of the staged table is equal
   bool step_pending = false;
   int skip_notify = -1;
   unsigned long long wait_ns = 200000000ull;
@@ -235,10 +236,11 @@ asap_status setup_mix(asap_ctx* c) {
   // aligned in shared memory (S >= 8 floats per row).
   c->box_rows = ((N + c->n_boxes - 1) / c->n_boxes + 3) / 4 * 4;
   c->rows_pad = c->n_boxes * c->box_rows;
-  int S = 128;
+  // Slab: S columns of all rows, about 32 KB (8 <= S <= 1024, a power of 2).
+  int S = 1024;
   while (S > 8 && static_cast<size_t>(c->rows_pad) * S * 4 > 32768) S >>= 1;
   int maxS = 8;
-  while (static_cast<int64_t>(maxS) * 2 <= c->ld && maxS < 128) maxS <<= 1;
+  while (static_cast<int64_t>(maxS) * 2 <= c->ld && maxS < 1024) maxS <<= 1;
   c->S = std::min(S, maxS);
   c->n_slabs = (c->ld + c->S - 1) / c->S;
   c->tab_kp1 = is_complete_kernel(c) ? 0 : c->k + 1;
@@ -248,7 +250,7 @@ asap_status setup_mix(asap_ctx* c) {
   for (int b = 0; b < 2; ++b) {
     cuuint64_t dims[2] = {static_cast<cuuint64_t>(c->ld), static_cast<cuuint64_t>(N)};
     cuuint64_t strides[1] = {static_cast<cuuint64_t>(c->ld) * 4};
-    cuuint32_t box[2] = {static_cast<cuuint32_t>(c->S), static_cast<cuuint32_t>(c->box_rows)};
+    cuuint32_t box[2] = {static_cast<cuuint32_t>(std::min(c->S, 256)), static_cast<cuuint32_t>(c->box_rows)};
     cuuint32_t estr[2] = {1, 1};
     CUresult r = enc(&c->tmap[b], CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, c->W[b], dims, strides, box, estr,
                      CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -292,9 +294,14 @@ asap_status configure_mix_launch(asap_ctx* c, bool fused) {
   const long long key = (complete ? 1 : 0) | (shadow ? 2 : 0) | (fused ? 4 : 0) |
                         (static_cast<long long>(c->tab_kp1) << 3) | (static_cast<long long>(region) << 12);
   if (key == c->configured_key) return ASAP_OK;
-  // Stages: as many as fit in ~200 KB of shared memory, 2 to 8.
-  const size_t stage = mix_stage_bytes(c->S, c->rows_pad, region);
-  c->stages = static_cast<int>(std::max<size_t>(2, std::min<size_t>(8, (200u << 10) / stage)));
+  // Stages: as many as fit in shared memory (the whole footprint, per-stage
+  // partial sums included), 2 to 8.
+  c->stages = 2;
+  for (int st = 8; st > 2; --st)
+    if (mix_smem_bytes(c->N, c->tab_kp1, c->S, c->rows_pad, st, region) <= (220u << 10)) {
+      c->stages = st;
+      break;
+    }
   c->mix_smem = mix_smem_bytes(c->N, c->tab_kp1, c->S, c->rows_pad, c->stages, region);
   if (c->mix_smem > (227u << 10)) return fail(c, ASAP_ERR_ARG, "reduce stages do not fit in shared memory");
   CU(mix_configure(complete, fused, c->tab_kp1, shadow, c->mix_smem), "configuring the reduce kernel");
@@ -394,6 +401,10 @@ asap_status prepare_graph(asap_ctx* c, int64_t r) {
   if (c->graph_ready_round == r) return ASAP_OK;
   asap_status s = graph_tables(c, r, &c->graph_nbr, &c->graph_wgt);
   if (s != ASAP_OK) return s;
+  c->graph_uniform = true;
+  if (c->kind == ASAP_GRAPH_EXPLICIT)
+    for (float w : c->ex_wgt)
+      if (w != c->ex_wgt[0]) c->graph_uniform = false;
   c->graph_ready_round = r;
   return ASAP_OK;
 }
@@ -1151,6 +1162,7 @@ asap_status asap_stochastic_reduce(asap_ctx* c) {
   if (s != ASAP_OK) return s;
   const int* nbr = c->graph_nbr;
   const float* wgt = c->graph_wgt;
+  const int uniform = c->graph_uniform ? 1 : 0;
   c->graph_ready_round = -1;
   MixArgs a = {};
   a.out = c->W[(r + 1) & 1];
@@ -1161,6 +1173,7 @@ asap_status asap_stochastic_reduce(asap_ctx* c) {
   a.nbr = nbr;
   a.wgt = wgt;
   a.wscale = (c->step_pending && sparse) ? (1.0f - c->lr * c->l2) : 1.0f;
+  a.uniform_w = uniform;
   a.S = c->S;
   a.rows_pad = c->rows_pad;
   a.box_rows = c->box_rows;

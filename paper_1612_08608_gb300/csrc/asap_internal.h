@@ -80,6 +80,7 @@ struct MixArgs {
   const int* nbr;              // [N][kp1]
   const float* wgt;            // [N][kp1]
   float wscale;                // (1 - eta l2) after a local step, else 1
+  int uniform_w;               // every weight of the table equals wgt[0]
   int S;                       // slab width (columns)
   int rows_pad;                // smem rows per slab (box_rows * n_boxes)
   int box_rows;
@@ -144,7 +145,7 @@ cudaError_t launch_margin(const SparseStepArgs& a, int N, int loss, int margin_c
 cudaError_t launch_update(const SparseStepArgs& a, int N, int update_ctas, cudaStream_t s);
 cudaError_t launch_gather_wv(const float* W, int64_t ld, const uint32_t* list, const int* slab_off, long long n_slabs,
                              int S, float* wv, int sm_count, cudaStream_t s);
-constexpr int kMixComputeWarps = 8;
+constexpr int kMixComputeWarps = 16;
 constexpr int kMixThreads = (kMixComputeWarps + 1) * 32;   // + one TMA producer warp
 cudaError_t launch_mix(const CUtensorMap& tmap, const MixArgs& a, bool complete, bool fused, int grid, size_t smem,
                        cudaStream_t s);

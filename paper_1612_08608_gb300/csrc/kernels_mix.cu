@@ -4,12 +4,12 @@
 // and the mean minibatch loss) and the NOTIFY-ACK bookkeeping of Section 4.
 //
 // Data movement.  W is [N][ld] fp32 (ld a multiple of 64).  The kernel is
-// persistent: CTA b walks column slabs b, b + grid, ...  A slab is S (<= 128)
-// columns of *all* N rows.  One producer warp brings slabs into a ring of
+// persistent: CTA b walks column slabs b, b + grid, ...  A slab is S columns
+// (8 to 1024, about 32 KB) of *all* N rows.  One producer warp brings slabs into a ring of
 // shared-memory stages with TMA 2-D tiled loads (one box per 256 rows), so
 // every element of W is read from HBM exactly once however many neighbours
-// use it; eight compute warps mix and write the outputs straight from
-// registers.  A stage goes back to the producer when all eight compute warps
+// use it; sixteen compute warps mix and write the outputs straight from
+// registers.  A stage goes back to the producer when all the compute warps
 // have arrived on its "empty" mbarrier: no CTA-wide barrier in steady state.
 //
 // Sparse models (FUSED): the local step left, per distinct (worker, column)
@@ -22,9 +22,10 @@
 //
 // Consensus error per column: with K the column's value in row 0 (a shift
 // against cancellation), sum_i (w_i - wbar)^2 = sum_i (w_i - K)^2 -
-// (sum_i (w_i - K))^2 / N.  Squares accumulate per thread in fp64; the
-// per-column sums are combined across warps by the producer warp when the
-// stage comes back.  The complete graph (all-reduce, equal weights) writes
+// (sum_i (w_i - K))^2 / N.  Squares accumulate per thread in fp32 (a few
+// dozen slabs per thread; GB300's fp64 pipe is narrow), the per-column sums
+// are combined across warps by the producer warp when the stage comes back,
+// and the block total is formed in fp64.  The complete graph (all-reduce, equal weights) writes
 // the column mean to every row and adds nothing.
 //
 // Protocol (Section 4, NOTIFY-ACK): before touching any input each CTA waits,
@@ -92,21 +93,38 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 
-// Bounded wait on an mbarrier phase; false if the limit ran out.
+// Bounded wait on an mbarrier phase; false if the limit ran out.  The timer
+// is read every 256 polls only (each try_wait already suspends the thread
+// for a while), so waiting warps take few issue slots.
 __device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity) {
   if (mbar_try_wait(bar, parity)) return true;
   const unsigned long long t0 = globaltimer_ns();
-  for (;;) {
+  for (unsigned n = 1;; ++n) {
     if (mbar_try_wait(bar, parity)) return true;
-    if (globaltimer_ns() - t0 > kTmaWaitNs) return false;
+    if ((n & 255u) == 0 && globaltimer_ns() - t0 > kTmaWaitNs) return false;
   }
 }
 
-__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, uint64_t* bar, int x, int y) {
+// L2 policy for the parameter stream: each element is read once and written
+// once per round, so it should not push the round's small lists out of L2.
+__device__ __forceinline__ uint64_t evict_first_policy() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+
+__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, uint64_t* bar, int x, int y,
+                                            uint64_t policy) {
   asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];"
-      :: "r"(smem_u32(dst)), "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_u32(bar))
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1, {%2, %3}], [%4], %5;"
+      :: "r"(smem_u32(dst)), "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_u32(bar)), "l"(policy)
       : "memory");
+}
+
+__device__ __forceinline__ void st_f4_hint(float* p, float4 v, uint64_t policy) {
+  asm volatile("st.global.L2::cache_hint.v4.f32 [%0], {%1, %2, %3, %4}, %5;"
+               :: "l"(p), "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w), "l"(policy) : "memory");
 }
 
 // Untiled bulk copy global -> shared (16-byte aligned, size a multiple of 16).
@@ -211,7 +229,7 @@ __device__ __forceinline__ MixSmem carve(unsigned char* raw, const MixArgs& a, i
   m.info = reinterpret_cast<int*>(base);
   base += 16 * a.stages;
   m.part = reinterpret_cast<float4*>(base);   // 16-byte aligned: every region above is a multiple of 16
-  base += 16 * static_cast<size_t>(a.stages) * kMixComputeWarps * (a.S / 4);
+  base += 16 * static_cast<size_t>(a.stages) * kCompute;
   m.nbr = reinterpret_cast<int*>(base);
   base += 4 * static_cast<size_t>(a.N) * kp1;
   m.wgt = reinterpret_cast<float*>(base);
@@ -227,8 +245,10 @@ __global__ void __launch_bounds__(kMixThreads, 1) k_mix(const __grid_constant__ 
   const int kp1 = KP1 > 0 ? KP1 : (KP1 == 0 ? a.kp1 : 0);
   MixSmem sm = carve(smem_raw, a, kp1);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int S = a.S, nq = S >> 2;
-  const int lq = __ffs(nq) - 1;              // nq is a power of two, <= 32
+  const int S = a.S, nq = S >> 2;            // column quads per slab, a power of two <= 256
+  const int lq = __ffs(nq) - 1;
+  const int QB = nq < 64 ? nq : 64;           // quads per TMA box row (a box spans <= 256 columns)
+  const int G = kCompute >> lq;               // row groups: compute threads that share a column quad
   const size_t slab_floats = static_cast<size_t>(a.rows_pad) * S;
   const size_t list_off = (slab_floats * 4 + 15) & ~static_cast<size_t>(15);
   const size_t list_bytes = (static_cast<size_t>(a.max_region) * 4 + 15) & ~static_cast<size_t>(15);
@@ -250,11 +270,11 @@ __global__ void __launch_bounds__(kMixThreads, 1) k_mix(const __grid_constant__ 
   __syncthreads();
   bool failed = sm.flags[0] != 0;
 
-  double s2 = 0.0;     // compute threads: sum of (w - K)^2;  producer lanes: sum of S1^2 / N
+  float s2 = 0.f;      // compute threads: sum of (w - K)^2;  producer lanes: -sum of S1^2 / N
   if (!failed) {
     if (KP1 >= 0) {
       for (int idx = tid; idx < a.N * kp1; idx += kMixThreads) {
-        sm.nbr[idx] = a.nbr[idx];
+        sm.nbr[idx] = a.nbr[idx] * QB;       // float4 offset of the neighbour's row within a box column
         sm.wgt[idx] = a.wgt[idx] * a.wscale;
       }
     }
@@ -271,24 +291,48 @@ __global__ void __launch_bounds__(kMixThreads, 1) k_mix(const __grid_constant__ 
     const long long n_my = (a.n_slabs - blockIdx.x + stride - 1) / stride;   // slabs of this CTA
     const float inv_n = 1.0f / static_cast<float>(a.N);
 
+    const uint64_t policy = evict_first_policy();
     if (warp == kProducerWarp) {
       // ================= producer warp =================
-      double term = 0.0;
+      float term = 0.f;
+      const float inv_n_term = 1.0f / static_cast<float>(a.N);
+      // List offsets of the next 32 slabs, one slab per lane, loaded ahead so
+      // that issuing a stage never waits on a global load.
+      int4 offs = make_int4(0, 0, 0, 0);
       for (long long it = 0; it < n_my + a.stages; ++it) {
+        if (FUSED && (it & 31) == 0 && it < n_my) {
+          const long long sl = blockIdx.x + (it + lane) * stride;
+          if (it + lane < n_my)
+            offs = make_int4(__ldg(a.upd_off + sl), __ldg(a.upd_off + sl + 1), __ldg(a.exp_off + sl),
+                             __ldg(a.exp_off + sl + 1));
+        }
+        int4 o = make_int4(0, 0, 0, 0);
+        if (FUSED) {
+          const int src = static_cast<int>(it & 31);
+          o.x = __shfl_sync(kFull, offs.x, src);
+          o.y = __shfl_sync(kFull, offs.y, src);
+          o.z = __shfl_sync(kFull, offs.z, src);
+          o.w = __shfl_sync(kFull, offs.w, src);
+        }
         if (it >= a.stages) {
           const long long done = it - a.stages;
           const int st = static_cast<int>(done % a.stages);
-          if (!mbar_wait_bounded(sm.empty + st, static_cast<uint32_t>((done / a.stages) & 1))) {
+          bool ok = (lane == 0) ? mbar_wait_bounded(sm.empty + st, static_cast<uint32_t>((done / a.stages) & 1))
+                                : true;
+          ok = __shfl_sync(kFull, ok, 0) != 0;   // warp-uniform outcome
+          __syncwarp();
+          if (!ok) {
             if (lane == 0) record_error(a.st, ASAP_ERR_CUDA, 0xfffffffeu, a.round);
             failed = true;
             break;
           }
-          if (KP1 >= 0 && lane < nq) {
-            const float4* p = sm.part + static_cast<size_t>(st) * kMixComputeWarps * nq;
-            float4 t = p[lane];
-            for (int w = 1; w < kMixComputeWarps; ++w) t = f4_add(t, p[w * nq + lane]);
-            term += (static_cast<double>(t.x) * t.x + static_cast<double>(t.y) * t.y +
-                     static_cast<double>(t.z) * t.z + static_cast<double>(t.w) * t.w) / a.N;
+          if (KP1 >= 0) {
+            const float4* p = sm.part + static_cast<size_t>(st) * kCompute;
+            for (int q = lane; q < nq; q += 32) {
+              float4 t = p[q];
+              for (int g = 1; g < G; ++g) t = f4_add(t, p[g * nq + q]);
+              term = fmaf(fmaf(t.x, t.x, fmaf(t.y, t.y, fmaf(t.z, t.z, t.w * t.w))), inv_n_term, term);
+            }
           }
           __syncwarp();
         }
@@ -299,10 +343,10 @@ __global__ void __launch_bounds__(kMixThreads, 1) k_mix(const __grid_constant__ 
           uint32_t bytes = static_cast<uint32_t>(a.n_boxes) * a.box_rows * S * 4u;
           int n_upd = 0, n_exp = 0, x0 = 0, u0 = 0;
           if (FUSED) {
-            u0 = a.upd_off[slab];
-            n_upd = a.upd_off[slab + 1] - u0;
-            x0 = a.exp_off[slab];
-            n_exp = a.exp_off[slab + 1] - x0;
+            u0 = o.x;
+            n_upd = o.y - o.x;
+            x0 = o.z;
+            n_exp = o.w - o.z;
             bytes += 8u * n_upd + 4u * n_exp;
           }
           int* info = sm.info + 4 * st;
@@ -310,9 +354,11 @@ __global__ void __launch_bounds__(kMixThreads, 1) k_mix(const __grid_constant__ 
           info[1] = n_exp;
           info[2] = x0;
           mbar_expect_tx(sm.full + st, bytes);
-          for (int b = 0; b < a.n_boxes; ++b)
-            tma_load_2d(base + static_cast<size_t>(b) * a.box_rows * S * 4, &tmap, sm.full + st,
-                        static_cast<int>(slab * S), b * a.box_rows);
+          // Slab layout in shared memory: [column box][row][QB quads].
+          for (int xb = 0; xb < nq / QB; ++xb)
+            for (int b = 0; b < a.n_boxes; ++b)
+              tma_load_2d(base + (static_cast<size_t>(xb) * a.rows_pad + static_cast<size_t>(b) * a.box_rows) * QB * 16,
+                          &tmap, sm.full + st, static_cast<int>(slab * S + xb * QB * 4), b * a.box_rows, policy);
           if (FUSED) {
             if (n_upd > 0) {
               bulk_load(base + list_off, a.upd_list + u0, 4u * n_upd, sm.full + st);
@@ -326,18 +372,21 @@ __global__ void __launch_bounds__(kMixThreads, 1) k_mix(const __grid_constant__ 
       s2 = -term;
     } else {
       // ================= compute warps =================
-      const int rows_w = (a.N - warp + kMixComputeWarps - 1) / kMixComputeWarps;   // rows i = warp + 8 r
-      const int pairs = rows_w << lq;
-      const int q_l = lane & (nq - 1);
+      // Thread t owns column quad q = t mod nq of every slab for the rows
+      // i = g, g + G, ... (g = t / nq): with ~32 KB slabs that is 4 rows.
+      const int q_t = tid & (nq - 1), g_t = tid >> lq;
+      const int qoff = (q_t / QB) * a.rows_pad * QB + (q_t % QB);   // float4 offset of (row 0, quad q_t)
+      const int rows_t = (a.N - g_t + G - 1) / G;
+      auto xq = [&](int q) { return (q / QB) * a.rows_pad * QB + (q % QB); };
       for (long long it = 0; it < n_my; ++it) {
         const long long slab = blockIdx.x + it * stride;
         const int st = static_cast<int>(it % a.stages);
-        bool ok = mbar_wait_bounded(sm.full + st, static_cast<uint32_t>((it / a.stages) & 1));
+        bool ok = __all_sync(kFull, mbar_wait_bounded(sm.full + st, static_cast<uint32_t>((it / a.stages) & 1)));
         unsigned char* base = sm.stage0 + st * sm.stage_bytes;
         float* x = reinterpret_cast<float*>(base);
         const float4* x4 = reinterpret_cast<const float4*>(base);
         const int* info = sm.info + 4 * st;
-        float4* part = sm.part + (static_cast<size_t>(st) * kMixComputeWarps + warp) * nq;
+        float4* part = sm.part + static_cast<size_t>(st) * kCompute;
         const long long c0 = slab * S;
         if (ok && FUSED) {
           // w_half = w - eta/B g on the slab (distinct (worker, column) per entry).
@@ -347,18 +396,18 @@ __global__ void __launch_bounds__(kMixThreads, 1) k_mix(const __grid_constant__ 
           for (int e = tid; e < n_upd; e += kCompute) {
             const uint32_t code = ul[e];
             if (code != kListPad) {
-              float* px = x + (code >> 16) * S + (code & 0xffffu);
+              const int i = static_cast<int>(code >> 16), cl = static_cast<int>(code & 0xffffu);
+              float* px = x + 4 * (i * QB + xq(cl >> 2)) + (cl & 3);
               *px = fmaf(-a.upd_scale, ug[e], *px);
             }
           }
         }
         if (FUSED && KP1 < 0) ok = !compute_bar_or(!ok);   // the update is visible to the column sums
         if (ok && KP1 < 0) {
-          // Complete graph: per-warp column sums over its rows.
+          // Complete graph: this thread's share of its column's sum.
           float4 cs = make_float4(0.f, 0.f, 0.f, 0.f);
-          for (int p = lane; p < pairs; p += 32) cs = f4_add(cs, x4[((warp + ((p >> lq) << 3)) << lq) + q_l]);
-          for (int o = nq; o < 32; o <<= 1) cs = f4_add(cs, f4_shfl_xor(cs, o));
-          if (lane < nq) part[lane] = cs;
+          for (int r = 0; r < rows_t; ++r) cs = f4_add(cs, x4[(g_t + r * G) * QB + qoff]);
+          part[tid] = cs;
         }
         if (FUSED || KP1 < 0) ok = !compute_bar_or(!ok);   // uniform decision; the update / sums are visible
         if (!ok) {
@@ -367,17 +416,20 @@ __global__ void __launch_bounds__(kMixThreads, 1) k_mix(const __grid_constant__ 
           break;
         }
         if constexpr (KP1 < 0) {
-          // Complete graph: column mean over all N rows, written to every row.
-          float4* p0 = sm.part + static_cast<size_t>(st) * kMixComputeWarps * nq;
-          float4 t = p0[q_l];
-          for (int w = 1; w < kMixComputeWarps; ++w) t = f4_add(t, p0[w * nq + q_l]);
-          const float sc = inv_n * a.wscale;
-          const float4 mean = make_float4(t.x * sc, t.y * sc, t.z * sc, t.w * sc);
-          for (int p = lane; p < pairs; p += 32) {
-            const int i = warp + ((p >> lq) << 3);
-            const long long c = c0 + 4 * q_l;
+          // Complete graph: column means (threads t < nq), then every row gets them.
+          if (tid < nq) {
+            float4 t = part[tid];
+            for (int g = 1; g < G; ++g) t = f4_add(t, part[g * nq + tid]);
+            const float sc = inv_n * a.wscale;
+            part[tid] = make_float4(t.x * sc, t.y * sc, t.z * sc, t.w * sc);
+          }
+          compute_bar();
+          const float4 mean = part[q_t];
+          for (int r = 0; r < rows_t; ++r) {
+            const int i = g_t + r * G;
+            const long long c = c0 + 4 * q_t;
             if (c < a.ld) {
-              *reinterpret_cast<float4*>(a.out + static_cast<int64_t>(i) * a.ld + c) = mean;
+              st_f4_hint(a.out + static_cast<int64_t>(i) * a.ld + c, mean, policy);
               if (SHADOW) {
                 __nv_bfloat162 lo = __floats2bfloat162_rn(mean.x, mean.y);
                 __nv_bfloat162 hi = __floats2bfloat162_rn(mean.z, mean.w);
@@ -389,36 +441,35 @@ __global__ void __launch_bounds__(kMixThreads, 1) k_mix(const __grid_constant__ 
             }
           }
           if (FUSED) {
-            // every lane needs the means of all columns: keep them in the partial slot of warp 0
-            compute_bar();
-            if (warp == 0 && lane < nq) p0[lane] = mean;   // p0 aliases warp 0's partials (read above)
-            compute_bar();
             const uint32_t* xl = reinterpret_cast<const uint32_t*>(base + list_off + 2 * list_bytes);
             const int n_exp = info[1], xbase = info[2];
-            const float* means = reinterpret_cast<const float*>(p0);
+            const float* means = reinterpret_cast<const float*>(part);
             for (int e = tid; e < n_exp; e += kCompute) {
               const uint32_t code = xl[e];
               if (code != kListPad) a.wv_out[xbase + e] = means[code & 0xffffu];
             }
           }
+          compute_bar();   // the means are read before the next slab's sums overwrite them
         } else {
-          const float4 K = x4[q_l];        // shift: row 0 of the (updated) slab
+          const float4 K = x4[qoff];        // shift: row 0 of the (updated) slab
           float4 s1 = make_float4(0.f, 0.f, 0.f, 0.f);
           float sq = 0.f;
-          for (int p = lane; p < pairs; p += 32) {
-            const int i = warp + ((p >> lq) << 3);
+          auto mix_one = [&](int i) -> float4 {
             const int* nb = sm.nbr + i * kp1;
             const float* wt = sm.wgt + i * kp1;
-            const float4 xa = x4[(nb[0] << lq) + q_l];
+            const float4 xa = x4[nb[0] + qoff];
             float4 acc = make_float4(wt[0] * xa.x, wt[0] * xa.y, wt[0] * xa.z, wt[0] * xa.w);
 #pragma unroll
             for (int m = 1; m < (KP1 > 0 ? KP1 : kMaxKp1Sparse); ++m) {
               if (KP1 == 0 && m >= kp1) break;
-              acc = f4_fma(wt[m], x4[(nb[m] << lq) + q_l], acc);
+              acc = f4_fma(wt[m], x4[nb[m] + qoff], acc);
             }
-            const long long c = c0 + 4 * q_l;
+            return acc;
+          };
+          auto emit = [&](int i, float4 acc) {
+            const long long c = c0 + 4 * q_t;
             if (c < a.ld) {
-              *reinterpret_cast<float4*>(a.out + static_cast<int64_t>(i) * a.ld + c) = acc;
+              st_f4_hint(a.out + static_cast<int64_t>(i) * a.ld + c, acc, policy);
               if (SHADOW) {
                 __nv_bfloat162 lo = __floats2bfloat162_rn(acc.x, acc.y);
                 __nv_bfloat162 hi = __floats2bfloat162_rn(acc.z, acc.w);
@@ -431,10 +482,18 @@ __global__ void __launch_bounds__(kMixThreads, 1) k_mix(const __grid_constant__ 
             const float dx = acc.x - K.x, dy = acc.y - K.y, dz = acc.z - K.z, dw = acc.w - K.w;
             s1 = f4_add(s1, make_float4(dx, dy, dz, dw));
             sq = fmaf(dx, dx, fmaf(dy, dy, fmaf(dz, dz, fmaf(dw, dw, sq))));
+          };
+          int r = 0;
+          for (; r + 1 < rows_t; r += 2) {      // two rows in flight
+            const int i0 = g_t + r * G, i1 = i0 + G;
+            const float4 a0 = mix_one(i0);
+            const float4 a1 = mix_one(i1);
+            emit(i0, a0);
+            emit(i1, a1);
           }
-          s2 += static_cast<double>(sq);
-          for (int o = nq; o < 32; o <<= 1) s1 = f4_add(s1, f4_shfl_xor(s1, o));
-          if (lane < nq) part[lane] = s1;
+          if (r < rows_t) emit(g_t + r * G, mix_one(g_t + r * G));
+          s2 += sq;
+          part[tid] = s1;
           if (FUSED) {
             // w_{t+1} at the next round's columns, recomputed with the same
             // operations in the same order as the stored outputs.
@@ -446,8 +505,9 @@ __global__ void __launch_bounds__(kMixThreads, 1) k_mix(const __grid_constant__ 
               const int i = static_cast<int>(code >> 16), cl = static_cast<int>(code & 0xffffu);
               const int* nb = sm.nbr + i * kp1;
               const float* wt = sm.wgt + i * kp1;
-              float v = wt[0] * x[nb[0] * S + cl];
-              for (int m = 1; m < kp1; ++m) v = fmaf(wt[m], x[nb[m] * S + cl], v);
+              const int xo = xq(cl >> 2), comp = cl & 3;
+              float v = wt[0] * x[4 * (nb[0] + xo) + comp];
+              for (int m = 1; m < kp1; ++m) v = fmaf(wt[m], x[4 * (nb[m] + xo) + comp], v);
               a.wv_out[xbase + e] = v;
             }
             asm volatile("fence.proxy.async.shared::cta;" ::: "memory");   // generic writes before the next TMA
@@ -460,7 +520,7 @@ __global__ void __launch_bounds__(kMixThreads, 1) k_mix(const __grid_constant__ 
   }
 
   // ---- per-CTA partial, ticket, and the last CTA's finalisation ----
-  const double csum = block_sum_f64(s2, sm.dscratch);
+  const double csum = block_sum_f64(static_cast<double>(s2), sm.dscratch);
   if (failed) atomicOr(&sm.flags[0], 1);
   __syncthreads();
   if (tid == 0) a.cons_part[blockIdx.x] = csum;
@@ -563,7 +623,7 @@ ASAP_HD size_t mix_stage_bytes(int S, int rows_pad, int max_region) {
 
 size_t mix_smem_bytes(int N, int kp1, int S, int rows_pad, int stages, int max_region) {
   return 1024 + mix_stage_bytes(S, rows_pad, max_region) * stages + 16 * stages + ((8 * (kMixThreads / 32) + 15) & ~15) + 16 +
-         16 * stages + 16 * static_cast<size_t>(stages) * kMixComputeWarps * (S / 4) + 8 * static_cast<size_t>(N) * kp1;
+         16 * stages + 16 * static_cast<size_t>(stages) * kMixComputeWarps * 32 + 8 * static_cast<size_t>(N) * kp1;
 }
 
 cudaError_t mix_configure(bool complete, bool fused, int kp1, bool shadow, size_t smem) {

@@ -2,7 +2,7 @@
 //
 // The step is split so that no kernel touches w at random addresses:
 //
-//   margin kernel   m_b = sum_e val_e * wv[pos_e]          (one warp per row)
+//   margin kernel   m_b = sum_e val_e * wv[pos_e]          (8 lanes per row)
 //                   r_b = d loss(y_b, m_b) / d m_b        (hinge or logistic)
 //   update kernel   g[p] = sum_{e : pos_e = p} r_{row_e} val_e   (column sums)
 //                   then NOTIFY ready[i] = t+1
@@ -16,8 +16,9 @@
 // below).  The reduce applies w_i[col] -= eta/B * g[pos] to the slab before
 // mixing it, so w_{t+1/2} never has to be written to HBM.
 //
-// Margin kernel: 128-bit loads of (pos, val), the L2-resident wv gathered,
-// a fixed butterfly sum.  Update kernel: entries sorted by (column, row) are
+// Margin kernel: 8 lanes per row (4 rows in flight per warp), 128-bit loads
+// of (pos, val), the L2-resident wv gathered, a fixed butterfly sum.
+// Update kernel: entries sorted by (column, row) are
 // cut into 32-entry chunks, one warp per chunk; a segmented warp scan sums
 // each column's run and the warp holding a run's first entry owns it,
 // finishing runs that cross into later chunks itself.  No atomics on data,
@@ -76,6 +77,8 @@ __device__ __forceinline__ void loss_and_r(float y, float m, float& l, float& r)
 
 template <int LOSS>
 __global__ void __launch_bounds__(kThreads) k_margin_loss(SparseStepArgs a) {
+  // 8 lanes per row, so that each warp keeps the loads of 4 rows in flight.
+  constexpr int kLanesPerRow = 8;
   const int i = blockIdx.y;
   const BatchDesc dsc = a.desc[i];
   const int* rp = reinterpret_cast<const int*>(a.block + dsc.rp);
@@ -84,12 +87,13 @@ __global__ void __launch_bounds__(kThreads) k_margin_loss(SparseStepArgs a) {
   const float4* val4 = reinterpret_cast<const float4*>(a.block + dsc.val);
   const float* wv = a.wv;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int row_end = min(a.B, static_cast<int>(blockIdx.x + 1) * kMarginRowsPerCta);
+  const int sub = lane / kLanesPerRow, sl = lane % kLanesPerRow;
+  const int b = blockIdx.x * kMarginRowsPerCta + warp * (32 / kLanesPerRow) + sub;   // 8 warps x 4 rows
   float lsum = 0.f;
-  for (int b = blockIdx.x * kMarginRowsPerCta + warp; b < row_end; b += kThreads / 32) {
+  float acc = 0.f;
+  if (b < a.B) {
     const int q0 = rp[b] >> 2, q1 = rp[b + 1] >> 2;
-    float acc = 0.f;
-    for (int q = q0 + lane; q < q1; q += 32) {
+    for (int q = q0 + sl; q < q1; q += kLanesPerRow) {
       const int4 p = ld_stream_i4(pos4 + q);
       const float4 v = ld_stream_f4(val4 + q);
       acc = fmaf(v.x, __ldg(wv + p.x), acc);
@@ -97,14 +101,18 @@ __global__ void __launch_bounds__(kThreads) k_margin_loss(SparseStepArgs a) {
       acc = fmaf(v.z, __ldg(wv + p.z), acc);
       acc = fmaf(v.w, __ldg(wv + p.w), acc);
     }
-    const float m = warp_sum(acc);
-    if (lane == 0) {
-      float l, r;
-      loss_and_r<LOSS>(y[b], m, l, r);
-      a.r[static_cast<int64_t>(i) * a.B + b] = r;
-      lsum += l;
-    }
   }
+#pragma unroll
+  for (int o = kLanesPerRow / 2; o > 0; o >>= 1) acc += __shfl_xor_sync(kFull, acc, o);
+  if (b < a.B && sl == 0) {
+    float l, r;
+    loss_and_r<LOSS>(y[b], acc, l, r);
+    a.r[static_cast<int64_t>(i) * a.B + b] = r;
+    lsum = l;
+  }
+  // fixed-order sum of the CTA's 32 row losses
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) lsum += __shfl_xor_sync(kFull, lsum, o);
   __shared__ float part[kThreads / 32];
   if (lane == 0) part[warp] = lsum;
   __syncthreads();
@@ -176,10 +184,11 @@ __global__ void __launch_bounds__(kThreads) k_column_sums(SparseStepArgs a) {
   }
 
   // NOTIFY: the last CTA of worker i publishes ready[i] = round + 1 once all
-  // of worker i's column sums are visible device-wide.
-  __threadfence();
+  // of worker i's column sums are visible device-wide.  The CTA barrier
+  // orders this CTA's writes before thread 0's fence, which is cumulative.
   __syncthreads();
   if (threadIdx.x == 0) {
+    __threadfence();
     const unsigned int done = atomicAdd(&a.worker_ticket[i], 1u);
     if (done == gridDim.x - 1) {
       a.worker_ticket[i] = 0u;

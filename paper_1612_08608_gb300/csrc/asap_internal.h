@@ -146,7 +146,9 @@ cudaError_t launch_update(const SparseStepArgs& a, int N, int update_ctas, cudaS
 cudaError_t launch_gather_wv(const float* W, int64_t ld, const uint32_t* list, const int* slab_off, long long n_slabs,
                              int S, float* wv, int sm_count, cudaStream_t s);
 constexpr int kMixComputeWarps = 16;
-constexpr int kMixThreads = (kMixComputeWarps + 1) * 32;   // + one TMA producer warp
+constexpr int kMixUpdaterWarps = 2;
+// compute warps + one TMA producer warp + the warps that apply the fused update
+constexpr int kMixThreads = (kMixComputeWarps + 1 + kMixUpdaterWarps) * 32;
 cudaError_t launch_mix(const CUtensorMap& tmap, const MixArgs& a, bool complete, bool fused, int grid, size_t smem,
                        cudaStream_t s);
 ASAP_HD size_t mix_stage_bytes(int S, int rows_pad, int max_region);

@@ -15,9 +15,10 @@
 // Sparse models (FUSED): the local step left, per distinct (worker, column)
 // of the minibatch, the column sum g of r_b x_b (kernels_sparse.cu).  The
 // producer also copies the slab's part of that list (and of the next
-// round's list) into the stage; the compute warps apply
-// w -= eta/B (1 - eta l2)^-1 g to the slab first -- so w_{t+1/2} exists only
-// in shared memory -- and after mixing they export w_{t+1} at the next
+// round's list) into the stage; once a slab has landed two updater warps
+// apply w -= eta/B (1 - eta l2)^-1 g to it and release it to the compute
+// warps through a "ready" mbarrier -- so w_{t+1/2} exists only in shared
+// memory -- and after mixing the compute warps export w_{t+1} at the next
 // round's columns, which is all the next margin kernel reads.
 //
 // Consensus error per column: with K the column's value in row 0 (a shift
@@ -51,6 +52,7 @@ constexpr unsigned kFull = 0xffffffffu;
 constexpr unsigned long long kTmaWaitNs = 2000000000ull;   // 2 s: a TMA load never takes this long
 constexpr int kCompute = kMixComputeWarps * 32;            // compute threads
 constexpr int kProducerWarp = kMixComputeWarps;
+constexpr int kUpdater0 = kMixComputeWarps + 1;             // first updater warp
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -169,11 +171,6 @@ __device__ __forceinline__ float4 f4_add(float4 a, float4 b) {
   return make_float4(a.x + b.x, a.y + b.y, a.z + b.z, a.w + b.w);
 }
 
-__device__ __forceinline__ float4 f4_shfl_xor(float4 v, int m) {
-  return make_float4(__shfl_xor_sync(kFull, v.x, m), __shfl_xor_sync(kFull, v.y, m), __shfl_xor_sync(kFull, v.z, m),
-                     __shfl_xor_sync(kFull, v.w, m));
-}
-
 // Sum over all threads of the block (kMixThreads); valid in thread 0.
 __device__ __forceinline__ double block_sum_f64(double v, double* scratch) {
 #pragma unroll
@@ -204,6 +201,7 @@ struct MixSmem {
   size_t stage_bytes;
   uint64_t* full;
   uint64_t* empty;
+  uint64_t* ready;   // FUSED: the producer has applied the slab's update
   float4* part;      // [stages][warps][nq]: per-warp column sums (consensus / complete-graph mean)
   int* info;         // [stages][4]: n_upd, n_exp, exp_base
   int* nbr;
@@ -212,8 +210,11 @@ struct MixSmem {
   int* flags;        // [0]: fail, [1]: last
 };
 
+// Shared-memory layout; every region starts 16-byte aligned (the slab
+// stages 1024-byte aligned).  mix_smem_bytes() mirrors it.
 __device__ __forceinline__ MixSmem carve(unsigned char* raw, const MixArgs& a, int kp1) {
   MixSmem m;
+  auto a16 = [](uintptr_t v) { return (v + 15) & ~static_cast<uintptr_t>(15); };
   uintptr_t base = (reinterpret_cast<uintptr_t>(raw) + 1023) & ~static_cast<uintptr_t>(1023);
   m.stage_bytes = mix_stage_bytes(a.S, a.rows_pad, a.max_region);
   m.stage0 = reinterpret_cast<unsigned char*>(base);
@@ -222,16 +223,18 @@ __device__ __forceinline__ MixSmem carve(unsigned char* raw, const MixArgs& a, i
   base += 8 * a.stages;
   m.empty = reinterpret_cast<uint64_t*>(base);
   base += 8 * a.stages;
+  m.ready = reinterpret_cast<uint64_t*>(base);
+  base = a16(base + 8 * a.stages);
   m.dscratch = reinterpret_cast<double*>(base);
-  base += (8 * (kMixThreads / 32) + 15) & ~15;
+  base = a16(base + 8 * (kMixThreads / 32));
   m.flags = reinterpret_cast<int*>(base);
-  base += 16;
+  base = a16(base + 16);
   m.info = reinterpret_cast<int*>(base);
-  base += 16 * a.stages;
-  m.part = reinterpret_cast<float4*>(base);   // 16-byte aligned: every region above is a multiple of 16
-  base += 16 * static_cast<size_t>(a.stages) * kCompute;
+  base = a16(base + 16 * a.stages);
+  m.part = reinterpret_cast<float4*>(base);
+  base = a16(base + 16 * static_cast<size_t>(a.stages) * kCompute);
   m.nbr = reinterpret_cast<int*>(base);
-  base += 4 * static_cast<size_t>(a.N) * kp1;
+  base = a16(base + 4 * static_cast<size_t>(a.N) * kp1);
   m.wgt = reinterpret_cast<float*>(base);
   return m;
 }
@@ -282,6 +285,7 @@ __global__ void __launch_bounds__(kMixThreads, 1) k_mix(const __grid_constant__ 
       for (int s = 0; s < a.stages; ++s) {
         mbar_init(sm.full + s, 1);
         mbar_init(sm.empty + s, kMixComputeWarps);
+        mbar_init(sm.ready + s, kMixUpdaterWarps);
       }
       asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
@@ -370,6 +374,39 @@ __global__ void __launch_bounds__(kMixThreads, 1) k_mix(const __grid_constant__ 
         __syncwarp();
       }
       s2 = -term;
+    } else if (warp >= kUpdater0) {
+      // ================= updater warps (FUSED) =================
+      // Once a slab has landed, apply w -= eta/B (1 - eta l2)^-1 g to it and
+      // release it to the compute warps.
+      if (FUSED) {
+        const int ut = tid - kUpdater0 * 32;
+        for (long long it = 0; it < n_my; ++it) {
+          const int st = static_cast<int>(it % a.stages);
+          const bool ok = __all_sync(kFull, mbar_wait_bounded(sm.full + st, static_cast<uint32_t>((it / a.stages) & 1)));
+          if (!ok) {
+            if (lane == 0) record_error(a.st, ASAP_ERR_CUDA, 0xfffffffdu, a.round);
+            failed = true;
+            break;
+          }
+          unsigned char* bj = sm.stage0 + st * sm.stage_bytes;
+          float* xj = reinterpret_cast<float*>(bj);
+          const uint32_t* ul = reinterpret_cast<const uint32_t*>(bj + list_off);
+          const float* ug = reinterpret_cast<const float*>(bj + list_off + list_bytes);
+          const int n_upd = sm.info[4 * st];
+          for (int e = ut; e < n_upd; e += kMixUpdaterWarps * 32) {
+            const uint32_t code = ul[e];
+            if (code != kListPad) {
+              const int i = static_cast<int>(code >> 16), cl = static_cast<int>(code & 0xffffu);
+              const int q = cl >> 2;
+              float* px = xj + 4 * (i * QB + (q / QB) * a.rows_pad * QB + (q % QB)) + (cl & 3);
+              *px = fmaf(-a.upd_scale, ug[e], *px);
+            }
+          }
+          asm volatile("fence.proxy.async.shared::cta;" ::: "memory");   // before this stage's next TMA
+          __syncwarp();
+          if (lane == 0) mbar_arrive(sm.ready + st);
+        }
+      }
     } else {
       // ================= compute warps =================
       // Thread t owns column quad q = t mod nq of every slab for the rows
@@ -381,35 +418,21 @@ __global__ void __launch_bounds__(kMixThreads, 1) k_mix(const __grid_constant__ 
       for (long long it = 0; it < n_my; ++it) {
         const long long slab = blockIdx.x + it * stride;
         const int st = static_cast<int>(it % a.stages);
-        bool ok = __all_sync(kFull, mbar_wait_bounded(sm.full + st, static_cast<uint32_t>((it / a.stages) & 1)));
+        bool ok = __all_sync(kFull, mbar_wait_bounded(FUSED ? sm.ready + st : sm.full + st,
+                                                      static_cast<uint32_t>((it / a.stages) & 1)));
         unsigned char* base = sm.stage0 + st * sm.stage_bytes;
         float* x = reinterpret_cast<float*>(base);
         const float4* x4 = reinterpret_cast<const float4*>(base);
         const int* info = sm.info + 4 * st;
         float4* part = sm.part + static_cast<size_t>(st) * kCompute;
         const long long c0 = slab * S;
-        if (ok && FUSED) {
-          // w_half = w - eta/B g on the slab (distinct (worker, column) per entry).
-          const uint32_t* ul = reinterpret_cast<const uint32_t*>(base + list_off);
-          const float* ug = reinterpret_cast<const float*>(base + list_off + list_bytes);
-          const int n_upd = info[0];
-          for (int e = tid; e < n_upd; e += kCompute) {
-            const uint32_t code = ul[e];
-            if (code != kListPad) {
-              const int i = static_cast<int>(code >> 16), cl = static_cast<int>(code & 0xffffu);
-              float* px = x + 4 * (i * QB + xq(cl >> 2)) + (cl & 3);
-              *px = fmaf(-a.upd_scale, ug[e], *px);
-            }
-          }
-        }
-        if (FUSED && KP1 < 0) ok = !compute_bar_or(!ok);   // the update is visible to the column sums
         if (ok && KP1 < 0) {
           // Complete graph: this thread's share of its column's sum.
           float4 cs = make_float4(0.f, 0.f, 0.f, 0.f);
           for (int r = 0; r < rows_t; ++r) cs = f4_add(cs, x4[(g_t + r * G) * QB + qoff]);
           part[tid] = cs;
         }
-        if (FUSED || KP1 < 0) ok = !compute_bar_or(!ok);   // uniform decision; the update / sums are visible
+        if (KP1 < 0) ok = !compute_bar_or(!ok);   // uniform decision; the column sums are visible
         if (!ok) {
           if (lane == 0) record_error(a.st, ASAP_ERR_CUDA, 0xffffffffu, a.round);
           failed = true;
@@ -510,7 +533,6 @@ __global__ void __launch_bounds__(kMixThreads, 1) k_mix(const __grid_constant__ 
               for (int m = 1; m < kp1; ++m) v = fmaf(wt[m], x[4 * (nb[m] + xo) + comp], v);
               a.wv_out[xbase + e] = v;
             }
-            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");   // generic writes before the next TMA
           }
         }
         __syncwarp();
@@ -622,8 +644,15 @@ ASAP_HD size_t mix_stage_bytes(int S, int rows_pad, int max_region) {
 }
 
 size_t mix_smem_bytes(int N, int kp1, int S, int rows_pad, int stages, int max_region) {
-  return 1024 + mix_stage_bytes(S, rows_pad, max_region) * stages + 16 * stages + ((8 * (kMixThreads / 32) + 15) & ~15) + 16 +
-         16 * stages + 16 * static_cast<size_t>(stages) * kMixComputeWarps * 32 + 8 * static_cast<size_t>(N) * kp1;
+  auto a16 = [](size_t v) { return (v + 15) & ~static_cast<size_t>(15); };
+  size_t b = 1024 + mix_stage_bytes(S, rows_pad, max_region) * stages;   // alignment slack + stages
+  b = a16(b + 24 * static_cast<size_t>(stages));                         // full / empty / ready
+  b = a16(b + 8 * (kMixThreads / 32));                                    // fp64 block scratch
+  b = a16(b + 16);                                                        // flags
+  b = a16(b + 16 * static_cast<size_t>(stages));                          // stage info
+  b = a16(b + 16 * static_cast<size_t>(stages) * kMixComputeWarps * 32);  // partial sums
+  b = a16(b + 4 * static_cast<size_t>(N) * kp1);                          // neighbour offsets
+  return b + 4 * static_cast<size_t>(N) * kp1;                            // weights
 }
 
 cudaError_t mix_configure(bool complete, bool fused, int kp1, bool shadow, size_t smem) {

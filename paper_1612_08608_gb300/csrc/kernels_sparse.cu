@@ -93,13 +93,40 @@ __global__ void __launch_bounds__(kThreads) k_margin_loss(SparseStepArgs a) {
   float acc = 0.f;
   if (b < a.B) {
     const int q0 = rp[b] >> 2, q1 = rp[b + 1] >> 2;
-    for (int q = q0 + sl; q < q1; q += kLanesPerRow) {
-      const int4 p = ld_stream_i4(pos4 + q);
-      const float4 v = ld_stream_f4(val4 + q);
-      acc = fmaf(v.x, __ldg(wv + p.x), acc);
-      acc = fmaf(v.y, __ldg(wv + p.y), acc);
-      acc = fmaf(v.z, __ldg(wv + p.z), acc);
-      acc = fmaf(v.w, __ldg(wv + p.w), acc);
+    // Four quads per lane per pass, all loads issued before the sums; the
+    // summation order is the sequential one (quad after quad).
+    constexpr int kU = 4;
+    for (int q = q0 + sl; q < q1; q += kU * kLanesPerRow) {
+      int4 p[kU];
+      float4 v[kU];
+#pragma unroll
+      for (int u = 0; u < kU; ++u) {
+        const int qq = q + u * kLanesPerRow;
+        if (qq < q1) {
+          p[u] = ld_stream_i4(pos4 + qq);
+          v[u] = ld_stream_f4(val4 + qq);
+        } else {
+          p[u] = make_int4(0, 0, 0, 0);
+          v[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+      }
+      float g[4 * kU];
+#pragma unroll
+      for (int u = 0; u < kU; ++u) {
+        g[4 * u + 0] = __ldg(wv + p[u].x);
+        g[4 * u + 1] = __ldg(wv + p[u].y);
+        g[4 * u + 2] = __ldg(wv + p[u].z);
+        g[4 * u + 3] = __ldg(wv + p[u].w);
+      }
+#pragma unroll
+      for (int u = 0; u < kU; ++u) {
+        if (q + u * kLanesPerRow < q1) {
+          acc = fmaf(v[u].x, g[4 * u + 0], acc);
+          acc = fmaf(v[u].y, g[4 * u + 1], acc);
+          acc = fmaf(v[u].z, g[4 * u + 2], acc);
+          acc = fmaf(v[u].w, g[4 * u + 3], acc);
+        }
+      }
     }
   }
 #pragma unroll
@@ -137,17 +164,32 @@ __global__ void __launch_bounds__(kThreads) k_column_sums(SparseStepArgs a) {
   const unsigned le_mask = (lane == 31) ? kFull : ((2u << lane) - 1u);
 
   const int n_chunks = (nnz + 31) >> 5;
-  for (int first = blockIdx.x * kUpdateChunksPerCta; first < n_chunks; first += gridDim.x * kUpdateChunksPerCta)
-  for (int j = warp; j < kUpdateChunksPerCta; j += kThreads / 32) {
-    const int chunk = first + j;
+  constexpr int kPerWarp = kUpdateChunksPerCta / (kThreads / 32);   // 4 chunks per warp per pass
+  for (int first = blockIdx.x * kUpdateChunksPerCta; first < n_chunks; first += gridDim.x * kUpdateChunksPerCta) {
+    // Load the warp's chunks first (independent), then scan them one by one.
+    int cv[kPerWarp], cpv[kPerWarp];
+    float pv[kPerWarp];
+#pragma unroll
+    for (int u = 0; u < kPerWarp; ++u) {
+      const int chunk = first + warp + u * (kThreads / 32);
+      const int e = chunk * 32 + lane;
+      const bool valid = chunk < n_chunks && e < nnz;
+      cv[u] = valid ? cpos[e] : -1;
+      cpv[u] = (lane == 0 && chunk < n_chunks && e > 0) ? cpos[e - 1] : -2;
+      pv[u] = valid ? cval[e] : 0.f;
+      if (valid) pv[u] *= r[crow[e]];
+    }
+#pragma unroll
+    for (int u = 0; u < kPerWarp; ++u) {
+    const int chunk = first + warp + u * (kThreads / 32);
     if (chunk >= n_chunks) break;                  // warp-uniform
     const int e = chunk * 32 + lane;
     const bool valid = e < nnz;
-    const int c = valid ? cpos[e] : -1;
+    const int c = cv[u];
     int cprev = __shfl_up_sync(kFull, c, 1);
-    if (lane == 0) cprev = (e > 0) ? cpos[e - 1] : -2;
+    if (lane == 0) cprev = cpv[u];
     const bool head = valid && (c != cprev);
-    float p = valid ? r[crow[e]] * cval[e] : 0.f;
+    float p = pv[u];
     const unsigned heads = __ballot_sync(kFull, head);
     const unsigned hl = heads & le_mask;
     const int start = hl ? (31 - __clz(hl)) : -1;   // first lane of this lane's run, -1: began earlier
@@ -180,6 +222,7 @@ __global__ void __launch_bounds__(kThreads) k_column_sums(SparseStepArgs a) {
         base += 32;
       }
       if (lane == 0) g[c31] = acc;
+    }
     }
   }
 

@@ -132,6 +132,7 @@ struct asap_ctx {
 
   CUtensorMap tmap[2];
   int S = 0, rows_pad = 0, box_rows = 0, n_boxes = 0, stages = 0;
+  int s_cap = 1024;                 // upper bound on the slab width (lowered for skewed column lists)
   bool fused_cfg = false;
   long long n_slabs = 0;
   int mix_grid = 0;
@@ -241,7 +242,7 @@ asap_status setup_mix(asap_ctx* c) {
   while (S > 8 && static_cast<size_t>(c->rows_pad) * S * 4 > 32768) S >>= 1;
   int maxS = 8;
   while (static_cast<int64_t>(maxS) * 2 <= c->ld && maxS < 1024) maxS <<= 1;
-  c->S = std::min(S, maxS);
+  c->S = std::min(std::min(S, maxS), c->s_cap);
   c->n_slabs = (c->ld + c->S - 1) / c->S;
   c->tab_kp1 = is_complete_kernel(c) ? 0 : c->k + 1;
   c->configured_key = -1;
@@ -765,8 +766,7 @@ asap_status asap_load_shards(asap_ctx* c, const int64_t* const* rowptr, const in
   if (!c || !rowptr || !col || !val || !y || !n_rows) return fail(c, ASAP_ERR_ARG, "NULL argument");
   if (c->loss != ASAP_LOSS_HINGE && c->loss != ASAP_LOSS_LOGISTIC)
     return fail(c, ASAP_ERR_ARG, "set a hinge or logistic model before loading CSR shards");
-  const int N = c->N, B = c->B, S = c->S;
-  const long long n_slabs = c->n_slabs;
+  const int N = c->N, B = c->B;
   int nb = -1;
   for (int i = 0; i < N; ++i) {
     if (!rowptr[i] || !col[i] || !val[i] || !y[i]) return fail(c, ASAP_ERR_ARG, "NULL shard pointer");
@@ -781,6 +781,12 @@ asap_status asap_load_shards(asap_ctx* c, const int64_t* const* rowptr, const in
   asap_status s0 = asap_sync(c);
   if (s0 != ASAP_OK) return s0;
   free_shards(c);
+  c->s_cap = 1024;
+  s0 = setup_mix(c);
+  if (s0 != ASAP_OK) return s0;
+  for (;;) {
+  const int S = c->S;
+  const long long n_slabs = c->n_slabs;
 
   // One block per minibatch index t: per worker the padded rows (pos, val),
   // labels and the entries sorted by (column, row); then the batch's
@@ -937,6 +943,19 @@ asap_status asap_load_shards(asap_ctx* c, const int64_t* const* rowptr, const in
   size_t total = 0;
   int max_nnz = 0, max_region = 0;
   int64_t max_list = 0;
+  for (int t = 0; t < nb; ++t)
+    if (built[t].err) return fail(c, ASAP_ERR_ARG, built[t].err);
+  for (int t = 0; t < nb; ++t) max_region = std::max(max_region, built[t].max_region);
+  // Two stages of the fused reduce (slab + three list regions each) must fit
+  // in shared memory; skewed column popularity calls for narrower slabs.
+  if (mix_smem_bytes(N, std::min(c->k + 1, kMaxKp1Sparse), S, c->rows_pad, 2, max_region) > (220u << 10)) {
+    if (S <= 8) return fail(c, ASAP_ERR_ARG, "a column slab's list does not fit in shared memory");
+    c->s_cap = S / 2;
+    asap_status sm = setup_mix(c);
+    if (sm != ASAP_OK) return sm;
+    continue;
+  }
+  max_region = 0;
   c->block_off.assign(nb, 0);
   c->block_bytes.assign(nb, 0);
   c->list_off.assign(nb, 0);
@@ -993,6 +1012,7 @@ asap_status asap_load_shards(asap_ctx* c, const int64_t* const* rowptr, const in
   c->update_ctas = update_ctas_for(max_nnz);
   c->configured_key = -1;
   return ASAP_OK;
+  }
 }
 
 asap_status asap_load_dense_shards(asap_ctx* c, const uint16_t* const* X, const int32_t* const* y,

@@ -260,6 +260,24 @@ def config(rows):
     return c
 
 
+def reduce_max(x, device="cpu"):
+    """Max of a per-rank scalar over all ranks (identity without a process
+    group).  gloo reduces CPU tensors, NCCL CUDA tensors."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return float(x)
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(world, units_per_step, steps, seconds_max):
+    """Units all ranks processed (each rank runs the same replica workload)
+    divided by the slowest rank's time."""
+    return world * units_per_step * steps / seconds_max
+
+
 def dist_env():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -336,11 +354,7 @@ def run_asap(args):
         torch.cuda.synchronize()
 
     def max_over_ranks(x):
-        if world == 1:
-            return x
-        t = torch.tensor([x], dtype=torch.float64, device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        return float(t.item())
+        return reduce_max(x, device="cuda")
 
     stream = torch.cuda.Stream()
     ctx = Context(w["N"], w["d"], graph_seed=w["graph_seed"], k=w["k"])
@@ -374,7 +388,7 @@ def run_asap(args):
             ctx.sync()
             t_e2e = max_over_ranks(time.perf_counter() - t0)
             graph_bytes = N * (w["k"] + 1) * 8 if w["regenerate"] else 0
-            e2e = {"value": world * units_per_step * K / t_e2e, "unit": "worker-samples/s",
+            e2e = {"value": whole_job_rate(world, units_per_step, K, t_e2e), "unit": "worker-samples/s",
                    "h2d_bytes_per_step": h2d / K + graph_bytes, "d2h_bytes_per_step": 8}
         ctx.set_shard_residency("device")
 
@@ -425,7 +439,7 @@ def run_asap(args):
             "peak_kind": kd["peak_kind"], "unit": kd["unit"], "frac": kd["frac"],
             "traffic": mix_traffic_per_launch() if (dom == "reduce" and w["name"] == "sparse_logistic_hashed")
             else None, "algorithmic_per_launch": kd["algorithmic_per_launch"], "mean_launch_ms": kd["mean_launch_ms"]}
-    value = world * units_per_step * K / (elapsed_ms * 1e-3)
+    value = whole_job_rate(world, units_per_step, K, elapsed_ms * 1e-3)
     line = {"metric": METRIC, "value": value, "unit": "worker-samples/s", "n_gpus": world, "steps": K,
             "warmup": Wm, "ms_per_step": elapsed_ms / K, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16 GEMM inputs, f32 accumulate and master" if dense else "f32",

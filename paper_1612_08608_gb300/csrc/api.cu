@@ -125,7 +125,7 @@ struct asap_ctx {
   uint16_t* RT = nullptr;    // [N][Cq*256][B] bf16
   int Cq = 0;
   int n_loss_part = 0;
-  CUtensorMap tmX, tmXT, tmR, tmWbf[2];
+  CUtensorMap tmX, tmXT, tmR, tmWbf[2], tmWf[2];
   bool dense_configured = false;
 
   cudaStream_t stream = nullptr, own_stream = nullptr, copy_stream = nullptr;
@@ -284,6 +284,15 @@ asap_status setup_dense_param_maps(asap_ctx* c) {
     cuuint32_t box[3] = {64, 256, 1};
     asap_status s = bf16_map(c, &c->tmWbf[b], c->Wbf[b], 3, dims, str, box);
     if (s != ASAP_OK) return s;
+    // fp32 master [N][C][d] for the gradient epilogue: boxes of 32 x 128 x 1, 128-byte swizzle.
+    EncodeTiledFn enc = get_encode_fn();
+    cuuint64_t strf[2] = {static_cast<cuuint64_t>(c->d) * 4, static_cast<cuuint64_t>(c->ld) * 4};
+    cuuint32_t boxf[3] = {32, 128, 1};
+    cuuint32_t estr[3] = {1, 1, 1};
+    CUresult rr = enc(&c->tmWf[b], CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, c->W[b], dims, strf, boxf, estr,
+                      CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                      CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (rr != CUDA_SUCCESS) return fail(c, ASAP_ERR_CUDA, "cuTensorMapEncodeTiled failed for the fp32 master");
   }
   return ASAP_OK;
 }
@@ -1126,7 +1135,7 @@ asap_status asap_local_step(asap_ctx* c) {
     CU(launch_dense_fwd(c->tmX, c->tmWbf[r & 1], f, c->N, c->stream), "launching the dense forward kernel");
     time_end(c);
     time_begin(c, ASAP_KERNEL_DENSE_GRAD);
-    CU(launch_dense_grad(c->tmR, c->tmXT, g, c->N, c->stream), "launching the dense gradient kernel");
+    CU(launch_dense_grad(c->tmR, c->tmXT, c->tmWf[r & 1], g, c->N, c->stream), "launching the dense gradient kernel");
     time_end(c);
     c->launches += 2;
     c->step_pending = true;

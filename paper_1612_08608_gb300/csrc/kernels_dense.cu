@@ -41,6 +41,12 @@ constexpr int kStages = 2;
 constexpr uint32_t kABytes = kTileM * kTileK * 2;   // 16 KB
 constexpr uint32_t kBBytes = kTileN * kTileK * 2;   // 32 KB
 constexpr uint32_t kTmemCols = 256;
+// Gradient epilogue: the fp32 master tile [128 classes x 256 features] is
+// staged in shared memory as 8 boxes of 32 columns (128-byte swizzled rows).
+constexpr int kWBoxCols = 32;
+constexpr uint32_t kWBoxBytes = kTileM * kWBoxCols * 4;          // 16 KB
+constexpr int kWBoxes = kTileN / kWBoxCols;                       // 8
+constexpr uint32_t kWTileBytes = kWBoxes * kWBoxBytes;            // 128 KB
 constexpr unsigned long long kWaitNs = 2000000000ull;
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
@@ -90,6 +96,11 @@ __device__ __forceinline__ void tma_3d(void* dst, const CUtensorMap* m, uint64_t
       "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], [%5];"
       :: "r"(smem_u32(dst)), "l"(reinterpret_cast<uint64_t>(m)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar))
       : "memory");
+}
+
+__device__ __forceinline__ void tma_store_3d(const CUtensorMap* m, const void* src, int x, int y, int z) {
+  asm volatile("cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%1, %2, %3}], [%4];"
+               :: "l"(reinterpret_cast<uint64_t>(m)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(src)) : "memory");
 }
 
 // --- tcgen05 -----------------------------------------------------------
@@ -189,6 +200,7 @@ struct GemmSmem {
   uint64_t* full;
   uint64_t* empty;
   uint64_t* accum;
+  uint64_t* wbar;       // gradient kernel: the staged master tile has landed
   uint32_t* tmem_slot;
   float* row_a;         // [128]
   float* row_b;         // [128]
@@ -196,9 +208,13 @@ struct GemmSmem {
   int* fail;
 };
 
-__device__ __forceinline__ GemmSmem carve(unsigned char* raw) {
+__device__ __forceinline__ uintptr_t align1024(const void* raw) {
+  return (reinterpret_cast<uintptr_t>(raw) + 1023) & ~static_cast<uintptr_t>(1023);
+}
+
+// Layout from a 1024-byte aligned address p.
+__device__ __forceinline__ GemmSmem carve_at(uintptr_t p) {
   GemmSmem s;
-  uintptr_t p = (reinterpret_cast<uintptr_t>(raw) + 1023) & ~static_cast<uintptr_t>(1023);
   s.a = reinterpret_cast<unsigned char*>(p);
   p += kStages * kABytes;
   s.b = reinterpret_cast<unsigned char*>(p);
@@ -206,7 +222,8 @@ __device__ __forceinline__ GemmSmem carve(unsigned char* raw) {
   s.full = reinterpret_cast<uint64_t*>(p);
   s.empty = s.full + kStages;
   s.accum = s.empty + kStages;
-  p += 8 * (2 * kStages + 1);
+  s.wbar = s.accum + 1;
+  p += 8 * (2 * kStages + 2);
   s.tmem_slot = reinterpret_cast<uint32_t*>(p);
   p += 16;
   s.row_a = reinterpret_cast<float*>(p);
@@ -218,6 +235,8 @@ __device__ __forceinline__ GemmSmem carve(unsigned char* raw) {
   s.fail = reinterpret_cast<int*>(p);
   return s;
 }
+
+__device__ __forceinline__ GemmSmem carve(unsigned char* raw) { return carve_at(align1024(raw)); }
 
 // The producer / MMA part shared by both GEMMs.  A tiles come from tmA at
 // (k, a_row), B tiles from tmB at (k, b_row[, b_z]) (3-D when b_is_3d).
@@ -278,6 +297,7 @@ __device__ __forceinline__ void setup(const GemmSmem& sm) {
       mbar_init(sm.empty + s, 1);
     }
     mbar_init(sm.accum, 1);
+    mbar_init(sm.wbar, 1);
     *sm.fail = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -380,22 +400,33 @@ __global__ void __launch_bounds__(kDenseThreads, 1)
 
 // ----------------------------------------------------------------------------
 // Gradient and update: G tile [128 classes x 256 features] = R^T X_b, then
-// W = (1 - eta l2) W - eta G on the fp32 master; the last CTA of a worker
-// publishes NOTIFY.  grid (d/256, ceil(C/128), N).
+// W = (1 - eta l2) W - eta G on the fp32 master.  The master tile is loaded
+// by TMA into shared memory at the start (overlapping the GEMM), updated
+// there and stored back by TMA; the 3-D map clips rows beyond C, so a tile
+// never touches the next worker's rows.  The last CTA of a worker publishes
+// NOTIFY.  grid (d/256, ceil(C/128), N), one CTA per SM.
 __global__ void __launch_bounds__(kDenseThreads, 1)
-    k_dense_grad(const __grid_constant__ CUtensorMap tmR, const __grid_constant__ CUtensorMap tmXT, DenseGradArgs a) {
+    k_dense_grad(const __grid_constant__ CUtensorMap tmR, const __grid_constant__ CUtensorMap tmXT,
+                 const __grid_constant__ CUtensorMap tmWf, DenseGradArgs a) {
   extern __shared__ unsigned char smem_raw[];
-  const GemmSmem sm = carve(smem_raw);
+  unsigned char* wtile = reinterpret_cast<unsigned char*>(align1024(smem_raw));
+  const GemmSmem sm = carve_at(reinterpret_cast<uintptr_t>(wtile) + kWTileBytes);
   const int nt = blockIdx.x, mt = blockIdx.y, i = blockIdx.z;
   const int warp = threadIdx.x >> 5;
   setup(sm);
   const uint32_t tmem = *sm.tmem_slot;
 
+  if (threadIdx.x == 0) {
+    mbar_expect_tx(sm.wbar, kWTileBytes);
+    for (int b = 0; b < kWBoxes; ++b)
+      tma_3d(wtile + b * kWBoxBytes, &tmWf, sm.wbar, nt * kTileN + b * kWBoxCols, mt * kTileM, i);
+  }
   const int a_row = i * a.Cq * kTileN + mt * kTileM;             // row of R^T
   const int b_row = (i * a.nb + a.t) * a.d + nt * kTileN;        // row of X^T
   gemm_mainloop(sm, &tmR, &tmXT, false, a_row, b_row, 0, a.B / kTileK, tmem, a.st, i, a.round);
 
-  const bool ok = __all_sync(0xffffffffu, mbar_wait(sm.accum, 0));
+  bool ok = __all_sync(0xffffffffu, mbar_wait(sm.accum, 0));
+  ok = __all_sync(0xffffffffu, ok && mbar_wait(sm.wbar, 0));
   if (!ok) {
     record_error(a.st, ASAP_ERR_CUDA, i, a.round);
     atomicOr(sm.fail, 1);
@@ -403,29 +434,37 @@ __global__ void __launch_bounds__(kDenseThreads, 1)
   __syncwarp();
   tc_fence_after();
   const uint32_t trow = tmem + (static_cast<uint32_t>(warp * 32) << 16);
-  const int c = mt * kTileM + threadIdx.x;                       // class row
+  const int r = threadIdx.x;                                     // row of the tile (class mt*128 + r)
   float g[32];
-  float* w = a.W + static_cast<int64_t>(i) * a.ld + static_cast<int64_t>(c) * a.d + nt * kTileN;
-  for (int ch = 0; ch < kTileN / 32; ++ch) {
-    if (ok) tmem_ld32(trow + ch * 32, g);
-    if (ok && c < a.C) {
-      float4* w4 = reinterpret_cast<float4*>(w + ch * 32);
+  if (ok) {
+    for (int ch = 0; ch < kWBoxes; ++ch) {
+      tmem_ld32(trow + ch * 32, g);
+      unsigned char* row = wtile + ch * kWBoxBytes + r * 128;
 #pragma unroll
       for (int j = 0; j < 8; ++j) {
-        float4 x = w4[j];
+        float4* p = reinterpret_cast<float4*>(row + ((j ^ (r & 7)) << 4));   // 128-byte swizzle
+        float4 x = *p;
         x.x = fmaf(-a.lr, g[4 * j + 0], a.decay * x.x);
         x.y = fmaf(-a.lr, g[4 * j + 1], a.decay * x.y);
         x.z = fmaf(-a.lr, g[4 * j + 2], a.decay * x.z);
         x.w = fmaf(-a.lr, g[4 * j + 3], a.decay * x.w);
-        w4[j] = x;
+        *p = x;
       }
     }
   }
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");   // the updated tile is visible to TMA
+  __syncthreads();
+  if (threadIdx.x == 0 && !*sm.fail) {
+    for (int b = 0; b < kWBoxes; ++b)
+      tma_store_3d(&tmWf, wtile + b * kWBoxBytes, nt * kTileN + b * kWBoxCols, mt * kTileM, i);
+    asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+    asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");       // written to global memory
+    asm volatile("fence.proxy.async.global;" ::: "memory");
+  }
   teardown(sm, tmem);
   // NOTIFY once every tile of worker i is written.
-  __threadfence();
-  __syncthreads();
   if (threadIdx.x == 0) {
+    __threadfence();
     const unsigned total = gridDim.x * gridDim.y;
     const unsigned done = atomicAdd(&a.worker_ticket[i], 1u);
     if (done == total - 1) {
@@ -440,8 +479,10 @@ __global__ void __launch_bounds__(kDenseThreads, 1)
 }  // namespace
 
 size_t dense_smem_bytes() {
-  return 1024 + kStages * (kABytes + kBBytes) + 8 * (2 * kStages + 1) + 16 + 8 * kTileM + 16 + 16;
+  return 1024 + kStages * (kABytes + kBBytes) + 8 * (2 * kStages + 2) + 16 + 8 * kTileM + 16 + 16;
 }
+
+size_t dense_grad_smem_bytes() { return dense_smem_bytes() + kWTileBytes; }
 
 cudaError_t dense_configure() {
   const int smem = static_cast<int>(dense_smem_bytes());
@@ -449,7 +490,8 @@ cudaError_t dense_configure() {
   if (e != cudaSuccess) return e;
   e = cudaFuncSetAttribute(k_dense_fwd, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   if (e != cudaSuccess) return e;
-  return cudaFuncSetAttribute(k_dense_grad, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  return cudaFuncSetAttribute(k_dense_grad, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              static_cast<int>(dense_grad_smem_bytes()));
 }
 
 cudaError_t launch_dense_fwd(const CUtensorMap& tmX, const CUtensorMap& tmW, const DenseFwdArgs& f, int N,
@@ -469,10 +511,10 @@ cudaError_t launch_dense_fwd(const CUtensorMap& tmX, const CUtensorMap& tmW, con
   return cudaLaunchKernelEx(&cfg, k_dense_fwd, tmX, tmW, f);
 }
 
-cudaError_t launch_dense_grad(const CUtensorMap& tmR, const CUtensorMap& tmXT, const DenseGradArgs& g, int N,
-                              cudaStream_t s) {
+cudaError_t launch_dense_grad(const CUtensorMap& tmR, const CUtensorMap& tmXT, const CUtensorMap& tmWf,
+                              const DenseGradArgs& g, int N, cudaStream_t s) {
   const dim3 g2(g.d / kTileN, (g.C + kTileM - 1) / kTileM, N);
-  k_dense_grad<<<g2, kDenseThreads, dense_smem_bytes(), s>>>(tmR, tmXT, g);
+  k_dense_grad<<<g2, kDenseThreads, dense_grad_smem_bytes(), s>>>(tmR, tmXT, tmWf, g);
   return cudaGetLastError();
 }
 

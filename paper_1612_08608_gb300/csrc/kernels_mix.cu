@@ -124,6 +124,18 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, u
       : "memory");
 }
 
+// The next round's w values (a few MB) should stay in L2 for the margin
+// kernel's gathers.
+__device__ __forceinline__ uint64_t evict_last_policy() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+
+__device__ __forceinline__ void st_f32_hint(float* p, float v, uint64_t policy) {
+  asm volatile("st.global.L2::cache_hint.f32 [%0], %1, %2;" :: "l"(p), "f"(v), "l"(policy) : "memory");
+}
+
 __device__ __forceinline__ void st_f4_hint(float* p, float4 v, uint64_t policy) {
   asm volatile("st.global.L2::cache_hint.v4.f32 [%0], {%1, %2, %3, %4}, %5;"
                :: "l"(p), "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w), "l"(policy) : "memory");
@@ -258,6 +270,9 @@ __global__ void __launch_bounds__(kMixThreads, 1) k_mix(const __grid_constant__ 
 
   if (tid == 0) { sm.flags[0] = 0; sm.flags[1] = 0; }
   __syncthreads();
+  // Programmatic dependent launch: the local step's kernels may still be
+  // running; everything below reads what they wrote.
+  asm volatile("griddepcontrol.wait;" ::: "memory");
 
   // ---- NOTIFY / ACK checks (time-limited waits) ----
   for (int j = tid; j < a.N; j += kMixThreads) {
@@ -412,6 +427,7 @@ __global__ void __launch_bounds__(kMixThreads, 1) k_mix(const __grid_constant__ 
       // Thread t owns column quad q = t mod nq of every slab for the rows
       // i = g, g + G, ... (g = t / nq): with ~32 KB slabs that is 4 rows.
       const int q_t = tid & (nq - 1), g_t = tid >> lq;
+      const uint64_t keep = evict_last_policy();
       const int qoff = (q_t / QB) * a.rows_pad * QB + (q_t % QB);   // float4 offset of (row 0, quad q_t)
       const int rows_t = (a.N - g_t + G - 1) / G;
       auto xq = [&](int q) { return (q / QB) * a.rows_pad * QB + (q % QB); };
@@ -531,7 +547,7 @@ __global__ void __launch_bounds__(kMixThreads, 1) k_mix(const __grid_constant__ 
               const int xo = xq(cl >> 2), comp = cl & 3;
               float v = wt[0] * x[4 * (nb[0] + xo) + comp];
               for (int m = 1; m < kp1; ++m) v = fmaf(wt[m], x[4 * (nb[m] + xo) + comp], v);
-              a.wv_out[xbase + e] = v;
+              st_f32_hint(a.wv_out + xbase + e, v, keep);
             }
           }
         }
@@ -596,8 +612,18 @@ struct MixKernel {
     return cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks, k_mix<KP1, SHADOW, FUSED>, kMixThreads, smem);
   }
   static cudaError_t launch(const CUtensorMap& tmap, const MixArgs& a, int grid, size_t smem, cudaStream_t s) {
-    k_mix<KP1, SHADOW, FUSED><<<grid, kMixThreads, smem, s>>>(tmap, a);
-    return cudaGetLastError();
+    // A programmatic dependent of the local step's last kernel.
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(kMixThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, k_mix<KP1, SHADOW, FUSED>, tmap, a);
   }
 };
 

@@ -57,6 +57,19 @@ __device__ __forceinline__ float4 ld_stream_f4(const float4* p) {
   return v;
 }
 
+// Gather of an exported w value, keeping the line in L2 (it is re-read by
+// other rows of the minibatch).
+__device__ __forceinline__ float ld_keep(const float* p, uint64_t policy) {
+  float v;
+  asm volatile("ld.global.nc.L2::cache_hint.f32 %0, [%1], %2;" : "=f"(v) : "l"(p), "l"(policy));
+  return v;
+}
+
+// Programmatic dependent launch: the next kernel in the stream may start its
+// CTAs now; this kernel waits here for the previous kernel's results.
+__device__ __forceinline__ void allow_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void wait_previous() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 __device__ __forceinline__ void st_release_u32(unsigned int* p, unsigned int v) {
   asm volatile("st.release.gpu.global.u32 [%0], %1;" :: "l"(p), "r"(v) : "memory");
 }
@@ -85,7 +98,10 @@ __global__ void __launch_bounds__(kThreads) k_margin_loss(SparseStepArgs a) {
   const float* y = reinterpret_cast<const float*>(a.block + dsc.y);
   const int4* pos4 = reinterpret_cast<const int4*>(a.block + dsc.posw);
   const float4* val4 = reinterpret_cast<const float4*>(a.block + dsc.val);
+  allow_dependents();
   const float* wv = a.wv;
+  uint64_t keep;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(keep));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int sub = lane / kLanesPerRow, sl = lane % kLanesPerRow;
   const int b = blockIdx.x * kMarginRowsPerCta + warp * (32 / kLanesPerRow) + sub;   // 8 warps x 4 rows
@@ -113,10 +129,10 @@ __global__ void __launch_bounds__(kThreads) k_margin_loss(SparseStepArgs a) {
       float g[4 * kU];
 #pragma unroll
       for (int u = 0; u < kU; ++u) {
-        g[4 * u + 0] = __ldg(wv + p[u].x);
-        g[4 * u + 1] = __ldg(wv + p[u].y);
-        g[4 * u + 2] = __ldg(wv + p[u].z);
-        g[4 * u + 3] = __ldg(wv + p[u].w);
+        g[4 * u + 0] = ld_keep(wv + p[u].x, keep);
+        g[4 * u + 1] = ld_keep(wv + p[u].y, keep);
+        g[4 * u + 2] = ld_keep(wv + p[u].z, keep);
+        g[4 * u + 3] = ld_keep(wv + p[u].w, keep);
       }
 #pragma unroll
       for (int u = 0; u < kU; ++u) {
@@ -152,6 +168,7 @@ __global__ void __launch_bounds__(kThreads) k_margin_loss(SparseStepArgs a) {
 }
 
 __global__ void __launch_bounds__(kThreads) k_column_sums(SparseStepArgs a) {
+  allow_dependents();
   const int i = blockIdx.y;
   const BatchDesc dsc = a.desc[i];
   const int nnz = dsc.nnz;
@@ -167,7 +184,7 @@ __global__ void __launch_bounds__(kThreads) k_column_sums(SparseStepArgs a) {
   constexpr int kPerWarp = kUpdateChunksPerCta / (kThreads / 32);   // 4 chunks per warp per pass
   for (int first = blockIdx.x * kUpdateChunksPerCta; first < n_chunks; first += gridDim.x * kUpdateChunksPerCta) {
     // Load the warp's chunks first (independent), then scan them one by one.
-    int cv[kPerWarp], cpv[kPerWarp];
+    int cv[kPerWarp], cpv[kPerWarp], rw[kPerWarp];
     float pv[kPerWarp];
 #pragma unroll
     for (int u = 0; u < kPerWarp; ++u) {
@@ -177,8 +194,12 @@ __global__ void __launch_bounds__(kThreads) k_column_sums(SparseStepArgs a) {
       cv[u] = valid ? cpos[e] : -1;
       cpv[u] = (lane == 0 && chunk < n_chunks && e > 0) ? cpos[e - 1] : -2;
       pv[u] = valid ? cval[e] : 0.f;
-      if (valid) pv[u] *= r[crow[e]];
+      rw[u] = valid ? crow[e] : -1;
     }
+    wait_previous();   // r comes from the margin kernel
+#pragma unroll
+    for (int u = 0; u < kPerWarp; ++u)
+      if (rw[u] >= 0) pv[u] *= r[rw[u]];
 #pragma unroll
     for (int u = 0; u < kPerWarp; ++u) {
     const int chunk = first + warp + u * (kThreads / 32);
@@ -270,9 +291,17 @@ cudaError_t launch_margin(const SparseStepArgs& a, int N, int loss, int margin_c
 }
 
 cudaError_t launch_update(const SparseStepArgs& a, int N, int update_ctas, cudaStream_t s) {
-  const dim3 g2(update_ctas, N);
-  k_column_sums<<<g2, kThreads, 0, s>>>(a);
-  return cudaGetLastError();
+  // Launched as a programmatic dependent of the margin kernel.
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(update_ctas, N);
+  cfg.blockDim = dim3(kThreads);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, k_column_sums, a);
 }
 
 cudaError_t launch_gather_wv(const float* W, int64_t ld, const uint32_t* list, const int* slab_off, long long n_slabs,

@@ -263,6 +263,8 @@ __global__ void __launch_bounds__(kMixThreads, 1) k_mix(const __grid_constant__ 
   const int S = a.S, nq = S >> 2;            // column quads per slab, a power of two <= 256
   const int lq = __ffs(nq) - 1;
   const int QB = nq < 64 ? nq : 64;           // quads per TMA box row (a box spans <= 256 columns)
+  const int lqb = __ffs(QB) - 1;
+  const int box_col = a.rows_pad << lqb;      // float4s per column box of a slab
   const int G = kCompute >> lq;               // row groups: compute threads that share a column quad
   const size_t slab_floats = static_cast<size_t>(a.rows_pad) * S;
   const size_t list_off = (slab_floats * 4 + 15) & ~static_cast<size_t>(15);
@@ -408,14 +410,29 @@ __global__ void __launch_bounds__(kMixThreads, 1) k_mix(const __grid_constant__ 
           const uint32_t* ul = reinterpret_cast<const uint32_t*>(bj + list_off);
           const float* ug = reinterpret_cast<const float*>(bj + list_off + list_bytes);
           const int n_upd = sm.info[4 * st];
-          for (int e = ut; e < n_upd; e += kMixUpdaterWarps * 32) {
-            const uint32_t code = ul[e];
-            if (code != kListPad) {
-              const int i = static_cast<int>(code >> 16), cl = static_cast<int>(code & 0xffffu);
-              const int q = cl >> 2;
-              float* px = xj + 4 * (i * QB + (q / QB) * a.rows_pad * QB + (q % QB)) + (cl & 3);
-              *px = fmaf(-a.upd_scale, ug[e], *px);
+          // Four entries per thread in flight: the (worker, column) pairs of
+          // one list are distinct, so the four read-modify-writes never alias.
+          constexpr int kUpd = kMixUpdaterWarps * 32, kU = 4;
+          for (int e0 = ut; e0 < n_upd; e0 += kU * kUpd) {
+            uint32_t code[kU];
+            float gv[kU], wv[kU] = {};
+            int off[kU];
+#pragma unroll
+            for (int u = 0; u < kU; ++u) {
+              const int e = e0 + u * kUpd;
+              code[u] = e < n_upd ? ul[e] : kListPad;
+              gv[u] = e < n_upd ? ug[e] : 0.f;
             }
+#pragma unroll
+            for (int u = 0; u < kU; ++u) {
+              const int i = static_cast<int>(code[u] >> 16), cl = static_cast<int>(code[u] & 0xffffu);
+              const int q = cl >> 2;
+              off[u] = 4 * ((i << lqb) + (q >> lqb) * box_col + (q & (QB - 1))) + (cl & 3);
+              if (code[u] != kListPad) wv[u] = xj[off[u]];
+            }
+#pragma unroll
+            for (int u = 0; u < kU; ++u)
+              if (code[u] != kListPad) xj[off[u]] = fmaf(-a.upd_scale, gv[u], wv[u]);
           }
           asm volatile("fence.proxy.async.shared::cta;" ::: "memory");   // before this stage's next TMA
           __syncwarp();
@@ -428,9 +445,9 @@ __global__ void __launch_bounds__(kMixThreads, 1) k_mix(const __grid_constant__ 
       // i = g, g + G, ... (g = t / nq): with ~32 KB slabs that is 4 rows.
       const int q_t = tid & (nq - 1), g_t = tid >> lq;
       const uint64_t keep = evict_last_policy();
-      const int qoff = (q_t / QB) * a.rows_pad * QB + (q_t % QB);   // float4 offset of (row 0, quad q_t)
+      const int qoff = (q_t >> lqb) * box_col + (q_t & (QB - 1));   // float4 offset of (row 0, quad q_t)
       const int rows_t = (a.N - g_t + G - 1) / G;
-      auto xq = [&](int q) { return (q / QB) * a.rows_pad * QB + (q % QB); };
+      auto xq = [&](int q) { return (q >> lqb) * box_col + (q & (QB - 1)); };
       for (long long it = 0; it < n_my; ++it) {
         const long long slab = blockIdx.x + it * stride;
         const int st = static_cast<int>(it % a.stages);

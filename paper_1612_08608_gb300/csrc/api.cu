@@ -304,10 +304,14 @@ asap_status configure_mix_launch(asap_ctx* c, bool fused) {
   const long long key = (complete ? 1 : 0) | (shadow ? 2 : 0) | (fused ? 4 : 0) |
                         (static_cast<long long>(c->tab_kp1) << 3) | (static_cast<long long>(region) << 12);
   if (key == c->configured_key) return ASAP_OK;
-  // Stages: as many as fit in shared memory (the whole footprint, per-stage
-  // partial sums included), 2 to 8.
+  // Stages of ~32 KB slabs: three keep enough bytes in flight per SM to
+  // stream at full rate; more only queue in the memory system (on GB300 the
+  // reduce alone and the dense reduce run 3-10 % faster with 3 than with 5).
+  // The fused reduce holds each slab longer (the update precedes the mix)
+  // and wants one more.  Fewer when the footprint does not fit.
+  const int want = fused ? 4 : 3;
   c->stages = 2;
-  for (int st = 8; st > 2; --st)
+  for (int st = want; st > 2; --st)
     if (mix_smem_bytes(c->N, c->tab_kp1, c->S, c->rows_pad, st, region) <= (220u << 10)) {
       c->stages = st;
       break;

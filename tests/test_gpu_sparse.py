@@ -89,6 +89,18 @@ def test_l2_regularised_logistic():
     _run_parity(ctx, sh, T, B, "logistic", lr, sched, l2=l2)
 
 
+@pytest.mark.parametrize("B", [12288, 12289])
+def test_large_minibatch(B):
+    # Minibatches of more than 12,000 rows: many margin and column-sum CTAs
+    # per worker, and column runs (the hot column is in every row) that span
+    # hundreds of 32-entry chunks.
+    N, d, lr, T = 3, 2000, 0.2, 2
+    sh = inputs.sparse_custom(seed=12, N=N, d=d, rows=2 * B, max_len=12, hot_col=5)
+    sched = rounds.graph_schedule("ring", N, 1)
+    ctx = _ctx(N, d, 1, 0, "ring", False, "hinge", B, lr, sh)
+    _run_parity(ctx, sh, T, B, "hinge", lr, sched)
+
+
 def test_single_worker_and_complete_graph():
     sh = inputs.sparse_custom(seed=6, N=1, d=200, rows=64, max_len=20)
     ctx = _ctx(1, 200, 0, 0, "identity", False, "hinge", 16, 0.2, sh)

@@ -1139,7 +1139,8 @@ asap_status asap_local_step(asap_ctx* c) {
     CU(launch_dense_fwd(c->tmX, c->tmWbf[r & 1], f, c->N, c->stream), "launching the dense forward kernel");
     time_end(c);
     time_begin(c, ASAP_KERNEL_DENSE_GRAD);
-    CU(launch_dense_grad(c->tmR, c->tmXT, c->tmWf[r & 1], g, c->N, c->stream), "launching the dense gradient kernel");
+    CU(launch_dense_grad(c->tmR, c->tmXT, c->tmWf[r & 1], g, c->N, c->sm_count, c->stream),
+       "launching the dense gradient kernel");
     time_end(c);
     c->launches += 2;
     c->step_pending = true;

@@ -126,6 +126,7 @@ struct DenseFwdArgs {
 
 struct DenseGradArgs {
   int C, Cq, d, B, nb, t;
+  int N;                       // workers (set by the launcher)
   float* W;                    // fp32 master [N][ld], worker row = C x d class-major
   int64_t ld;
   float lr;
@@ -160,7 +161,7 @@ cudaError_t dense_configure();
 cudaError_t launch_dense_fwd(const CUtensorMap& tmX, const CUtensorMap& tmW, const DenseFwdArgs& f, int N,
                              cudaStream_t s);
 cudaError_t launch_dense_grad(const CUtensorMap& tmR, const CUtensorMap& tmXT, const CUtensorMap& tmWf,
-                              const DenseGradArgs& g, int N, cudaStream_t s);
+                              const DenseGradArgs& g, int N, int sm_count, cudaStream_t s);
 cudaError_t launch_cast_bf16(const float* src, uint16_t* dst, int64_t n, cudaStream_t s);
 
 }  // namespace asap

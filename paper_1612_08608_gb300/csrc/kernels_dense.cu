@@ -6,12 +6,13 @@
 //   gradient G = R^T X_b           [C x d], fp32 accumulate
 //            W_half = (1 - eta l2) W - eta G    (fp32 master, in place), then NOTIFY
 //
-// Both GEMMs: one CTA per 128 x 256 output tile, 4 warps.  Warp 0 lane 0
-// issues TMA loads (128-byte swizzled, K-major tiles of 64 bf16) into a ring
-// of stages guarded by full/empty mbarriers; warp 1 lane 0 issues
-// tcgen05.mma (M=128, N=256, K=16, bf16 x bf16 -> fp32 in TMEM) and commits
-// each stage back to its empty barrier; all four warps then read the
-// accumulator out of TMEM (warp w owns TMEM lanes 32w..32w+31, i.e. rows).
+// Both GEMMs use 128 x 256 output tiles.  One lane issues TMA loads
+// (128-byte swizzled, K-major tiles of 64 bf16) into a ring of stages guarded
+// by full/empty mbarriers; another issues tcgen05.mma (M=128, N=256, K=16,
+// bf16 x bf16 -> fp32 in TMEM) and commits each stage back to its empty
+// barrier; four warps read the accumulator out of TMEM (a warp reaches the
+// TMEM lanes 32 (w mod 4) .. + 31, i.e. tile rows).  The forward kernel is one
+// CTA per tile (4 warps); the gradient kernel is persistent (below).
 //
 // Softmax needs all C logits of a row, more than one CTA's 256 TMEM
 // columns: the forward kernel runs as a cluster of ceil(C/256) CTAs along
@@ -41,19 +42,17 @@ constexpr int kTileK = 64;                  // one 128-byte swizzle row of bf16
 // share an SM (2 x 100 KB of shared memory, 2 x 256 TMEM columns), so one's
 // softmax epilogue overlaps the other's main loop: on GB300 that beats one
 // CTA with a 4-stage ring (109 us against 152 us at N=32, d=2048, C=1000).
-// The gradient kernel also holds the 128 KB master tile: one CTA per SM.
+// The persistent gradient kernel overlaps its epilogue itself (one CTA per SM).
 constexpr int kFwdStages = 2;
 constexpr int kFwdCtasPerSm = 2;
-constexpr int kGradStages = 2;
+constexpr int kGradStages = 3;
 constexpr uint32_t kABytes = kTileM * kTileK * 2;   // 16 KB
 constexpr uint32_t kBBytes = kTileN * kTileK * 2;   // 32 KB
 constexpr uint32_t kTmemCols = 256;
-// Gradient epilogue: the fp32 master tile [128 classes x 256 features] is
-// staged in shared memory as 8 boxes of 32 columns (128-byte swizzled rows).
+// Gradient epilogue: the fp32 master tile [128 classes x 256 features] passes
+// through shared memory as 8 chunks of 32 columns (128-byte swizzled rows).
 constexpr int kWBoxCols = 32;
 constexpr uint32_t kWBoxBytes = kTileM * kWBoxCols * 4;          // 16 KB
-constexpr int kWBoxes = kTileN / kWBoxCols;                       // 8
-constexpr uint32_t kWTileBytes = kWBoxes * kWBoxBytes;            // 128 KB
 constexpr unsigned long long kWaitNs = 2000000000ull;
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
@@ -207,7 +206,6 @@ struct GemmSmem {
   uint64_t* full;
   uint64_t* empty;
   uint64_t* accum;
-  uint64_t* wbar;       // gradient kernel: the staged master tile has landed
   uint32_t* tmem_slot;
   float* row_a;         // [128]
   float* row_b;         // [128]
@@ -230,7 +228,6 @@ __device__ __forceinline__ GemmSmem carve_at(uintptr_t p) {
   s.full = reinterpret_cast<uint64_t*>(p);
   s.empty = s.full + ST;
   s.accum = s.empty + ST;
-  s.wbar = s.accum + 1;
   p += 8 * (2 * ST + 2);
   s.tmem_slot = reinterpret_cast<uint32_t*>(p);
   p += 16;
@@ -313,7 +310,6 @@ __device__ __forceinline__ void setup(const GemmSmem& sm) {
       mbar_init(sm.empty + s, 1);
     }
     mbar_init(sm.accum, 1);
-    mbar_init(sm.wbar, 1);
     *sm.fail = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -416,87 +412,282 @@ __global__ void __launch_bounds__(kDenseThreads, kFwdCtasPerSm)
 
 // ----------------------------------------------------------------------------
 // Gradient and update: G tile [128 classes x 256 features] = R^T X_b, then
-// W = (1 - eta l2) W - eta G on the fp32 master.  The master tile is loaded
-// by TMA into shared memory at the start (overlapping the GEMM), updated
-// there and stored back by TMA; the 3-D map clips rows beyond C, so a tile
-// never touches the next worker's rows.  The last CTA of a worker publishes
-// NOTIFY.  grid (d/256, ceil(C/128), N), one CTA per SM.
-__global__ void __launch_bounds__(kDenseThreads, 1)
+// W = (1 - eta l2) W - eta G on the fp32 master.
+//
+// Persistent and warp-specialised, one CTA per SM walking tiles
+// blockIdx.x, blockIdx.x + gridDim.x, ...:
+//   warp 0      TMA producer of the operand ring (R^T and X^T k-tiles);
+//   warp 1      tcgen05.mma issuer into one of two TMEM accumulators
+//               (2 x 256 columns), so tile n+1's GEMM runs while tile n's
+//               epilogue drains the other;
+//   warps 2-5   epilogue: the master tile is streamed through shared memory
+//               in 16 KB chunks of 128 rows x 32 columns (TMA load, update
+//               in place, TMA store), several chunk loads in flight.
+// The 3-D master map clips rows beyond C, so a tile never touches the next
+// worker's rows.  A worker's NOTIFY is published by the CTA that completes
+// its last tile, once that tile's stores are complete (checked one tile
+// later, so that waiting for store completion never stalls the epilogue).
+constexpr int kGradThreads = 192;
+constexpr int kEpi0 = 2;                                  // first epilogue warp
+constexpr int kWBufs = 5;                                 // master chunks in shared memory
+constexpr int kChunksPerTile = kTileN / kWBoxCols;        // 8
+constexpr uint32_t kGradTmemCols = 2 * kTmemCols;        // two accumulators
+
+struct GradSmem {
+  unsigned char* a;      // kGradStages x kABytes
+  unsigned char* b;      // kGradStages x kBBytes
+  unsigned char* w;      // kWBufs x kWBoxBytes
+  uint64_t* full;        // [kGradStages]
+  uint64_t* empty;       // [kGradStages]
+  uint64_t* acc_full;    // [2]
+  uint64_t* acc_empty;   // [2]
+  uint64_t* wfull;       // [kWBufs]
+  uint32_t* tmem_slot;
+  int* fail;
+};
+
+constexpr size_t grad_smem_bytes() {
+  return 1024 + static_cast<size_t>(kGradStages) * (kABytes + kBBytes) + static_cast<size_t>(kWBufs) * kWBoxBytes +
+         8 * (2 * kGradStages + 4 + kWBufs) + 16 + 16;
+}
+
+__device__ __forceinline__ GradSmem grad_carve(unsigned char* raw) {
+  uintptr_t p = align1024(raw);
+  GradSmem s;
+  s.a = reinterpret_cast<unsigned char*>(p);
+  p += kGradStages * kABytes;
+  s.b = reinterpret_cast<unsigned char*>(p);
+  p += kGradStages * kBBytes;
+  s.w = reinterpret_cast<unsigned char*>(p);
+  p += kWBufs * kWBoxBytes;
+  s.full = reinterpret_cast<uint64_t*>(p);
+  s.empty = s.full + kGradStages;
+  s.acc_full = s.empty + kGradStages;
+  s.acc_empty = s.acc_full + 2;
+  s.wfull = s.acc_empty + 2;
+  p += 8 * (2 * kGradStages + 4 + kWBufs);
+  s.tmem_slot = reinterpret_cast<uint32_t*>(p);
+  p += 16;
+  s.fail = reinterpret_cast<int*>(p);
+  return s;
+}
+
+// Barrier among the four epilogue warps that also returns the OR of `v`.
+__device__ __forceinline__ bool epi_bar_or(bool v) {
+  uint32_t r;
+  asm volatile(
+      "{\n .reg .pred p, q;\n setp.ne.u32 p, %1, 0;\n bar.red.or.pred q, 1, 128, p;\n selp.u32 %0, 1, 0, q;\n}"
+      : "=r"(r) : "r"(static_cast<uint32_t>(v)) : "memory");
+  return r != 0;
+}
+
+__device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
+
+struct GradTile {
+  int i, mt, nt;
+};
+
+__device__ __forceinline__ GradTile grad_tile(long long tau, int MT, int NT) {
+  GradTile t;
+  const long long per = static_cast<long long>(MT) * NT;
+  t.i = static_cast<int>(tau / per);
+  const int rem = static_cast<int>(tau - static_cast<long long>(t.i) * per);
+  t.mt = rem / NT;
+  t.nt = rem - t.mt * NT;
+  return t;
+}
+
+__global__ void __launch_bounds__(kGradThreads, 1)
     k_dense_grad(const __grid_constant__ CUtensorMap tmR, const __grid_constant__ CUtensorMap tmXT,
                  const __grid_constant__ CUtensorMap tmWf, DenseGradArgs a) {
   extern __shared__ unsigned char smem_raw[];
-  unsigned char* wtile = reinterpret_cast<unsigned char*>(align1024(smem_raw));
-  const GemmSmem sm = carve_at<kGradStages>(reinterpret_cast<uintptr_t>(wtile) + kWTileBytes);
-  const int nt = blockIdx.x, mt = blockIdx.y, i = blockIdx.z;
-  const int warp = threadIdx.x >> 5;
-  setup<kGradStages>(sm);
+  const GradSmem sm = grad_carve(smem_raw);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int MT = (a.C + kTileM - 1) / kTileM, NT = a.d / kTileN;
+  const long long total = static_cast<long long>(a.N) * MT * NT;
+  const int n_tiles = total > blockIdx.x ? static_cast<int>((total - blockIdx.x + gridDim.x - 1) / gridDim.x) : 0;
+  const int k_tiles = a.B / kTileK;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kGradStages; ++s) {
+      mbar_init(sm.full + s, 1);
+      mbar_init(sm.empty + s, 1);
+    }
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(sm.acc_full + s, 1);
+      mbar_init(sm.acc_empty + s, 4);   // one arrival per epilogue warp
+    }
+    for (int s = 0; s < kWBufs; ++s) mbar_init(sm.wfull + s, 1);
+    *sm.fail = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) tmem_alloc(sm.tmem_slot, kGradTmemCols);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
   const uint32_t tmem = *sm.tmem_slot;
 
-  if (threadIdx.x == 0) {
-    mbar_expect_tx(sm.wbar, kWTileBytes);
-    for (int b = 0; b < kWBoxes; ++b)
-      tma_3d(wtile + b * kWBoxBytes, &tmWf, sm.wbar, nt * kTileN + b * kWBoxCols, mt * kTileM, i);
-  }
-  const int a_row = i * a.Cq * kTileN + mt * kTileM;             // row of R^T
-  const int b_row = (i * a.nb + a.t) * a.d + nt * kTileN;        // row of X^T
-  gemm_mainloop<kGradStages>(sm, &tmR, &tmXT, false, a_row, b_row, 0, a.B / kTileK, tmem, a.st, i, a.round);
-
-  bool ok = __all_sync(0xffffffffu, mbar_wait(sm.accum, 0));
-  ok = __all_sync(0xffffffffu, ok && mbar_wait(sm.wbar, 0));
-  if (!ok) {
-    record_error(a.st, ASAP_ERR_CUDA, i, a.round);
-    atomicOr(sm.fail, 1);
-  }
-  __syncwarp();
-  tc_fence_after();
-  const uint32_t trow = tmem + (static_cast<uint32_t>(warp * 32) << 16);
-  const int r = threadIdx.x;                                     // row of the tile (class mt*128 + r)
-  float g[32];
-  if (ok) {
-    for (int ch = 0; ch < kWBoxes; ++ch) {
-      tmem_ld32(trow + ch * 32, g);
-      unsigned char* row = wtile + ch * kWBoxBytes + r * 128;
-#pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        float4* p = reinterpret_cast<float4*>(row + ((j ^ (r & 7)) << 4));   // 128-byte swizzle
-        float4 x = *p;
-        x.x = fmaf(-a.lr, g[4 * j + 0], a.decay * x.x);
-        x.y = fmaf(-a.lr, g[4 * j + 1], a.decay * x.y);
-        x.z = fmaf(-a.lr, g[4 * j + 2], a.decay * x.z);
-        x.w = fmaf(-a.lr, g[4 * j + 3], a.decay * x.w);
-        *p = x;
+  if (warp == 0) {
+    // ---------------- TMA producer ----------------
+    if (lane == 0) {
+      long long g = 0;   // k-tile counter over all of this CTA's tiles
+      bool ok = true;
+      for (int n = 0; n < n_tiles && ok; ++n) {
+        const GradTile t = grad_tile(blockIdx.x + static_cast<long long>(n) * gridDim.x, MT, NT);
+        const int a_row = t.i * a.Cq * kTileN + t.mt * kTileM;          // row of R^T
+        const int b_row = (t.i * a.nb + a.t) * a.d + t.nt * kTileN;     // row of X^T
+        for (int kt = 0; kt < k_tiles; ++kt, ++g) {
+          const int s = static_cast<int>(g % kGradStages);
+          if (g >= kGradStages && !mbar_wait(sm.empty + s, static_cast<uint32_t>(((g / kGradStages) - 1) & 1))) {
+            record_error(a.st, ASAP_ERR_CUDA, t.i, a.round);
+            atomicOr(sm.fail, 1);
+            ok = false;
+            break;
+          }
+          mbar_expect_tx(sm.full + s, kABytes + kBBytes);
+          tma_2d(sm.a + s * kABytes, &tmR, sm.full + s, kt * kTileK, a_row);
+          tma_2d(sm.b + s * kBBytes, &tmXT, sm.full + s, kt * kTileK, b_row);
+        }
       }
     }
-  }
-  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");   // the updated tile is visible to TMA
-  __syncthreads();
-  if (threadIdx.x == 0 && !*sm.fail) {
-    for (int b = 0; b < kWBoxes; ++b)
-      tma_store_3d(&tmWf, wtile + b * kWBoxBytes, nt * kTileN + b * kWBoxCols, mt * kTileM, i);
-    asm volatile("cp.async.bulk.commit_group;" ::: "memory");
-    asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");       // written to global memory
-    asm volatile("fence.proxy.async.global;" ::: "memory");
-  }
-  teardown(sm, tmem);
-  // NOTIFY once every tile of worker i is written.
-  if (threadIdx.x == 0) {
-    __threadfence();
-    const unsigned total = gridDim.x * gridDim.y;
-    const unsigned done = atomicAdd(&a.worker_ticket[i], 1u);
-    if (done == total - 1) {
-      a.worker_ticket[i] = 0u;
+    __syncwarp();
+  } else if (warp == 1) {
+    // ---------------- MMA issuer ----------------
+    if (lane == 0) {
+      constexpr uint32_t idesc = idesc_bf16(kTileM, kTileN);
+      long long g = 0;
+      bool ok = true;
+      for (int n = 0; n < n_tiles && ok; ++n) {
+        const int ab = n & 1;
+        if (n >= 2 && !mbar_wait(sm.acc_empty + ab, static_cast<uint32_t>(((n >> 1) - 1) & 1))) {
+          record_error(a.st, ASAP_ERR_CUDA, 0xfffffffcu, a.round);
+          atomicOr(sm.fail, 1);
+          break;
+        }
+        tc_fence_after();
+        const uint32_t acc = tmem + static_cast<uint32_t>(ab) * kTmemCols;
+        for (int kt = 0; kt < k_tiles; ++kt, ++g) {
+          const int s = static_cast<int>(g % kGradStages);
+          if (!mbar_wait(sm.full + s, static_cast<uint32_t>((g / kGradStages) & 1))) {
+            record_error(a.st, ASAP_ERR_CUDA, 0xfffffffcu, a.round);
+            atomicOr(sm.fail, 1);
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+#pragma unroll
+          for (int kk = 0; kk < kTileK / 16; ++kk) {
+            const uint64_t ad = smem_desc_sw128(sm.a + s * kABytes + kk * 32);
+            const uint64_t bd = smem_desc_sw128(sm.b + s * kBBytes + kk * 32);
+            umma_bf16(acc, ad, bd, idesc, (kt | kk) != 0 ? 1u : 0u);
+          }
+          umma_commit(sm.empty + s);
+        }
+        if (ok) umma_commit(sm.acc_full + ab);
+      }
+    }
+    __syncwarp();
+  } else {
+    // ---------------- epilogue (warps 2-5) ----------------
+    const int et = threadIdx.x - kEpi0 * 32;                  // 0..127
+    const int quarter = warp & 3;                             // TMEM lanes 32*quarter .. +31
+    const int r = quarter * 32 + lane;                        // tile row (class mt*128 + r)
+    const bool issuer = et == 0;
+    const long long n_chunks = static_cast<long long>(n_tiles) * kChunksPerTile;
+    auto load_chunk = [&](long long h) {
+      const int b = static_cast<int>(h % kWBufs);
+      const GradTile t = grad_tile(blockIdx.x + (h / kChunksPerTile) * gridDim.x, MT, NT);
+      const int c = static_cast<int>(h % kChunksPerTile);
+      mbar_expect_tx(sm.wfull + b, kWBoxBytes);
+      tma_3d(sm.w + b * kWBoxBytes, &tmWf, sm.wfull + b, t.nt * kTileN + c * kWBoxCols, t.mt * kTileM, t.i);
+    };
+    auto notify = [&](int n) {   // tile n's stores are complete
+      const GradTile t = grad_tile(blockIdx.x + static_cast<long long>(n) * gridDim.x, MT, NT);
+      asm volatile("fence.proxy.async.global;" ::: "memory");
       __threadfence();
-      if (i != a.skip_worker) asm volatile("st.release.gpu.global.u32 [%0], %1;" :: "l"(a.ready + i),
-                                           "r"(a.round + 1u) : "memory");
+      const unsigned per = static_cast<unsigned>(MT * NT);
+      const unsigned done = atomicAdd(&a.worker_ticket[t.i], 1u);
+      if (done == per - 1) {
+        a.worker_ticket[t.i] = 0u;
+        __threadfence();
+        if (t.i != a.skip_worker)
+          asm volatile("st.release.gpu.global.u32 [%0], %1;" :: "l"(a.ready + t.i), "r"(a.round + 1u) : "memory");
+      }
+    };
+    if (issuer)
+      for (long long h = 0; h < n_chunks && h < kWBufs - 1; ++h) load_chunk(h);
+    bool failed = false;
+    int done_tiles = 0;
+    for (int n = 0; n < n_tiles && !failed; ++n) {
+      const int ab = n & 1;
+      bool ok = mbar_wait(sm.acc_full + ab, static_cast<uint32_t>((n >> 1) & 1));
+      if (epi_bar_or(!ok)) {
+        if (issuer) record_error(a.st, ASAP_ERR_CUDA, 0xfffffffbu, a.round);
+        failed = true;
+        break;
+      }
+      tc_fence_after();
+      const uint32_t trow = tmem + (static_cast<uint32_t>(quarter * 32) << 16) + static_cast<uint32_t>(ab) * kTmemCols;
+      for (int c = 0; c < kChunksPerTile; ++c) {
+        const long long h = static_cast<long long>(n) * kChunksPerTile + c;
+        const int b = static_cast<int>(h % kWBufs);
+        ok = mbar_wait(sm.wfull + b, static_cast<uint32_t>((h / kWBufs) & 1));
+        if (epi_bar_or(!ok)) {
+          if (issuer) record_error(a.st, ASAP_ERR_CUDA, 0xfffffffau, a.round);
+          failed = true;
+          break;
+        }
+        float gv[32];
+        tmem_ld32(trow + c * kWBoxCols, gv);
+        unsigned char* row = sm.w + b * kWBoxBytes + r * 128;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          float4* p = reinterpret_cast<float4*>(row + ((j ^ (r & 7)) << 4));   // 128-byte swizzle
+          float4 x = *p;
+          x.x = fmaf(-a.lr, gv[4 * j + 0], a.decay * x.x);
+          x.y = fmaf(-a.lr, gv[4 * j + 1], a.decay * x.y);
+          x.z = fmaf(-a.lr, gv[4 * j + 2], a.decay * x.z);
+          x.w = fmaf(-a.lr, gv[4 * j + 3], a.decay * x.w);
+          *p = x;
+        }
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");   // the updated chunk is visible to TMA
+        epi_bar();
+        if (issuer) {
+          const GradTile t = grad_tile(blockIdx.x + static_cast<long long>(n) * gridDim.x, MT, NT);
+          tma_store_3d(&tmWf, sm.w + b * kWBoxBytes, t.nt * kTileN + c * kWBoxCols, t.mt * kTileM, t.i);
+          asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+          // The previous chunk's store has read its buffer: reuse it.
+          asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+          if (h + kWBufs - 1 < n_chunks) load_chunk(h + kWBufs - 1);
+        }
+      }
+      if (failed) break;
+      // This accumulator may be overwritten by tile n+2.
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" :: "r"(smem_u32(sm.acc_empty + ab))
+                                  : "memory");
+      if (issuer && n >= 1) {
+        asm volatile("cp.async.bulk.wait_group 8;" ::: "memory");   // tile n-1's stores are complete
+        notify(n - 1);
+      }
+      done_tiles = n + 1;
+    }
+    if (issuer) {
+      asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+      if (!failed && done_tiles > 0) notify(done_tiles - 1);
     }
   }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) tmem_dealloc(tmem, kGradTmemCols);
 }
 
 }  // namespace
 
 size_t dense_smem_bytes() { return gemm_smem_bytes(kFwdStages); }
 
-size_t dense_grad_smem_bytes() { return gemm_smem_bytes(kGradStages) + kWTileBytes; }
+size_t dense_grad_smem_bytes() { return grad_smem_bytes(); }
 
 cudaError_t dense_configure() {
   const int smem = static_cast<int>(dense_smem_bytes());
@@ -526,9 +717,13 @@ cudaError_t launch_dense_fwd(const CUtensorMap& tmX, const CUtensorMap& tmW, con
 }
 
 cudaError_t launch_dense_grad(const CUtensorMap& tmR, const CUtensorMap& tmXT, const CUtensorMap& tmWf,
-                              const DenseGradArgs& g, int N, cudaStream_t s) {
-  const dim3 g2(g.d / kTileN, (g.C + kTileM - 1) / kTileM, N);
-  k_dense_grad<<<g2, kDenseThreads, dense_grad_smem_bytes(), s>>>(tmR, tmXT, tmWf, g);
+                              const DenseGradArgs& g, int N, int sm_count, cudaStream_t s) {
+  DenseGradArgs ga = g;
+  ga.N = N;
+  const long long tiles = static_cast<long long>(N) * ((g.C + kTileM - 1) / kTileM) * (g.d / kTileN);
+  const int grid = static_cast<int>(tiles < sm_count ? tiles : sm_count);
+  if (grid < 1) return cudaSuccess;
+  k_dense_grad<<<grid, kGradThreads, dense_grad_smem_bytes(), s>>>(tmR, tmXT, tmWf, ga);
   return cudaGetLastError();
 }
 

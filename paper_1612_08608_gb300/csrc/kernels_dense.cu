@@ -420,15 +420,19 @@ __global__ void __launch_bounds__(kDenseThreads, kFwdCtasPerSm)
 //   warp 1      tcgen05.mma issuer into one of two TMEM accumulators
 //               (2 x 256 columns), so tile n+1's GEMM runs while tile n's
 //               epilogue drains the other;
-//   warps 2-5   epilogue: the master tile is streamed through shared memory
-//               in 16 KB chunks of 128 rows x 32 columns (TMA load, update
-//               in place, TMA store), several chunk loads in flight.
+//   warps 2-5   epilogue: each thread updates one row of a 16 KB chunk of
+//               the master tile (128 rows x 32 columns) in shared memory and
+//               the warp arrives on the chunk's "updated" mbarrier;
+//   warp 6      master I/O: TMA loads of the chunks (up to kWBufs ahead),
+//               TMA stores of the updated ones, NOTIFY.
+// The epilogue warps never wait on each other or on a store; the I/O warp
+// alone waits for stores to finish reading a buffer before reloading it.
 // The 3-D master map clips rows beyond C, so a tile never touches the next
 // worker's rows.  A worker's NOTIFY is published by the CTA that completes
 // its last tile, once that tile's stores are complete (checked one tile
-// later, so that waiting for store completion never stalls the epilogue).
-constexpr int kGradThreads = 192;
-constexpr int kEpi0 = 2;                                  // first epilogue warp
+// later, so that the I/O warp keeps loading meanwhile).
+constexpr int kGradThreads = 224;
+constexpr int kIoWarp = 6;
 constexpr int kWBufs = 5;                                 // master chunks in shared memory
 constexpr int kChunksPerTile = kTileN / kWBoxCols;        // 8
 constexpr uint32_t kGradTmemCols = 2 * kTmemCols;        // two accumulators
@@ -441,14 +445,15 @@ struct GradSmem {
   uint64_t* empty;       // [kGradStages]
   uint64_t* acc_full;    // [2]
   uint64_t* acc_empty;   // [2]
-  uint64_t* wfull;       // [kWBufs]
+  uint64_t* wfull;       // [kWBufs]: chunk loaded
+  uint64_t* wupd;        // [kWBufs]: chunk updated by the four epilogue warps
   uint32_t* tmem_slot;
   int* fail;
 };
 
 constexpr size_t grad_smem_bytes() {
   return 1024 + static_cast<size_t>(kGradStages) * (kABytes + kBBytes) + static_cast<size_t>(kWBufs) * kWBoxBytes +
-         8 * (2 * kGradStages + 4 + kWBufs) + 16 + 16;
+         8 * (2 * kGradStages + 4 + 2 * kWBufs) + 16 + 16;
 }
 
 __device__ __forceinline__ GradSmem grad_carve(unsigned char* raw) {
@@ -465,23 +470,13 @@ __device__ __forceinline__ GradSmem grad_carve(unsigned char* raw) {
   s.acc_full = s.empty + kGradStages;
   s.acc_empty = s.acc_full + 2;
   s.wfull = s.acc_empty + 2;
-  p += 8 * (2 * kGradStages + 4 + kWBufs);
+  s.wupd = s.wfull + kWBufs;
+  p += 8 * (2 * kGradStages + 4 + 2 * kWBufs);
   s.tmem_slot = reinterpret_cast<uint32_t*>(p);
   p += 16;
   s.fail = reinterpret_cast<int*>(p);
   return s;
 }
-
-// Barrier among the four epilogue warps that also returns the OR of `v`.
-__device__ __forceinline__ bool epi_bar_or(bool v) {
-  uint32_t r;
-  asm volatile(
-      "{\n .reg .pred p, q;\n setp.ne.u32 p, %1, 0;\n bar.red.or.pred q, 1, 128, p;\n selp.u32 %0, 1, 0, q;\n}"
-      : "=r"(r) : "r"(static_cast<uint32_t>(v)) : "memory");
-  return r != 0;
-}
-
-__device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
 
 struct GradTile {
   int i, mt, nt;
@@ -517,7 +512,10 @@ __global__ void __launch_bounds__(kGradThreads, 1)
       mbar_init(sm.acc_full + s, 1);
       mbar_init(sm.acc_empty + s, 4);   // one arrival per epilogue warp
     }
-    for (int s = 0; s < kWBufs; ++s) mbar_init(sm.wfull + s, 1);
+    for (int s = 0; s < kWBufs; ++s) {
+      mbar_init(sm.wfull + s, 1);
+      mbar_init(sm.wupd + s, 4);
+    }
     *sm.fail = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -587,42 +585,74 @@ __global__ void __launch_bounds__(kGradThreads, 1)
       }
     }
     __syncwarp();
+  } else if (warp == kIoWarp) {
+    // ---------------- master I/O ----------------
+    if (lane == 0) {
+      const long long n_chunks = static_cast<long long>(n_tiles) * kChunksPerTile;
+      auto chunk_xyz = [&](long long h, int& x, int& y, int& z) {
+        const GradTile t = grad_tile(blockIdx.x + (h / kChunksPerTile) * gridDim.x, MT, NT);
+        x = t.nt * kTileN + static_cast<int>(h % kChunksPerTile) * kWBoxCols;
+        y = t.mt * kTileM;
+        z = t.i;
+      };
+      auto load_chunk = [&](long long h) {
+        const int b = static_cast<int>(h % kWBufs);
+        int x, y, z;
+        chunk_xyz(h, x, y, z);
+        mbar_expect_tx(sm.wfull + b, kWBoxBytes);
+        tma_3d(sm.w + b * kWBoxBytes, &tmWf, sm.wfull + b, x, y, z);
+      };
+      auto notify = [&](int n) {   // tile n's stores are complete
+        const GradTile t = grad_tile(blockIdx.x + static_cast<long long>(n) * gridDim.x, MT, NT);
+        asm volatile("fence.proxy.async.global;" ::: "memory");
+        __threadfence();
+        const unsigned per = static_cast<unsigned>(MT * NT);
+        const unsigned done = atomicAdd(&a.worker_ticket[t.i], 1u);
+        if (done == per - 1) {
+          a.worker_ticket[t.i] = 0u;
+          __threadfence();
+          if (t.i != a.skip_worker)
+            asm volatile("st.release.gpu.global.u32 [%0], %1;" :: "l"(a.ready + t.i), "r"(a.round + 1u) : "memory");
+        }
+      };
+      for (long long h = 0; h < n_chunks && h < kWBufs; ++h) load_chunk(h);
+      bool ok = true;
+      for (long long h = 0; h < n_chunks; ++h) {
+        const int b = static_cast<int>(h % kWBufs);
+        if (!mbar_wait(sm.wupd + b, static_cast<uint32_t>((h / kWBufs) & 1))) {
+          record_error(a.st, ASAP_ERR_CUDA, 0xfffffffau, a.round);
+          atomicOr(sm.fail, 1);
+          ok = false;
+          break;
+        }
+        int x, y, z;
+        chunk_xyz(h, x, y, z);
+        tma_store_3d(&tmWf, sm.w + b * kWBoxBytes, x, y, z);
+        asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+        const long long n = h / kChunksPerTile;
+        if (h % kChunksPerTile == kChunksPerTile - 1 && n >= 1) {
+          asm volatile("cp.async.bulk.wait_group 8;" ::: "memory");   // tile n-1's stores are complete
+          notify(static_cast<int>(n - 1));
+        }
+        // Reload the previous chunk's buffer once its store has read it.
+        if (h >= 1 && h - 1 + kWBufs < n_chunks) {
+          asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+          load_chunk(h - 1 + kWBufs);
+        }
+      }
+      asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+      if (ok && n_tiles > 0) notify(n_tiles - 1);
+    }
+    __syncwarp();
   } else {
     // ---------------- epilogue (warps 2-5) ----------------
-    const int et = threadIdx.x - kEpi0 * 32;                  // 0..127
     const int quarter = warp & 3;                             // TMEM lanes 32*quarter .. +31
     const int r = quarter * 32 + lane;                        // tile row (class mt*128 + r)
-    const bool issuer = et == 0;
-    const long long n_chunks = static_cast<long long>(n_tiles) * kChunksPerTile;
-    auto load_chunk = [&](long long h) {
-      const int b = static_cast<int>(h % kWBufs);
-      const GradTile t = grad_tile(blockIdx.x + (h / kChunksPerTile) * gridDim.x, MT, NT);
-      const int c = static_cast<int>(h % kChunksPerTile);
-      mbar_expect_tx(sm.wfull + b, kWBoxBytes);
-      tma_3d(sm.w + b * kWBoxBytes, &tmWf, sm.wfull + b, t.nt * kTileN + c * kWBoxCols, t.mt * kTileM, t.i);
-    };
-    auto notify = [&](int n) {   // tile n's stores are complete
-      const GradTile t = grad_tile(blockIdx.x + static_cast<long long>(n) * gridDim.x, MT, NT);
-      asm volatile("fence.proxy.async.global;" ::: "memory");
-      __threadfence();
-      const unsigned per = static_cast<unsigned>(MT * NT);
-      const unsigned done = atomicAdd(&a.worker_ticket[t.i], 1u);
-      if (done == per - 1) {
-        a.worker_ticket[t.i] = 0u;
-        __threadfence();
-        if (t.i != a.skip_worker)
-          asm volatile("st.release.gpu.global.u32 [%0], %1;" :: "l"(a.ready + t.i), "r"(a.round + 1u) : "memory");
-      }
-    };
-    if (issuer)
-      for (long long h = 0; h < n_chunks && h < kWBufs - 1; ++h) load_chunk(h);
     bool failed = false;
-    int done_tiles = 0;
     for (int n = 0; n < n_tiles && !failed; ++n) {
       const int ab = n & 1;
-      bool ok = mbar_wait(sm.acc_full + ab, static_cast<uint32_t>((n >> 1) & 1));
-      if (epi_bar_or(!ok)) {
-        if (issuer) record_error(a.st, ASAP_ERR_CUDA, 0xfffffffbu, a.round);
+      if (!__all_sync(0xffffffffu, mbar_wait(sm.acc_full + ab, static_cast<uint32_t>((n >> 1) & 1)))) {
+        if (lane == 0) record_error(a.st, ASAP_ERR_CUDA, 0xfffffffbu, a.round);
         failed = true;
         break;
       }
@@ -631,9 +661,8 @@ __global__ void __launch_bounds__(kGradThreads, 1)
       for (int c = 0; c < kChunksPerTile; ++c) {
         const long long h = static_cast<long long>(n) * kChunksPerTile + c;
         const int b = static_cast<int>(h % kWBufs);
-        ok = mbar_wait(sm.wfull + b, static_cast<uint32_t>((h / kWBufs) & 1));
-        if (epi_bar_or(!ok)) {
-          if (issuer) record_error(a.st, ASAP_ERR_CUDA, 0xfffffffau, a.round);
+        if (!__all_sync(0xffffffffu, mbar_wait(sm.wfull + b, static_cast<uint32_t>((h / kWBufs) & 1)))) {
+          if (lane == 0) record_error(a.st, ASAP_ERR_CUDA, 0xfffffffbu, a.round);
           failed = true;
           break;
         }
@@ -650,16 +679,10 @@ __global__ void __launch_bounds__(kGradThreads, 1)
           x.w = fmaf(-a.lr, gv[4 * j + 3], a.decay * x.w);
           *p = x;
         }
-        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");   // the updated chunk is visible to TMA
-        epi_bar();
-        if (issuer) {
-          const GradTile t = grad_tile(blockIdx.x + static_cast<long long>(n) * gridDim.x, MT, NT);
-          tma_store_3d(&tmWf, sm.w + b * kWBoxBytes, t.nt * kTileN + c * kWBoxCols, t.mt * kTileM, t.i);
-          asm volatile("cp.async.bulk.commit_group;" ::: "memory");
-          // The previous chunk's store has read its buffer: reuse it.
-          asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
-          if (h + kWBufs - 1 < n_chunks) load_chunk(h + kWBufs - 1);
-        }
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");   // the updated rows are visible to TMA
+        __syncwarp();
+        if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" :: "r"(smem_u32(sm.wupd + b))
+                                    : "memory");
       }
       if (failed) break;
       // This accumulator may be overwritten by tile n+2.
@@ -667,15 +690,6 @@ __global__ void __launch_bounds__(kGradThreads, 1)
       __syncwarp();
       if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" :: "r"(smem_u32(sm.acc_empty + ab))
                                   : "memory");
-      if (issuer && n >= 1) {
-        asm volatile("cp.async.bulk.wait_group 8;" ::: "memory");   // tile n-1's stores are complete
-        notify(n - 1);
-      }
-      done_tiles = n + 1;
-    }
-    if (issuer) {
-      asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
-      if (!failed && done_tiles > 0) notify(done_tiles - 1);
     }
   }
   tc_fence_before();

@@ -163,8 +163,9 @@ def make_shards(rows, seed):
 
 
 def kernel_work(sh):
-    """Algorithmic work of one launch of each kernel kind: (unit, amount, bound).
-    Sparse byte counts use the mean minibatch over a sample of batches."""
+    """Algorithmic work of one launch of each kernel kind: (unit, amount, bound)
+    or (unit, amount, bound, flops) when a memory-bound kernel also runs a
+    GEMM.  Sparse byte counts use the mean minibatch over a sample of batches."""
     import numpy as np
     w = WORKLOAD
     N, B, d = w["N"], w["B"], w["d"]
@@ -173,7 +174,10 @@ def kernel_work(sh):
     if w["loss"] == "softmax":
         C = w["C"]
         out["dense_fwd"] = ("TFLOP/s", 2.0 * N * B * C * d, "tensor")
-        out["dense_grad"] = ("TFLOP/s", 2.0 * N * C * d * B, "tensor")
+        # The gradient GEMM carries the fused fp32 master update (read + write
+        # 8 B per parameter) plus its bf16 operands R^T and X_b^T: HBM-bound.
+        cpad = (C + 255) // 256 * 256
+        out["dense_grad"] = ("GB/s", 8.0 * N * C * d + 2.0 * N * B * (cpad + d), "hbm", 2.0 * N * C * d * B)
         out["reduce"] = ("GB/s", 10.0 * N * ld, "hbm")     # fp32 read + write, bf16 copy write
         return out
     rng = np.random.default_rng(0)
@@ -421,7 +425,8 @@ def run_asap(args):
     pk = peaks_all()
     work = kernel_work(sh)
     kernels = {}
-    for name, (unit, amount, bound) in work.items():
+    for name, wk in work.items():
+        unit, amount, bound = wk[:3]
         n, ms = times[name]
         if n == 0:
             continue
@@ -433,6 +438,10 @@ def run_asap(args):
                          "frac": achieved / peak, "mean_launch_ms": mean_ms, "launches": n,
                          "share": ms / max(1e-9, sum(v[1] for v in times.values())),
                          "algorithmic_per_launch": amount}
+        if len(wk) > 3:   # the GEMM inside a memory-bound kernel, against the tensor peak
+            tf = wk[3] / (mean_ms * 1e-3) / 1e12
+            kernels[name]["tensor_tflops"] = tf
+            kernels[name]["tensor_frac"] = tf / pk["tensor"][0]
     dom = max(kernels, key=lambda k: kernels[k]["share"])
     kd = kernels[dom]
     roof = {"kernel": dom, "bound": kd["bound"], "achieved": kd["achieved"], "peak": kd["peak"],

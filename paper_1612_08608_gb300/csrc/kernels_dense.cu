@@ -45,7 +45,7 @@ constexpr int kTileK = 64;                  // one 128-byte swizzle row of bf16
 // The persistent gradient kernel overlaps its epilogue itself (one CTA per SM).
 constexpr int kFwdStages = 2;
 constexpr int kFwdCtasPerSm = 2;
-constexpr int kGradStages = 3;
+constexpr int kGradStages = 2;
 constexpr uint32_t kABytes = kTileM * kTileK * 2;   // 16 KB
 constexpr uint32_t kBBytes = kTileN * kTileK * 2;   // 32 KB
 constexpr uint32_t kTmemCols = 256;
@@ -433,7 +433,11 @@ __global__ void __launch_bounds__(kDenseThreads, kFwdCtasPerSm)
 // later, so that the I/O warp keeps loading meanwhile).
 constexpr int kGradThreads = 224;
 constexpr int kIoWarp = 6;
-constexpr int kWBufs = 5;                                 // master chunks in shared memory
+// Master chunks in shared memory: the kernel is bound by master bytes in
+// flight, so they take what the 2-stage operand ring leaves (GB300, N=32,
+// d=2048, C=1000: 3 stages + 5 chunks 135 us, 2 + 8 129 us, 4 + 2 224 us;
+// extra L2 prefetches of later chunks were slower still).
+constexpr int kWBufs = 8;
 constexpr int kChunksPerTile = kTileN / kWBoxCols;        // 8
 constexpr uint32_t kGradTmemCols = 2 * kTmemCols;        // two accumulators
 

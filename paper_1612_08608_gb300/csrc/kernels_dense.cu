@@ -49,6 +49,7 @@ constexpr int kGradStages = 2;
 constexpr uint32_t kABytes = kTileM * kTileK * 2;   // 16 KB
 constexpr uint32_t kBBytes = kTileN * kTileK * 2;   // 32 KB
 constexpr uint32_t kTmemCols = 256;
+constexpr uint32_t kRtBoxBytes = 128 * 64 * 2;      // R^T box: 128 classes x 64 batch rows of bf16 (16 KB)
 // Gradient epilogue: the fp32 master tile [128 classes x 256 features] passes
 // through shared memory as 8 chunks of 32 columns (128-byte swizzled rows).
 constexpr int kWBoxCols = 32;
@@ -102,6 +103,11 @@ __device__ __forceinline__ void tma_3d(void* dst, const CUtensorMap* m, uint64_t
       "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], [%5];"
       :: "r"(smem_u32(dst)), "l"(reinterpret_cast<uint64_t>(m)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar))
       : "memory");
+}
+
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap* m, const void* src, int x, int y) {
+  asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];"
+               :: "l"(reinterpret_cast<uint64_t>(m)), "r"(x), "r"(y), "r"(smem_u32(src)) : "memory");
 }
 
 __device__ __forceinline__ void tma_store_3d(const CUtensorMap* m, const void* src, int x, int y, int z) {
@@ -329,7 +335,8 @@ __device__ __forceinline__ void teardown(const GemmSmem& sm, uint32_t tmem) {
 // Forward: logits, softmax across the cluster, R^T, loss partials.
 // grid (Cq, B/128, N), cluster (Cq, 1, 1); CTA rank q owns classes [256q, 256q+256).
 __global__ void __launch_bounds__(kDenseThreads, kFwdCtasPerSm)
-    k_dense_fwd(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmW, DenseFwdArgs a) {
+    k_dense_fwd(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmW,
+                const __grid_constant__ CUtensorMap tmR, DenseFwdArgs a) {
   extern __shared__ unsigned char smem_raw[];
   const GemmSmem sm = carve<kFwdStages>(smem_raw);
   const int q = blockIdx.x, mt = blockIdx.y, i = blockIdx.z;
@@ -353,50 +360,67 @@ __global__ void __launch_bounds__(kDenseThreads, kFwdCtasPerSm)
   const int yb = a.y[(i * a.nb + a.t) * a.B + b];
   const int c0 = q * kTileN;
   float v[32];
-  float m = -INFINITY;
+  // One pass over this CTA's classes: running max m and sum of exp(z - m),
+  // rescaled whenever the max grows; and the label's logit.
+  float m = -INFINITY, s = 0.f, zy = 0.f;
   if (ok) {
     for (int ch = 0; ch < kTileN / 32; ++ch) {
       tmem_ld32(trow + ch * 32, v);
+      float cm = m;
 #pragma unroll
       for (int j = 0; j < 32; ++j)
-        if (c0 + ch * 32 + j < a.C) m = fmaxf(m, v[j]);
+        if (c0 + ch * 32 + j < a.C) cm = fmaxf(cm, v[j]);
+      if (cm > -INFINITY) s *= __expf(m - cm);   // m = -inf: s is still 0
+#pragma unroll
+      for (int j = 0; j < 32; ++j) {
+        const int c = c0 + ch * 32 + j;
+        if (c < a.C) s += __expf(v[j] - cm);
+        if (c == yb) zy = v[j];
+      }
+      m = cm;
     }
   }
   sm.row_a[threadIdx.x] = m;
+  sm.row_b[threadIdx.x] = s;
   cluster_sync();
   const uint32_t nr = cluster_size();
   float gmax = -INFINITY;
   for (uint32_t r = 0; r < nr; ++r) gmax = fmaxf(gmax, ld_dsmem_f32(sm.row_a + threadIdx.x, r));
-  float s = 0.f, zy = 0.f;
+  float S = 0.f;
+  for (uint32_t r = 0; r < nr; ++r) {
+    const float mr = ld_dsmem_f32(sm.row_a + threadIdx.x, r);
+    if (mr > -INFINITY) S += ld_dsmem_f32(sm.row_b + threadIdx.x, r) * __expf(mr - gmax);
+  }
+  const float invS = 1.0f / S;
+  // R^T tile [256 classes x 128 rows] in bf16, staged in the operand stages
+  // (free once the accumulator is complete) as four 128-byte-swizzled boxes
+  // of 128 classes x 64 rows -- the layout of the R^T map -- then stored by TMA.
+  unsigned char* rt_tile = sm.a;
   if (ok) {
+    const int jb = threadIdx.x & 63;                              // row within its box
+    unsigned char* col = rt_tile + (threadIdx.x >> 6) * kRtBoxBytes + ((jb & 7) << 1);
     for (int ch = 0; ch < kTileN / 32; ++ch) {
       tmem_ld32(trow + ch * 32, v);
 #pragma unroll
       for (int j = 0; j < 32; ++j) {
-        const int c = c0 + ch * 32 + j;
-        if (c < a.C) s += __expf(v[j] - gmax);
-        if (c == yb) zy = v[j];
+        const int cl = ch * 32 + j, c = c0 + cl;                  // class within the tile / overall
+        float r = 0.f;
+        if (c < a.C) r = (__expf(v[j] - gmax) * invS - (c == yb ? 1.f : 0.f)) * a.inv_B;
+        const int row = cl & 127;
+        *reinterpret_cast<__nv_bfloat16*>(col + (cl >> 7) * 2 * kRtBoxBytes + row * 128 +
+                                          ((((jb >> 3) ^ (row & 7))) << 4)) = __float2bfloat16_rn(r);
       }
     }
   }
-  sm.row_b[threadIdx.x] = s;
-  cluster_sync();
-  float S = 0.f;
-  for (uint32_t r = 0; r < nr; ++r) S += ld_dsmem_f32(sm.row_b + threadIdx.x, r);
-  const float invS = 1.0f / S;
-  if (ok) {
-    __nv_bfloat16* rt = reinterpret_cast<__nv_bfloat16*>(a.RT) +
-                        (static_cast<int64_t>(i) * a.Cq * kTileN + c0) * a.B + b;
-    for (int ch = 0; ch < kTileN / 32; ++ch) {
-      tmem_ld32(trow + ch * 32, v);
-#pragma unroll
-      for (int j = 0; j < 32; ++j) {
-        const int c = c0 + ch * 32 + j;
-        float r = 0.f;
-        if (c < a.C) r = (__expf(v[j] - gmax) * invS - (c == yb ? 1.f : 0.f)) * a.inv_B;
-        rt[static_cast<int64_t>(ch * 32 + j) * a.B] = __float2bfloat16_rn(r);
-      }
-    }
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");   // the staged tile is visible to TMA
+  __syncthreads();
+  if (threadIdx.x == 0 && ok) {
+    const int y0 = i * a.Cq * kTileN + c0;                       // R^T row of this tile's first class
+    for (int h = 0; h < 2; ++h)
+      for (int bx = 0; bx < 2; ++bx)
+        tma_store_2d(&tmR, rt_tile + (h * 2 + bx) * kRtBoxBytes, mt * kTileM + bx * 64, y0 + h * 128);
+    asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+    asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
   }
   // loss of the rows whose label falls in this CTA's classes
   float l = (ok && yb >= c0 && yb < c0 + kTileN) ? (gmax + __logf(S) - zy) : 0.f;
@@ -717,8 +741,8 @@ cudaError_t dense_configure() {
                               static_cast<int>(dense_grad_smem_bytes()));
 }
 
-cudaError_t launch_dense_fwd(const CUtensorMap& tmX, const CUtensorMap& tmW, const DenseFwdArgs& f, int N,
-                             cudaStream_t s) {
+cudaError_t launch_dense_fwd(const CUtensorMap& tmX, const CUtensorMap& tmW, const CUtensorMap& tmR,
+                             const DenseFwdArgs& f, int N, cudaStream_t s) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(f.Cq, f.B / kTileM, N);
   cfg.blockDim = dim3(kDenseThreads, 1, 1);
@@ -731,7 +755,7 @@ cudaError_t launch_dense_fwd(const CUtensorMap& tmX, const CUtensorMap& tmW, con
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, k_dense_fwd, tmX, tmW, f);
+  return cudaLaunchKernelEx(&cfg, k_dense_fwd, tmX, tmW, tmR, f);
 }
 
 cudaError_t launch_dense_grad(const CUtensorMap& tmR, const CUtensorMap& tmXT, const CUtensorMap& tmWf,

@@ -116,6 +116,7 @@ struct MixArgs {
 // Arguments of the dense softmax-regression step (kernels_dense.cu).
 struct DenseFwdArgs {
   int C, Cq, d, B, nb, t;      // Cq = ceil(C / 256) CTAs per cluster
+  int N;                       // workers (set by the launcher)
   const int* y;                // [N][nb*B] class ids
   uint16_t* RT;                // [N][Cq*256][B] bf16: R^T
   float* loss_part;            // [N][B/128][Cq]

@@ -6,13 +6,13 @@
 //   gradient G = R^T X_b           [C x d], fp32 accumulate
 //            W_half = (1 - eta l2) W - eta G    (fp32 master, in place), then NOTIFY
 //
-// Both GEMMs use 128 x 256 output tiles.  One lane issues TMA loads
-// (128-byte swizzled, K-major tiles of 64 bf16) into a ring of stages guarded
-// by full/empty mbarriers; another issues tcgen05.mma (M=128, N=256, K=16,
-// bf16 x bf16 -> fp32 in TMEM) and commits each stage back to its empty
-// barrier; four warps read the accumulator out of TMEM (a warp reaches the
-// TMEM lanes 32 (w mod 4) .. + 31, i.e. tile rows).  The forward kernel is one
-// CTA per tile (4 warps); the gradient kernel is persistent (below).
+// Both GEMMs use 128 x 256 output tiles and are persistent and
+// warp-specialised: one lane issues TMA loads (128-byte swizzled, K-major
+// tiles of 64 bf16) into a ring of stages guarded by full/empty mbarriers;
+// another issues tcgen05.mma (M=128, N=256, K=16, bf16 x bf16 -> fp32 in
+// TMEM) into one of two accumulators and commits each stage back to its empty
+// barrier; four epilogue warps drain the other accumulator meanwhile (a warp
+// reaches the TMEM lanes 32 (w mod 4) .. + 31, i.e. tile rows).
 //
 // Softmax needs all C logits of a row, more than one CTA's 256 TMEM
 // columns: the forward kernel runs as a cluster of ceil(C/256) CTAs along
@@ -34,17 +34,11 @@ namespace asap {
 
 namespace {
 
-constexpr int kDenseThreads = 128;
 constexpr int kTileM = 128;
 constexpr int kTileN = 256;
 constexpr int kTileK = 64;                  // one 128-byte swizzle row of bf16
-// Operand stages of the TMA -> tcgen05 ring (48 KB each).  Two forward CTAs
-// share an SM (2 x 100 KB of shared memory, 2 x 256 TMEM columns), so one's
-// softmax epilogue overlaps the other's main loop: on GB300 that beats one
-// CTA with a 4-stage ring (109 us against 152 us at N=32, d=2048, C=1000).
-// The persistent gradient kernel overlaps its epilogue itself (one CTA per SM).
-constexpr int kFwdStages = 2;
-constexpr int kFwdCtasPerSm = 2;
+// Operand stages of the TMA -> tcgen05 rings (48 KB each).
+constexpr int kFwdStages = 3;
 constexpr int kGradStages = 2;
 constexpr uint32_t kABytes = kTileM * kTileK * 2;   // 16 KB
 constexpr uint32_t kBBytes = kTileN * kTileK * 2;   // 32 KB
@@ -192,246 +186,331 @@ __device__ __forceinline__ void cluster_sync() {
   asm volatile("barrier.cluster.arrive.release.aligned;\nbarrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
 
-__device__ __forceinline__ uint32_t cluster_size() {
-  uint32_t r;
-  asm volatile("mov.u32 %0, %%cluster_nctarank;" : "=r"(r));
-  return r;
-}
-
-__device__ __forceinline__ float ld_dsmem_f32(const float* local, uint32_t rank) {
+// Store to the shared memory of cluster CTA `rank`, at `local`'s offset.
+__device__ __forceinline__ void st_dsmem_f32(float* local, uint32_t rank, float v) {
   uint32_t remote;
   asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(local)), "r"(rank));
-  float v;
-  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(remote) : "memory");
-  return v;
+  asm volatile("st.shared::cluster.f32 [%0], %1;" :: "r"(remote), "f"(v) : "memory");
 }
-
-struct GemmSmem {
-  unsigned char* a;     // stages x kABytes
-  unsigned char* b;     // stages x kBBytes
-  uint64_t* full;
-  uint64_t* empty;
-  uint64_t* accum;
-  uint32_t* tmem_slot;
-  float* row_a;         // [128]
-  float* row_b;         // [128]
-  float* red;           // [4]
-  int* fail;
-};
 
 __device__ __forceinline__ uintptr_t align1024(const void* raw) {
   return (reinterpret_cast<uintptr_t>(raw) + 1023) & ~static_cast<uintptr_t>(1023);
 }
 
-// Layout from a 1024-byte aligned address p, with ST operand stages.
-template <int ST>
-__device__ __forceinline__ GemmSmem carve_at(uintptr_t p) {
-  GemmSmem s;
+// Relaxed arrival on the mbarrier at `local`'s offset in the shared memory of
+// cluster CTA `rank` (order earlier writes with a release fence first).
+__device__ __forceinline__ void mbar_arrive_cluster_relaxed(uint64_t* local, uint32_t rank) {
+  uint32_t remote;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(local)), "r"(rank));
+  asm volatile("mbarrier.arrive.relaxed.cluster.shared::cluster.b64 _, [%0];" :: "r"(remote) : "memory");
+}
+
+// Time-limited wait on a local mbarrier whose arrivals come from other CTAs
+// of the cluster (acquire at cluster scope: their prior writes are visible).
+__device__ __forceinline__ bool mbar_wait_cluster(uint64_t* bar, uint32_t parity) {
+  const unsigned long long t0 = now_ns();
+  for (;;) {
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n"
+        " selp.u32 %0, 1, 0, p;\n}"
+        : "=r"(ok) : "r"(smem_u32(bar)), "r"(parity) : "memory");
+    if (ok) return true;
+    if (now_ns() - t0 > kWaitNs) return false;
+  }
+}
+
+// Barrier among the epilogue warps (barrier 1) that also returns the OR of
+// `v` over them, so that they take every decision together.
+constexpr int kEpiWarps = 8;                           // forward epilogue warps: two per TMEM lane quarter
+constexpr int kEpiParts = kEpiWarps / 4;               // column parts of a row
+constexpr int kEpiChunks = kTileN / 32 / kEpiParts;    // 32-column chunks per epilogue thread
+
+__device__ __forceinline__ bool epi_bar_or(bool v) {
+  uint32_t r;
+  asm volatile(
+      "{\n .reg .pred p, q;\n setp.ne.u32 p, %1, 0;\n bar.red.or.pred q, 1, %2, p;\n selp.u32 %0, 1, 0, q;\n}"
+      : "=r"(r) : "r"(static_cast<uint32_t>(v)), "n"(kEpiWarps * 32) : "memory");
+  return r != 0;
+}
+
+__device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, %0;" :: "n"(kEpiWarps * 32) : "memory"); }
+
+// ----------------------------------------------------------------------------
+// Forward: logits, softmax across the cluster, R^T, loss partials.
+//
+// Persistent clusters of Cq = ceil(C/256) CTAs, one CTA per SM; CTA rank q
+// owns classes [256q, 256q+256) of every row tile (i, mt) its cluster walks
+// (row tiles cluster, cluster + n_clusters, ...).  Per CTA:
+//   warp 0      TMA producer of the operand ring (X and W k-tiles);
+//   warp 1      tcgen05.mma issuer into one of two TMEM accumulators, so the
+//               next row tile's GEMM runs while this one's epilogue drains;
+//   warps 2-9   epilogue, two threads per row (128 columns each): a single
+//               pass over their logits gives a running max m and sum of
+//               exp(z - m); each thread stores its (m, s) into every cluster
+//               CTA's double-buffered slot (remote shared-memory stores, then
+//               a release arrival on that CTA's "full" mbarrier; "free"
+//               mbarriers guard a slot's reuse), so that the combination
+//               reads local shared memory; then R = (softmax - onehot) / B is
+//               staged as the R^T tile and written by TMA.
+constexpr int kFwdThreads = (2 + kEpiWarps) * 32;
+constexpr int kMaxCq = 4;                                       // C <= 1024
+constexpr int kStatsSlot = kMaxCq * kEpiParts * 2 * kTileM;     // floats per stats slot
+
+struct FwdSmem {
+  unsigned char* a;      // kFwdStages x kABytes
+  unsigned char* b;      // kFwdStages x kBBytes
+  unsigned char* rt;     // R^T tile staging: 4 boxes of kRtBoxBytes
+  float* stats;          // [2 slots][kMaxCq source CTAs][kEpiParts][2: m, s][128 rows]
+  uint64_t* full;        // [kFwdStages]
+  uint64_t* empty;       // [kFwdStages]
+  uint64_t* acc_full;    // [2]
+  uint64_t* acc_empty;   // [2]
+  uint64_t* st_full;     // [2]: every cluster CTA's (m, s) of the slot are written
+  uint64_t* st_free;     // [2]: every cluster CTA has read the slot
+  uint32_t* tmem_slot;
+  float* red;            // [kEpiWarps]
+};
+
+constexpr size_t fwd_smem_bytes() {
+  return 1024 + static_cast<size_t>(kFwdStages) * (kABytes + kBBytes) + 4 * static_cast<size_t>(kRtBoxBytes) +
+         4 * kStatsSlot * 2 + 8 * (2 * kFwdStages + 8) + 16 + 4 * kEpiWarps;
+}
+
+__device__ __forceinline__ FwdSmem fwd_carve(unsigned char* raw) {
+  uintptr_t p = align1024(raw);
+  FwdSmem s;
   s.a = reinterpret_cast<unsigned char*>(p);
-  p += ST * kABytes;
+  p += kFwdStages * kABytes;
   s.b = reinterpret_cast<unsigned char*>(p);
-  p += ST * kBBytes;
+  p += kFwdStages * kBBytes;
+  s.rt = reinterpret_cast<unsigned char*>(p);
+  p += 4 * kRtBoxBytes;
+  s.stats = reinterpret_cast<float*>(p);
+  p += 4 * kStatsSlot * 2;
   s.full = reinterpret_cast<uint64_t*>(p);
-  s.empty = s.full + ST;
-  s.accum = s.empty + ST;
-  p += 8 * (2 * ST + 2);
+  s.empty = s.full + kFwdStages;
+  s.acc_full = s.empty + kFwdStages;
+  s.acc_empty = s.acc_full + 2;
+  s.st_full = s.acc_empty + 2;
+  s.st_free = s.st_full + 2;
+  p += 8 * (2 * kFwdStages + 8);
   s.tmem_slot = reinterpret_cast<uint32_t*>(p);
   p += 16;
-  s.row_a = reinterpret_cast<float*>(p);
-  p += 4 * kTileM;
-  s.row_b = reinterpret_cast<float*>(p);
-  p += 4 * kTileM;
   s.red = reinterpret_cast<float*>(p);
-  p += 16;
-  s.fail = reinterpret_cast<int*>(p);
   return s;
 }
 
-template <int ST>
-__device__ __forceinline__ GemmSmem carve(unsigned char* raw) { return carve_at<ST>(align1024(raw)); }
-
-// Bytes of dynamic shared memory for ST stages (alignment slack included).
-constexpr size_t gemm_smem_bytes(int st) {
-  return 1024 + static_cast<size_t>(st) * (kABytes + kBBytes) + 8 * (2 * st + 2) + 16 + 8 * kTileM + 16 + 16;
-}
-
-// The producer / MMA part shared by both GEMMs.  A tiles come from tmA at
-// (k, a_row), B tiles from tmB at (k, b_row[, b_z]) (3-D when b_is_3d).
-template <int ST>
-__device__ void gemm_mainloop(const GemmSmem& sm, const CUtensorMap* tmA, const CUtensorMap* tmB, bool b_is_3d,
-                              int a_row, int b_row, int b_z, int k_tiles, uint32_t tmem, DevState* st,
-                              unsigned worker, unsigned round) {
+__global__ void __launch_bounds__(kFwdThreads, 1)
+    k_dense_fwd(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmW,
+                const __grid_constant__ CUtensorMap tmR, DenseFwdArgs a) {
+  extern __shared__ unsigned char smem_raw[];
+  const FwdSmem sm = fwd_carve(smem_raw);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int Cq = a.Cq, q = static_cast<int>(blockIdx.x) % Cq, cl_id = static_cast<int>(blockIdx.x) / Cq;
+  const int n_clusters = static_cast<int>(gridDim.x) / Cq;
+  const int MT = a.B / kTileM;
+  const int total = a.N * MT;                                   // row tiles
+  const int n_my = total > cl_id ? (total - cl_id + n_clusters - 1) / n_clusters : 0;
+  const int k_tiles = a.d / kTileK;
+  const int c0 = q * kTileN;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kFwdStages; ++s) {
+      mbar_init(sm.full + s, 1);
+      mbar_init(sm.empty + s, 1);
+    }
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(sm.acc_full + s, 1);
+      mbar_init(sm.acc_empty + s, kEpiWarps);            // one arrival per epilogue warp
+      mbar_init(sm.st_full + s, kEpiWarps * Cq);         // every epilogue warp of every cluster CTA
+      mbar_init(sm.st_free + s, kEpiWarps * Cq);
+    }
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) tmem_alloc(sm.tmem_slot, 2 * kTmemCols);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  cluster_sync();   // every CTA's barriers exist before any remote arrival
+  const uint32_t tmem = *sm.tmem_slot;
+
   if (warp == 0) {
+    // ---------------- TMA producer ----------------
     if (lane == 0) {
-      for (int kt = 0; kt < k_tiles; ++kt) {
-        const int s = kt % ST;
-        if (kt >= ST && !mbar_wait(sm.empty + s, ((kt / ST) - 1) & 1)) {
-          record_error(st, ASAP_ERR_CUDA, worker, round);
-          atomicOr(sm.fail, 1);
-          break;
+      long long g = 0;
+      bool ok = true;
+      for (int n = 0; n < n_my && ok; ++n) {
+        const int rt_i = cl_id + n * n_clusters, i = rt_i / MT, mt = rt_i - i * MT;
+        const int row0 = (i * a.nb + a.t) * a.B + mt * kTileM;   // row of X
+        for (int kt = 0; kt < k_tiles; ++kt, ++g) {
+          const int s = static_cast<int>(g % kFwdStages);
+          if (g >= kFwdStages && !mbar_wait(sm.empty + s, static_cast<uint32_t>(((g / kFwdStages) - 1) & 1))) {
+            record_error(a.st, ASAP_ERR_CUDA, i, a.round);
+            ok = false;
+            break;
+          }
+          mbar_expect_tx(sm.full + s, kABytes + kBBytes);
+          tma_2d(sm.a + s * kABytes, &tmX, sm.full + s, kt * kTileK, row0);
+          tma_3d(sm.b + s * kBBytes, &tmW, sm.full + s, kt * kTileK, c0, i);
         }
-        mbar_expect_tx(sm.full + s, kABytes + kBBytes);
-        tma_2d(sm.a + s * kABytes, tmA, sm.full + s, kt * kTileK, a_row);
-        if (b_is_3d)
-          tma_3d(sm.b + s * kBBytes, tmB, sm.full + s, kt * kTileK, b_row, b_z);
-        else
-          tma_2d(sm.b + s * kBBytes, tmB, sm.full + s, kt * kTileK, b_row);
       }
     }
     __syncwarp();
   } else if (warp == 1) {
+    // ---------------- MMA issuer ----------------
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_bf16(kTileM, kTileN);
+      long long g = 0;
       bool ok = true;
-      for (int kt = 0; kt < k_tiles; ++kt) {
-        const int s = kt % ST;
-        if (!mbar_wait(sm.full + s, (kt / ST) & 1)) {
-          record_error(st, ASAP_ERR_CUDA, worker, round);
-          atomicOr(sm.fail, 1);
-          ok = false;
+      for (int n = 0; n < n_my && ok; ++n) {
+        const int ab = n & 1;
+        if (n >= 2 && !mbar_wait(sm.acc_empty + ab, static_cast<uint32_t>(((n >> 1) - 1) & 1))) {
+          record_error(a.st, ASAP_ERR_CUDA, 0xfffffff9u, a.round);
           break;
         }
         tc_fence_after();
+        const uint32_t acc = tmem + static_cast<uint32_t>(ab) * kTmemCols;
+        for (int kt = 0; kt < k_tiles; ++kt, ++g) {
+          const int s = static_cast<int>(g % kFwdStages);
+          if (!mbar_wait(sm.full + s, static_cast<uint32_t>((g / kFwdStages) & 1))) {
+            record_error(a.st, ASAP_ERR_CUDA, 0xfffffff9u, a.round);
+            ok = false;
+            break;
+          }
+          tc_fence_after();
 #pragma unroll
-        for (int kk = 0; kk < kTileK / 16; ++kk) {
-          const uint64_t ad = smem_desc_sw128(sm.a + s * kABytes + kk * 32);
-          const uint64_t bd = smem_desc_sw128(sm.b + s * kBBytes + kk * 32);
-          umma_bf16(tmem, ad, bd, idesc, (kt | kk) != 0 ? 1u : 0u);
+          for (int kk = 0; kk < kTileK / 16; ++kk) {
+            const uint64_t ad = smem_desc_sw128(sm.a + s * kABytes + kk * 32);
+            const uint64_t bd = smem_desc_sw128(sm.b + s * kBBytes + kk * 32);
+            umma_bf16(acc, ad, bd, idesc, (kt | kk) != 0 ? 1u : 0u);
+          }
+          umma_commit(sm.empty + s);
         }
-        umma_commit(sm.empty + s);
+        if (ok) umma_commit(sm.acc_full + ab);
       }
-      if (ok) umma_commit(sm.accum);
     }
     __syncwarp();
-  }
-}
-
-template <int ST>
-__device__ __forceinline__ void setup(const GemmSmem& sm) {
-  const int warp = threadIdx.x >> 5;
-  if (threadIdx.x == 0) {
-    for (int s = 0; s < ST; ++s) {
-      mbar_init(sm.full + s, 1);
-      mbar_init(sm.empty + s, 1);
+  } else {
+    // ---------------- epilogue (warps 2 .. 2 + kEpiWarps - 1) ----------------
+    const int ew = warp - 2;
+    const int quarter = warp & 3;                               // TMEM lanes 32*quarter .. +31
+    const int part = ew >> 2;                                   // columns [128 part, 128 part + 128)
+    const int r = quarter * 32 + lane;                          // row within the tile
+    const int ch0 = part * kEpiChunks;
+    const bool issuer = ew == 0 && lane == 0;
+    const int jb = r & 63;                                      // row within its R^T box
+    unsigned char* rt_col = sm.rt + (r >> 6) * kRtBoxBytes + ((jb & 7) << 1);
+    float v[32];
+    for (int n = 0; n < n_my; ++n) {
+      const int ab = n & 1, slot = n & 1;
+      const int rt_i = cl_id + n * n_clusters, i = rt_i / MT, mt = rt_i - i * MT;
+      bool ok = mbar_wait(sm.acc_full + ab, static_cast<uint32_t>((n >> 1) & 1));
+      if (epi_bar_or(!ok)) {
+        if (issuer) record_error(a.st, ASAP_ERR_CUDA, 0xfffffff8u, a.round);
+        break;
+      }
+      tc_fence_after();
+      const uint32_t trow = tmem + (static_cast<uint32_t>(quarter * 32) << 16) + static_cast<uint32_t>(ab) * kTmemCols;
+      const int yb = a.y[(i * a.nb + a.t) * a.B + mt * kTileM + r];
+      // One pass: running max and rescaled exp-sum over this thread's columns.
+      float m = -INFINITY, s = 0.f, zy = 0.f;
+      for (int ch = ch0; ch < ch0 + kEpiChunks; ++ch) {
+        tmem_ld32(trow + ch * 32, v);
+        float cm = m;
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+          if (c0 + ch * 32 + j < a.C) cm = fmaxf(cm, v[j]);
+        if (cm > -INFINITY) s *= __expf(m - cm);
+#pragma unroll
+        for (int j = 0; j < 32; ++j) {
+          const int c = c0 + ch * 32 + j;
+          if (c < a.C) s += __expf(v[j] - cm);
+          if (c == yb) zy = v[j];
+        }
+        m = cm;
+      }
+      // Exchange (m, s) with the cluster: every peer must have read its slot of
+      // tile n-2 before this thread writes into it again.
+      ok = n < 2 || mbar_wait_cluster(sm.st_free + slot, static_cast<uint32_t>(((n >> 1) - 1) & 1));
+      if (epi_bar_or(!ok)) {
+        if (issuer) record_error(a.st, ASAP_ERR_CUDA, 0xfffffff7u, a.round);
+        break;
+      }
+      float* slot_stats = sm.stats + slot * kStatsSlot;
+      float* mine = slot_stats + (q * kEpiParts + part) * 2 * kTileM + r;   // this thread's entry, in every CTA
+      for (int p = 0; p < Cq; ++p) {
+        st_dsmem_f32(mine, static_cast<uint32_t>(p), m);
+        st_dsmem_f32(mine + kTileM, static_cast<uint32_t>(p), s);
+      }
+      __syncwarp();
+      if (lane == 0) {
+        // One release fence for the warp's stores, then relaxed arrivals.
+        asm volatile("fence.acq_rel.cluster;" ::: "memory");
+        for (int p = 0; p < Cq; ++p) mbar_arrive_cluster_relaxed(sm.st_full + slot, static_cast<uint32_t>(p));
+      }
+      ok = mbar_wait_cluster(sm.st_full + slot, static_cast<uint32_t>((n >> 1) & 1));
+      if (epi_bar_or(!ok)) {
+        if (issuer) record_error(a.st, ASAP_ERR_CUDA, 0xfffffff6u, a.round);
+        break;
+      }
+      float gmax = -INFINITY;
+      for (int e = 0; e < Cq * kEpiParts; ++e) gmax = fmaxf(gmax, slot_stats[e * 2 * kTileM + r]);
+      float S = 0.f;
+      for (int e = 0; e < Cq * kEpiParts; ++e) {
+        const float mp = slot_stats[e * 2 * kTileM + r];
+        if (mp > -INFINITY) S += slot_stats[(e * 2 + 1) * kTileM + r] * __expf(mp - gmax);
+      }
+      // Our slot is read: peers may refill it for tile n+2.
+      __syncwarp();
+      if (lane == 0)
+        for (int p = 0; p < Cq; ++p) mbar_arrive_cluster_relaxed(sm.st_free + slot, static_cast<uint32_t>(p));
+      const float invS = 1.0f / S;
+      // R^T tile in the staging boxes (the previous tile's store has read them:
+      // the issuer waited for that before the barrier at the top of this tile).
+      for (int ch = ch0; ch < ch0 + kEpiChunks; ++ch) {
+        tmem_ld32(trow + ch * 32, v);
+#pragma unroll
+        for (int j = 0; j < 32; ++j) {
+          const int cl = ch * 32 + j, c = c0 + cl;
+          float rv = 0.f;
+          if (c < a.C) rv = (__expf(v[j] - gmax) * invS - (c == yb ? 1.f : 0.f)) * a.inv_B;
+          const int row = cl & 127;
+          *reinterpret_cast<__nv_bfloat16*>(rt_col + (cl >> 7) * 2 * kRtBoxBytes + row * 128 +
+                                            (((jb >> 3) ^ (row & 7)) << 4)) = __float2bfloat16_rn(rv);
+        }
+      }
+      // The accumulator is free for tile n+2.
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" :: "r"(smem_u32(sm.acc_empty + ab))
+                                  : "memory");
+      // loss of the rows whose label falls in this thread's classes
+      const int lo = c0 + ch0 * 32;
+      float l = (yb >= lo && yb < lo + kEpiChunks * 32) ? (gmax + __logf(S) - zy) : 0.f;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
+      if (lane == 0) sm.red[ew] = l;
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");   // the staged tile is visible to TMA
+      epi_bar();
+      if (issuer) {
+        const int y0 = i * Cq * kTileN + c0;                       // R^T row of this tile's first class
+        for (int h = 0; h < 2; ++h)
+          for (int bx = 0; bx < 2; ++bx)
+            tma_store_2d(&tmR, sm.rt + (h * 2 + bx) * kRtBoxBytes, mt * kTileM + bx * 64, y0 + h * 128);
+        asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+        float lt = 0.f;
+        for (int w2 = 0; w2 < kEpiWarps; ++w2) lt += sm.red[w2];
+        a.loss_part[(static_cast<int64_t>(i) * MT + mt) * Cq + q] = lt;
+        asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");   // staging boxes reusable
+      }
     }
-    mbar_init(sm.accum, 1);
-    *sm.fail = 0;
-    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    if (issuer) asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
   }
-  if (warp == 1) tmem_alloc(sm.tmem_slot, kTmemCols);
   tc_fence_before();
   __syncthreads();
-  tc_fence_after();
-}
-
-__device__ __forceinline__ void teardown(const GemmSmem& sm, uint32_t tmem) {
-  tc_fence_before();
-  __syncthreads();
-  if ((threadIdx.x >> 5) == 1) tmem_dealloc(tmem, kTmemCols);
-}
-
-// ----------------------------------------------------------------------------
-// Forward: logits, softmax across the cluster, R^T, loss partials.
-// grid (Cq, B/128, N), cluster (Cq, 1, 1); CTA rank q owns classes [256q, 256q+256).
-__global__ void __launch_bounds__(kDenseThreads, kFwdCtasPerSm)
-    k_dense_fwd(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmW,
-                const __grid_constant__ CUtensorMap tmR, DenseFwdArgs a) {
-  extern __shared__ unsigned char smem_raw[];
-  const GemmSmem sm = carve<kFwdStages>(smem_raw);
-  const int q = blockIdx.x, mt = blockIdx.y, i = blockIdx.z;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  setup<kFwdStages>(sm);
-  const uint32_t tmem = *sm.tmem_slot;
-
-  const int row0 = (i * a.nb + a.t) * a.B + mt * kTileM;        // row of X
-  gemm_mainloop<kFwdStages>(sm, &tmX, &tmW, true, row0, q * kTileN, i, a.d / kTileK, tmem, a.st, i, a.round);
-
-  // ---- epilogue: thread = batch row ----
-  const bool ok = __all_sync(0xffffffffu, mbar_wait(sm.accum, 0));
-  if (!ok) {
-    record_error(a.st, ASAP_ERR_CUDA, i, a.round);
-    atomicOr(sm.fail, 1);
-  }
-  __syncwarp();
-  tc_fence_after();
-  const uint32_t trow = tmem + (static_cast<uint32_t>(warp * 32) << 16);
-  const int b = mt * kTileM + threadIdx.x;                       // row within the batch
-  const int yb = a.y[(i * a.nb + a.t) * a.B + b];
-  const int c0 = q * kTileN;
-  float v[32];
-  // One pass over this CTA's classes: running max m and sum of exp(z - m),
-  // rescaled whenever the max grows; and the label's logit.
-  float m = -INFINITY, s = 0.f, zy = 0.f;
-  if (ok) {
-    for (int ch = 0; ch < kTileN / 32; ++ch) {
-      tmem_ld32(trow + ch * 32, v);
-      float cm = m;
-#pragma unroll
-      for (int j = 0; j < 32; ++j)
-        if (c0 + ch * 32 + j < a.C) cm = fmaxf(cm, v[j]);
-      if (cm > -INFINITY) s *= __expf(m - cm);   // m = -inf: s is still 0
-#pragma unroll
-      for (int j = 0; j < 32; ++j) {
-        const int c = c0 + ch * 32 + j;
-        if (c < a.C) s += __expf(v[j] - cm);
-        if (c == yb) zy = v[j];
-      }
-      m = cm;
-    }
-  }
-  sm.row_a[threadIdx.x] = m;
-  sm.row_b[threadIdx.x] = s;
-  cluster_sync();
-  const uint32_t nr = cluster_size();
-  float gmax = -INFINITY;
-  for (uint32_t r = 0; r < nr; ++r) gmax = fmaxf(gmax, ld_dsmem_f32(sm.row_a + threadIdx.x, r));
-  float S = 0.f;
-  for (uint32_t r = 0; r < nr; ++r) {
-    const float mr = ld_dsmem_f32(sm.row_a + threadIdx.x, r);
-    if (mr > -INFINITY) S += ld_dsmem_f32(sm.row_b + threadIdx.x, r) * __expf(mr - gmax);
-  }
-  const float invS = 1.0f / S;
-  // R^T tile [256 classes x 128 rows] in bf16, staged in the operand stages
-  // (free once the accumulator is complete) as four 128-byte-swizzled boxes
-  // of 128 classes x 64 rows -- the layout of the R^T map -- then stored by TMA.
-  unsigned char* rt_tile = sm.a;
-  if (ok) {
-    const int jb = threadIdx.x & 63;                              // row within its box
-    unsigned char* col = rt_tile + (threadIdx.x >> 6) * kRtBoxBytes + ((jb & 7) << 1);
-    for (int ch = 0; ch < kTileN / 32; ++ch) {
-      tmem_ld32(trow + ch * 32, v);
-#pragma unroll
-      for (int j = 0; j < 32; ++j) {
-        const int cl = ch * 32 + j, c = c0 + cl;                  // class within the tile / overall
-        float r = 0.f;
-        if (c < a.C) r = (__expf(v[j] - gmax) * invS - (c == yb ? 1.f : 0.f)) * a.inv_B;
-        const int row = cl & 127;
-        *reinterpret_cast<__nv_bfloat16*>(col + (cl >> 7) * 2 * kRtBoxBytes + row * 128 +
-                                          ((((jb >> 3) ^ (row & 7))) << 4)) = __float2bfloat16_rn(r);
-      }
-    }
-  }
-  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");   // the staged tile is visible to TMA
-  __syncthreads();
-  if (threadIdx.x == 0 && ok) {
-    const int y0 = i * a.Cq * kTileN + c0;                       // R^T row of this tile's first class
-    for (int h = 0; h < 2; ++h)
-      for (int bx = 0; bx < 2; ++bx)
-        tma_store_2d(&tmR, rt_tile + (h * 2 + bx) * kRtBoxBytes, mt * kTileM + bx * 64, y0 + h * 128);
-    asm volatile("cp.async.bulk.commit_group;" ::: "memory");
-    asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
-  }
-  // loss of the rows whose label falls in this CTA's classes
-  float l = (ok && yb >= c0 && yb < c0 + kTileN) ? (gmax + __logf(S) - zy) : 0.f;
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
-  if (lane == 0) sm.red[warp] = l;
-  cluster_sync();   // no CTA leaves while its row maxima / sums may still be read
-  if (threadIdx.x == 0)
-    a.loss_part[(static_cast<int64_t>(i) * gridDim.y + mt) * gridDim.x + q] =
-        sm.red[0] + sm.red[1] + sm.red[2] + sm.red[3];
-  teardown(sm, tmem);
+  cluster_sync();   // no CTA leaves while peers may still read its slots or arrive on its barriers
+  if (warp == 1) tmem_dealloc(tmem, 2 * kTmemCols);
 }
 
 // ----------------------------------------------------------------------------
@@ -727,7 +806,7 @@ __global__ void __launch_bounds__(kGradThreads, 1)
 
 }  // namespace
 
-size_t dense_smem_bytes() { return gemm_smem_bytes(kFwdStages); }
+size_t dense_smem_bytes() { return fwd_smem_bytes(); }
 
 size_t dense_grad_smem_bytes() { return grad_smem_bytes(); }
 
@@ -741,11 +820,43 @@ cudaError_t dense_configure() {
                               static_cast<int>(dense_grad_smem_bytes()));
 }
 
+// Clusters of `cq` forward CTAs that fit on the device at once (cached).
+static int fwd_active_clusters(int cq) {
+  static int cache[5] = {0, 0, 0, 0, 0};
+  if (cq < 1 || cq > 4) return 0;
+  if (cache[cq] == 0) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(cq, 1, 1);
+    cfg.blockDim = dim3(kFwdThreads, 1, 1);
+    cfg.dynamicSmemBytes = dense_smem_bytes();
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = cq;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, k_dense_fwd, &cfg) != cudaSuccess || n < 1) {
+      cudaGetLastError();
+      n = 1;
+    }
+    cache[cq] = n;
+  }
+  return cache[cq];
+}
+
 cudaError_t launch_dense_fwd(const CUtensorMap& tmX, const CUtensorMap& tmW, const CUtensorMap& tmR,
                              const DenseFwdArgs& f, int N, cudaStream_t s) {
+  DenseFwdArgs fa = f;
+  fa.N = N;
+  const int row_tiles = N * (f.B / kTileM);
+  int clusters = fwd_active_clusters(f.Cq);
+  if (clusters > row_tiles) clusters = row_tiles;
+  if (clusters < 1) return cudaSuccess;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(f.Cq, f.B / kTileM, N);
-  cfg.blockDim = dim3(kDenseThreads, 1, 1);
+  cfg.gridDim = dim3(f.Cq * clusters, 1, 1);
+  cfg.blockDim = dim3(kFwdThreads, 1, 1);
   cfg.dynamicSmemBytes = dense_smem_bytes();
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
@@ -755,7 +866,7 @@ cudaError_t launch_dense_fwd(const CUtensorMap& tmX, const CUtensorMap& tmW, con
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, k_dense_fwd, tmX, tmW, tmR, f);
+  return cudaLaunchKernelEx(&cfg, k_dense_fwd, tmX, tmW, tmR, fa);
 }
 
 cudaError_t launch_dense_grad(const CUtensorMap& tmR, const CUtensorMap& tmXT, const CUtensorMap& tmWf,

@@ -1136,7 +1136,7 @@ asap_status asap_local_step(asap_ctx* c) {
     g.round = static_cast<unsigned>(r);
     c->skip_notify = -1;
     time_begin(c, ASAP_KERNEL_DENSE_FWD);
-    CU(launch_dense_fwd(c->tmX, c->tmWbf[r & 1], c->tmR, f, c->N, c->stream), "launching the dense forward kernel");
+    CU(launch_dense_fwd(c->tmX, c->tmWbf[r & 1], f, c->N, c->stream), "launching the dense forward kernel");
     time_end(c);
     time_begin(c, ASAP_KERNEL_DENSE_GRAD);
     CU(launch_dense_grad(c->tmR, c->tmXT, c->tmWf[r & 1], g, c->N, c->sm_count, c->stream),

@@ -159,8 +159,8 @@ cudaError_t mix_configure(bool complete, bool fused, int kp1, bool shadow, size_
 cudaError_t mix_occupancy(bool complete, bool fused, int kp1, bool shadow, size_t smem, int* blocks);
 size_t dense_smem_bytes();
 cudaError_t dense_configure();
-cudaError_t launch_dense_fwd(const CUtensorMap& tmX, const CUtensorMap& tmW, const CUtensorMap& tmR,
-                             const DenseFwdArgs& f, int N, cudaStream_t s);
+cudaError_t launch_dense_fwd(const CUtensorMap& tmX, const CUtensorMap& tmW, const DenseFwdArgs& f, int N,
+                             cudaStream_t s);
 cudaError_t launch_dense_grad(const CUtensorMap& tmR, const CUtensorMap& tmXT, const CUtensorMap& tmWf,
                               const DenseGradArgs& g, int N, int sm_count, cudaStream_t s);
 cudaError_t launch_cast_bf16(const float* src, uint16_t* dst, int64_t n, cudaStream_t s);

@@ -38,12 +38,11 @@ constexpr int kTileM = 128;
 constexpr int kTileN = 256;
 constexpr int kTileK = 64;                  // one 128-byte swizzle row of bf16
 // Operand stages of the TMA -> tcgen05 rings (48 KB each).
-constexpr int kFwdStages = 3;
+constexpr int kFwdStages = 4;
 constexpr int kGradStages = 2;
 constexpr uint32_t kABytes = kTileM * kTileK * 2;   // 16 KB
 constexpr uint32_t kBBytes = kTileN * kTileK * 2;   // 32 KB
 constexpr uint32_t kTmemCols = 256;
-constexpr uint32_t kRtBoxBytes = 128 * 64 * 2;      // R^T box: 128 classes x 64 batch rows of bf16 (16 KB)
 // Gradient epilogue: the fp32 master tile [128 classes x 256 features] passes
 // through shared memory as 8 chunks of 32 columns (128-byte swizzled rows).
 constexpr int kWBoxCols = 32;
@@ -97,11 +96,6 @@ __device__ __forceinline__ void tma_3d(void* dst, const CUtensorMap* m, uint64_t
       "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], [%5];"
       :: "r"(smem_u32(dst)), "l"(reinterpret_cast<uint64_t>(m)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar))
       : "memory");
-}
-
-__device__ __forceinline__ void tma_store_2d(const CUtensorMap* m, const void* src, int x, int y) {
-  asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];"
-               :: "l"(reinterpret_cast<uint64_t>(m)), "r"(x), "r"(y), "r"(smem_u32(src)) : "memory");
 }
 
 __device__ __forceinline__ void tma_store_3d(const CUtensorMap* m, const void* src, int x, int y, int z) {
@@ -252,7 +246,7 @@ __device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, %0;" :: "n
 //               a release arrival on that CTA's "full" mbarrier; "free"
 //               mbarriers guard a slot's reuse), so that the combination
 //               reads local shared memory; then R = (softmax - onehot) / B is
-//               staged as the R^T tile and written by TMA.
+//               written to R^T from registers.
 constexpr int kFwdThreads = (2 + kEpiWarps) * 32;
 constexpr int kMaxCq = 4;                                       // C <= 1024
 constexpr int kStatsSlot = kMaxCq * kEpiParts * 2 * kTileM;     // floats per stats slot
@@ -260,7 +254,6 @@ constexpr int kStatsSlot = kMaxCq * kEpiParts * 2 * kTileM;     // floats per st
 struct FwdSmem {
   unsigned char* a;      // kFwdStages x kABytes
   unsigned char* b;      // kFwdStages x kBBytes
-  unsigned char* rt;     // R^T tile staging: 4 boxes of kRtBoxBytes
   float* stats;          // [2 slots][kMaxCq source CTAs][kEpiParts][2: m, s][128 rows]
   uint64_t* full;        // [kFwdStages]
   uint64_t* empty;       // [kFwdStages]
@@ -273,8 +266,7 @@ struct FwdSmem {
 };
 
 constexpr size_t fwd_smem_bytes() {
-  return 1024 + static_cast<size_t>(kFwdStages) * (kABytes + kBBytes) + 4 * static_cast<size_t>(kRtBoxBytes) +
-         4 * kStatsSlot * 2 + 8 * (2 * kFwdStages + 8) + 16 + 4 * kEpiWarps;
+  return 1024 + static_cast<size_t>(kFwdStages) * (kABytes + kBBytes) + 4 * kStatsSlot * 2 + 8 * (2 * kFwdStages + 8) + 16 + 4 * kEpiWarps;
 }
 
 __device__ __forceinline__ FwdSmem fwd_carve(unsigned char* raw) {
@@ -284,8 +276,6 @@ __device__ __forceinline__ FwdSmem fwd_carve(unsigned char* raw) {
   p += kFwdStages * kABytes;
   s.b = reinterpret_cast<unsigned char*>(p);
   p += kFwdStages * kBBytes;
-  s.rt = reinterpret_cast<unsigned char*>(p);
-  p += 4 * kRtBoxBytes;
   s.stats = reinterpret_cast<float*>(p);
   p += 4 * kStatsSlot * 2;
   s.full = reinterpret_cast<uint64_t*>(p);
@@ -302,8 +292,7 @@ __device__ __forceinline__ FwdSmem fwd_carve(unsigned char* raw) {
 }
 
 __global__ void __launch_bounds__(kFwdThreads, 1)
-    k_dense_fwd(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmW,
-                const __grid_constant__ CUtensorMap tmR, DenseFwdArgs a) {
+    k_dense_fwd(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmW, DenseFwdArgs a) {
   extern __shared__ unsigned char smem_raw[];
   const FwdSmem sm = fwd_carve(smem_raw);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -399,8 +388,6 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
     const int r = quarter * 32 + lane;                          // row within the tile
     const int ch0 = part * kEpiChunks;
     const bool issuer = ew == 0 && lane == 0;
-    const int jb = r & 63;                                      // row within its R^T box
-    unsigned char* rt_col = sm.rt + (r >> 6) * kRtBoxBytes + ((jb & 7) << 1);
     float v[32];
     for (int n = 0; n < n_my; ++n) {
       const int ab = n & 1, slot = n & 1;
@@ -466,8 +453,10 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
       if (lane == 0)
         for (int p = 0; p < Cq; ++p) mbar_arrive_cluster_relaxed(sm.st_free + slot, static_cast<uint32_t>(p));
       const float invS = 1.0f / S;
-      // R^T tile in the staging boxes (the previous tile's store has read them:
-      // the issuer waited for that before the barrier at the top of this tile).
+      // R^T: this thread's row of the tile, class after class (a warp writes 64
+      // contiguous bytes per class).
+      __nv_bfloat16* rt = reinterpret_cast<__nv_bfloat16*>(a.RT) +
+                          (static_cast<int64_t>(i) * Cq * kTileN + c0) * a.B + mt * kTileM + r;
       for (int ch = ch0; ch < ch0 + kEpiChunks; ++ch) {
         tmem_ld32(trow + ch * 32, v);
 #pragma unroll
@@ -475,9 +464,7 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
           const int cl = ch * 32 + j, c = c0 + cl;
           float rv = 0.f;
           if (c < a.C) rv = (__expf(v[j] - gmax) * invS - (c == yb ? 1.f : 0.f)) * a.inv_B;
-          const int row = cl & 127;
-          *reinterpret_cast<__nv_bfloat16*>(rt_col + (cl >> 7) * 2 * kRtBoxBytes + row * 128 +
-                                            (((jb >> 3) ^ (row & 7)) << 4)) = __float2bfloat16_rn(rv);
+          rt[static_cast<int64_t>(cl) * a.B] = __float2bfloat16_rn(rv);
         }
       }
       // The accumulator is free for tile n+2.
@@ -491,21 +478,14 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
       if (lane == 0) sm.red[ew] = l;
-      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");   // the staged tile is visible to TMA
       epi_bar();
       if (issuer) {
-        const int y0 = i * Cq * kTileN + c0;                       // R^T row of this tile's first class
-        for (int h = 0; h < 2; ++h)
-          for (int bx = 0; bx < 2; ++bx)
-            tma_store_2d(&tmR, sm.rt + (h * 2 + bx) * kRtBoxBytes, mt * kTileM + bx * 64, y0 + h * 128);
-        asm volatile("cp.async.bulk.commit_group;" ::: "memory");
         float lt = 0.f;
         for (int w2 = 0; w2 < kEpiWarps; ++w2) lt += sm.red[w2];
         a.loss_part[(static_cast<int64_t>(i) * MT + mt) * Cq + q] = lt;
-        asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");   // staging boxes reusable
       }
+      epi_bar();   // sm.red is rewritten by the next tile
     }
-    if (issuer) asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
   }
   tc_fence_before();
   __syncthreads();
@@ -846,8 +826,8 @@ static int fwd_active_clusters(int cq) {
   return cache[cq];
 }
 
-cudaError_t launch_dense_fwd(const CUtensorMap& tmX, const CUtensorMap& tmW, const CUtensorMap& tmR,
-                             const DenseFwdArgs& f, int N, cudaStream_t s) {
+cudaError_t launch_dense_fwd(const CUtensorMap& tmX, const CUtensorMap& tmW, const DenseFwdArgs& f, int N,
+                             cudaStream_t s) {
   DenseFwdArgs fa = f;
   fa.N = N;
   const int row_tiles = N * (f.B / kTileM);
@@ -866,7 +846,7 @@ cudaError_t launch_dense_fwd(const CUtensorMap& tmX, const CUtensorMap& tmW, con
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, k_dense_fwd, tmX, tmW, tmR, fa);
+  return cudaLaunchKernelEx(&cfg, k_dense_fwd, tmX, tmW, fa);
 }
 
 cudaError_t launch_dense_grad(const CUtensorMap& tmR, const CUtensorMap& tmXT, const CUtensorMap& tmWf,

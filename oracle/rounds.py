@@ -30,30 +30,41 @@ def graph_schedule(kind: str, N: int, k: int, graph_seed: int = 0, regenerate: b
     return lambda rnd: graphs.build_graph(kind, N, k, graph_seed, rnd)
 
 
-def sparse_round(W, shards, t, B, loss, lr, nbr, wgt, l2=0.0, flips=None):
+def sparse_round(W, shards, t, B, loss, lr, nbr, wgt, l2=0.0, flips=None, tau=1, lr_at=None):
     """One round from W_t (any float array [N, d]); returns
-    (W_{t+1} fp64, mean loss at W_t, consensus error of W_{t+1})."""
+    (W_{t+1} fp64, mean minibatch loss, consensus error of W_{t+1}).
+
+    Each worker takes ``tau`` local steps before the reduce (Section 4: the
+    replicas communicate after processing a few examples): step j of round t
+    is global step k = t*tau + j, on minibatch k and at rate lr_at(k) (``lr``
+    when lr_at is None).  The loss is the workers' mean minibatch loss of the
+    round's last step, at its pre-step model.  ``flips`` maps a worker to the
+    hinge rows of its last step whose subgradient branch is inverted."""
     N = W.shape[0]
     H = np.empty(W.shape, dtype=np.float64)
     losses = []
     for i in range(N):
-        h, lval, _ = sgd.sparse_worker_step(
-            np.asarray(W[i], dtype=np.float64), shards.rowptr[i], shards.col[i], shards.val[i],
-            shards.y[i], t, B, loss, lr, l2, (flips or {}).get(i, ()))
+        h = np.asarray(W[i], dtype=np.float64)
+        for j in range(tau):
+            k = t * tau + j
+            eta = lr if lr_at is None else lr_at(k)
+            fl = (flips or {}).get(i, ()) if j == tau - 1 else ()
+            h, lval, _ = sgd.sparse_worker_step(h, shards.rowptr[i], shards.col[i], shards.val[i],
+                                                shards.y[i], k, B, loss, eta, l2, fl)
         H[i] = h
         losses.append(lval)
     Wn = reduce.stochastic_reduce(H, nbr, wgt)
     return Wn, float(np.mean(losses)), reduce.consensus_error(Wn)
 
 
-def run_sparse(shards, T, B, loss, lr, graph, W0=None, l2=0.0, t0=0):
+def run_sparse(shards, T, B, loss, lr, graph, W0=None, l2=0.0, t0=0, tau=1, lr_at=None):
     """Free-running trajectory: returns (W_T fp64, losses[T], consensus[T])."""
     N, d = shards.N, shards.d
     W = np.zeros((N, d)) if W0 is None else np.asarray(W0, dtype=np.float64)
     losses, cons = [], []
     for t in range(t0, t0 + T):
         nbr, wgt = graph(t)
-        W, lval, c = sparse_round(W, shards, t, B, loss, lr, nbr, wgt, l2)
+        W, lval, c = sparse_round(W, shards, t, B, loss, lr, nbr, wgt, l2, tau=tau, lr_at=lr_at)
         losses.append(lval)
         cons.append(c)
     return W, np.array(losses), np.array(cons)

@@ -71,6 +71,17 @@ def sparse_gradient(rowptr, col, val, r, b0, B, d):
     return np.bincount(col[lo:hi], weights=r[row_of] * val[lo:hi].astype(np.float64), minlength=d) / B
 
 
+def learning_rate(kind: str, eta0: float, gamma: float, k: int) -> float:
+    """eta_k of local step k (Eq. A.1 writes the rate as eta_t): ``constant``
+    keeps eta0; ``inverse`` is eta0 / (1 + gamma k), the decreasing rate of
+    Bottou's SVM-SGD, which the paper's SVM experiments use (Section 5)."""
+    if kind == "constant":
+        return float(eta0)
+    if kind == "inverse":
+        return float(eta0) / (1.0 + float(gamma) * k)
+    raise ValueError("unknown learning-rate schedule %r" % kind)
+
+
 def local_step(w, g, lr, l2=0.0):
     """Eq. A.1 first line, with an optional L2 term in f_i."""
     w = np.asarray(w, dtype=np.float64)

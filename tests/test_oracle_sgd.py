@@ -11,6 +11,9 @@
 * Eq. A.2: with d = 1, w_0 = 0 and a fixed gradient sequence,
   w_t = -sum_k eta_k P^{t-k} g_k, which fixes the order "SGD, then reduce".
 * The early-exit permutation sampler is uniform over admissible layers.
+* Learning-rate schedules at literal values; two local steps per round by
+  hand (inverse rate, with and without L2); one worker with tau local steps
+  equals textbook minibatch SGD over the global step sequence.
 """
 import itertools
 import math
@@ -229,3 +232,51 @@ def test_admissible_layer_sampler_is_uniform():
     exp = accepted / len(admissible)
     chi2 = sum((c - exp) ** 2 / exp for c in counts.values())
     assert chi2 < 25.0
+
+
+def test_learning_rate_schedules():
+    assert [sgd.learning_rate("constant", 0.3, 7.0, k) for k in (0, 1, 50)] == [0.3, 0.3, 0.3]
+    # eta0 / (1 + gamma k) with eta0 = 0.5, gamma = 0.25
+    assert [sgd.learning_rate("inverse", 0.5, 0.25, k) for k in (0, 4, 12)] == [0.5, 0.25, 0.125]
+    with pytest.raises(ValueError):
+        sgd.learning_rate("step", 0.5, 0.1, 0)
+
+
+def test_hand_computed_two_local_steps_per_round():
+    # One worker, rows x0 = {0: 1} (y=+1), x1 = {1: 2} (y=-1), B = 1, tau = 2,
+    # eta_k = 0.5 / (1 + k): eta_0 = 0.5 on row 0, eta_1 = 0.25 on row 1.
+    # step 0: m = 0, y m = 0 < 1 -> r = -1, g = [-1, 0] -> w = [0.5, 0]
+    # step 1: m = 2 * 0 = 0, y m = 0 < 1 -> r = +1, g = [0, 2] -> w = [0.5, -0.5]
+    # with l2 = 0.2: step 1 scales w by (1 - 0.25 * 0.2) = 0.95 first: [0.475, -0.5]
+    sh = inputs.SparseShards(d=2)
+    sh.rowptr.append(np.array([0, 1, 2], np.int64))
+    sh.col.append(np.array([0, 1], np.int32))
+    sh.val.append(np.array([1.0, 2.0], np.float32))
+    sh.y.append(np.array([1.0, -1.0], np.float32))
+    sched = rounds.graph_schedule("identity", 1, 0)
+    lr_at = lambda k: sgd.learning_rate("inverse", 0.5, 1.0, k)
+    W, losses, _ = rounds.run_sparse(sh, 1, 1, "hinge", None, sched, tau=2, lr_at=lr_at)
+    assert W[0] == pytest.approx([0.5, -0.5], abs=1e-15)
+    assert losses[0] == pytest.approx(1.0, abs=1e-15)      # the last step's loss: max(0, 1 - 0)
+    W, _, _ = rounds.run_sparse(sh, 1, 1, "hinge", None, sched, l2=0.2, tau=2, lr_at=lr_at)
+    assert W[0] == pytest.approx([0.475, -0.5], abs=1e-15)
+
+
+def test_local_steps_are_textbook_sgd_over_global_steps():
+    sh = inputs.sparse_custom(seed=5, N=1, d=20, rows=60, max_len=8)
+    B, tau, T, eta0, gamma = 10, 3, 4, 0.4, 0.2
+    sched = rounds.graph_schedule("identity", 1, 0)
+    lr_at = lambda k: sgd.learning_rate("inverse", eta0, gamma, k)
+    Wo, _, _ = rounds.run_sparse(sh, T, B, "logistic", None, sched, tau=tau, lr_at=lr_at)
+    Xd = np.zeros((60, 20))
+    for r in range(60):
+        a, b = sh.rowptr[0][r], sh.rowptr[0][r + 1]
+        Xd[r, sh.col[0][a:b]] = sh.val[0][a:b]
+    y = sh.y[0].astype(np.float64)
+    w = np.zeros(20)
+    for k in range(T * tau):                     # global step k: minibatch k mod 6, rate eta0 / (1 + gamma k)
+        b0 = (k % 6) * B
+        Xb, yb = Xd[b0:b0 + B], y[b0:b0 + B]
+        s = 1.0 / (1.0 + np.exp(yb * (Xb @ w)))
+        w = w - eta0 / (1.0 + gamma * k) / B * (Xb.T @ (-yb * s))
+    assert Wo[0] == pytest.approx(w, abs=1e-14)

@@ -118,6 +118,25 @@ asap_status asap_set_mixing(asap_ctx* ctx, const int32_t* nbr, const float* wgt)
  * model clears the shards and resets W to 0. */
 asap_status asap_set_model(asap_ctx* ctx, asap_loss loss, int num_classes, int batch, float lr, float l2);
 
+/* Learning-rate schedules for asap_set_schedule. */
+typedef enum {
+  ASAP_LR_CONSTANT = 0, /* eta_k = lr                                   */
+  ASAP_LR_INVERSE = 1   /* eta_k = lr / (1 + gamma k)  (Bottou's SVM-SGD) */
+} asap_lr_schedule;
+
+/* Local steps per round and the learning-rate schedule.  Eq. A.1 writes the
+ * rate as eta_t; Section 4 has the replicas exchange parameters "after
+ * processing a few data examples".  Each round runs local_steps (>= 1)
+ * minibatch steps per worker before the reduce: step j of round t is global
+ * step k = t * local_steps + j, on minibatch k mod nb, at rate eta_k;
+ * asap_local_step runs all of them and the round's loss metric is its last
+ * step's.  The L2 shrink of the intermediate steps is kept as one scale per
+ * round (all workers take the same steps) and applied in the reduce.
+ * SOFTMAX models take the schedule with local_steps = 1 only.  Defaults:
+ * 1, ASAP_LR_CONSTANT.  Keeps W, shards and the round counter; the
+ * minibatch of a round follows the new local_steps from the next call on. */
+asap_status asap_set_schedule(asap_ctx* ctx, int local_steps, asap_lr_schedule kind, float gamma);
+
 /* Stream for all device work of this context (a cudaStream_t, e.g.
  * torch.cuda.current_stream().cuda_stream).  NULL selects the context's own
  * non-blocking stream (the default). */

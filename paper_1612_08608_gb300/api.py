@@ -14,6 +14,7 @@ STATUS = {0: "ASAP_OK", 1: "ASAP_ERR_ARG", 2: "ASAP_ERR_CUDA", 3: "ASAP_ERR_OOM"
 GRAPH = {"ring": 1, "root": 2, "random_regular": 3, "complete": 4, "explicit": 5, "identity": 6}
 LOSS = {"none": 0, "hinge": 1, "logistic": 2, "softmax": 3}
 RESIDENCY = {"device": 0, "host": 1}
+LR_SCHEDULE = {"constant": 0, "inverse": 1}
 
 
 class AsapError(RuntimeError):
@@ -72,6 +73,12 @@ class Context:
     def set_model(self, loss: str, batch: int, lr: float, num_classes: int = 1, l2: float = 0.0):
         self._c(self._lib.asap_set_model(self._h, LOSS[loss], num_classes, batch, lr, l2))
         self.P = self.d * (num_classes if loss == "softmax" else 1)
+
+    def set_schedule(self, local_steps: int = 1, lr_schedule: str = "constant", gamma: float = 0.0):
+        """local_steps minibatch steps per worker per round; learning rate
+        ``constant`` (eta_k = lr) or ``inverse`` (eta_k = lr / (1 + gamma k)),
+        k = round * local_steps + step."""
+        self._c(self._lib.asap_set_schedule(self._h, int(local_steps), LR_SCHEDULE[lr_schedule], float(gamma)))
 
     def set_stream(self, stream):
         """stream: a torch.cuda.Stream, an integer cudaStream_t, or None."""

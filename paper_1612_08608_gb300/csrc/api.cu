@@ -70,6 +70,14 @@ struct asap_ctx {
   asap_loss loss = ASAP_LOSS_NONE;
   int C = 1, B = 0;
   float lr = 0.f, l2 = 0.f;
+  // schedule: local steps per round, eta_k = lr (constant) or lr / (1 + gamma k)
+  int tau = 1;
+  int lr_kind = ASAP_LR_CONSTANT;
+  float lr_gamma = 0.f;
+  // left by the last local step for the fused reduce
+  float pend_wscale = 1.f;          // true w = pend_wscale * stored values
+  float pend_upd = 0.f;             // eta / (B pend_wscale)
+  int64_t pend_k = 0;               // global step of the last local step
   int64_t P = 0, ld = 0;
 
   float* W[2] = {nullptr, nullptr};
@@ -107,7 +115,7 @@ struct asap_ctx {
   int64_t max_list = 0;
   float* wv = nullptr;              // w at the current round's list positions
   float* gsum = nullptr;            // column sums at the current round's list positions
-  int64_t wv_round = -1;            // round whose list wv holds (-1: none)
+  int64_t wv_step = -1;             // global local step whose column list wv holds (-1: none)
   // host residency: a round reads its own block and the next one
   static constexpr int kStaging = 3;
   unsigned char* staging[kStaging] = {nullptr, nullptr, nullptr};
@@ -209,7 +217,7 @@ void free_shards(asap_ctx* c) {
   c->list_len.clear();
   c->max_region = 0;
   c->max_list = 0;
-  c->wv_round = -1;
+  c->wv_step = -1;
   c->nb = 0;
 }
 
@@ -464,6 +472,12 @@ asap_status sync_all(asap_ctx* c) {
 // Make round r's batch block available on the device (host residency).
 // Slot r % 3; a slot is rewritten only after the last kernel that reads its
 // previous block (the reduce of that block's own round) has finished.
+// eta_k of global local step k.
+float lr_at(const asap_ctx* c, int64_t k) {
+  if (c->lr_kind == ASAP_LR_INVERSE) return static_cast<float>(c->lr / (1.0 + c->lr_gamma * static_cast<double>(k)));
+  return c->lr;
+}
+
 asap_status stage_block(asap_ctx* c, int64_t r) {
   const int slot = static_cast<int>(r % asap_ctx::kStaging);
   if (c->staged_round[slot] == r) return ASAP_OK;
@@ -720,6 +734,21 @@ asap_status asap_set_model(asap_ctx* c, asap_loss loss, int num_classes, int bat
   }
   if (c->n_loss_part > 0)
     CU(cudaMalloc(&c->loss_part, 4 * static_cast<size_t>(c->n_loss_part)), "allocating step scratch");
+  return ASAP_OK;
+}
+
+asap_status asap_set_schedule(asap_ctx* c, int local_steps, asap_lr_schedule kind, float gamma) {
+  if (!c) return fail(nullptr, ASAP_ERR_ARG, "ctx is NULL");
+  if (local_steps < 1 || local_steps > 4096) return fail(c, ASAP_ERR_ARG, "local_steps must be in [1, 4096]");
+  if (kind != ASAP_LR_CONSTANT && kind != ASAP_LR_INVERSE) return fail(c, ASAP_ERR_ARG, "unknown schedule");
+  if (!(gamma >= 0.f) || !std::isfinite(gamma)) return fail(c, ASAP_ERR_ARG, "gamma must be finite and >= 0");
+  if (c->step_pending) return fail(c, ASAP_ERR_ARG, "a local step is pending: reduce first");
+  if (c->loss == ASAP_LOSS_SOFTMAX && local_steps != 1)
+    return fail(c, ASAP_ERR_ARG, "softmax models take one local step per round");
+  c->tau = local_steps;
+  c->lr_kind = kind;
+  c->lr_gamma = gamma;
+  c->wv_step = -1;   // the step numbering may change: gather at the next step
   return ASAP_OK;
 }
 
@@ -1021,7 +1050,7 @@ asap_status asap_load_shards(asap_ctx* c, const int64_t* const* rowptr, const in
   c->max_nnz = max_nnz;
   c->max_region = max_region;
   c->max_list = max_list;
-  c->wv_round = -1;
+  c->wv_step = -1;
   c->update_ctas = update_ctas_for(max_nnz);
   c->configured_key = -1;
   return ASAP_OK;
@@ -1103,6 +1132,7 @@ asap_status asap_local_step(asap_ctx* c) {
   const int64_t r = c->round;
   const int t = static_cast<int>(r % c->nb);
   if (c->loss == ASAP_LOSS_SOFTMAX) {
+    if (c->tau != 1) return fail(c, ASAP_ERR_ARG, "softmax models take one local step per round");
     asap_status sg = prepare_graph(c, r);
     if (sg != ASAP_OK) return sg;
     DenseFwdArgs f;
@@ -1127,8 +1157,9 @@ asap_status asap_local_step(asap_ctx* c) {
     g.t = t;
     g.W = c->W[r & 1];
     g.ld = c->ld;
-    g.lr = c->lr;
-    g.decay = 1.0f - c->lr * c->l2;
+    const float eta = lr_at(c, r);
+    g.lr = eta;
+    g.decay = 1.0f - eta * c->l2;
     g.ready = c->ready;
     g.worker_ticket = c->ticket;
     g.skip_worker = c->skip_notify;
@@ -1146,41 +1177,78 @@ asap_status asap_local_step(asap_ctx* c) {
     c->step_pending = true;
     return ASAP_OK;
   }
-  const unsigned char* block = nullptr;
-  asap_status sb = block_of(c, r, &block);
-  if (sb != ASAP_OK) return sb;
-  if (c->wv_round != r) {
-    // No exported w values for this round's columns (parameters came from
-    // the host): gather them once.
-    CU(launch_gather_wv(c->W[r & 1], c->ld, reinterpret_cast<const uint32_t*>(block + c->list_off[t]),
-                        reinterpret_cast<const int*>(block + c->soff_off[t]), c->n_slabs, c->S, c->wv, c->sm_count,
-                        c->stream),
-       "launching the gather kernel");
-    c->launches += 1;
-    c->wv_round = r;
+  // tau local steps: step j is global step k = r tau + j on minibatch k mod nb.
+  // L2 shrinks every worker's w by the same (1 - eta_k l2) per step, kept as
+  // one scale s (true w = s * stored values) until the reduce applies it.
+  float s_scale = 1.0f;
+  for (int j = 0; j < c->tau; ++j) {
+    const int64_t k = r * c->tau + j;
+    const int tk = static_cast<int>(k % c->nb);
+    const bool last = j == c->tau - 1;
+    const unsigned char* block = nullptr;
+    asap_status sb = block_of(c, k, &block);
+    if (sb != ASAP_OK) return sb;
+    if (c->wv_step != k) {
+      // No exported w values for this step's columns (parameters came from
+      // the host, or an earlier local step of the round changed them): gather.
+      CU(launch_gather_wv(c->W[r & 1], c->ld, reinterpret_cast<const uint32_t*>(block + c->list_off[tk]),
+                          reinterpret_cast<const int*>(block + c->soff_off[tk]), c->n_slabs, c->S, c->wv,
+                          c->sm_count, c->stream),
+         "launching the gather kernel");
+      c->launches += 1;
+      c->wv_step = k;
+    }
+    SparseStepArgs a;
+    a.block = block;
+    a.desc = c->d_desc + static_cast<size_t>(tk) * c->N;
+    a.wv = c->wv;
+    a.gsum = c->gsum;
+    a.r = c->r_scr;
+    a.loss_part = c->loss_part;
+    a.ready = c->ready;
+    a.worker_ticket = c->ticket;
+    a.B = c->B;
+    a.round = static_cast<unsigned>(r);
+    a.mscale = s_scale;
+    a.notify = last ? 1 : 0;
+    a.skip_worker = last ? c->skip_notify : -1;
+    if (last) {
+      c->skip_notify = -1;
+      asap_status sg = prepare_graph(c, r);   // upload a regenerated graph ahead of the reduce
+      if (sg != ASAP_OK) return sg;
+    }
+    time_begin(c, ASAP_KERNEL_MARGIN);
+    CU(launch_margin(a, c->N, c->loss, c->margin_ctas, c->stream), "launching the margin kernel");
+    time_end(c);
+    time_begin(c, ASAP_KERNEL_UPDATE);
+    CU(launch_update(a, c->N, c->update_ctas, c->stream), "launching the update kernel");
+    time_end(c);
+    c->launches += 2;
+    const float eta = lr_at(c, k);
+    const float s_next = s_scale * (1.0f - eta * c->l2);
+    const float upd = eta / (static_cast<float>(c->B) * s_next);
+    if (!last) {
+      // w_stored -= eta / (B s') g at the step's columns; the reduce applies
+      // the round's last update itself.
+      CU(launch_apply_update(c->W[r & 1], c->ld, reinterpret_cast<const uint32_t*>(block + c->list_off[tk]),
+                             reinterpret_cast<const int*>(block + c->soff_off[tk]), c->n_slabs, c->S, c->gsum, upd,
+                             c->sm_count, c->stream),
+         "launching the local update kernel");
+      c->launches += 1;
+      if (c->residency == ASAP_SHARDS_HOST) {
+        const int slot = static_cast<int>(k % asap_ctx::kStaging);
+        CU(cudaEventRecord(c->free_ev[slot], c->stream), "staging event");   // block k is no longer read
+        c->free_recorded[slot] = true;
+        asap_status ss = stage_block(c, k + 2);                                 // prefetch
+        if (ss != ASAP_OK) return ss;
+      }
+    } else {
+      c->pend_wscale = s_next;
+      c->pend_upd = upd;
+      c->pend_k = k;
+    }
+    s_scale = s_next;
   }
-  SparseStepArgs a;
-  a.block = block;
-  a.desc = c->d_desc + static_cast<size_t>(t) * c->N;
-  a.wv = c->wv;
-  a.gsum = c->gsum;
-  a.r = c->r_scr;
-  a.loss_part = c->loss_part;
-  a.ready = c->ready;
-  a.worker_ticket = c->ticket;
-  a.B = c->B;
-  a.round = static_cast<unsigned>(r);
-  a.skip_worker = c->skip_notify;
-  c->skip_notify = -1;
-  asap_status sg = prepare_graph(c, r);   // upload a regenerated graph ahead of the reduce
-  if (sg != ASAP_OK) return sg;
-  time_begin(c, ASAP_KERNEL_MARGIN);
-  CU(launch_margin(a, c->N, c->loss, c->margin_ctas, c->stream), "launching the margin kernel");
-  time_end(c);
-  time_begin(c, ASAP_KERNEL_UPDATE);
-  CU(launch_update(a, c->N, c->update_ctas, c->stream), "launching the update kernel");
-  time_end(c);
-  c->launches += 2;
   c->step_pending = true;
   return ASAP_OK;
 }
@@ -1206,7 +1274,7 @@ asap_status asap_stochastic_reduce(asap_ctx* c) {
   a.kp1 = c->tab_kp1;
   a.nbr = nbr;
   a.wgt = wgt;
-  a.wscale = (c->step_pending && sparse) ? (1.0f - c->lr * c->l2) : 1.0f;
+  a.wscale = (c->step_pending && sparse) ? c->pend_wscale : 1.0f;
   a.uniform_w = uniform;
   a.S = c->S;
   a.rows_pad = c->rows_pad;
@@ -1217,15 +1285,16 @@ asap_status asap_stochastic_reduce(asap_ctx* c) {
   if (fused) {
     const unsigned char* bt = nullptr;
     const unsigned char* bn = nullptr;
-    s = block_of(c, r, &bt);
+    const int64_t kl = c->pend_k;            // the round's last local step; the next round starts at kl + 1
+    s = block_of(c, kl, &bt);
     if (s != ASAP_OK) return s;
-    s = block_of(c, r + 1, &bn);
+    s = block_of(c, kl + 1, &bn);
     if (s != ASAP_OK) return s;
-    const int t = static_cast<int>(r % c->nb), tn = static_cast<int>((r + 1) % c->nb);
+    const int t = static_cast<int>(kl % c->nb), tn = static_cast<int>((kl + 1) % c->nb);
     a.upd_list = reinterpret_cast<const uint32_t*>(bt + c->list_off[t]);
     a.upd_off = reinterpret_cast<const int*>(bt + c->soff_off[t]);
     a.gsum = c->gsum;
-    a.upd_scale = c->lr / (static_cast<float>(c->B) * (1.0f - c->lr * c->l2));
+    a.upd_scale = c->pend_upd;
     a.exp_list = reinterpret_cast<const uint32_t*>(bn + c->list_off[tn]);
     a.exp_off = reinterpret_cast<const int*>(bn + c->soff_off[tn]);
     a.wv_out = c->wv;
@@ -1250,12 +1319,12 @@ asap_status asap_stochastic_reduce(asap_ctx* c) {
      "launching the stochastic reduce");
   time_end(c);
   c->launches += 1;
-  c->wv_round = fused ? r + 1 : -1;
+  c->wv_step = fused ? c->pend_k + 1 : -1;
   if (fused && c->residency == ASAP_SHARDS_HOST) {
-    const int slot = static_cast<int>(r % asap_ctx::kStaging);
-    CU(cudaEventRecord(c->free_ev[slot], c->stream), "staging event");   // block r is no longer read
+    const int slot = static_cast<int>(c->pend_k % asap_ctx::kStaging);
+    CU(cudaEventRecord(c->free_ev[slot], c->stream), "staging event");   // block pend_k is no longer read
     c->free_recorded[slot] = true;
-    s = stage_block(c, r + 2);                                            // prefetch
+    s = stage_block(c, c->pend_k + 2);                                    // prefetch
     if (s != ASAP_OK) return s;
   }
   c->round = r + 1;
@@ -1303,7 +1372,7 @@ asap_status asap_write_params(asap_ctx* c, const float* host_in, int64_t round) 
     c->launches += 1;
     CU(cudaStreamSynchronize(c->stream), "bf16 copy");
   }
-  c->wv_round = -1;
+  c->wv_step = -1;
   return reset_protocol(c, round);
 }
 

@@ -68,6 +68,8 @@ struct SparseStepArgs {
   int B;
   unsigned int round;
   int skip_worker;             // fault injection: do not NOTIFY this worker
+  float mscale;                // true w = mscale * (stored values): margins are scaled by it
+  int notify;                  // the column sums publish NOTIFY (last local step of the round)
 };
 
 // Arguments of the stochastic reduce.
@@ -145,6 +147,8 @@ asap_status build_graph_host(asap_graph_kind kind, int N, int k, uint64_t seed, 
 // Launchers (kernels_*.cu).  Each returns the cudaError_t of the launch.
 cudaError_t launch_margin(const SparseStepArgs& a, int N, int loss, int margin_ctas, cudaStream_t s);
 cudaError_t launch_update(const SparseStepArgs& a, int N, int update_ctas, cudaStream_t s);
+cudaError_t launch_apply_update(float* W, int64_t ld, const uint32_t* list, const int* slab_off, long long n_slabs,
+                                int S, const float* gsum, float scale, int sm_count, cudaStream_t s);
 cudaError_t launch_gather_wv(const float* W, int64_t ld, const uint32_t* list, const int* slab_off, long long n_slabs,
                              int S, float* wv, int sm_count, cudaStream_t s);
 constexpr int kMixComputeWarps = 16;

@@ -149,7 +149,7 @@ __global__ void __launch_bounds__(kThreads) k_margin_loss(SparseStepArgs a) {
   for (int o = kLanesPerRow / 2; o > 0; o >>= 1) acc += __shfl_xor_sync(kFull, acc, o);
   if (b < a.B && sl == 0) {
     float l, r;
-    loss_and_r<LOSS>(y[b], acc, l, r);
+    loss_and_r<LOSS>(y[b], acc * a.mscale, l, r);
     a.r[static_cast<int64_t>(i) * a.B + b] = r;
     lsum = l;
   }
@@ -257,7 +257,7 @@ __global__ void __launch_bounds__(kThreads) k_column_sums(SparseStepArgs a) {
     if (done == gridDim.x - 1) {
       a.worker_ticket[i] = 0u;
       __threadfence();
-      if (i != a.skip_worker) st_release_u32(&a.ready[i], a.round + 1u);
+      if (a.notify && i != a.skip_worker) st_release_u32(&a.ready[i], a.round + 1u);
     }
   }
 }
@@ -279,7 +279,34 @@ __global__ void __launch_bounds__(kThreads) k_gather_wv(const float* __restrict_
   }
 }
 
+// W[i][s*S + cl] -= scale * g[e] for every entry {i << 16 | cl} of a slab-major
+// column list: the update of a local step that is not the round's last (the
+// last one is applied inside the stochastic reduce).  The entries of a list
+// are distinct, so every parameter is written by one thread.
+__global__ void __launch_bounds__(kThreads) k_apply_update(float* __restrict__ W, int64_t ld,
+                                                          const uint32_t* __restrict__ list,
+                                                          const int* __restrict__ slab_off, long long n_slabs, int S,
+                                                          const float* __restrict__ g, float scale) {
+  for (long long s = blockIdx.x; s < n_slabs; s += gridDim.x) {
+    const int a0 = slab_off[s], a1 = slab_off[s + 1];
+    for (int e = a0 + threadIdx.x; e < a1; e += blockDim.x) {
+      const uint32_t code = list[e];
+      if (code == kListPad) continue;
+      const int i = static_cast<int>(code >> 16), cl = static_cast<int>(code & 0xffffu);
+      float* p = W + static_cast<int64_t>(i) * ld + s * S + cl;
+      *p = fmaf(-scale, g[e], *p);
+    }
+  }
+}
+
 }  // namespace
+
+cudaError_t launch_apply_update(float* W, int64_t ld, const uint32_t* list, const int* slab_off, long long n_slabs,
+                                int S, const float* gsum, float scale, int sm_count, cudaStream_t s) {
+  const int grid = static_cast<int>(n_slabs < 4LL * sm_count ? n_slabs : 4LL * sm_count);
+  k_apply_update<<<grid > 0 ? grid : 1, kThreads, 0, s>>>(W, ld, list, slab_off, n_slabs, S, gsum, scale);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_margin(const SparseStepArgs& a, int N, int loss, int margin_ctas, cudaStream_t s) {
   const dim3 g1(margin_ctas, N);

@@ -28,10 +28,11 @@ def hinge_near_ties(W, shards, t, B, tol=1e-5):
     return out
 
 
-def sparse_round_matching(W_t, W_gpu_next, shards, t, B, loss, lr, nbr, wgt, tol, l2=0.0):
+def sparse_round_matching(W_t, W_gpu_next, shards, t, B, loss, lr, nbr, wgt, tol, l2=0.0, tau=1, lr_at=None):
     """Oracle round from the GPU's W_t; on hinge corner rows accept either
-    subgradient.  Returns (rel_err, oracle loss, oracle consensus)."""
-    ties = hinge_near_ties(W_t, shards, t, B) if loss == "hinge" else {}
+    subgradient (one local step per round only).  Returns (rel_err, oracle
+    loss, oracle consensus)."""
+    ties = hinge_near_ties(W_t, shards, t, B) if (loss == "hinge" and tau == 1) else {}
     cands = [{}]
     if ties:
         flat = [(i, r) for i, rows in ties.items() for r in rows]
@@ -45,7 +46,8 @@ def sparse_round_matching(W_t, W_gpu_next, shards, t, B, loss, lr, nbr, wgt, tol
             cands.append(f)
     best = None
     for flips in cands:
-        Wn, lval, cons = rounds.sparse_round(W_t, shards, t, B, loss, lr, nbr, wgt, l2=l2, flips=flips)
+        Wn, lval, cons = rounds.sparse_round(W_t, shards, t, B, loss, lr, nbr, wgt, l2=l2, flips=flips, tau=tau,
+                                             lr_at=lr_at)
         e = rel_err_rows(W_gpu_next, Wn)
         if best is None or e < best[0]:
             best = (e, lval, cons)

@@ -29,7 +29,7 @@ def _ctx(N, d, k, seed, kind, regen, loss, B, lr, shards, explicit=None, residen
     return ctx
 
 
-def _run_parity(ctx, shards, T, B, loss, lr, sched, l2=0.0, check_graph=True):
+def _run_parity(ctx, shards, T, B, loss, lr, sched, l2=0.0, check_graph=True, tau=1, lr_at=None):
     losses_gpu = []
     W_t, _ = ctx.read_params()
     for t in range(T):
@@ -41,7 +41,7 @@ def _run_parity(ctx, shards, T, B, loss, lr, sched, l2=0.0, check_graph=True):
         W_n, rnd = ctx.read_params()
         assert rnd == t + 1
         err, lref, cref = sparse_round_matching(W_t.astype(np.float64), W_n, shards, t, B, loss, lr, nbr, wgt,
-                                                TOL, l2=l2)
+                                                TOL, l2=l2, tau=tau, lr_at=lr_at)
         assert err <= TOL, (t, err)
         lg, cg = ctx.read_metrics(t, 1)
         assert abs(lg[0] - lref) <= 1e-5 * max(1.0, abs(lref)), (t, lg[0], lref)
@@ -99,6 +99,48 @@ def test_large_minibatch(B):
     sched = rounds.graph_schedule("ring", N, 1)
     ctx = _ctx(N, d, 1, 0, "ring", False, "hinge", B, lr, sh)
     _run_parity(ctx, sh, T, B, "hinge", lr, sched)
+
+
+@pytest.mark.parametrize("residency", ["device", "host"])
+def test_local_steps_inverse_rate_l2(residency):
+    # tau = 3 local steps per round (the intermediate updates and the L2
+    # shrink kept as one scale until the reduce), eta_k = 0.5 / (1 + 0.1 k),
+    # a graph regenerated every round.
+    from oracle import sgd
+    N, d, B, T, tau, l2 = 6, 1000, 32, 4, 3, 0.05
+    sh = inputs.sparse_custom(seed=21, N=N, d=d, rows=10 * B, max_len=40, hot_col=3)
+    sched = rounds.graph_schedule("random_regular", N, 2, graph_seed=4, regenerate=True)
+    ctx = _ctx(N, d, 2, 4, "random_regular", True, "logistic", B, 0.5, sh, residency=residency, l2=l2)
+    ctx.set_schedule(local_steps=tau, lr_schedule="inverse", gamma=0.1)
+    lr_at = lambda k: sgd.learning_rate("inverse", 0.5, 0.1, k)
+    lg = _run_parity(ctx, sh, T, B, "logistic", None, sched, l2=l2, tau=tau, lr_at=lr_at)
+    _, lref, _ = rounds.run_sparse(sh, T, B, "logistic", None, sched, l2=l2, tau=tau, lr_at=lr_at)
+    assert np.abs(lg - lref).max() <= 1e-4
+    assert ctx.kernel_launches() == (4 * tau - 1) * T + 1    # margins, sums, update, gather per step
+
+
+def test_inverse_rate_hinge_one_step():
+    from oracle import sgd
+    N, d, B, T = 5, 400, 24, 5
+    sh = inputs.sparse_custom(seed=22, N=N, d=d, rows=4 * B, max_len=25)
+    sched = rounds.graph_schedule("ring", N, 1)
+    ctx = _ctx(N, d, 1, 0, "ring", False, "hinge", B, 0.8, sh)
+    ctx.set_schedule(local_steps=1, lr_schedule="inverse", gamma=0.5)
+    _run_parity(ctx, sh, T, B, "hinge", None, sched, lr_at=lambda k: sgd.learning_rate("inverse", 0.8, 0.5, k))
+
+
+def test_schedule_argument_errors():
+    from paper_1612_08608_gb300 import AsapError, Context
+    ctx = Context(4, 256, graph_seed=0, k=1)
+    ctx.set_model("softmax", batch=128, lr=0.1, num_classes=10)
+    with pytest.raises(AsapError):
+        ctx.set_schedule(local_steps=2)
+    ctx.set_schedule(local_steps=1, lr_schedule="inverse", gamma=0.2)
+    ctx.set_model("logistic", batch=16, lr=0.1)
+    with pytest.raises(AsapError):
+        ctx.set_schedule(local_steps=0)
+    with pytest.raises(AsapError):
+        ctx.set_schedule(local_steps=2, gamma=-1.0)
 
 
 def test_single_worker_and_complete_graph():

@@ -51,6 +51,7 @@ WORKLOADS = {
                           loss="softmax", graph="root", regenerate=False, graph_seed=0),
 }
 WORKLOAD = WORKLOADS["sparse_logistic_hashed"]
+SCHED = {"tau": 1, "kind": "constant", "gamma": 0.0}   # local steps per round, learning-rate schedule
 PROFILE = os.path.join(ROOT, "profiles", "stochastic_reduce_sparse_logistic_hashed.txt")
 MIX_SOURCE = os.path.join(ROOT, "paper_1612_08608_gb300", "csrc", "kernels_mix.cu")
 
@@ -65,6 +66,9 @@ def parse():
     ap.add_argument("--workload", default="sparse_logistic_hashed", choices=sorted(WORKLOADS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--local-steps", type=int, default=1, help="minibatch steps per worker per round (sparse)")
+    ap.add_argument("--lr-schedule", default="constant", choices=["constant", "inverse"])
+    ap.add_argument("--gamma", type=float, default=0.0, help="eta_k = lr / (1 + gamma k) for --lr-schedule inverse")
     return ap.parse_args()
 
 
@@ -204,28 +208,38 @@ def _sched():
     return rounds.graph_schedule(w["graph"], w["N"], w["k"], w["graph_seed"], w["regenerate"])
 
 
+def _lr_at(k):
+    from oracle import sgd
+    return sgd.learning_rate(SCHED["kind"], WORKLOAD["lr"], SCHED["gamma"], k)
+
+
 def oracle_round_sample(sh, W, t, workers):
-    """The oracle on a sample of one round: the local step and the reduce
+    """The oracle on a sample of one round: the local steps and the reduce
     row of each listed worker (neighbours' half-steps taken from W when not
     in the sample).  Returns the worker-samples processed."""
     import numpy as np
     from oracle import sgd
     w = WORKLOAD
+    tau = SCHED["tau"]
     nbr, wgt = _sched()(t)
     H = {}
     for i in workers:
         if w["loss"] == "softmax":
             Wm = W[i].astype(np.float32).reshape(w["C"], w["d"])
-            H[i] = sgd.softmax_worker_step(Wm, sh.X[i], sh.y[i], t, w["B"], w["lr"])[0].reshape(-1)
+            H[i] = sgd.softmax_worker_step(Wm, sh.X[i], sh.y[i], t, w["B"], _lr_at(t))[0].reshape(-1)
         else:
-            H[i], _, _ = sgd.sparse_worker_step(W[i], sh.rowptr[i], sh.col[i], sh.val[i], sh.y[i], t, w["B"],
-                                                w["loss"], w["lr"])
+            h = W[i]
+            for j in range(tau):
+                k = t * tau + j
+                h, _, _ = sgd.sparse_worker_step(h, sh.rowptr[i], sh.col[i], sh.val[i], sh.y[i], k, w["B"],
+                                                 w["loss"], _lr_at(k))
+            H[i] = h
     for i in workers:
         acc = np.zeros(W.shape[1])
         for m in range(nbr.shape[1]):
             j = int(nbr[i, m])
             acc += wgt[i, m] * (H[j] if j in H else W[j])
-    return len(workers) * w["B"]
+    return len(workers) * w["B"] * (1 if w["loss"] == "softmax" else tau)
 
 
 def cpu_baseline(sh):
@@ -237,12 +251,13 @@ def cpu_baseline(sh):
     W = np.zeros((w["N"], P))
     nbr, wgt = _sched()(0)
     t0 = time.perf_counter()
+    tau = 1 if w["loss"] == "softmax" else SCHED["tau"]
     if w["loss"] == "softmax":
         rounds.softmax_round(W.astype(np.float32), sh, 0, w["B"], w["lr"], nbr, wgt)
     else:
-        rounds.sparse_round(W, sh, 0, w["B"], w["loss"], w["lr"], nbr, wgt)
+        rounds.sparse_round(W, sh, 0, w["B"], w["loss"], None, nbr, wgt, tau=tau, lr_at=_lr_at)
     dt = time.perf_counter() - t0
-    return {"value": w["N"] * w["B"] / dt, "unit": "worker-samples/s", "cores": 1,
+    return {"value": w["N"] * w["B"] * tau / dt, "unit": "worker-samples/s", "cores": 1,
             "kind": "oracle", "sample": "one full round (%d workers' SGD steps, the reduce and both metrics), "
                                         "numpy fp64%s; %.1f s" % (w["N"], ", BLAS matmuls" if w["loss"] == "softmax"
                                                                    else ", single thread", dt)}
@@ -253,7 +268,9 @@ def config(rows):
     c = {"workload": w["name"], "N_workers": w["N"], "d": w["d"], "B": w["B"], "rows_per_worker": rows,
          "loss": w["loss"], "lr": w["lr"],
          "graph": "%s k=%d%s" % (w["graph"], w["k"], ", regenerated every round" if w["regenerate"] else ""),
-         "parallelism": "independent replicas, one per GPU"}
+         "parallelism": "independent replicas, one per GPU",
+         "local_steps": SCHED["tau"], "lr_schedule": SCHED["kind"] if SCHED["kind"] == "constant"
+         else "lr / (1 + %g k)" % SCHED["gamma"]}
     if "nnz" in w:
         c["nnz_per_row"] = w["nnz"]
     if "C" in w:
@@ -363,10 +380,11 @@ def run_asap(args):
     stream = torch.cuda.Stream()
     ctx = Context(w["N"], w["d"], graph_seed=w["graph_seed"], k=w["k"])
     ctx.set_model(w["loss"], batch=w["B"], lr=w["lr"], num_classes=w.get("C", 1))
+    ctx.set_schedule(local_steps=SCHED["tau"], lr_schedule=SCHED["kind"], gamma=SCHED["gamma"])
     ctx.set_graph(w["graph"], regenerate=w["regenerate"])
     ctx.set_stream(stream)
     N, B, K, Wm = w["N"], w["B"], args.steps, args.warmup
-    units_per_step = N * B
+    units_per_step = N * B * SCHED["tau"]
 
     # ---- end to end: shards in pinned host memory, metrics read back ----
     e2e = None
@@ -471,6 +489,9 @@ def main():
     global WORKLOAD
     args = parse()
     WORKLOAD = WORKLOADS[args.workload]
+    SCHED.update(tau=args.local_steps, kind=args.lr_schedule, gamma=args.gamma)
+    if WORKLOAD["loss"] == "softmax" and args.local_steps != 1:
+        raise SystemExit("dense_softmax takes one local step per round")
     if args.impl == "reference":
         run_reference(args)
     else:

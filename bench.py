@@ -199,6 +199,9 @@ def kernel_work(sh):
     out["margin"] = ("GB/s", 8.0 * pad + 4.0 * nnz + 8.0 * N * B, "hbm")
     out["update"] = ("GB/s", 10.0 * nnz + 8.0 * touched + 4.0 * N * B, "hbm")
     out["reduce"] = ("GB/s", 8.0 * N * ld, "hbm")
+    # local steps before the round's last: the update scatter and the next gather
+    out["apply"] = ("GB/s", 16.0 * touched, "hbm")    # list + column sum read, w read + write per column
+    out["gather"] = ("GB/s", 12.0 * touched, "hbm")   # list + w read, w value written per column
     return out
 
 

@@ -227,7 +227,9 @@ typedef enum {
   ASAP_KERNEL_REDUCE = 2,     /* stochastic reduce + ACK + metrics (a5-a7, a9)  */
   ASAP_KERNEL_DENSE_FWD = 3,  /* dense logits, softmax, R^T (a3')               */
   ASAP_KERNEL_DENSE_GRAD = 4, /* dense gradient GEMM + update + NOTIFY (a3')    */
-  ASAP_KERNEL_KINDS = 5
+  ASAP_KERNEL_APPLY = 5,      /* update of a local step before the round's last */
+  ASAP_KERNEL_GATHER = 6,     /* w at a step's columns from the stored W        */
+  ASAP_KERNEL_KINDS = 7
 } asap_kernel_kind;
 
 /* Per-kernel timing: while enabled, every kernel launch of the context is

@@ -161,7 +161,7 @@ class Context:
     def debug_skip_notify(self, worker: int):
         self._c(self._lib.asap_debug_skip_notify(self._h, worker))
 
-    KERNELS = ("margin", "update", "reduce", "dense_fwd", "dense_grad")
+    KERNELS = ("margin", "update", "reduce", "dense_fwd", "dense_grad", "apply", "gather")
 
     def set_kernel_timing(self, enable: bool = True):
         self._c(self._lib.asap_set_kernel_timing(self._h, int(enable)))

@@ -1191,10 +1191,12 @@ asap_status asap_local_step(asap_ctx* c) {
     if (c->wv_step != k) {
       // No exported w values for this step's columns (parameters came from
       // the host, or an earlier local step of the round changed them): gather.
+      time_begin(c, ASAP_KERNEL_GATHER);
       CU(launch_gather_wv(c->W[r & 1], c->ld, reinterpret_cast<const uint32_t*>(block + c->list_off[tk]),
                           reinterpret_cast<const int*>(block + c->soff_off[tk]), c->n_slabs, c->S, c->wv,
                           c->sm_count, c->stream),
          "launching the gather kernel");
+      time_end(c);
       c->launches += 1;
       c->wv_step = k;
     }
@@ -1230,10 +1232,12 @@ asap_status asap_local_step(asap_ctx* c) {
     if (!last) {
       // w_stored -= eta / (B s') g at the step's columns; the reduce applies
       // the round's last update itself.
+      time_begin(c, ASAP_KERNEL_APPLY);
       CU(launch_apply_update(c->W[r & 1], c->ld, reinterpret_cast<const uint32_t*>(block + c->list_off[tk]),
                              reinterpret_cast<const int*>(block + c->soff_off[tk]), c->n_slabs, c->S, c->gsum, upd,
                              c->sm_count, c->stream),
          "launching the local update kernel");
+      time_end(c);
       c->launches += 1;
       if (c->residency == ASAP_SHARDS_HOST) {
         const int slot = static_cast<int>(k % asap_ctx::kStaging);

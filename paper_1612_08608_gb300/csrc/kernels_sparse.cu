@@ -262,19 +262,32 @@ __global__ void __launch_bounds__(kThreads) k_column_sums(SparseStepArgs a) {
   }
 }
 
-// wv[e] = W[i][s*S + cl] for every entry e of the round's column list
-// (parameters written from the host have no exported copy yet).
+// wv[e] = W[i][s*S + cl] for every entry e of a step's column list
+// (parameters written from the host, or changed by an earlier local step of
+// the round, have no exported copy).  One warp per slab, four entries per
+// lane in flight.
 __global__ void __launch_bounds__(kThreads) k_gather_wv(const float* __restrict__ W, int64_t ld,
                                                        const uint32_t* __restrict__ list,
                                                        const int* __restrict__ slab_off, long long n_slabs, int S,
                                                        float* __restrict__ wv) {
-  for (long long s = blockIdx.x; s < n_slabs; s += gridDim.x) {
+  constexpr int kU = 4;
+  const int lane = threadIdx.x & 31;
+  const long long nw = static_cast<long long>(gridDim.x) * (kThreads / 32);
+  for (long long s = static_cast<long long>(blockIdx.x) * (kThreads / 32) + (threadIdx.x >> 5); s < n_slabs;
+       s += nw) {
     const int a0 = slab_off[s], a1 = slab_off[s + 1];
-    for (int e = a0 + threadIdx.x; e < a1; e += blockDim.x) {
-      const uint32_t code = list[e];
-      if (code == kListPad) continue;
-      const int i = static_cast<int>(code >> 16), cl = static_cast<int>(code & 0xffffu);
-      wv[e] = W[static_cast<int64_t>(i) * ld + s * S + cl];
+    const float* Ws = W + s * S;
+    for (int e0 = a0 + lane; e0 < a1; e0 += kU * 32) {
+      uint32_t code[kU];
+      float v[kU];
+#pragma unroll
+      for (int u = 0; u < kU; ++u) code[u] = e0 + 32 * u < a1 ? list[e0 + 32 * u] : kListPad;
+#pragma unroll
+      for (int u = 0; u < kU; ++u)
+        v[u] = code[u] != kListPad ? Ws[static_cast<int64_t>(code[u] >> 16) * ld + (code[u] & 0xffffu)] : 0.f;
+#pragma unroll
+      for (int u = 0; u < kU; ++u)
+        if (code[u] != kListPad) wv[e0 + 32 * u] = v[u];
     }
   }
 }
@@ -282,29 +295,53 @@ __global__ void __launch_bounds__(kThreads) k_gather_wv(const float* __restrict_
 // W[i][s*S + cl] -= scale * g[e] for every entry {i << 16 | cl} of a slab-major
 // column list: the update of a local step that is not the round's last (the
 // last one is applied inside the stochastic reduce).  The entries of a list
-// are distinct, so every parameter is written by one thread.
+// are distinct, so every parameter is written by one thread.  One warp per
+// slab, four entries per lane in flight.
 __global__ void __launch_bounds__(kThreads) k_apply_update(float* __restrict__ W, int64_t ld,
                                                           const uint32_t* __restrict__ list,
                                                           const int* __restrict__ slab_off, long long n_slabs, int S,
                                                           const float* __restrict__ g, float scale) {
-  for (long long s = blockIdx.x; s < n_slabs; s += gridDim.x) {
+  constexpr int kU = 4;
+  const int lane = threadIdx.x & 31;
+  const long long nw = static_cast<long long>(gridDim.x) * (kThreads / 32);
+  for (long long s = static_cast<long long>(blockIdx.x) * (kThreads / 32) + (threadIdx.x >> 5); s < n_slabs;
+       s += nw) {
     const int a0 = slab_off[s], a1 = slab_off[s + 1];
-    for (int e = a0 + threadIdx.x; e < a1; e += blockDim.x) {
-      const uint32_t code = list[e];
-      if (code == kListPad) continue;
-      const int i = static_cast<int>(code >> 16), cl = static_cast<int>(code & 0xffffu);
-      float* p = W + static_cast<int64_t>(i) * ld + s * S + cl;
-      *p = fmaf(-scale, g[e], *p);
+    float* Ws = W + s * S;
+    for (int e0 = a0 + lane; e0 < a1; e0 += kU * 32) {
+      uint32_t code[kU];
+      float gv[kU], wv[kU];
+#pragma unroll
+      for (int u = 0; u < kU; ++u) {
+        const bool in = e0 + 32 * u < a1;
+        code[u] = in ? list[e0 + 32 * u] : kListPad;
+        gv[u] = in ? g[e0 + 32 * u] : 0.f;
+      }
+#pragma unroll
+      for (int u = 0; u < kU; ++u)
+        wv[u] = code[u] != kListPad ? Ws[static_cast<int64_t>(code[u] >> 16) * ld + (code[u] & 0xffffu)] : 0.f;
+#pragma unroll
+      for (int u = 0; u < kU; ++u)
+        if (code[u] != kListPad)
+          Ws[static_cast<int64_t>(code[u] >> 16) * ld + (code[u] & 0xffffu)] = fmaf(-scale, gv[u], wv[u]);
     }
   }
 }
 
 }  // namespace
 
+// One warp per slab; at most one wave of 8-warp CTAs.
+static int slab_warp_grid(long long n_slabs, int sm_count) {
+  const long long ctas = (n_slabs + kThreads / 32 - 1) / (kThreads / 32);
+  const long long cap = 8LL * sm_count;
+  const long long g = ctas < cap ? ctas : cap;
+  return static_cast<int>(g > 0 ? g : 1);
+}
+
 cudaError_t launch_apply_update(float* W, int64_t ld, const uint32_t* list, const int* slab_off, long long n_slabs,
                                 int S, const float* gsum, float scale, int sm_count, cudaStream_t s) {
-  const int grid = static_cast<int>(n_slabs < 4LL * sm_count ? n_slabs : 4LL * sm_count);
-  k_apply_update<<<grid > 0 ? grid : 1, kThreads, 0, s>>>(W, ld, list, slab_off, n_slabs, S, gsum, scale);
+  k_apply_update<<<slab_warp_grid(n_slabs, sm_count), kThreads, 0, s>>>(W, ld, list, slab_off, n_slabs, S, gsum,
+                                                                        scale);
   return cudaGetLastError();
 }
 
@@ -333,8 +370,7 @@ cudaError_t launch_update(const SparseStepArgs& a, int N, int update_ctas, cudaS
 
 cudaError_t launch_gather_wv(const float* W, int64_t ld, const uint32_t* list, const int* slab_off, long long n_slabs,
                              int S, float* wv, int sm_count, cudaStream_t s) {
-  const int grid = static_cast<int>(n_slabs < 4LL * sm_count ? n_slabs : 4LL * sm_count);
-  k_gather_wv<<<grid > 0 ? grid : 1, kThreads, 0, s>>>(W, ld, list, slab_off, n_slabs, S, wv);
+  k_gather_wv<<<slab_warp_grid(n_slabs, sm_count), kThreads, 0, s>>>(W, ld, list, slab_off, n_slabs, S, wv);
   return cudaGetLastError();
 }
 

@@ -176,6 +176,34 @@ def test_sparse_logistic_hashed_full_shapes():
     _run_parity(ctx, sh, T, B, "logistic", lr, sched)
 
 
+def test_local_steps_full_shapes():
+    # The bench's hashed workload with 4 local steps per round, eta_k =
+    # 0.1 / (1 + 0.001 k) and a small L2 term: 2 rounds over 8 minibatches.
+    from oracle import sgd
+    N, d, B, T, tau, l2 = 64, 1 << 20, 512, 2, 4, 1e-4
+    sh = inputs.sparse_logistic_hashed(seed=0, N=N, rows=tau * T * B)
+    sched = rounds.graph_schedule("random_regular", N, 4, graph_seed=0, regenerate=True)
+    ctx = _ctx(N, d, 4, 0, "random_regular", True, "logistic", B, 0.1, sh, l2=l2)
+    ctx.set_schedule(local_steps=tau, lr_schedule="inverse", gamma=0.001)
+    _run_parity(ctx, sh, T, B, "logistic", None, sched, l2=l2, tau=tau,
+                lr_at=lambda k: sgd.learning_rate("inverse", 0.1, 0.001, k))
+
+
+def test_local_steps_complete_graph_and_single_worker():
+    # The complete graph's column-mean path and a lone worker (identity
+    # graph) with the per-round L2 scale of several local steps.
+    sh = inputs.sparse_custom(seed=23, N=8, d=500, rows=6 * 16, max_len=20)
+    ctx = _ctx(8, 500, 7, 0, "complete", False, "logistic", 16, 0.3, sh, l2=0.05)
+    ctx.set_schedule(local_steps=2)
+    _run_parity(ctx, sh, 3, 16, "logistic", 0.3, rounds.graph_schedule("complete", 8, 7), l2=0.05, tau=2)
+    W, _ = ctx.read_params()
+    assert np.abs(W - W[0]).max() <= 1e-6 * np.abs(W).max()
+    sh = inputs.sparse_custom(seed=24, N=1, d=300, rows=9 * 16, max_len=20)
+    ctx = _ctx(1, 300, 0, 0, "identity", False, "logistic", 16, 0.3, sh, l2=0.05)
+    ctx.set_schedule(local_steps=3)
+    _run_parity(ctx, sh, 3, 16, "logistic", 0.3, rounds.graph_schedule("identity", 1, 0), l2=0.05, tau=3)
+
+
 def test_notify_timeout_is_reported_and_recoverable():
     from paper_1612_08608_gb300 import AsapError
     sh = inputs.sparse_custom(seed=3, N=4, d=100, rows=64, max_len=10)

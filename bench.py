@@ -52,8 +52,11 @@ WORKLOADS = {
 }
 WORKLOAD = WORKLOADS["sparse_logistic_hashed"]
 SCHED = {"tau": 1, "kind": "constant", "gamma": 0.0}   # local steps per round, learning-rate schedule
-PROFILE = os.path.join(ROOT, "profiles", "stochastic_reduce_sparse_logistic_hashed.txt")
-MIX_SOURCE = os.path.join(ROOT, "paper_1612_08608_gb300", "csrc", "kernels_mix.cu")
+# (workload, kernel) -> (ncu summary holding its DRAM bytes per launch, kernel source the summary was taken on)
+TRAFFIC = {
+    ("sparse_logistic_hashed", "reduce"): ("stochastic_reduce_sparse_logistic_hashed.txt", "kernels_mix.cu"),
+    ("dense_softmax", "dense_grad"): ("dense_gemms_dense_softmax.txt", "kernels_dense.cu"),
+}
 
 
 def parse():
@@ -82,14 +85,17 @@ def peaks():
         return 6800.0, "fallback"
 
 
-def mix_traffic_per_launch():
-    """DRAM bytes per reduce launch from the committed ncu summary, or None
-    when the kernel source changed since it was captured."""
+def traffic_per_launch(workload, kernel):
+    """DRAM bytes per launch of the kernel from its committed ncu summary, or
+    None when there is none or the kernel source changed since it was taken."""
+    if (workload, kernel) not in TRAFFIC:
+        return None
+    prof, source = TRAFFIC[(workload, kernel)]
     try:
-        txt = open(PROFILE).read()
+        txt = open(os.path.join(ROOT, "profiles", prof)).read()
     except OSError:
         return None
-    src = hashlib.sha256(open(MIX_SOURCE, "rb").read()).hexdigest()[:16]
+    src = hashlib.sha256(open(os.path.join(ROOT, "paper_1612_08608_gb300", "csrc", source), "rb").read()).hexdigest()[:16]
     vals = {}
     for line in txt.splitlines():
         if ":" in line:
@@ -467,8 +473,8 @@ def run_asap(args):
     kd = kernels[dom]
     roof = {"kernel": dom, "bound": kd["bound"], "achieved": kd["achieved"], "peak": kd["peak"],
             "peak_kind": kd["peak_kind"], "unit": kd["unit"], "frac": kd["frac"],
-            "traffic": mix_traffic_per_launch() if (dom == "reduce" and w["name"] == "sparse_logistic_hashed")
-            else None, "algorithmic_per_launch": kd["algorithmic_per_launch"], "mean_launch_ms": kd["mean_launch_ms"]}
+            "traffic": traffic_per_launch(w["name"], dom),
+            "algorithmic_per_launch": kd["algorithmic_per_launch"], "mean_launch_ms": kd["mean_launch_ms"]}
     value = whole_job_rate(world, units_per_step, K, elapsed_ms * 1e-3)
     line = {"metric": METRIC, "value": value, "unit": "worker-samples/s", "n_gpus": world, "steps": K,
             "warmup": Wm, "ms_per_step": elapsed_ms / K, "higher_is_better": True, "scaling": "weak",

@@ -85,6 +85,18 @@ def peaks():
         return 6800.0, "fallback"
 
 
+def code_fingerprint(path):
+    """sha256 (16 hex digits) of a source file with // comments and blank
+    lines removed: a comment edit leaves it, any code change alters it."""
+    import re
+    lines = []
+    for line in open(path, encoding="utf-8").read().splitlines():
+        line = re.sub(r"//.*$", "", line).rstrip()
+        if line:
+            lines.append(line)
+    return hashlib.sha256("\n".join(lines).encode()).hexdigest()[:16]
+
+
 def traffic_per_launch(workload, kernel):
     """DRAM bytes per launch of the kernel from its committed ncu summary, or
     None when there is none or the kernel source changed since it was taken."""
@@ -95,13 +107,13 @@ def traffic_per_launch(workload, kernel):
         txt = open(os.path.join(ROOT, "profiles", prof)).read()
     except OSError:
         return None
-    src = hashlib.sha256(open(os.path.join(ROOT, "paper_1612_08608_gb300", "csrc", source), "rb").read()).hexdigest()[:16]
+    src = code_fingerprint(os.path.join(ROOT, "paper_1612_08608_gb300", "csrc", source))
     vals = {}
     for line in txt.splitlines():
         if ":" in line:
             k, v = line.split(":", 1)
             vals[k.strip()] = v.strip()
-    if vals.get("kernel_source_sha256_16") != src:
+    if vals.get("kernel_code_sha256_16") != src:
         return None
     try:
         return float(vals["dram_bytes_per_launch"])

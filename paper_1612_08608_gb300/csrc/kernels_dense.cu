@@ -11,8 +11,9 @@
 // tiles of 64 bf16) into a ring of stages guarded by full/empty mbarriers;
 // another issues tcgen05.mma (M=128, N=256, K=16, bf16 x bf16 -> fp32 in
 // TMEM) into one of two accumulators and commits each stage back to its empty
-// barrier; four epilogue warps drain the other accumulator meanwhile (a warp
-// reaches the TMEM lanes 32 (w mod 4) .. + 31, i.e. tile rows).
+// barrier; epilogue warps (eight in the forward kernel, four in the gradient
+// kernel) drain the other accumulator meanwhile (a warp reaches the TMEM
+// lanes 32 (w mod 4) .. + 31, i.e. tile rows).
 //
 // Softmax needs all C logits of a row, more than one CTA's 256 TMEM
 // columns: the forward kernel runs as a cluster of ceil(C/256) CTAs along

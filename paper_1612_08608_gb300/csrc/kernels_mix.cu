@@ -16,9 +16,11 @@
 // of the minibatch, the column sum g of r_b x_b (kernels_sparse.cu).  The
 // producer also copies the slab's part of that list (and of the next
 // round's list) into the stage; once a slab has landed two updater warps
-// apply w -= eta/B (1 - eta l2)^-1 g to it and release it to the compute
-// warps through a "ready" mbarrier -- so w_{t+1/2} exists only in shared
-// memory -- and after mixing the compute warps export w_{t+1} at the next
+// apply the round's last local update to it, w -= eta / (B s) g, and release
+// it to the compute warps through a "ready" mbarrier -- so w_{t+1/2} exists
+// only in shared memory.  s is the round's L2 shrink, prod_j (1 - eta_j l2)
+// over its local steps, which also scales the mixing weights (true w =
+// s * stored w).  After mixing the compute warps export w_{t+1} at the next
 // round's columns, which is all the next margin kernel reads.
 //
 // Consensus error per column: with K the column's value in row 0 (a shift

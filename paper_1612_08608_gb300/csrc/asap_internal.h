@@ -81,7 +81,7 @@ struct MixArgs {
   int kp1;                     // neighbours per row (sparse kind)
   const int* nbr;              // [N][kp1]
   const float* wgt;            // [N][kp1]
-  float wscale;                // (1 - eta l2) after a local step, else 1
+  float wscale;                // the round's L2 shrink prod_j (1 - eta_j l2) after local steps, else 1
   int uniform_w;               // every weight of the table equals wgt[0]
   int S;                       // slab width (columns)
   int rows_pad;                // smem rows per slab (box_rows * n_boxes)
@@ -93,7 +93,7 @@ struct MixArgs {
   const uint32_t* upd_list;    // this round's column list (slab-major)
   const int* upd_off;          // [n_slabs + 1] slab regions of upd_list
   const float* gsum;           // column sums at upd_list positions
-  float upd_scale;             // eta / (B (1 - eta l2))
+  float upd_scale;             // eta / (B wscale) of the round's last local step
   const uint32_t* exp_list;    // next round's column list
   const int* exp_off;          // [n_slabs + 1]
   float* wv_out;               // w_{t+1} at exp_list positions

@@ -184,7 +184,7 @@ __global__ void __launch_bounds__(kThreads) k_column_sums(SparseStepArgs a) {
   constexpr int kPerWarp = kUpdateChunksPerCta / (kThreads / 32);   // 4 chunks per warp per pass
   for (int first = blockIdx.x * kUpdateChunksPerCta; first < n_chunks; first += gridDim.x * kUpdateChunksPerCta) {
     // Load the warp's chunks first (independent), then scan them one by one.
-    int cv[kPerWarp], cpv[kPerWarp], rw[kPerWarp];
+    int cv[kPerWarp], cpv[kPerWarp], cnx[kPerWarp], rw[kPerWarp];
     float pv[kPerWarp];
 #pragma unroll
     for (int u = 0; u < kPerWarp; ++u) {
@@ -193,6 +193,8 @@ __global__ void __launch_bounds__(kThreads) k_column_sums(SparseStepArgs a) {
       const bool valid = chunk < n_chunks && e < nnz;
       cv[u] = valid ? cpos[e] : -1;
       cpv[u] = (lane == 0 && chunk < n_chunks && e > 0) ? cpos[e - 1] : -2;
+      // the entry after the chunk: does lane 31's run continue past it?
+      cnx[u] = (lane == 31 && chunk < n_chunks && e + 1 < nnz) ? cpos[e + 1] : -3;
       pv[u] = valid ? cval[e] : 0.f;
       rw[u] = valid ? crow[e] : -1;
     }
@@ -230,7 +232,7 @@ __global__ void __launch_bounds__(kThreads) k_column_sums(SparseStepArgs a) {
     const float p31 = __shfl_sync(kFull, p, 31);
     if (c31 >= 0 && start31 >= 0) {
       const int e31 = chunk * 32 + 31;
-      bool cont = (e31 + 1 < nnz) && (cpos[e31 + 1] == c31);
+      bool cont = (e31 + 1 < nnz) && (__shfl_sync(kFull, cnx[u], 31) == c31);
       float acc = p31;
       int base = e31 + 1;
       while (cont) {

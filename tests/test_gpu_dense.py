@@ -6,7 +6,7 @@ error per worker per round (bf16-input GEMM path), loss within 1e-4."""
 import numpy as np
 import pytest
 
-from oracle import rounds
+from oracle import rounds, sgd
 from paper_1612_08608_gb300 import inputs
 from parity import rel_err_rows
 
@@ -15,12 +15,14 @@ pytestmark = pytest.mark.gpu
 TOL = 1e-3
 
 
-def _run(N, d, C, B, lr, k, kind, T, seed=0, l2=0.0, w0_scale=0.0):
+def _run(N, d, C, B, lr, k, kind, T, seed=0, l2=0.0, w0_scale=0.0, gamma=None):
     from paper_1612_08608_gb300 import Context
     sh = inputs.dense_softmax(seed=seed, N=N, d=d, C=C, rows=T * B)
     ctx = Context(N, d, graph_seed=seed, k=k)
     ctx.set_model("softmax", batch=B, lr=lr, num_classes=C, l2=l2)
     ctx.set_graph(kind)
+    if gamma is not None:
+        ctx.set_schedule(local_steps=1, lr_schedule="inverse", gamma=gamma)
     ctx.load_dense_shards(sh)
     sched = rounds.graph_schedule(kind, N, k, graph_seed=seed)
     W_t, _ = ctx.read_params()
@@ -33,7 +35,8 @@ def _run(N, d, C, B, lr, k, kind, T, seed=0, l2=0.0, w0_scale=0.0):
         W_n, rnd = ctx.read_params()
         assert rnd == t + 1
         nbr, wgt = sched(t)
-        ref, lref, cref = rounds.softmax_round(W_t, sh, t, B, lr, nbr, wgt, l2=l2)
+        eta = lr if gamma is None else sgd.learning_rate("inverse", lr, gamma, t)
+        ref, lref, cref = rounds.softmax_round(W_t, sh, t, B, eta, nbr, wgt, l2=l2)
         err = rel_err_rows(W_n, ref)
         assert err <= TOL, (t, err)
         lg, cg = ctx.read_metrics(t, 1)
@@ -62,6 +65,11 @@ def test_dense_cluster_geometries(C, B):
     # restatement in the kernel's fp32 order differs from the oracle by
     # 3.7e-3 there, as the GPU does).
     _run(N=3, d=256, C=C, B=B, lr=0.2, k=1, kind="ring", T=2, seed=3, w0_scale=0.05)
+
+
+def test_dense_inverse_rate_l2():
+    # eta_t = 0.5 / (1 + 0.5 t) on the dense path (one local step per round)
+    _run(N=4, d=256, C=20, B=128, lr=0.5, k=1, kind="ring", T=4, seed=4, l2=0.02, gamma=0.5)
 
 
 def test_dense_softmax_full_size():

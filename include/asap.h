@@ -220,6 +220,25 @@ asap_status asap_set_wait_limit_ns(asap_ctx* ctx, uint64_t ns);
  * runs into its wait limit.  worker = -1 clears the injection. */
 asap_status asap_debug_skip_notify(asap_ctx* ctx, int worker);
 
+/* Host only, for tests (no device needed): the image asap_load_shards builds
+ * for minibatch t -- the index structure of Section 4's per-worker updates
+ * laid out for the stochastic reduce's column slabs (no counterpart in the
+ * paper beyond that).  Shards as in asap_load_shards; batch: B rows;
+ * slab_cols: the slab width S (a power of two, 8 to 1024); the column list
+ * covers ceil(round_up(d, 64) / S) slabs.  The image is written to `image`
+ * (cap bytes; *image_bytes receives its size; ASAP_ERR_ARG when it does not
+ * fit).  desc_out (N*9 int64), per worker: byte offsets of the padded row
+ * starts (int32 [B+1]), labels (float [B]), list positions and values of
+ * the padded entries (int32 / float [nnz_pad]), the (column, row)-sorted
+ * list positions, values and rows (int32 / float / uint16 [nnz]), then
+ * nnz_pad and nnz.  list_out (3 int64): byte offsets of the slab-major list
+ * of distinct (worker << 16 | column in slab) codes and of its slab offsets
+ * (int32 [n_slabs + 1]), and the list length in entries. */
+asap_status asap_debug_batch_image(int N, int64_t d, int batch, int slab_cols, int t, const int64_t* const* rowptr,
+                                   const int32_t* const* col, const float* const* val, const float* const* y,
+                                   unsigned char* image, int64_t cap, int64_t* image_bytes, int64_t* desc_out,
+                                   int64_t* list_out);
+
 /* Kernel kinds for per-kernel timing. */
 typedef enum {
   ASAP_KERNEL_MARGIN = 0,     /* sparse margins + loss derivative (a2)          */

@@ -46,6 +46,29 @@ def build_graph(kind: str, N: int, k: int, graph_seed: int = 0, rnd: int = 0) ->
     return out
 
 
+def debug_batch_image(shards, batch: int, slab_cols: int, t: int):
+    """The image asap_load_shards builds for minibatch t (host only, for
+    tests): (image bytes uint8, desc [N, 9] int64, (list byte offset, slab
+    offsets byte offset, list length))."""
+    lib = load_library()
+    rp = [np.ascontiguousarray(a, dtype=np.int64) for a in shards.rowptr]
+    cl = [np.ascontiguousarray(a, dtype=np.int32) for a in shards.col]
+    vl = [np.ascontiguousarray(a, dtype=np.float32) for a in shards.val]
+    yl = [np.ascontiguousarray(a, dtype=np.float32) for a in shards.y]
+    N = len(rp)
+    args = (N, shards.d, batch, slab_cols, t, _ptr_array(rp), _ptr_array(cl), _ptr_array(vl), _ptr_array(yl))
+    size = C.c_int64()
+    desc = np.empty((N, 9), dtype=np.int64)
+    lst = np.empty(3, dtype=np.int64)
+    st = lib.asap_debug_batch_image(*args, None, 0, C.byref(size), _ptr(desc), _ptr(lst))
+    if st != 1:                       # anything but "buffer too small" is a real error
+        _check(lib, None, st)
+    img = np.empty(size.value, dtype=np.uint8)
+    _check(lib, None, lib.asap_debug_batch_image(*args, _ptr(img), img.shape[0], C.byref(size), _ptr(desc),
+                                                 _ptr(lst)))
+    return img, desc, (int(lst[0]), int(lst[1]), int(lst[2]))
+
+
 class Context:
     """N simulated workers on the current CUDA device (see include/asap.h)."""
 

@@ -469,15 +469,160 @@ asap_status sync_all(asap_ctx* c) {
   return check_device_error(c);
 }
 
-// Make round r's batch block available on the device (host residency).
-// Slot r % 3; a slot is rewritten only after the last kernel that reads its
-// previous block (the reduce of that block's own round) has finished.
+// The device image of minibatch t (host only): per worker the padded rows
+// (list position, value) and labels, and the entries sorted by (column, row);
+// then the batch's slab-major list of distinct (worker, column) pairs and its
+// slab offsets.  Used by asap_load_shards and, for tests, asap_debug_batch_image.
+struct BatchImage {
+  std::vector<unsigned char> img;
+  std::vector<BatchDesc> desc;
+  size_t list_off = 0, soff_off = 0;
+  int64_t list_len = 0;
+  int max_region = 0, max_nnz = 0;
+  const char* err = nullptr;
+};
+
+void build_batch_image(int N, int B, int64_t d, int S, long long n_slabs, int t, const int64_t* const* rowptr,
+                       const int32_t* const* col, const float* const* val, const float* const* y, BatchImage& bt) {
+  std::vector<std::vector<uint64_t>> keys(N);
+  std::vector<std::vector<int32_t>> ucol(N), run_of(N), upos(N);
+  std::vector<int64_t> nnz(N, 0), nnz_pad(N, 0);
+  for (int i = 0; i < N; ++i) {
+    const int64_t* rp = rowptr[i];
+    const int64_t r0 = static_cast<int64_t>(t) * B;
+    const int64_t a0 = rp[r0], a1 = rp[r0 + B];
+    nnz[i] = a1 - a0;
+    for (int b = 0; b < B; ++b) nnz_pad[i] += (rp[r0 + b + 1] - rp[r0 + b] + 3) / 4 * 4;
+    if (nnz_pad[i] > (1ll << 30)) { bt.err = "a minibatch holds more than 2^30 entries"; return; }
+    std::vector<uint64_t>& k = keys[i];
+    k.resize(nnz[i]);
+    for (int64_t e = 0; e < nnz[i]; ++e) {
+      const int32_t cc = col[i][a0 + e];
+      if (cc < 0 || cc >= d) { bt.err = "column id out of range [0, d)"; return; }
+      k[e] = (static_cast<uint64_t>(static_cast<uint32_t>(cc)) << 32) | static_cast<uint64_t>(e);
+    }
+    std::sort(k.begin(), k.end());   // by column, then by entry (= by row)
+    run_of[i].resize(nnz[i]);
+    for (int64_t e = 0; e < nnz[i]; ++e) {
+      const int32_t cc = static_cast<int32_t>(k[e] >> 32);
+      if (e == 0 || cc != static_cast<int32_t>(k[e - 1] >> 32)) ucol[i].push_back(cc);
+      run_of[i][e] = static_cast<int32_t>(ucol[i].size()) - 1;
+    }
+    bt.max_nnz = std::max<int>(bt.max_nnz, static_cast<int>(nnz[i]));
+  }
+  // Slab-major positions.
+  std::vector<int32_t> cnt(static_cast<size_t>(n_slabs) * N, 0);
+  for (int i = 0; i < N; ++i)
+    for (int32_t cc : ucol[i]) cnt[static_cast<size_t>(cc / S) * N + i]++;
+  std::vector<int32_t> soff(n_slabs + 1), start(static_cast<size_t>(n_slabs) * N);
+  int64_t tot = 0;
+  for (long long sl = 0; sl < n_slabs; ++sl) {
+    soff[sl] = static_cast<int32_t>(tot);
+    int64_t acc = tot;
+    for (int i = 0; i < N; ++i) {
+      start[static_cast<size_t>(sl) * N + i] = static_cast<int32_t>(acc);
+      acc += cnt[static_cast<size_t>(sl) * N + i];
+    }
+    const int64_t n = acc - tot, np = (n + 3) / 4 * 4;
+    bt.max_region = std::max<int>(bt.max_region, static_cast<int>(np));
+    tot += np;
+    if (tot >= (1ll << 31)) { bt.err = "column list of a minibatch too long"; return; }
+  }
+  soff[n_slabs] = static_cast<int32_t>(tot);
+  std::vector<uint32_t> list(tot, kListPad);
+  for (int i = 0; i < N; ++i) {
+    upos[i].resize(ucol[i].size());
+    for (size_t u = 0; u < ucol[i].size(); ++u) {
+      const int32_t cc = ucol[i][u];
+      const int sl = cc / S;
+      const int32_t pos = start[static_cast<size_t>(sl) * N + i]++;
+      list[pos] = (static_cast<uint32_t>(i) << 16) | static_cast<uint32_t>(cc - sl * S);
+      upos[i][u] = pos;
+    }
+  }
+  // Layout of the block image.
+  bt.desc.resize(N);
+  size_t off = 0;
+  for (int i = 0; i < N; ++i) {
+    BatchDesc& dd = bt.desc[i];
+    dd.rp = static_cast<int64_t>(off);
+    off = align_up(off + 4 * static_cast<size_t>(B + 1), 16);
+    dd.y = static_cast<int64_t>(off);
+    off = align_up(off + 4 * static_cast<size_t>(B), 16);
+    dd.posw = static_cast<int64_t>(off);
+    off += 4 * static_cast<size_t>(nnz_pad[i]);
+    dd.val = static_cast<int64_t>(off);
+    off += 4 * static_cast<size_t>(nnz_pad[i]);
+    dd.cpos = static_cast<int64_t>(off);
+    off = align_up(off + 4 * static_cast<size_t>(nnz[i]), 16);
+    dd.cval = static_cast<int64_t>(off);
+    off = align_up(off + 4 * static_cast<size_t>(nnz[i]), 16);
+    dd.crow = static_cast<int64_t>(off);
+    off = align_up(off + 2 * static_cast<size_t>(nnz[i]), 16);
+    dd.nnz_pad = static_cast<int32_t>(nnz_pad[i]);
+    dd.nnz = static_cast<int32_t>(nnz[i]);
+  }
+  bt.list_off = off;
+  off = align_up(off + 4 * static_cast<size_t>(tot), 16);
+  bt.soff_off = off;
+  off = align_up(off + 4 * static_cast<size_t>(n_slabs + 1), 256);
+  bt.list_len = tot;
+  bt.img.assign(off, 0);
+  unsigned char* base = bt.img.data();
+  std::memcpy(base + bt.list_off, list.data(), 4 * list.size());
+  std::memcpy(base + bt.soff_off, soff.data(), 4 * soff.size());
+  for (int i = 0; i < N; ++i) {
+    const BatchDesc& dd = bt.desc[i];
+    int32_t* rp_o = reinterpret_cast<int32_t*>(base + dd.rp);
+    float* y_o = reinterpret_cast<float*>(base + dd.y);
+    int32_t* pw_o = reinterpret_cast<int32_t*>(base + dd.posw);
+    float* val_o = reinterpret_cast<float*>(base + dd.val);
+    int32_t* cp_o = reinterpret_cast<int32_t*>(base + dd.cpos);
+    float* cv_o = reinterpret_cast<float*>(base + dd.cval);
+    uint16_t* cr_o = reinterpret_cast<uint16_t*>(base + dd.crow);
+    const int64_t* rp = rowptr[i];
+    const int64_t r0 = static_cast<int64_t>(t) * B, a0 = rp[r0];
+    // list position of every entry (row-major), through the sort
+    std::vector<int32_t> epos(nnz[i]);
+    std::vector<uint16_t> erow(nnz[i]);
+    for (int b = 0; b < B; ++b)
+      for (int64_t e = rp[r0 + b] - a0; e < rp[r0 + b + 1] - a0; ++e) erow[e] = static_cast<uint16_t>(b);
+    for (int64_t e = 0; e < nnz[i]; ++e) {
+      const int64_t k = static_cast<int64_t>(keys[i][e] & 0xffffffffu);
+      const int32_t pos = upos[i][run_of[i][e]];
+      epos[k] = pos;
+      cp_o[e] = pos;
+      cv_o[e] = val[i][a0 + k];
+      cr_o[e] = erow[k];
+    }
+    int32_t q = 0;
+    for (int b = 0; b < B; ++b) {
+      rp_o[b] = q;
+      y_o[b] = y[i][r0 + b];
+      for (int64_t e = rp[r0 + b] - a0; e < rp[r0 + b + 1] - a0; ++e) {
+        pw_o[q] = epos[e];
+        val_o[q] = val[i][a0 + e];
+        ++q;
+      }
+      while (q & 3) {   // pad the row to a multiple of 4 entries (value 0)
+        pw_o[q] = 0;
+        val_o[q] = 0.f;
+        ++q;
+      }
+    }
+    rp_o[B] = q;
+  }
+}
+
 // eta_k of global local step k.
 float lr_at(const asap_ctx* c, int64_t k) {
   if (c->lr_kind == ASAP_LR_INVERSE) return static_cast<float>(c->lr / (1.0 + c->lr_gamma * static_cast<double>(k)));
   return c->lr;
 }
 
+// Make the block of global local step r available on the device (host residency).
+// Slot r % 3; a slot is rewritten only after the last kernel that reads its
+// previous block (the step's update, or the reduce of its round) has finished.
 asap_status stage_block(asap_ctx* c, int64_t r) {
   const int slot = static_cast<int>(r % asap_ctx::kStaging);
   if (c->staged_round[slot] == r) return ASAP_OK;
@@ -515,6 +660,34 @@ extern "C" {
 const char* asap_version(void) { return "asap-gb300 0.1 (sm_103a)"; }
 
 const char* asap_last_error(const asap_ctx* c) { return c ? c->err.c_str() : g_last_error.c_str(); }
+
+asap_status asap_debug_batch_image(int N, int64_t d, int batch, int slab_cols, int t, const int64_t* const* rowptr,
+                                   const int32_t* const* col, const float* const* val, const float* const* y,
+                                   unsigned char* image, int64_t cap, int64_t* image_bytes, int64_t* desc_out,
+                                   int64_t* list_out) {
+  if (N < 1 || N > kMaxWorkers || d < 1 || batch < 1 || batch > 65535 || t < 0 || !rowptr || !col || !val || !y ||
+      !image_bytes || !desc_out || !list_out)
+    return fail(nullptr, ASAP_ERR_ARG, "bad arguments to asap_debug_batch_image");
+  if (slab_cols < 8 || slab_cols > 1024 || (slab_cols & (slab_cols - 1)))
+    return fail(nullptr, ASAP_ERR_ARG, "slab_cols must be a power of two in [8, 1024]");
+  const int64_t ld = (d + 63) / 64 * 64;
+  const long long n_slabs = (ld + slab_cols - 1) / slab_cols;
+  BatchImage bt;
+  build_batch_image(N, batch, d, slab_cols, n_slabs, t, rowptr, col, val, y, bt);
+  if (bt.err) return fail(nullptr, ASAP_ERR_ARG, bt.err);
+  *image_bytes = static_cast<int64_t>(bt.img.size());
+  if (!image || cap < static_cast<int64_t>(bt.img.size())) return fail(nullptr, ASAP_ERR_ARG, "image buffer too small");
+  std::memcpy(image, bt.img.data(), bt.img.size());
+  for (int i = 0; i < N; ++i) {
+    const BatchDesc& q = bt.desc[i];
+    const int64_t v[9] = {q.rp, q.y, q.posw, q.val, q.cpos, q.cval, q.crow, q.nnz_pad, q.nnz};
+    std::memcpy(desc_out + 9 * static_cast<size_t>(i), v, sizeof v);
+  }
+  list_out[0] = static_cast<int64_t>(bt.list_off);
+  list_out[1] = static_cast<int64_t>(bt.soff_off);
+  list_out[2] = bt.list_len;
+  return ASAP_OK;
+}
 
 asap_status asap_build_graph(asap_graph_kind kind, int N, int k, uint64_t graph_seed, int64_t round,
                              int32_t* nbr_out) {
@@ -830,149 +1003,8 @@ asap_status asap_load_shards(asap_ctx* c, const int64_t* const* rowptr, const in
   const int S = c->S;
   const long long n_slabs = c->n_slabs;
 
-  // One block per minibatch index t: per worker the padded rows (pos, val),
-  // labels and the entries sorted by (column, row); then the batch's
-  // slab-major list of distinct (worker, column) pairs and its slab offsets.
-  struct Built {
-    std::vector<unsigned char> img;
-    std::vector<BatchDesc> desc;
-    size_t list_off = 0, soff_off = 0;
-    int64_t list_len = 0;
-    int max_region = 0, max_nnz = 0;
-    const char* err = nullptr;
-  };
-  std::vector<Built> built(nb);
-  auto build_batch = [&](int t) {
-    Built& bt = built[t];
-    std::vector<std::vector<uint64_t>> keys(N);
-    std::vector<std::vector<int32_t>> ucol(N), run_of(N), upos(N);
-    std::vector<int64_t> nnz(N, 0), nnz_pad(N, 0);
-    for (int i = 0; i < N; ++i) {
-      const int64_t* rp = rowptr[i];
-      const int64_t r0 = static_cast<int64_t>(t) * B;
-      const int64_t a0 = rp[r0], a1 = rp[r0 + B];
-      nnz[i] = a1 - a0;
-      for (int b = 0; b < B; ++b) nnz_pad[i] += (rp[r0 + b + 1] - rp[r0 + b] + 3) / 4 * 4;
-      if (nnz_pad[i] > (1ll << 30)) { bt.err = "a minibatch holds more than 2^30 entries"; return; }
-      std::vector<uint64_t>& k = keys[i];
-      k.resize(nnz[i]);
-      for (int64_t e = 0; e < nnz[i]; ++e) {
-        const int32_t cc = col[i][a0 + e];
-        if (cc < 0 || cc >= c->d) { bt.err = "column id out of range [0, d)"; return; }
-        k[e] = (static_cast<uint64_t>(static_cast<uint32_t>(cc)) << 32) | static_cast<uint64_t>(e);
-      }
-      std::sort(k.begin(), k.end());   // by column, then by entry (= by row)
-      run_of[i].resize(nnz[i]);
-      for (int64_t e = 0; e < nnz[i]; ++e) {
-        const int32_t cc = static_cast<int32_t>(k[e] >> 32);
-        if (e == 0 || cc != static_cast<int32_t>(k[e - 1] >> 32)) ucol[i].push_back(cc);
-        run_of[i][e] = static_cast<int32_t>(ucol[i].size()) - 1;
-      }
-      bt.max_nnz = std::max<int>(bt.max_nnz, static_cast<int>(nnz[i]));
-    }
-    // Slab-major positions.
-    std::vector<int32_t> cnt(static_cast<size_t>(n_slabs) * N, 0);
-    for (int i = 0; i < N; ++i)
-      for (int32_t cc : ucol[i]) cnt[static_cast<size_t>(cc / S) * N + i]++;
-    std::vector<int32_t> soff(n_slabs + 1), start(static_cast<size_t>(n_slabs) * N);
-    int64_t tot = 0;
-    for (long long sl = 0; sl < n_slabs; ++sl) {
-      soff[sl] = static_cast<int32_t>(tot);
-      int64_t acc = tot;
-      for (int i = 0; i < N; ++i) {
-        start[static_cast<size_t>(sl) * N + i] = static_cast<int32_t>(acc);
-        acc += cnt[static_cast<size_t>(sl) * N + i];
-      }
-      const int64_t n = acc - tot, np = (n + 3) / 4 * 4;
-      bt.max_region = std::max<int>(bt.max_region, static_cast<int>(np));
-      tot += np;
-      if (tot >= (1ll << 31)) { bt.err = "column list of a minibatch too long"; return; }
-    }
-    soff[n_slabs] = static_cast<int32_t>(tot);
-    std::vector<uint32_t> list(tot, kListPad);
-    for (int i = 0; i < N; ++i) {
-      upos[i].resize(ucol[i].size());
-      for (size_t u = 0; u < ucol[i].size(); ++u) {
-        const int32_t cc = ucol[i][u];
-        const int sl = cc / S;
-        const int32_t pos = start[static_cast<size_t>(sl) * N + i]++;
-        list[pos] = (static_cast<uint32_t>(i) << 16) | static_cast<uint32_t>(cc - sl * S);
-        upos[i][u] = pos;
-      }
-    }
-    // Layout of the block image.
-    bt.desc.resize(N);
-    size_t off = 0;
-    for (int i = 0; i < N; ++i) {
-      BatchDesc& dd = bt.desc[i];
-      dd.rp = static_cast<int64_t>(off);
-      off = align_up(off + 4 * static_cast<size_t>(B + 1), 16);
-      dd.y = static_cast<int64_t>(off);
-      off = align_up(off + 4 * static_cast<size_t>(B), 16);
-      dd.posw = static_cast<int64_t>(off);
-      off += 4 * static_cast<size_t>(nnz_pad[i]);
-      dd.val = static_cast<int64_t>(off);
-      off += 4 * static_cast<size_t>(nnz_pad[i]);
-      dd.cpos = static_cast<int64_t>(off);
-      off = align_up(off + 4 * static_cast<size_t>(nnz[i]), 16);
-      dd.cval = static_cast<int64_t>(off);
-      off = align_up(off + 4 * static_cast<size_t>(nnz[i]), 16);
-      dd.crow = static_cast<int64_t>(off);
-      off = align_up(off + 2 * static_cast<size_t>(nnz[i]), 16);
-      dd.nnz_pad = static_cast<int32_t>(nnz_pad[i]);
-      dd.nnz = static_cast<int32_t>(nnz[i]);
-    }
-    bt.list_off = off;
-    off = align_up(off + 4 * static_cast<size_t>(tot), 16);
-    bt.soff_off = off;
-    off = align_up(off + 4 * static_cast<size_t>(n_slabs + 1), 256);
-    bt.list_len = tot;
-    bt.img.assign(off, 0);
-    unsigned char* base = bt.img.data();
-    std::memcpy(base + bt.list_off, list.data(), 4 * list.size());
-    std::memcpy(base + bt.soff_off, soff.data(), 4 * soff.size());
-    for (int i = 0; i < N; ++i) {
-      const BatchDesc& dd = bt.desc[i];
-      int32_t* rp_o = reinterpret_cast<int32_t*>(base + dd.rp);
-      float* y_o = reinterpret_cast<float*>(base + dd.y);
-      int32_t* pw_o = reinterpret_cast<int32_t*>(base + dd.posw);
-      float* val_o = reinterpret_cast<float*>(base + dd.val);
-      int32_t* cp_o = reinterpret_cast<int32_t*>(base + dd.cpos);
-      float* cv_o = reinterpret_cast<float*>(base + dd.cval);
-      uint16_t* cr_o = reinterpret_cast<uint16_t*>(base + dd.crow);
-      const int64_t* rp = rowptr[i];
-      const int64_t r0 = static_cast<int64_t>(t) * B, a0 = rp[r0];
-      // list position of every entry (row-major), through the sort
-      std::vector<int32_t> epos(nnz[i]);
-      std::vector<uint16_t> erow(nnz[i]);
-      for (int b = 0; b < B; ++b)
-        for (int64_t e = rp[r0 + b] - a0; e < rp[r0 + b + 1] - a0; ++e) erow[e] = static_cast<uint16_t>(b);
-      for (int64_t e = 0; e < nnz[i]; ++e) {
-        const int64_t k = static_cast<int64_t>(keys[i][e] & 0xffffffffu);
-        const int32_t pos = upos[i][run_of[i][e]];
-        epos[k] = pos;
-        cp_o[e] = pos;
-        cv_o[e] = val[i][a0 + k];
-        cr_o[e] = erow[k];
-      }
-      int32_t q = 0;
-      for (int b = 0; b < B; ++b) {
-        rp_o[b] = q;
-        y_o[b] = y[i][r0 + b];
-        for (int64_t e = rp[r0 + b] - a0; e < rp[r0 + b + 1] - a0; ++e) {
-          pw_o[q] = epos[e];
-          val_o[q] = val[i][a0 + e];
-          ++q;
-        }
-        while (q & 3) {   // pad the row to a multiple of 4 entries (value 0)
-          pw_o[q] = 0;
-          val_o[q] = 0.f;
-          ++q;
-        }
-      }
-      rp_o[B] = q;
-    }
-  };
+  std::vector<BatchImage> built(nb);
+  auto build_batch = [&](int t) { build_batch_image(N, B, c->d, S, n_slabs, t, rowptr, col, val, y, built[t]); };
   {
     const unsigned nthr = std::max(1u, std::min(32u, std::thread::hardware_concurrency()));
     std::vector<std::thread> pool;

@@ -14,7 +14,8 @@ Printed JSON line (rank 0):
   e2e        -- the same metric through the public API with the shards in
                 pinned host memory: every round copies its minibatch block
                 host->device (overlapped with the previous round) and reads
-                the round's metrics back device->host
+                the round's metrics back device->host while the next round
+                runs
   roofline   -- the stochastic-reduce kernel (the dominant kernel): 8 N d
                 algorithmic bytes per launch / its mean CUDA-event duration
   cpu_baseline -- the CPU oracle as it stands, one full round of the same
@@ -424,15 +425,21 @@ def run_asap(args):
             r0 = Wm
             barrier()
             t0 = time.perf_counter()
+            # Round s's loss and consensus error are read back while round
+            # s + 1 runs (the read waits for round s only); the last one
+            # after the loop, inside the timed region.
             for s in range(K):
                 h2d += ctx.shard_block_bytes(r0 + s)
                 ctx.round(1)
-                ctx.read_metrics(r0 + s, 1)
+                if s > 0:
+                    ctx.read_metrics(r0 + s - 1, 1)
+            ctx.read_metrics(r0 + K - 1, 1)
             ctx.sync()
             t_e2e = max_over_ranks(time.perf_counter() - t0)
             graph_bytes = N * (w["k"] + 1) * 8 if w["regenerate"] else 0
+            # d2h per step: loss and consensus error (8 B) and the device error word (4 B)
             e2e = {"value": whole_job_rate(world, units_per_step, K, t_e2e), "unit": "worker-samples/s",
-                   "h2d_bytes_per_step": h2d / K + graph_bytes, "d2h_bytes_per_step": 8}
+                   "h2d_bytes_per_step": h2d / K + graph_bytes, "d2h_bytes_per_step": 12}
         ctx.set_shard_residency("device")
 
     # ---- device resident: the kernel-level number ----

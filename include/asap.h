@@ -196,7 +196,12 @@ asap_status asap_write_params(asap_ctx* ctx, const float* host_in, int64_t round
  * over workers of the minibatch loss at the pre-step parameters (NaN for a
  * reduce-only round) and the consensus error ||W_{t+1} - 1 wbar^T||_F.
  * The last 65536 rounds are kept.  Either output pointer may be NULL.
- * Syncing. */
+ * Waits only until round first_round + count - 1 is complete when that is
+ * one of the last 64 rounds launched since the last asap_write_params
+ * (rounds queued after it keep running, so a caller may read round t's
+ * metrics while round t+1 runs); otherwise, and for count = 0, it
+ * synchronises fully.  A device error recorded by then is reported after a
+ * full drain, as by asap_sync. */
 asap_status asap_read_metrics(asap_ctx* ctx, int64_t first_round, int64_t count, float* loss_out,
                               float* consensus_out);
 

@@ -137,6 +137,12 @@ struct asap_ctx {
   bool dense_configured = false;
 
   cudaStream_t stream = nullptr, own_stream = nullptr, copy_stream = nullptr;
+  // An event recorded after every round's reduce (a ring), so that a metrics
+  // read waits for its own rounds only while later rounds keep the GPU busy.
+  static constexpr int kRoundEvents = 64;
+  cudaEvent_t round_ev[kRoundEvents] = {};
+  int64_t round_ev_round[kRoundEvents] = {};   // round recorded in each slot, -1: none
+  cudaStream_t read_stream = nullptr;
 
   CUtensorMap tmap[2];
   int S = 0, rows_pad = 0, box_rows = 0, n_boxes = 0, stages = 0;
@@ -346,6 +352,7 @@ asap_status reset_protocol(asap_ctx* c, int64_t rnd) {
   c->round = rnd;
   c->step_pending = false;
   c->graph_ready_round = -1;
+  for (int i = 0; i < asap_ctx::kRoundEvents; ++i) c->round_ev_round[i] = -1;
   return ASAP_OK;
 }
 
@@ -720,7 +727,12 @@ asap_status asap_create(int N, int64_t d, uint64_t graph_seed, int k, asap_ctx**
   CU(cudaDeviceGetAttribute(&c->sm_count, cudaDevAttrMultiProcessorCount, c->dev), "querying SM count");
   CU(cudaStreamCreateWithFlags(&c->own_stream, cudaStreamNonBlocking), "creating a stream");
   CU(cudaStreamCreateWithFlags(&c->copy_stream, cudaStreamNonBlocking), "creating a copy stream");
+  CU(cudaStreamCreateWithFlags(&c->read_stream, cudaStreamNonBlocking), "creating a read stream");
   c->stream = c->own_stream;
+  for (int i = 0; i < asap_ctx::kRoundEvents; ++i) {
+    CU(cudaEventCreateWithFlags(&c->round_ev[i], cudaEventDisableTiming), "creating events");
+    c->round_ev_round[i] = -1;
+  }
   for (int i = 0; i < kGraphRing; ++i) {
     CU(cudaEventCreateWithFlags(&c->slot_ev[i], cudaEventDisableTiming), "creating events");
     c->slot_used[i] = false;
@@ -795,6 +807,12 @@ void asap_destroy(asap_ctx* c) {
   for (int b = 0; b < asap_ctx::kStaging; ++b) {
     if (c->staged_ev[b]) cudaEventDestroy(c->staged_ev[b]);
     if (c->free_ev[b]) cudaEventDestroy(c->free_ev[b]);
+  }
+  for (int i = 0; i < asap_ctx::kRoundEvents; ++i)
+    if (c->round_ev[i]) cudaEventDestroy(c->round_ev[i]);
+  if (c->read_stream) {
+    cudaStreamSynchronize(c->read_stream);
+    cudaStreamDestroy(c->read_stream);
   }
   if (c->own_stream) cudaStreamDestroy(c->own_stream);
   if (c->copy_stream) cudaStreamDestroy(c->copy_stream);
@@ -1355,6 +1373,9 @@ asap_status asap_stochastic_reduce(asap_ctx* c) {
      "launching the stochastic reduce");
   time_end(c);
   c->launches += 1;
+  const int ev = static_cast<int>(r % asap_ctx::kRoundEvents);
+  CU(cudaEventRecord(c->round_ev[ev], c->stream), "round event");
+  c->round_ev_round[ev] = r;
   c->wv_step = fused ? c->pend_k + 1 : -1;
   if (fused && c->residency == ASAP_SHARDS_HOST) {
     const int slot = static_cast<int>(c->pend_k % asap_ctx::kStaging);
@@ -1416,15 +1437,37 @@ asap_status asap_read_metrics(asap_ctx* c, int64_t first, int64_t count, float* 
   if (!c || first < 0 || count < 0) return fail(c, ASAP_ERR_ARG, "bad argument");
   if (first + count > c->round || first < c->round - kMetricsCap)
     return fail(c, ASAP_ERR_ARG, "rounds outside the kept metrics window");
-  asap_status s = sync_all(c);
-  if (s != ASAP_OK) return s;
+  const int64_t last = first + count - 1;
+  const int ev = static_cast<int>((count > 0 ? last : 0) % asap_ctx::kRoundEvents);
+  if (count == 0 || c->round_ev_round[ev] != last) {
+    // No event for the last requested round: drain everything.
+    asap_status s = sync_all(c);
+    if (s != ASAP_OK) return s;
+  } else {
+    // Wait for round `last` only; rounds queued after it keep running.  A
+    // device error recorded by then is reported after a full drain.
+    CU(cudaStreamWaitEvent(c->read_stream, c->round_ev[ev], 0), "waiting for the round");
+    unsigned code = 0;
+    CU(cudaMemcpyAsync(&code, &c->st->err_code, 4, cudaMemcpyDeviceToHost, c->read_stream), "reading device state");
+    CU(cudaStreamSynchronize(c->read_stream), "waiting for the round");
+    if (code != 0) {
+      asap_status s = sync_all(c);
+      if (s != ASAP_OK) return s;
+    }
+  }
+  // Pageable destinations: each copy returns once it is done.
   for (int64_t r = first; r < first + count;) {
     const int64_t slot = r % kMetricsCap;
     const int64_t n = std::min<int64_t>(first + count - r, kMetricsCap - slot);
-    if (loss_out) CU(cudaMemcpy(loss_out + (r - first), c->m_loss + slot, 4 * n, cudaMemcpyDeviceToHost), "metrics");
-    if (cons_out) CU(cudaMemcpy(cons_out + (r - first), c->m_cons + slot, 4 * n, cudaMemcpyDeviceToHost), "metrics");
+    if (loss_out)
+      CU(cudaMemcpyAsync(loss_out + (r - first), c->m_loss + slot, 4 * n, cudaMemcpyDeviceToHost, c->read_stream),
+         "metrics");
+    if (cons_out)
+      CU(cudaMemcpyAsync(cons_out + (r - first), c->m_cons + slot, 4 * n, cudaMemcpyDeviceToHost, c->read_stream),
+         "metrics");
     r += n;
   }
+  CU(cudaStreamSynchronize(c->read_stream), "metrics");
   return ASAP_OK;
 }
 

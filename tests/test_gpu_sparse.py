@@ -224,6 +224,44 @@ def test_notify_timeout_is_reported_and_recoverable():
     assert rnd == 3 and np.isfinite(W3).all()
 
 
+@pytest.mark.parametrize("residency", ["device", "host"])
+def test_lagged_metric_reads_match_a_full_sync(residency):
+    # Round t's metrics read while round t+1 runs (the read waits for round t
+    # only) equal those read after a full drain.
+    sh = inputs.sparse_custom(seed=12, N=8, d=3000, rows=256, max_len=60, hot_col=3)
+    ctx = _ctx(8, 3000, 2, 4, "random_regular", True, "logistic", 64, 0.3, sh, residency=residency)
+    T = 7
+    lagged = []
+    for t in range(T):
+        ctx.round(1)
+        if t > 0:
+            lagged.append(ctx.read_metrics(t - 1, 1))
+    lagged.append(ctx.read_metrics(T - 1, 1))
+    ctx.sync()
+    loss, cons = ctx.read_metrics(0, T)
+    assert np.array_equal(np.concatenate([m[0] for m in lagged]), loss)
+    assert np.array_equal(np.concatenate([m[1] for m in lagged]), cons)
+    assert np.isfinite(loss).all() and np.isfinite(cons).all()
+
+
+def test_lagged_metric_read_reports_a_timeout():
+    from paper_1612_08608_gb300 import AsapError
+    sh = inputs.sparse_custom(seed=3, N=4, d=100, rows=64, max_len=10)
+    ctx = _ctx(4, 100, 1, 0, "ring", False, "logistic", 16, 0.1, sh)
+    ctx.round(1)
+    W1, _ = ctx.read_params()
+    ctx.set_wait_limit_ns(20_000_000)         # 20 ms
+    ctx.debug_skip_notify(1)
+    ctx.round(1)
+    with pytest.raises(AsapError) as ei:
+        ctx.read_metrics(1, 1)
+    assert ei.value.name == "ASAP_ERR_TIMEOUT"
+    ctx.write_params(W1, 1)
+    ctx.round(1)
+    loss, cons = ctx.read_metrics(1, 1)
+    assert np.isfinite(loss).all() and np.isfinite(cons).all()
+
+
 def test_two_runs_bit_identical():
     sh = inputs.sparse_custom(seed=8, N=8, d=3000, rows=256, max_len=60, hot_col=3)
     outs = []

@@ -228,7 +228,8 @@ asap_status asap_debug_skip_notify(asap_ctx* ctx, int worker);
 /* Host only, for tests (no device needed): the image asap_load_shards builds
  * for minibatch t -- the index structure of Section 4's per-worker updates
  * laid out for the stochastic reduce's column slabs (no counterpart in the
- * paper beyond that).  Shards as in asap_load_shards; batch: B rows;
+ * paper beyond that).  Shards as in asap_load_shards, each with at least
+ * (t + 1) * batch rows (not checked: there is no row count here); batch: B rows;
  * slab_cols: the slab width S (a power of two, 8 to 1024); the column list
  * covers ceil(round_up(d, 64) / S) slabs.  The image is written to `image`
  * (cap bytes; *image_bytes receives its size; ASAP_ERR_ARG when it does not

@@ -56,6 +56,8 @@ def debug_batch_image(shards, batch: int, slab_cols: int, t: int):
     vl = [np.ascontiguousarray(a, dtype=np.float32) for a in shards.val]
     yl = [np.ascontiguousarray(a, dtype=np.float32) for a in shards.y]
     N = len(rp)
+    if t < 0 or any((t + 1) * batch > a.shape[0] - 1 for a in rp):
+        raise ValueError("minibatch %d of %d rows is past the end of a shard" % (t, batch))
     args = (N, shards.d, batch, slab_cols, t, _ptr_array(rp), _ptr_array(cl), _ptr_array(vl), _ptr_array(yl))
     size = C.c_int64()
     desc = np.empty((N, 9), dtype=np.int64)

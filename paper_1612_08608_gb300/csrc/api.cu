@@ -705,24 +705,12 @@ asap_status asap_build_graph(asap_graph_kind kind, int N, int k, uint64_t graph_
   return ASAP_OK;
 }
 
-asap_status asap_create(int N, int64_t d, uint64_t graph_seed, int k, asap_ctx** out) {
-  if (!out) return fail(nullptr, ASAP_ERR_ARG, "out is NULL");
-  *out = nullptr;
-  if (N < 1 || N > kMaxWorkers || d < 1 || k < 0 || k > N - 1)
-    return fail(nullptr, ASAP_ERR_ARG, "need 1 <= N <= 1024, d >= 1, 0 <= k <= N-1");
-  std::unique_ptr<asap_ctx> holder(new asap_ctx());
-  asap_ctx* c = holder.get();
-  c->N = N;
-  c->d = d;
-  c->seed = graph_seed;
-  c->k = k;
-  c->kind = (k == 0) ? ASAP_GRAPH_IDENTITY
-            : (k == N - 1) ? ASAP_GRAPH_COMPLETE
-            : (k == 1) ? ASAP_GRAPH_RING
-                       : ASAP_GRAPH_RANDOM_REGULAR;
-  if (c->kind == ASAP_GRAPH_RANDOM_REGULAR && k + 1 > kMaxKp1Sparse)
-    return fail(nullptr, ASAP_ERR_ARG, "k+1 > 32 is supported only for the complete graph");
-  c->P = d;
+// Streams, events, flags, metrics and the parameter buffers of a new
+// context.  On failure asap_create hands the partly built context to
+// asap_destroy, which frees whatever exists.
+static asap_status init_ctx(asap_ctx* c) {
+  const int N = c->N, k = c->k;
+  c->P = c->d;
   CU(cudaGetDevice(&c->dev), "cudaGetDevice");
   CU(cudaDeviceGetAttribute(&c->sm_count, cudaDevAttrMultiProcessorCount, c->dev), "querying SM count");
   CU(cudaStreamCreateWithFlags(&c->own_stream, cudaStreamNonBlocking), "creating a stream");
@@ -761,12 +749,28 @@ asap_status asap_create(int N, int64_t d, uint64_t graph_seed, int k, asap_ctx**
   CU(cudaHostAlloc(&c->h_nbr, ring * 4, cudaHostAllocDefault), "allocating pinned graph slots");
   CU(cudaHostAlloc(&c->h_wgt, ring * 4, cudaHostAllocDefault), "allocating pinned graph slots");
   asap_status s = alloc_params(c);
-  if (s != ASAP_OK) {
-    g_last_error = c->err;
-    asap_destroy(holder.release());
-    return s;
-  }
-  s = upload_fixed_graph(c);
+  if (s != ASAP_OK) return s;
+  return upload_fixed_graph(c);
+}
+
+asap_status asap_create(int N, int64_t d, uint64_t graph_seed, int k, asap_ctx** out) {
+  if (!out) return fail(nullptr, ASAP_ERR_ARG, "out is NULL");
+  *out = nullptr;
+  if (N < 1 || N > kMaxWorkers || d < 1 || k < 0 || k > N - 1)
+    return fail(nullptr, ASAP_ERR_ARG, "need 1 <= N <= 1024, d >= 1, 0 <= k <= N-1");
+  std::unique_ptr<asap_ctx> holder(new asap_ctx());
+  asap_ctx* c = holder.get();
+  c->N = N;
+  c->d = d;
+  c->seed = graph_seed;
+  c->k = k;
+  c->kind = (k == 0) ? ASAP_GRAPH_IDENTITY
+            : (k == N - 1) ? ASAP_GRAPH_COMPLETE
+            : (k == 1) ? ASAP_GRAPH_RING
+                       : ASAP_GRAPH_RANDOM_REGULAR;
+  if (c->kind == ASAP_GRAPH_RANDOM_REGULAR && k + 1 > kMaxKp1Sparse)
+    return fail(nullptr, ASAP_ERR_ARG, "k+1 > 32 is supported only for the complete graph");
+  asap_status s = init_ctx(c);
   if (s != ASAP_OK) {
     g_last_error = c->err;
     asap_destroy(holder.release());

@@ -54,3 +54,19 @@ def test_graph_builder_rejects_bad_kinds(lib):
     for kind, N, k in [("ring", 4, 2), ("root", 3, 2), ("complete", 5, 3), ("random_regular", 4, 0)]:
         with pytest.raises(AsapError):
             build_graph(kind, N, k)
+
+
+def test_create_rejects_bad_sizes_and_reports_a_missing_device(lib):
+    import ctypes as C
+    h = C.c_void_p()
+    for N, d, k in [(0, 10, 0), (4, 0, 1), (4, 10, 4), (4, 10, -1), (2000, 10, 1), (64, 10, 40)]:
+        assert lib.asap_create(N, d, 0, k, C.byref(h)) == 1, (N, d, k)   # ASAP_ERR_ARG
+        assert not h.value
+        assert lib.asap_last_error(None)
+    import torch
+    if torch.cuda.is_available():
+        pytest.skip("a device is present")
+    # No device: the context's first CUDA call fails; nothing is returned.
+    assert lib.asap_create(4, 10, 0, 1, C.byref(h)) == 2                  # ASAP_ERR_CUDA
+    assert not h.value
+    assert lib.asap_last_error(None)

@@ -74,3 +74,9 @@ def test_batch_image_rejects_bad_slab_width():
     sh = inputs.sparse_custom(seed=1, N=2, d=100, rows=16, max_len=5)
     with pytest.raises(AsapError):
         debug_batch_image(sh, 8, 48, 0)
+
+
+def test_batch_image_rejects_a_minibatch_past_the_shard():
+    sh = inputs.sparse_custom(seed=1, N=2, d=100, rows=16, max_len=5)
+    with pytest.raises(ValueError):
+        debug_batch_image(sh, 8, 64, 2)

@@ -1021,93 +1021,95 @@ asap_status asap_load_shards(asap_ctx* c, const int64_t* const* rowptr, const in
   c->s_cap = 1024;
   s0 = setup_mix(c);
   if (s0 != ASAP_OK) return s0;
+  // Build every minibatch's image; narrow the slabs and rebuild while a
+  // slab's column list is too long for the fused reduce's shared memory.
   for (;;) {
-  const int S = c->S;
-  const long long n_slabs = c->n_slabs;
+    const int S = c->S;
+    const long long n_slabs = c->n_slabs;
 
-  std::vector<BatchImage> built(nb);
-  auto build_batch = [&](int t) { build_batch_image(N, B, c->d, S, n_slabs, t, rowptr, col, val, y, built[t]); };
-  {
-    const unsigned nthr = std::max(1u, std::min(32u, std::thread::hardware_concurrency()));
-    std::vector<std::thread> pool;
-    for (unsigned w = 0; w < nthr; ++w)
-      pool.emplace_back([&, w]() {
-        for (int t = static_cast<int>(w); t < nb; t += static_cast<int>(nthr)) build_batch(t);
-      });
-    for (auto& th : pool) th.join();
-  }
-  size_t total = 0;
-  int max_nnz = 0, max_region = 0;
-  int64_t max_list = 0;
-  for (int t = 0; t < nb; ++t)
-    if (built[t].err) return fail(c, ASAP_ERR_ARG, built[t].err);
-  for (int t = 0; t < nb; ++t) max_region = std::max(max_region, built[t].max_region);
-  // Two stages of the fused reduce (slab + three list regions each) must fit
-  // in shared memory; skewed column popularity calls for narrower slabs.
-  if (mix_smem_bytes(N, std::min(c->k + 1, kMaxKp1Sparse), S, c->rows_pad, 2, max_region) > (220u << 10)) {
-    if (S <= 8) return fail(c, ASAP_ERR_ARG, "a column slab's list does not fit in shared memory");
-    c->s_cap = S / 2;
-    asap_status sm = setup_mix(c);
-    if (sm != ASAP_OK) return sm;
-    continue;
-  }
-  max_region = 0;
-  c->block_off.assign(nb, 0);
-  c->block_bytes.assign(nb, 0);
-  c->list_off.assign(nb, 0);
-  c->soff_off.assign(nb, 0);
-  c->list_len.assign(nb, 0);
-  std::vector<BatchDesc> desc(static_cast<size_t>(nb) * N);
-  for (int t = 0; t < nb; ++t) {
-    if (built[t].err) return fail(c, ASAP_ERR_ARG, built[t].err);
-    c->block_off[t] = total;
-    c->block_bytes[t] = built[t].img.size();
-    c->list_off[t] = built[t].list_off;
-    c->soff_off[t] = built[t].soff_off;
-    c->list_len[t] = built[t].list_len;
-    total += built[t].img.size();
-    max_nnz = std::max(max_nnz, built[t].max_nnz);
-    max_region = std::max(max_region, built[t].max_region);
-    max_list = std::max(max_list, built[t].list_len);
-    std::copy(built[t].desc.begin(), built[t].desc.end(), desc.begin() + static_cast<size_t>(t) * N);
-  }
-  if (c->residency == ASAP_SHARDS_HOST) {
-    CU(cudaHostAlloc(&c->pool, total, cudaHostAllocDefault), "allocating pinned shard memory");
-    c->pool_pinned = true;
-    size_t mb = 0;
-    for (int t = 0; t < nb; ++t) {
-      std::memcpy(c->pool + c->block_off[t], built[t].img.data(), built[t].img.size());
-      mb = std::max(mb, built[t].img.size());
-      std::vector<unsigned char>().swap(built[t].img);
+    std::vector<BatchImage> built(nb);
+    auto build_batch = [&](int t) { build_batch_image(N, B, c->d, S, n_slabs, t, rowptr, col, val, y, built[t]); };
+    {
+      const unsigned nthr = std::max(1u, std::min(32u, std::thread::hardware_concurrency()));
+      std::vector<std::thread> pool;
+      for (unsigned w = 0; w < nthr; ++w)
+        pool.emplace_back([&, w]() {
+          for (int t = static_cast<int>(w); t < nb; t += static_cast<int>(nthr)) build_batch(t);
+        });
+      for (auto& th : pool) th.join();
     }
-    c->staging_bytes = mb;
-    for (int b = 0; b < asap_ctx::kStaging; ++b) CU(cudaMalloc(&c->staging[b], mb), "allocating staging buffers");
-  } else {
-    CU(cudaMalloc(&c->pool, total), "allocating device shard memory");
-    c->pool_pinned = false;
-    for (int t = 0; t < nb; ++t) {
-      CU(cudaMemcpy(c->pool + c->block_off[t], built[t].img.data(), built[t].img.size(), cudaMemcpyHostToDevice),
-         "copying shards to the device");
-      std::vector<unsigned char>().swap(built[t].img);
+    size_t total = 0;
+    int max_nnz = 0, max_region = 0;
+    int64_t max_list = 0;
+    for (int t = 0; t < nb; ++t)
+      if (built[t].err) return fail(c, ASAP_ERR_ARG, built[t].err);
+    for (int t = 0; t < nb; ++t) max_region = std::max(max_region, built[t].max_region);
+    // Two stages of the fused reduce (slab + three list regions each) must fit
+    // in shared memory; skewed column popularity calls for narrower slabs.
+    if (mix_smem_bytes(N, std::min(c->k + 1, kMaxKp1Sparse), S, c->rows_pad, 2, max_region) > (220u << 10)) {
+      if (S <= 8) return fail(c, ASAP_ERR_ARG, "a column slab's list does not fit in shared memory");
+      c->s_cap = S / 2;
+      asap_status sm = setup_mix(c);
+      if (sm != ASAP_OK) return sm;
+      continue;
     }
-  }
-  c->pool_bytes = total;
-  CU(cudaMalloc(&c->d_desc, desc.size() * sizeof(BatchDesc)), "allocating batch descriptors");
-  CU(cudaMemcpy(c->d_desc, desc.data(), desc.size() * sizeof(BatchDesc), cudaMemcpyHostToDevice),
-     "copying batch descriptors");
-  const size_t lb = 4 * static_cast<size_t>(std::max<int64_t>(max_list, 4));
-  CU(cudaMalloc(&c->wv, lb), "allocating the list value buffer");
-  CU(cudaMalloc(&c->gsum, lb), "allocating the column-sum buffer");
-  CU(cudaMemset(c->wv, 0, lb), "zeroing the list value buffer");
-  CU(cudaMemset(c->gsum, 0, lb), "zeroing the column-sum buffer");
-  c->nb = nb;
-  c->max_nnz = max_nnz;
-  c->max_region = max_region;
-  c->max_list = max_list;
-  c->wv_step = -1;
-  c->update_ctas = update_ctas_for(max_nnz);
-  c->configured_key = -1;
-  return ASAP_OK;
+    max_region = 0;
+    c->block_off.assign(nb, 0);
+    c->block_bytes.assign(nb, 0);
+    c->list_off.assign(nb, 0);
+    c->soff_off.assign(nb, 0);
+    c->list_len.assign(nb, 0);
+    std::vector<BatchDesc> desc(static_cast<size_t>(nb) * N);
+    for (int t = 0; t < nb; ++t) {
+      if (built[t].err) return fail(c, ASAP_ERR_ARG, built[t].err);
+      c->block_off[t] = total;
+      c->block_bytes[t] = built[t].img.size();
+      c->list_off[t] = built[t].list_off;
+      c->soff_off[t] = built[t].soff_off;
+      c->list_len[t] = built[t].list_len;
+      total += built[t].img.size();
+      max_nnz = std::max(max_nnz, built[t].max_nnz);
+      max_region = std::max(max_region, built[t].max_region);
+      max_list = std::max(max_list, built[t].list_len);
+      std::copy(built[t].desc.begin(), built[t].desc.end(), desc.begin() + static_cast<size_t>(t) * N);
+    }
+    if (c->residency == ASAP_SHARDS_HOST) {
+      CU(cudaHostAlloc(&c->pool, total, cudaHostAllocDefault), "allocating pinned shard memory");
+      c->pool_pinned = true;
+      size_t mb = 0;
+      for (int t = 0; t < nb; ++t) {
+        std::memcpy(c->pool + c->block_off[t], built[t].img.data(), built[t].img.size());
+        mb = std::max(mb, built[t].img.size());
+        std::vector<unsigned char>().swap(built[t].img);
+      }
+      c->staging_bytes = mb;
+      for (int b = 0; b < asap_ctx::kStaging; ++b) CU(cudaMalloc(&c->staging[b], mb), "allocating staging buffers");
+    } else {
+      CU(cudaMalloc(&c->pool, total), "allocating device shard memory");
+      c->pool_pinned = false;
+      for (int t = 0; t < nb; ++t) {
+        CU(cudaMemcpy(c->pool + c->block_off[t], built[t].img.data(), built[t].img.size(), cudaMemcpyHostToDevice),
+           "copying shards to the device");
+        std::vector<unsigned char>().swap(built[t].img);
+      }
+    }
+    c->pool_bytes = total;
+    CU(cudaMalloc(&c->d_desc, desc.size() * sizeof(BatchDesc)), "allocating batch descriptors");
+    CU(cudaMemcpy(c->d_desc, desc.data(), desc.size() * sizeof(BatchDesc), cudaMemcpyHostToDevice),
+       "copying batch descriptors");
+    const size_t lb = 4 * static_cast<size_t>(std::max<int64_t>(max_list, 4));
+    CU(cudaMalloc(&c->wv, lb), "allocating the list value buffer");
+    CU(cudaMalloc(&c->gsum, lb), "allocating the column-sum buffer");
+    CU(cudaMemset(c->wv, 0, lb), "zeroing the list value buffer");
+    CU(cudaMemset(c->gsum, 0, lb), "zeroing the column-sum buffer");
+    c->nb = nb;
+    c->max_nnz = max_nnz;
+    c->max_region = max_region;
+    c->max_list = max_list;
+    c->wv_step = -1;
+    c->update_ctas = update_ctas_for(max_nnz);
+    c->configured_key = -1;
+    return ASAP_OK;
   }
 }
 

@@ -249,6 +249,11 @@ __global__ void __launch_bounds__(kThreads) k_column_sums(SparseStepArgs a) {
     }
   }
 
+  // A CTA without chunks has not waited for the margin kernel yet.  Were no
+  // CTA to wait (an all-empty minibatch), this grid could complete before the
+  // margin kernel, and the reduce would read its loss partials too early.
+  wait_previous();
+
   // NOTIFY: the last CTA of worker i publishes ready[i] = round + 1 once all
   // of worker i's column sums are visible device-wide.  The CTA barrier
   // orders this CTA's writes before thread 0's fence, which is cumulative.

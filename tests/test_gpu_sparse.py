@@ -81,6 +81,21 @@ def test_ragged_edge_cases(loss, residency):
     _run_parity(ctx, sh, T, B, loss, lr, sched)
 
 
+def test_all_empty_minibatch():
+    # Minibatch 1 has no entries on any worker: margins 0, no column sums, the
+    # loss of every row at m = 0.
+    N, d, B, lr, T = 4, 300, 16, 0.5, 4
+    rng = np.random.default_rng(21)
+    lengths = [rng.integers(1, 20, 3 * B) for _ in range(N)]
+    for ln in lengths:
+        ln[B:2 * B] = 0
+    sh = inputs.sparse_custom(seed=13, N=N, d=d, rows=3 * B, lengths=lengths)
+    sched = rounds.graph_schedule("ring", N, 1)
+    ctx = _ctx(N, d, 1, 0, "ring", False, "logistic", B, lr, sh)
+    lg = _run_parity(ctx, sh, T, B, "logistic", lr, sched)
+    assert abs(lg[1] - np.log(2.0)) <= 1e-6
+
+
 def test_l2_regularised_logistic():
     N, d, B, lr, l2, T = 5, 300, 40, 0.3, 0.1, 5
     sh = inputs.sparse_custom(seed=4, N=N, d=d, rows=3 * B, max_len=30)

@@ -114,7 +114,7 @@ asap_status asap_set_mixing(asap_ctx* ctx, const int32_t* nbr, const float* wgt)
  * batch: minibatch rows B per worker per round (round t uses rows
  * [(t mod nb) B, (t mod nb) B + B), nb = floor(rows / B)); lr: eta (> 0);
  * l2: coefficient of (l2/2) ||w||^2 in f_i (0 <= lr*l2 < 1).
- * SOFTMAX requires d % 64 == 0, B % 128 == 0, C <= 1024.  Re-setting the
+ * SOFTMAX requires d % 256 == 0, B % 128 == 0, 2 <= C <= 1024.  Re-setting the
  * model clears the shards and resets W to 0. */
 asap_status asap_set_model(asap_ctx* ctx, asap_loss loss, int num_classes, int batch, float lr, float l2);
 
@@ -168,8 +168,11 @@ asap_status asap_load_dense_shards(asap_ctx* ctx, const uint16_t* const* X_bf16,
                                    const int64_t* n_rows);
 
 /* Eq. A.1 first line for every worker, then NOTIFY (ready[i] = t+1).
- * Async.  Between this call and asap_stochastic_reduce the current buffer
- * holds w_{t+1/2} (divided by (1 - lr*l2) when l2 > 0). */
+ * Async.  Between this call and asap_stochastic_reduce, for SOFTMAX models
+ * the current buffer holds w_{t+1/2}.  For hinge / logistic models it holds
+ * w_t with every local step but the round's last applied (values scaled by
+ * the inverse L2 shrink of those steps); the last step's update is applied
+ * by the reduce to each column slab it loads, so w_{t+1/2} is never stored. */
 asap_status asap_local_step(asap_ctx* ctx);
 
 /* Eq. A.1 second line for every worker: wait for the in-neighbours' NOTIFY,

@@ -216,7 +216,9 @@ def kernel_work(sh):
         touched += np.unique(sh.col[i][rp[0]:rp[-1]]).shape[0]
     nnz, pad, touched = nnz * N / samples, pad * N / samples, touched * N / samples
     out["margin"] = ("GB/s", 8.0 * pad + 4.0 * nnz + 8.0 * N * B, "hbm")
-    out["update"] = ("GB/s", 10.0 * nnz + 8.0 * touched + 4.0 * N * B, "hbm")
+    # entries (list position, value, row: 10 B), one fp32 sum written per
+    # distinct (worker, column), the margin kernel's r read once
+    out["update"] = ("GB/s", 10.0 * nnz + 4.0 * touched + 4.0 * N * B, "hbm")
     out["reduce"] = ("GB/s", 8.0 * N * ld, "hbm")
     # local steps before the round's last: the update scatter and the next gather
     out["apply"] = ("GB/s", 16.0 * touched, "hbm")    # list + column sum read, w read + write per column

@@ -70,7 +70,7 @@ typedef enum {
 
 typedef enum {
   ASAP_LOSS_NONE = 0,     /* no local step: the context only mixes              */
-  ASAP_LOSS_HINGE = 1,    /* linear SVM, l = max(0, 1 - y m) (Section 5)         */
+  ASAP_LOSS_HINGE = 1,    /* linear SVM, l = max(0, 1 - y m) (Section 6)         */
   ASAP_LOSS_LOGISTIC = 2, /* l = ln(1 + exp(-y m))                              */
   ASAP_LOSS_SOFTMAX = 3   /* dense softmax regression on bf16 features          */
 } asap_loss;
@@ -92,8 +92,8 @@ typedef enum {
 asap_status asap_create(int N, int64_t d, uint64_t graph_seed, int k, asap_ctx** out);
 
 /* Choose the graph kind, and whether a new graph is drawn from
- * (graph_seed, round) every round (Section 3.1: graphs should be "easy to
- * generate", including re-configuration).  The kind must match k (RING: 1,
+ * (graph_seed, round) every round (Section 3.1 wants graphs that are cheap
+ * to build, so that they can be rebuilt, e.g. around a failure).  The kind must match k (RING: 1,
  * ROOT: 2, COMPLETE: N-1, IDENTITY: 0).  RANDOM_REGULAR construction:
  * SplitMix64 seeded with graph_seed ^ (0x9E3779B97F4A7C15 * (round+1));
  * a uniform random Hamiltonian cycle (Fisher-Yates), then k-1 permutation
@@ -125,8 +125,8 @@ typedef enum {
 } asap_lr_schedule;
 
 /* Local steps per round and the learning-rate schedule.  Eq. A.1 writes the
- * rate as eta_t; Section 4 has the replicas exchange parameters "after
- * processing a few data examples".  Each round runs local_steps (>= 1)
+ * rate as eta_t; in Section 5 each replica trains on a handful of local
+ * examples between two exchanges.  Each round runs local_steps (>= 1)
  * minibatch steps per worker before the reduce: step j of round t is global
  * step k = t * local_steps + j, on minibatch k mod nb, at rate eta_k;
  * asap_local_step runs all of them and the round's loss metric is its last
@@ -209,7 +209,7 @@ asap_status asap_read_metrics(asap_ctx* ctx, int64_t first_round, int64_t count,
                               float* consensus_out);
 
 /* Counters of the NOTIFY-ACK protocol since creation: reduces performed,
- * in-neighbour inputs whose round stamp matched (Section 5.2 reports the
+ * in-neighbour inputs whose round stamp matched (Section 6.2 reports the
  * share of such consistent reduces), and waits that ran out.  Syncing. */
 asap_status asap_read_counters(asap_ctx* ctx, uint64_t* reduces, uint64_t* consistent_inputs,
                                uint64_t* timeouts);
@@ -229,7 +229,7 @@ asap_status asap_set_wait_limit_ns(asap_ctx* ctx, uint64_t ns);
 asap_status asap_debug_skip_notify(asap_ctx* ctx, int worker);
 
 /* Host only, for tests (no device needed): the image asap_load_shards builds
- * for minibatch t -- the index structure of Section 4's per-worker updates
+ * for minibatch t -- the index structure of Section 5's per-worker updates
  * laid out for the stochastic reduce's column slabs (no counterpart in the
  * paper beyond that).  Shards as in asap_load_shards, each with at least
  * (t + 1) * batch rows (not checked: there is no row count here); batch: B rows;

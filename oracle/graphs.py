@@ -3,8 +3,9 @@
 Paper passages followed:
 * Section 3.1 and Fig. 2: the all-reduce (complete) graph, the chain graph,
   and the "root" expander in which node i sends to i+1 and to i+sqrt(N).
-* Section 3.1 ("easy to generate ... re-configuration in case of a failure"):
-  a graph is produced from a seed, and may be produced anew every round.
+* Section 3.1 (such graphs are cheap to build, so a failed node can be
+  routed around by building a new one): a graph is produced from a seed,
+  and may be produced anew every round.
 * Appendix A, "Network requirement": A_ij = 1 iff (j, i) is an edge, self
   included; P = diag(d_in)^-1 A; P must be doubly stochastic, i.e. every node
   has the same in- and out-degree.

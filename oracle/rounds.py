@@ -7,7 +7,8 @@ takes w_0 = 0).  Per round the oracle records the mean over workers of the
 minibatch loss at the pre-step model and the consensus error after the reduce.
 
 ``graph`` is a callable rnd -> (nbr, wgt) so that a graph regenerated every
-round (Section 3.1, "easy to generate") and a fixed one look the same here.
+round (Section 3.1: such graphs are cheap to build afresh) and a fixed one
+look the same here.
 """
 from __future__ import annotations
 
@@ -34,8 +35,8 @@ def sparse_round(W, shards, t, B, loss, lr, nbr, wgt, l2=0.0, flips=None, tau=1,
     """One round from W_t (any float array [N, d]); returns
     (W_{t+1} fp64, mean minibatch loss, consensus error of W_{t+1}).
 
-    Each worker takes ``tau`` local steps before the reduce (Section 4: the
-    replicas communicate after processing a few examples): step j of round t
+    Each worker takes ``tau`` local steps before the reduce (Section 5: the
+    replicas exchange models after a handful of local examples): step j of round t
     is global step k = t*tau + j, on minibatch k and at rate lr_at(k) (``lr``
     when lr_at is None).  The loss is the workers' mean minibatch loss of the
     round's last step, at its pre-step model.  ``flips`` maps a worker to the

@@ -2,9 +2,9 @@
 
 Paper passages followed:
 * Eq. A.1, first line: w_{t+1/2} = w_t - eta_t * grad f_i(w_t).
-* Section 4 (Implementation): each replica updates its local model after
-  processing a few data examples, then communicates.
-* Section 5: the linear SVM of Bottou's SVM-SGD (hinge loss).
+* Section 5 (Implementation): each replica trains its own model on a
+  handful of local examples between two exchanges.
+* Section 6 (Evaluation): the linear SVM of Bottou's SVM-SGD (hinge loss).
 
 Readings where the paper is silent (stated in the design notes):
 * minibatch of round t = rows [(t mod nb) B, (t mod nb) B + B) of the
@@ -74,7 +74,7 @@ def sparse_gradient(rowptr, col, val, r, b0, B, d):
 def learning_rate(kind: str, eta0: float, gamma: float, k: int) -> float:
     """eta_k of local step k (Eq. A.1 writes the rate as eta_t): ``constant``
     keeps eta0; ``inverse`` is eta0 / (1 + gamma k), the decreasing rate of
-    Bottou's SVM-SGD, which the paper's SVM experiments use (Section 5)."""
+    Bottou's SVM-SGD, which the paper's SVM experiments use (Section 6)."""
     if kind == "constant":
         return float(eta0)
     if kind == "inverse":

@@ -12,7 +12,8 @@
 //                   rejection; SplitMix64 (Steele, Lea & Flood 2014) seeded
 //                   by graph_seed ^ (gamma * (round + 1)).
 // The paper fixes no construction for random expanders; this one is cheap
-// enough to redo every round on the host ("easy to generate", Section 3.1).
+// enough to redo every round on the host (Section 3.1 asks for graphs that
+// are cheap to build).
 #include <algorithm>
 #include <cstdint>
 #include <vector>

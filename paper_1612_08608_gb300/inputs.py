@@ -6,7 +6,7 @@ mixing or graph construction), so the CPU oracle and the CUDA path can both
 be fed from it without sharing any of the computation they are compared on.
 
 The paper trains linear SVMs on RCV1, webspam and splice-site and a CNN on
-CIFAR-10 (Section 5, "Evaluation").  None of those datasets is available here;
+CIFAR-10 (Section 6, "Evaluation").  None of those datasets is available here;
 the generators below stand in for them with the same shapes, sparsity
 patterns and value distributions:
 

@@ -1,6 +1,6 @@
 """Graph comparison on one GB300: rounds, time and bytes to a target loss.
 
-Section 5 compares ASAP's stochastic reduce over sparse graphs with the
+Section 6.1 compares ASAP's stochastic reduce over sparse graphs with the
 all-reduce: sparse graphs need about as many iterations, while each worker
 receives only its k in-neighbours' models per round instead of all N-1.
 Here every graph runs the same workers, shards and model settings.  The

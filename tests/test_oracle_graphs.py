@@ -5,7 +5,7 @@ the mathematics fix (no GPU).
 * Fisher-Yates uniformity (brute force over all permutations of 3).
 * Every graph kind: in-degree = out-degree = k+1, so P is doubly stochastic
   (Appendix A, "Network requirement").
-* Spectral gap against the values printed in Fig. 2 / Section 5.1 and against
+* Spectral gap against the values printed in Fig. 2 / Section 6.1 and against
   circulant closed forms (Appendix A, "Spectral Gap").
 * Mixing preserves the worker average; the consensus error contracts by at
   least sigma_2(P) per round (Appendix A's Perron-Frobenius bound).

@@ -14,6 +14,10 @@
 * Learning-rate schedules at literal values; two local steps per round by
   hand (inverse rate, with and without L2); one worker with tau local steps
   equals textbook minibatch SGD over the global step sequence.
+* A hand-computed softmax step from a W that bf16 cannot represent: the
+  logits read RNE_bf16(W), R is rounded to bf16, the fp32 master is updated.
+* rounds.softmax_round against a restatement with dense matrices (step with
+  torch's bf16 casts, then P H with P written out, the loss and consensus).
 """
 import itertools
 import math
@@ -280,3 +284,75 @@ def test_local_steps_are_textbook_sgd_over_global_steps():
         s = 1.0 / (1.0 + np.exp(yb * (Xb @ w)))
         w = w - eta0 / (1.0 + gamma * k) / B * (Xb.T @ (-yb * s))
     assert Wo[0] == pytest.approx(w, abs=1e-14)
+
+
+def test_hand_computed_softmax_step_reads_w_in_bf16():
+    # C = 2 classes, d = 3, one row x = [1, 2, -1] (exact in bf16) of class 0,
+    # B = 1, eta = 0.5.  W is not representable in bf16, so the logits use
+    # RNE_bf16(W) while the update applies to the fp32 master:
+    #   W[0] = [1 + 2^-8, 0.75 + 3 2^-10, -0.5 - 2^-11]
+    #     -> [1 (tie, to even), 0.75 + 2^-8, -0.5]
+    #   W[1] = [1 + 3 2^-8, -(2^-4 + 2^-13), 0.25 + 2^-10]
+    #     -> [1 + 2^-6 (tie, to even), -2^-4, 0.25 (tie, to even)]
+    # z = [1 + 1.5 + 2^-7 + 0.5, 1 + 2^-6 - 2^-3 - 0.25] = [3.0078125, 0.640625]
+    # p1 = 1 / (1 + e^{2.3671875}) = 0.0857093..., p0 = 1 - p1
+    # R = (p - e_0) / 1 = [p0 - 1, p1] = [-0.0857093..., 0.0857093...]; in bf16
+    #   0.0857093 / 2^-11 = 175.53 -> 176 2^-11 = 0.0859375, so R = [-0.0859375, 0.0859375]
+    # H[c] = W[c] - 0.5 R_c x:
+    #   H[0] = W[0] + 0.04296875 [1, 2, -1] = [1.046875, 0.8388671875, -0.54345703125]
+    #   H[1] = W[1] - 0.04296875 [1, 2, -1] = [0.96875, -0.1485595703125, 0.2939453125]
+    # loss = ln(1 + e^{z1 - z0}) = log1p(exp(-2.3671875))
+    W = np.array([[1 + 2 ** -8, 0.75 + 3 * 2 ** -10, -0.5 - 2 ** -11],
+                  [1 + 3 * 2 ** -8, -(2 ** -4 + 2 ** -13), 0.25 + 2 ** -10]], np.float32)
+    assert np.array_equal(W.astype(np.float64), [[1.00390625, 0.7529296875, -0.50048828125],
+                                                 [1.01171875, -0.0626220703125, 0.2509765625]])
+    Xbits = np.array([[0x3F80, 0x4000, 0xBF80]], np.uint16)       # bf16 bits of 1, 2, -1
+    y = np.array([0], np.int32)
+    H, loss = sgd.softmax_worker_step(W, Xbits, y, 0, 1, 0.5)
+    assert H == pytest.approx(np.array([[1.046875, 0.8388671875, -0.54345703125],
+                                        [0.96875, -0.1485595703125, 0.2939453125]]), abs=1e-15)
+    assert loss == pytest.approx(math.log1p(math.exp(-2.3671875)), abs=1e-15)
+    # The three plausible slips each move H: reading W unrounded, rounding the
+    # master before the update, or skipping the bf16 rounding of R.
+    Hu, _ = sgd.softmax_worker_step(W, Xbits, y, 0, 1, 0.5, mirror_bf16=False)
+    assert np.abs(Hu - H).max() > 1e-4
+
+
+def test_softmax_round_is_step_then_reduce_as_dense_matrices():
+    # rounds.softmax_round against a restatement with dense matrices: per
+    # worker the logits from the bf16-rounded model (torch's bf16 cast), the
+    # softmax residual rounded to bf16, the fp32 master updated with an L2
+    # term; then W' = P H with P written out, the mean loss and
+    # ||W' - 1 wbar^T||_F.
+    import torch
+    N, d, C, B, t, lr, l2 = 3, 8, 4, 4, 1, 0.3, 0.05
+    sh = inputs.dense_softmax(seed=5, N=N, d=d, C=C, rows=2 * B)
+    rng = np.random.default_rng(2)
+    W = (0.3 * rng.standard_normal((N, C * d))).astype(np.float32)
+    nbr = np.array([[0, 2], [0, 1], [1, 2]])                 # ring: i <- i-1, weights 1/2
+    wgt = np.full((3, 2), 0.5)
+    P = np.zeros((3, 3))
+    P[0, 0] = P[0, 2] = P[1, 0] = P[1, 1] = P[2, 1] = P[2, 2] = 0.5
+
+    def bf16(a):
+        return torch.from_numpy(np.asarray(a, np.float32)).to(torch.bfloat16).to(torch.float64).numpy()
+
+    H = np.zeros((N, C * d))
+    losses = []
+    for i in range(N):
+        X = bf16(np.asarray(torch.from_numpy(sh.X[i].view(np.int16)).view(torch.bfloat16).float()))[B:2 * B]
+        yb = sh.y[i][B:2 * B]
+        Wm = W[i].reshape(C, d).astype(np.float64)
+        Z = X @ bf16(W[i].reshape(C, d)).T
+        lse = np.logaddexp.reduce(Z, axis=1)
+        losses.append(np.mean(lse - Z[np.arange(B), yb]))
+        R = np.exp(Z - lse[:, None])
+        R[np.arange(B), yb] -= 1.0
+        R = bf16(R / B)
+        H[i] = (Wm - lr * (R.T @ X + l2 * Wm)).reshape(-1)
+    Wn = P @ H
+    cons = np.sqrt(((Wn - Wn.mean(axis=0)) ** 2).sum())
+    got, lval, c = rounds.softmax_round(W, sh, t, B, lr, nbr, wgt, l2=l2)
+    assert got == pytest.approx(Wn, abs=1e-13)
+    assert lval == pytest.approx(np.mean(losses), abs=1e-13)
+    assert c == pytest.approx(cons, abs=1e-13)

@@ -195,6 +195,17 @@ asap_status asap_read_params(asap_ctx* ctx, float* host_out, int64_t* round_out)
  * (resume from a checkpoint, or a custom W_0).  Synchronous. */
 asap_status asap_write_params(asap_ctx* ctx, const float* host_in, int64_t round);
 
+/* Set W_t from device memory: dev_in holds N rows of P floats with row
+ * stride ld_in (>= P), on the context's device; the round counter becomes
+ * `round`.  For parameters that already live in HBM (a resume, or inputs
+ * drawn on the device), without a host round trip.  Synchronous. */
+asap_status asap_write_params_device(asap_ctx* ctx, const float* dev_in, int64_t ld_in, int64_t round);
+
+/* Copy columns [first, first + count) of every worker's current
+ * parameters W_t to host_out (N rows of count floats, row-major): a sample
+ * of the model without reading all N x P values.  Syncing. */
+asap_status asap_read_param_columns(asap_ctx* ctx, int64_t first, int64_t count, float* host_out);
+
 /* Per-round metrics of rounds [first_round, first_round + count): the mean
  * over workers of the minibatch loss at the pre-step parameters (NaN for a
  * reduce-only round) and the consensus error ||W_{t+1} - 1 wbar^T||_F.
@@ -286,7 +297,8 @@ asap_status asap_build_graph(asap_graph_kind kind, int N, int k, uint64_t graph_
  * is the reduce of asap_stochastic_reduce without a context.
  * All pointers are device pointers owned by the caller: W_in, W_out
  * N rows of `ld` floats (row stride ld, ld >= d, ld % 4 == 0, 16-byte
- * aligned, not aliased; columns [d, ld) are mixed too); nbr / wgt N*kp1
+ * aligned, the two ranges of N*ld floats not overlapping; columns [d, ld)
+ * are mixed too); nbr / wgt N*kp1
  * int32 / float (row i = the ids in [0, N) and weights of worker i's
  * inputs, summed in the given order; ids outside [0, N) are clamped into
  * range, never read out of bounds); consensus_out one float, set to
@@ -298,7 +310,10 @@ asap_status asap_build_graph(asap_graph_kind kind, int N, int k, uint64_t graph_
  * (about 256 KB) is a file-scope device array that every GPU loading this
  * library holds until the process exits.  The first call on each device
  * looks up that array's device address (cudaGetSymbolAddress) with the
- * device current, so make that first call before any stream capture.  Every
+ * device current, so make that first call before any stream capture.  The
+ * address is kept per device together with the id of the CUDA context it
+ * was found in; a call from a different context (after cudaDeviceReset, or
+ * a host framework that reset its primary context) looks it up again.  Every
  * call shares the array and clears what must start at zero; calls that
  * overlap on the GPU (other streams, other threads) race on it and must be
  * serialised by the caller.  Async on cuda_stream (NULL: legacy default

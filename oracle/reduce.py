@@ -25,6 +25,13 @@ def stochastic_reduce(H, nbr, wgt):
     return W
 
 
+def reduce_with_matrix(H, P):
+    """The same reduce written as one product W = P H with the dense N x N
+    mixing matrix P (Appendix A); a library matmul serves as the step, so
+    the fp64 summation order is the library's."""
+    return np.asarray(P, dtype=np.float64) @ np.asarray(H, dtype=np.float64)
+
+
 def consensus_error(W) -> float:
     """||W - 1 wbar^T||_F with wbar the mean over workers (rows)."""
     W = np.asarray(W, dtype=np.float64)

@@ -87,6 +87,23 @@ def softmax_round(W, shards, t, B, lr, nbr, wgt, l2=0.0, mirror_bf16=True):
     return Wn, float(np.mean(losses)), reduce.consensus_error(Wn)
 
 
+def run_softmax(shards, T, B, lr, graph, W0=None, l2=0.0, t0=0, lr_at=None):
+    """Free-running dense trajectory from W0 (default 0); the master weights
+    are fp32 between rounds, as on the tensor-core path.  Returns
+    (W_T fp64, losses[T], consensus[T])."""
+    N, P = shards.N, shards.C * shards.d
+    W = np.zeros((N, P), np.float32) if W0 is None else np.asarray(W0, dtype=np.float32)
+    losses, cons = [], []
+    for t in range(t0, t0 + T):
+        nbr, wgt = graph(t)
+        eta = lr if lr_at is None else lr_at(t)
+        Wn, lval, c = softmax_round(W, shards, t, B, eta, nbr, wgt, l2)
+        W = Wn.astype(np.float32)
+        losses.append(lval)
+        cons.append(c)
+    return Wn, np.array(losses), np.array(cons)
+
+
 def mixing_rounds(W0, T, graph, t0=0):
     """Stochastic reduce alone, T times; returns (W_T fp64, consensus[T])."""
     W = np.asarray(W0, dtype=np.float64)

@@ -115,10 +115,11 @@ def bf16_to_f64(bits) -> np.ndarray:
     return (np.asarray(bits, dtype=np.uint16).astype(np.uint32) << 16).view(np.float32).astype(np.float64)
 
 
-def softmax_worker_step(Wm, Xbits, y, t, B, lr, mirror_bf16=True, l2=0.0):
-    """Dense softmax regression for one worker.  Wm: [C, d] float32 master
-    weights; Xbits: [rows, d] bf16 bits; y: [rows] class ids.  Returns
-    (W_{t+1/2} fp64 [C, d], mean loss at W_t)."""
+def softmax_residual(Wm, Xbits, y, t, B, mirror_bf16=True):
+    """The minibatch of round t for one worker: returns (X_b fp64 [B, d],
+    R = (softmax(X_b Wread^T) - onehot(y_b)) / B fp64 [B, C] before any
+    rounding, mean loss at W_t).  Wread = RNE_bf16(Wm) when mirroring the
+    tensor-core path, else Wm."""
     b0, _ = batch_window(t, Xbits.shape[0], B)
     X = bf16_to_f64(Xbits[b0:b0 + B])
     yb = np.asarray(y[b0:b0 + B], dtype=np.int64)
@@ -131,9 +132,16 @@ def softmax_worker_step(Wm, Xbits, y, t, B, lr, mirror_bf16=True, l2=0.0):
     loss = lse - Z[np.arange(B), yb]
     Pm = E / S
     Pm[np.arange(B), yb] -= 1.0
-    R = Pm / B
+    return X, Pm / B, float(loss.mean())
+
+
+def softmax_worker_step(Wm, Xbits, y, t, B, lr, mirror_bf16=True, l2=0.0):
+    """Dense softmax regression for one worker.  Wm: [C, d] float32 master
+    weights; Xbits: [rows, d] bf16 bits; y: [rows] class ids.  Returns
+    (W_{t+1/2} fp64 [C, d], mean loss at W_t)."""
+    X, R, loss = softmax_residual(Wm, Xbits, y, t, B, mirror_bf16)
     if mirror_bf16:
         R = rne_bf16(R.astype(np.float32)).astype(np.float64)
     G = R.T @ X                                       # [C, d]
     H = np.asarray(Wm, dtype=np.float64) - lr * (G + l2 * np.asarray(Wm, dtype=np.float64))
-    return H, float(loss.mean())
+    return H, loss

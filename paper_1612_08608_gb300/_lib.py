@@ -33,6 +33,8 @@ SIGNATURES = {
     "asap_sync": (C.c_int, [_P]),
     "asap_read_params": (C.c_int, [_P, _P, C.POINTER(C.c_int64)]),
     "asap_write_params": (C.c_int, [_P, _P, C.c_int64]),
+    "asap_write_params_device": (C.c_int, [_P, _P, C.c_int64, C.c_int64]),
+    "asap_read_param_columns": (C.c_int, [_P, C.c_int64, C.c_int64, _P]),
     "asap_read_metrics": (C.c_int, [_P, C.c_int64, C.c_int64, _P, _P]),
     "asap_read_counters": (C.c_int, [_P, C.POINTER(C.c_uint64), C.POINTER(C.c_uint64), C.POINTER(C.c_uint64)]),
     "asap_get_graph": (C.c_int, [_P, C.c_int64, _P, _P]),

@@ -163,6 +163,20 @@ class Context:
         assert W.shape == (self.N, self.P)
         self._c(self._lib.asap_write_params(self._h, _ptr(W), rnd))
 
+    def write_params_device(self, W, rnd: int = 0):
+        """W: a CUDA tensor (float32, N x P with unit column stride) on the
+        context's device; copied device to device."""
+        assert W.dtype.itemsize == 4 and W.dim() == 2 and W.shape[0] == self.N and W.shape[1] >= self.P
+        assert W.stride(1) == 1 and W.is_cuda
+        self._c(self._lib.asap_write_params_device(self._h, C.c_void_p(W.data_ptr()), W.stride(0), rnd))
+
+    def read_param_columns(self, first: int, count: int, out: Optional[np.ndarray] = None):
+        """Columns [first, first + count) of every worker's parameters."""
+        if out is None:
+            out = np.empty((self.N, count), dtype=np.float32)
+        self._c(self._lib.asap_read_param_columns(self._h, first, count, _ptr(out)))
+        return out
+
     def read_metrics(self, first: int, count: int):
         loss = np.empty(count, dtype=np.float32)
         cons = np.empty(count, dtype=np.float32)

@@ -1439,6 +1439,32 @@ asap_status asap_write_params(asap_ctx* c, const float* host_in, int64_t round) 
   return reset_protocol(c, round);
 }
 
+asap_status asap_write_params_device(asap_ctx* c, const float* dev_in, int64_t ld_in, int64_t round) {
+  if (!c || !dev_in || round < 0 || ld_in < c->P) return fail(c, ASAP_ERR_ARG, "bad argument");
+  asap_status s = sync_all(c);
+  if (s != ASAP_OK) return s;
+  float* dst = c->W[round & 1];
+  CU(cudaMemcpy2DAsync(dst, c->ld * 4, dev_in, ld_in * 4, c->P * 4, c->N, cudaMemcpyDeviceToDevice, c->stream),
+     "writing parameters");
+  if (c->Wbf[round & 1]) {
+    CU(launch_cast_bf16(dst, c->Wbf[round & 1], static_cast<int64_t>(c->N) * c->ld, c->stream), "bf16 copy");
+    c->launches += 1;
+  }
+  CU(cudaStreamSynchronize(c->stream), "writing parameters");
+  c->wv_step = -1;
+  return reset_protocol(c, round);
+}
+
+asap_status asap_read_param_columns(asap_ctx* c, int64_t first, int64_t count, float* host_out) {
+  if (!c || !host_out || first < 0 || count < 1 || first + count > c->P) return fail(c, ASAP_ERR_ARG, "bad argument");
+  asap_status s = sync_all(c);
+  if (s != ASAP_OK) return s;
+  CU(cudaMemcpy2D(host_out, count * 4, c->W[c->round & 1] + first, c->ld * 4, count * 4, c->N,
+                  cudaMemcpyDeviceToHost),
+     "reading parameter columns");
+  return ASAP_OK;
+}
+
 asap_status asap_read_metrics(asap_ctx* c, int64_t first, int64_t count, float* loss_out, float* cons_out) {
   if (!c || first < 0 || count < 0) return fail(c, ASAP_ERR_ARG, "bad argument");
   if (first + count > c->round || first < c->round - kMetricsCap)

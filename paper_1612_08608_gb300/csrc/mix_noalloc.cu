@@ -15,6 +15,7 @@
 // instead of a TMA pipeline, no NOTIFY-ACK flags and at most 256 workers;
 // the arithmetic (weights applied in row order, column means from the
 // input, fp64 partial sums) is the same.
+#include <cuda.h>
 #include <cuda_runtime.h>
 
 #include <algorithm>
@@ -141,7 +142,8 @@ __global__ void __launch_bounds__(kThreads) k_mix_noalloc(const NoAllocArgs a) {
     __syncthreads();   // the slab buffer is reused by the next slab
   }
 
-  // The last CTA sums the per-slab partials in slab order.
+  // The last CTA sums the per-slab partials in a fixed order (the result does
+  // not depend on which CTA finishes last).
   __threadfence();
   __syncthreads();
   if (tid == 0) flag[0] = (atomicAdd(a.ticket, 1u) == gridDim.x - 1) ? 1 : 0;
@@ -160,7 +162,38 @@ __global__ void __launch_bounds__(kThreads) k_mix_noalloc(const NoAllocArgs a) {
 struct DeviceSlot {
   void* scratch = nullptr;
   int sm_count = 0;
+  unsigned long long ctx_id = 0;   // the CUDA context the address belongs to
 };
+
+// Unique id of the calling thread's current CUDA context (0: none current).
+// A device reset, or a host framework that resets its primary context,
+// reloads this library's module at a new address; the id tells the cached
+// scratch address apart from a stale one.  The driver entry points are
+// looked up through the runtime, so the library needs no link to libcuda.
+unsigned long long current_context_id() {
+  typedef CUresult (*GetCurrentFn)(CUcontext*);
+  typedef CUresult (*GetIdFn)(CUcontext, unsigned long long*);
+  static GetCurrentFn get_current = nullptr;
+  static GetIdFn get_id = nullptr;
+  static bool looked_up = false;
+  if (!looked_up) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 4000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      get_current = reinterpret_cast<GetCurrentFn>(p);
+    p = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      get_id = reinterpret_cast<GetIdFn>(p);
+    looked_up = true;
+  }
+  CUcontext ctx = nullptr;
+  unsigned long long id = 0;
+  if (!get_current || !get_id || get_current(&ctx) != CUDA_SUCCESS || !ctx || get_id(ctx, &id) != CUDA_SUCCESS)
+    return 0;
+  return id;
+}
 
 std::mutex g_noalloc_mu;
 DeviceSlot g_noalloc_dev[kNoAllocMaxDevices];
@@ -177,11 +210,18 @@ extern "C" asap_status asap_mix_noalloc(const float* W_in, float* W_out, int N, 
                                         void* cuda_stream) {
   if (!W_in || !W_out || !nbr || !wgt || !consensus_out)
     return reject(ASAP_ERR_ARG, "asap_mix_noalloc: NULL pointer");
-  if (W_in == W_out) return reject(ASAP_ERR_ARG, "asap_mix_noalloc: W_in and W_out must not alias");
   if (N < 1 || N > kNoAllocMaxN) return reject(ASAP_ERR_ARG, "asap_mix_noalloc: need 1 <= N <= 256");
   if (kp1 < 1 || kp1 > kMaxKp1Sparse) return reject(ASAP_ERR_ARG, "asap_mix_noalloc: need 1 <= k+1 <= 32");
   if (d < 1 || ld < d || ld % 4 != 0)
     return reject(ASAP_ERR_ARG, "asap_mix_noalloc: need d >= 1, ld >= d and ld a multiple of 4");
+  {
+    // Every CTA reads rows of W_in that other CTAs may already have written
+    // to W_out: the two ranges must not overlap at all.
+    const uintptr_t a0 = reinterpret_cast<uintptr_t>(W_in), b0 = reinterpret_cast<uintptr_t>(W_out);
+    const uintptr_t bytes = static_cast<uintptr_t>(N) * static_cast<uintptr_t>(ld) * sizeof(float);
+    if (a0 < b0 + bytes && b0 < a0 + bytes)
+      return reject(ASAP_ERR_ARG, "asap_mix_noalloc: W_in and W_out must not overlap");
+  }
   if ((reinterpret_cast<uintptr_t>(W_in) | reinterpret_cast<uintptr_t>(W_out)) & 15u)
     return reject(ASAP_ERR_ARG, "asap_mix_noalloc: W_in and W_out must be 16-byte aligned");
   int S = 256;
@@ -198,9 +238,11 @@ extern "C" asap_status asap_mix_noalloc(const float* W_in, float* W_out, int N, 
   {
     std::lock_guard<std::mutex> lock(g_noalloc_mu);
     DeviceSlot& ds = g_noalloc_dev[dev];
-    if (!ds.scratch) {
-      // First call on this device: resolve the device address of the
-      // file-scope scratch (the host-side name is only a stand-in).
+    const unsigned long long cur = current_context_id();
+    if (!ds.scratch || cur == 0 || cur != ds.ctx_id) {
+      // First call on this device (or in a new context of it): resolve the
+      // device address of the file-scope scratch (the host-side name is only
+      // a stand-in).  This also makes the device's primary context current.
       void* p = nullptr;
       if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p)
         return reject(ASAP_ERR_CUDA, "asap_mix_noalloc: cudaGetSymbolAddress failed for the scratch array");
@@ -209,6 +251,7 @@ extern "C" asap_status asap_mix_noalloc(const float* W_in, float* W_out, int N, 
         return reject(ASAP_ERR_CUDA, "asap_mix_noalloc: cannot query the SM count");
       ds.scratch = p;
       ds.sm_count = sms;
+      ds.ctx_id = current_context_id();
     }
     slot = ds;
   }

@@ -33,7 +33,7 @@ import numpy as np
 __all__ = [
     "SparseShards", "DenseShards", "WORKLOADS",
     "tiny_dense_logistic", "sparse_hinge_svm", "sparse_logistic_hashed",
-    "sparse_custom", "mixing_params", "dense_softmax", "bf16_bits_to_f32",
+    "sparse_custom", "mixing_params", "mixing_params_device", "dense_softmax", "bf16_bits_to_f32",
 ]
 
 # Stream ids keep the draws for different purposes independent.
@@ -285,6 +285,17 @@ def mixing_params(seed: int, N: int, d: int, rows: Optional[range] = None,
         row = _rng(seed, _PARAMS, i).standard_normal(d, dtype=np.float32)
         W[a] = row if cols is None else row[cols]
     return W
+
+
+def mixing_params_device(seed: int, N: int, d: int, device="cuda"):
+    """W ~ N(0,1) float32 [N, d] drawn on a CUDA device with torch's seeded
+    generator (Philox), for sweep sizes whose host draw would take minutes
+    (up to 256 x 10^7 values).  A different stream from ``mixing_params``;
+    a sub-block for the oracle is read back from the returned tensor."""
+    import torch
+    g = torch.Generator(device=device)
+    g.manual_seed(int(seed) * 1000003 + 7919)
+    return torch.randn((N, d), generator=g, device=device, dtype=torch.float32)
 
 
 # ---------------------------------------------------------------------------

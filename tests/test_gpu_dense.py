@@ -1,23 +1,31 @@
 """GPU parity of the dense softmax-regression round (tcgen05 bf16 GEMMs with
 fp32 accumulation, softmax across a cluster, fp32 master update, then the
 stochastic reduce writing the next round's bf16 copy) against the oracle,
-which mirrors the bf16 rounding points.  Tolerance: 1e-3 normwise relative
-error per worker per round (bf16-input GEMM path), loss within 1e-4."""
+which mirrors the bf16 rounding points.
+
+Protocol, every round: the local step is checked on its own (the half-step
+W_{t+1/2} is read before the reduce) against the oracle restarted from the
+GPU's W_t -- 1e-3 normwise relative error per worker, accepting either bf16
+rounding of residual entries within fp32 reach of a bf16 midpoint -- then the
+reduce is checked against P times the GPU's half-step (fp32 mixing, 1e-5),
+and the round's loss within 1e-4.  Free-running loss trajectories stay
+within 1e-4 absolute of the oracle's."""
 import numpy as np
 import pytest
 
-from oracle import rounds, sgd
+from oracle import reduce, rounds, sgd
 from paper_1612_08608_gb300 import inputs
-from parity import rel_err_rows
+from parity import rel_err_rows, softmax_half_step_matching
 
 pytestmark = pytest.mark.gpu
 
 TOL = 1e-3
 
 
-def _run(N, d, C, B, lr, k, kind, T, seed=0, l2=0.0, w0_scale=0.0, gamma=None):
+def _run(N, d, C, B, lr, k, kind, T, seed=0, l2=0.0, w0_scale=0.0, gamma=None, rows=None, trajectory=False,
+         per_round=None):
     from paper_1612_08608_gb300 import Context
-    sh = inputs.dense_softmax(seed=seed, N=N, d=d, C=C, rows=T * B)
+    sh = inputs.dense_softmax(seed=seed, N=N, d=d, C=C, rows=rows or T * B)
     ctx = Context(N, d, graph_seed=seed, k=k)
     ctx.set_model("softmax", batch=B, lr=lr, num_classes=C, l2=l2)
     ctx.set_graph(kind)
@@ -25,54 +33,84 @@ def _run(N, d, C, B, lr, k, kind, T, seed=0, l2=0.0, w0_scale=0.0, gamma=None):
         ctx.set_schedule(local_steps=1, lr_schedule="inverse", gamma=gamma)
     ctx.load_dense_shards(sh)
     sched = rounds.graph_schedule(kind, N, k, graph_seed=seed)
+    lr_at = None if gamma is None else (lambda t: sgd.learning_rate("inverse", lr, gamma, t))
     W_t, _ = ctx.read_params()
     assert W_t.shape == (N, C * d) and not W_t.any()
+    W0 = None
     if w0_scale:
         W_t = (w0_scale * np.random.default_rng(seed).standard_normal(W_t.shape)).astype(np.float32)
         ctx.write_params(W_t, 0)
+        W0 = W_t.copy()
+    losses, flips = [], 0
     for t in range(T):
-        ctx.round(1)
+        nbr, wgt = sched(t)
+        eta = lr if lr_at is None else lr_at(t)
+        ctx.local_step()
+        H, rnd = ctx.read_params()                    # W_{t+1/2}: the reduce has not run yet
+        assert rnd == t
+        # every worker's half-step, or (per_round = m) m workers per round in
+        # rotation plus all of them in the first and the last round
+        check = range(N) if (per_round is None or t in (0, T - 1)) else \
+            [(t * per_round + j) % N for j in range(per_round)]
+        lref = []
+        for i in check:
+            err, li, f = softmax_half_step_matching(W_t[i].reshape(C, d), H[i].reshape(C, d), sh.X[i], sh.y[i], t,
+                                                    B, eta, l2, TOL)
+            assert err <= TOL, (t, i, err)
+            lref.append(li)
+            flips += f
+        ctx.stochastic_reduce()
         W_n, rnd = ctx.read_params()
         assert rnd == t + 1
-        nbr, wgt = sched(t)
-        eta = lr if gamma is None else sgd.learning_rate("inverse", lr, gamma, t)
-        ref, lref, cref = rounds.softmax_round(W_t, sh, t, B, eta, nbr, wgt, l2=l2)
-        err = rel_err_rows(W_n, ref)
-        assert err <= TOL, (t, err)
+        mixed = reduce.stochastic_reduce(H.astype(np.float64), nbr, wgt)
+        assert rel_err_rows(W_n, mixed) <= 1e-5, t
         lg, cg = ctx.read_metrics(t, 1)
-        assert abs(lg[0] - lref) <= 1e-4 * max(1.0, abs(lref)), (t, lg[0], lref)
+        if len(lref) == N:
+            assert abs(lg[0] - np.mean(lref)) <= 1e-4 * max(1.0, abs(np.mean(lref))), (t, lg[0], np.mean(lref))
+        cref = reduce.consensus_error(mixed)
         assert abs(cg[0] - cref) <= 2e-3 * cref + 1e-7, (t, cg[0], cref)
+        losses.append(lg[0])
         W_t = W_n
-    return ctx
+    if trajectory:
+        _, lfree, _ = rounds.run_softmax(sh, T, B, lr, sched, W0=W0, l2=l2, lr_at=lr_at)
+        assert np.abs(np.array(losses) - lfree).max() <= 1e-4, np.abs(np.array(losses) - lfree).max()
+    return ctx, flips
 
 
 def test_dense_small_one_cluster_cta():
-    _run(N=4, d=256, C=10, B=128, lr=0.5, k=1, kind="ring", T=3)
+    _run(N=4, d=256, C=10, B=128, lr=0.5, k=1, kind="ring", T=3, trajectory=True)
 
 
 def test_dense_ragged_classes_two_cluster_ctas_l2():
-    _run(N=6, d=512, C=300, B=256, lr=0.3, k=2, kind="random_regular", T=3, seed=2, l2=0.01)
+    _run(N=6, d=512, C=300, B=256, lr=0.3, k=2, kind="random_regular", T=3, seed=2, l2=0.01, trajectory=True)
 
 
 @pytest.mark.parametrize("C,B", [(600, 256), (1024, 384)])
-def test_dense_cluster_geometries(C, B):
+def test_dense_cluster_geometries_from_zero(C, B):
     # Forward clusters of three CTAs (C=600) and of four full class tiles
-    # with an odd number of row tiles (C=1024, B=384).  Random initial
-    # parameters: from W = 0, every class absent from the first minibatch
-    # gets the same row, their logits and residuals in the next round are
-    # exactly equal, and one fp32-versus-fp64 rounding decision at the bf16
-    # cast of R moves hundreds of them together by one bf16 ulp (a CPU
-    # restatement in the kernel's fp32 order differs from the oracle by
-    # 3.7e-3 there, as the GPU does).
+    # with an odd number of row tiles (C=1024, B=384), from W = 0: every
+    # class absent from the first minibatch gets the same row, so in the
+    # next round their residuals are exactly equal and one rounding decision
+    # at the bf16 cast of R moves all of them together -- the tie-aware check
+    # accepts either rounding there.
+    _run(N=3, d=256, C=C, B=B, lr=0.2, k=1, kind="ring", T=3, seed=3)
+
+
+@pytest.mark.parametrize("C,B", [(600, 256), (1024, 384)])
+def test_dense_cluster_geometries_random_start(C, B):
     _run(N=3, d=256, C=C, B=B, lr=0.2, k=1, kind="ring", T=2, seed=3, w0_scale=0.05)
 
 
 def test_dense_inverse_rate_l2():
     # eta_t = 0.5 / (1 + 0.5 t) on the dense path (one local step per round)
-    _run(N=4, d=256, C=20, B=128, lr=0.5, k=1, kind="ring", T=4, seed=4, l2=0.02, gamma=0.5)
+    _run(N=4, d=256, C=20, B=128, lr=0.5, k=1, kind="ring", T=4, seed=4, l2=0.02, gamma=0.5, trajectory=True)
 
 
-def test_dense_softmax_full_size():
-    # N=32 workers, d=2048 bf16 features, C=1000 classes, B=512, root graph.
-    ctx = _run(N=32, d=2048, C=1000, B=512, lr=0.1, k=2, kind="root", T=3)
+def test_dense_softmax_full_size_50_rounds():
+    # N=32 workers, d=2048 bf16 features, C=1000 classes, B=512, root graph,
+    # 25,600 rows per worker (one pass in 50 rounds).  Every round: the
+    # reduce of all workers, the half-step of four workers in rotation (all
+    # 32 in the first and the last round); then the free-running loss
+    # trajectory against the oracle's.
+    ctx, _ = _run(N=32, d=2048, C=1000, B=512, lr=0.1, k=2, kind="root", T=50, trajectory=True, per_round=4)
     assert ctx.read_counters()["timeouts"] == 0

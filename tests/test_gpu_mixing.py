@@ -1,8 +1,12 @@
 """GPU parity of the stochastic reduce alone (W <- P W, 20 rounds) against
-the oracle: N in {8, 32, 128, 256}, d in {1e5, 1e6, 1e7}, k in {1, 2, 4,
-N-1}.  At d = 1e5 every round is checked in full; above, the oracle follows
-a seeded subset of 65,536 columns exactly (the reduce acts on each column on
-its own) and the consensus error is checked against the Appendix A bound."""
+the oracle over the whole sweep: N in {8, 32, 128, 256}, d in {1e5, 1e6,
+1e7}, k in {1, 2, 4, N-1}; random regular graphs are drawn anew every round.
+Every round is checked on its own (the oracle restarted from the GPU's W_t,
+1e-5 normwise per worker).  At d = 1e5 all columns are compared; above, the
+oracle follows 65,536 columns in eight seeded blocks (the reduce acts on each
+column on its own), the GPU's consensus error must contract by sigma_2(P_t)
+every round (Appendix A), and where W fits a host copy the last round's
+consensus error is checked in full."""
 import numpy as np
 import pytest
 
@@ -13,34 +17,44 @@ from parity import rel_err_rows
 pytestmark = pytest.mark.gpu
 
 TOL = 1e-5
+NS = [8, 32, 128, 256]
+KS = [1, 2, 4, "N-1"]
 
 
 def _kind(N, k):
     return {1: "ring", N - 1: "complete"}.get(k, "random_regular")
 
 
-def _ctx(N, d, k, regen=False):
+def _ctx(N, d, k):
     from paper_1612_08608_gb300 import Context
     ctx = Context(N, d, graph_seed=1, k=k)
-    ctx.set_graph(_kind(N, k), regenerate=regen and _kind(N, k) == "random_regular")
-    return ctx
+    ctx.set_graph(_kind(N, k), regenerate=_kind(N, k) == "random_regular")
+    return ctx, rounds.graph_schedule(_kind(N, k), N, k, graph_seed=1, regenerate=_kind(N, k) == "random_regular")
 
 
-@pytest.mark.parametrize("N", [8, 32, 128, 256])
-@pytest.mark.parametrize("k", [1, 2, 4, "N-1"])
+def _oracle_reduce(W, nbr, wgt):
+    # the per-row form for sparse graphs; the product with P for the
+    # complete graph (N^2 row operations otherwise)
+    if nbr.shape[1] > 8:
+        return reduce.reduce_with_matrix(W, graphs.mixing_matrix(nbr, wgt))
+    return reduce.stochastic_reduce(W, nbr, wgt)
+
+
+@pytest.mark.parametrize("N", NS)
+@pytest.mark.parametrize("k", KS)
 def test_mixing_every_round_d1e5(N, k):
     k = N - 1 if k == "N-1" else k
     d, T = 100000, 20
     W0 = inputs.mixing_params(seed=0, N=N, d=d)
-    ctx = _ctx(N, d, k, regen=True)
+    ctx, sched = _ctx(N, d, k)
     ctx.write_params(W0, 0)
-    sched = rounds.graph_schedule(_kind(N, k), N, k, graph_seed=1, regenerate=_kind(N, k) == "random_regular")
     W_t = W0.astype(np.float64)
     for t in range(T):
         ctx.stochastic_reduce()
         W_n, _ = ctx.read_params()
         nbr, wgt = sched(t)
-        ref = reduce.stochastic_reduce(W_t, nbr, wgt)
+        assert np.array_equal(ctx.get_graph(t)[0], nbr)
+        ref = _oracle_reduce(W_t, nbr, wgt)
         assert rel_err_rows(W_n, ref) <= TOL, t
         loss, cons = ctx.read_metrics(t, 1)
         assert np.isnan(loss[0])
@@ -49,29 +63,41 @@ def test_mixing_every_round_d1e5(N, k):
         W_t = W_n.astype(np.float64)
 
 
-@pytest.mark.parametrize("N,d,k", [(8, 1000000, 2), (32, 1000000, 4), (128, 1000000, 1), (256, 1000000, 255),
-                                   (8, 10000000, 1), (32, 10000000, 2), (128, 10000000, 4), (256, 10000000, 4),
-                                   (256, 10000000, 255)])
-def test_mixing_large_column_subset(N, d, k):
-    T = 20
-    cols = np.sort(np.random.default_rng(N * 7 + k).choice(d, 65536, replace=False))
-    W0 = inputs.mixing_params(seed=0, N=N, d=d)
-    ctx = _ctx(N, d, k)
-    ctx.write_params(W0, 0)
+@pytest.mark.parametrize("d", [1000000, 10000000])
+@pytest.mark.parametrize("N", NS)
+@pytest.mark.parametrize("k", KS)
+def test_mixing_every_round_large_d(d, N, k):
+    import torch
+    k = N - 1 if k == "N-1" else k
+    T, nblk, blk = 20, 8, 8192
+    ctx, sched = _ctx(N, d, k)
+    W0 = inputs.mixing_params_device(seed=N * 31 + k, N=N, d=d)
+    starts = np.sort(np.random.default_rng(N * 7 + k).choice(d // blk, nblk, replace=False)) * blk
+    starts[-1] = d - blk                          # the ragged tail of the last slab
+    sub = torch.cat([W0[:, s:s + blk] for s in starts], dim=1).cpu().numpy().astype(np.float64)
+    ctx.write_params_device(W0, 0)
     del W0
-    ctx.round(T)
-    sched = rounds.graph_schedule(_kind(N, k), N, k, graph_seed=1)
-    Wsub, _ = rounds.mixing_rounds(inputs.mixing_params(seed=0, N=N, d=d, cols=cols), T, sched)
-    W_T, rnd = ctx.read_params()
-    assert rnd == T
-    assert rel_err_rows(W_T[:, cols], Wsub) <= 1e-4
-    _, cons = ctx.read_metrics(0, T)
-    nbr, wgt = sched(0)
-    s2 = 1.0 - graphs.spectral_gap(graphs.mixing_matrix(nbr, wgt))
-    prev = None
+    torch.cuda.empty_cache()
+    out = np.empty((N, blk), np.float32)
+    prev_cons = None
     for t in range(T):
-        if prev is not None and prev > 1e-3 * cons[0]:
-            assert cons[t] <= s2 * prev * (1 + 1e-4) + 1e-6 * cons[0], t
-        prev = cons[t]
-    full = reduce.consensus_error(W_T)
-    assert abs(cons[T - 1] - full) <= 1e-3 * max(full, 1e-3 * cons[0])
+        ctx.stochastic_reduce()
+        got = np.concatenate([ctx.read_param_columns(int(s), blk, out).copy() for s in starts], axis=1)
+        nbr, wgt = sched(t)
+        assert np.array_equal(ctx.get_graph(t)[0], nbr)
+        ref = _oracle_reduce(sub, nbr, wgt)
+        assert rel_err_rows(got, ref) <= TOL, t
+        _, cons = ctx.read_metrics(t, 1)
+        s2 = 1.0 - graphs.spectral_gap(graphs.mixing_matrix(nbr, wgt))
+        if prev_cons is not None and prev_cons > 1e-5 * first_cons:
+            assert cons[0] <= s2 * prev_cons * (1 + 1e-4) + 1e-6 * first_cons, (t, cons[0], s2, prev_cons)
+        if prev_cons is None:
+            first_cons = cons[0]
+        prev_cons = cons[0]
+        sub = got.astype(np.float64)
+    if N * d <= 320000000:
+        W_T, rnd = ctx.read_params()
+        assert rnd == T
+        full = reduce.consensus_error(W_T)
+        assert abs(prev_cons - full) <= 1e-3 * max(full, 1e-3 * first_cons)
+    ctx.close()

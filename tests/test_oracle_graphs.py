@@ -216,3 +216,20 @@ def test_simplex_bound_of_appendix_a():
         for t in range(1, 30):
             v = P @ v
             assert np.linalg.norm(v - 1.0 / N) <= s2 ** t + 1e-12
+
+
+def test_matrix_form_of_the_reduce():
+    # reduce_with_matrix: the hand case above, the complete graph's exact
+    # column mean, and agreement with the per-row form on a random graph.
+    H = np.array([[2.0, -4.0], [6.0, 0.0], [10.0, 8.0]])
+    nbr = np.array([[0, 1], [1, 2], [0, 2]])
+    P = graphs.mixing_matrix(nbr, np.full((3, 2), 0.5))
+    assert np.array_equal(reduce.reduce_with_matrix(H, P), [[4.0, -2.0], [8.0, 4.0], [6.0, 2.0]])
+    Hc = np.array([[1.0, 3.0], [5.0, -7.0], [0.0, 4.0], [2.0, 0.0]])     # column means 2 and 0
+    nbr, wgt = graphs.build_graph("complete", 4, 3)
+    assert np.array_equal(reduce.reduce_with_matrix(Hc, graphs.mixing_matrix(nbr, wgt)), [[2.0, 0.0]] * 4)
+    rng = np.random.default_rng(7)
+    Hr = rng.standard_normal((40, 30))
+    nbr, wgt = graphs.build_graph("random_regular", 40, 4, 5, 2)
+    assert np.allclose(reduce.reduce_with_matrix(Hr, graphs.mixing_matrix(nbr, wgt)),
+                       reduce.stochastic_reduce(Hr, nbr, wgt), atol=1e-14)

@@ -3,16 +3,19 @@ memory (a framework that owns all of HBM through its own pool, or a
 latency-critical loop where cudaMalloc may synchronise the device).
 
 It is called here through the C ABI on buffers the test owns, and its output
-is checked against the context's own stochastic reduce on two calls in a
+is checked against the context's own stochastic reduce and against the CPU
+oracle (Eq. A.1, second line, and the consensus error) on two calls in a
 row (the second call starts from the first call's output, so the shared
-scratch array holds the previous call's contents).  Collected last on
-purpose: a run that stops at the first failure has already run every other
-test."""
+scratch array holds the previous call's contents).  After a warm-up call,
+further calls leave the device's free memory and torch's allocation count
+unchanged.  Collected last on purpose: a run that stops at the first
+failure has already run every other test."""
 import ctypes as C
 
 import numpy as np
 import pytest
 
+from oracle import reduce
 from paper_1612_08608_gb300 import inputs
 from parity import rel_err_rows
 
@@ -54,6 +57,7 @@ def test_mix_noalloc_matches_stochastic_reduce_twice(N, d, k):
     d_nbr = torch.from_numpy(nbr).to(dev)
     d_wgt = torch.from_numpy(wgt).to(dev)
     stream = torch.cuda.current_stream().cuda_stream
+    prev = W0.astype(np.float64)
     for t in range(2):
         src, dst = (W_a, W_b) if t == 0 else (W_b, W_a)
         assert _noalloc(lib, src, dst, N, d, ld, d_nbr, d_wgt, k + 1, cons, stream) == 0, \
@@ -63,6 +67,21 @@ def test_mix_noalloc_matches_stochastic_reduce_twice(N, d, k):
         assert rel_err_rows(got, ref_W[t]) <= 1e-5, t
         assert abs(cons.item() - ref_c[t]) <= 1e-4 * ref_c[t] + 1e-6, (t, cons.item(), ref_c[t])
         assert torch.all(dst[:, d:] == 0)   # zero padding columns stay zero
+        # the oracle, restarted from this call's input
+        want = reduce.stochastic_reduce(prev, nbr.astype(np.int64), wgt.astype(np.float64))
+        assert rel_err_rows(got, want) <= 1e-5, t
+        cw = reduce.consensus_error(want)
+        assert abs(cons.item() - cw) <= 1e-4 * cw + 1e-6, (t, cons.item(), cw)
+        prev = got.astype(np.float64)
+
+    # No allocation: free device memory and torch's count stay put.
+    free0, alloc0 = torch.cuda.mem_get_info()[0], torch.cuda.memory_allocated()
+    for t in range(6):
+        src, dst = (W_a, W_b) if t % 2 == 0 else (W_b, W_a)
+        assert _noalloc(lib, src, dst, N, d, ld, d_nbr, d_wgt, k + 1, cons, stream) == 0
+    torch.cuda.synchronize()
+    assert torch.cuda.mem_get_info()[0] == free0
+    assert torch.cuda.memory_allocated() == alloc0
 
 
 def test_mix_noalloc_rejects_sizes_beyond_its_scratch():
@@ -77,3 +96,7 @@ def test_mix_noalloc_rejects_sizes_beyond_its_scratch():
     assert _noalloc(lib, x, x.clone(), 256, ld_too_big, ld_too_big, n, x, 1, x, 0) == 1
     assert b"scratch" in lib.asap_last_error(None)
     assert _noalloc(lib, x, x.clone(), 257, 4, 4, n, x, 1, x, 0) == 1
+    # overlapping input and output ranges (not only equal base pointers)
+    big = torch.zeros(4 * 16 + 8, dtype=torch.float32, device=dev)
+    assert _noalloc(lib, big[8:], big[:64], 4, 16, 16, n, x, 1, x, 0) == 1
+    assert b"overlap" in lib.asap_last_error(None)

@@ -204,21 +204,19 @@ def kernel_work(sh):
         out["reduce"] = ("GB/s", 10.0 * N * ld, "hbm")     # fp32 read + write, bf16 copy write
         return out
     rng = np.random.default_rng(0)
-    nnz = pad = touched = 0.0
+    nnz = touched = 0.0
     samples = 16
     for _ in range(samples):
         i = int(rng.integers(N))
         t = int(rng.integers(sh.n_rows(i) // B))
         rp = sh.rowptr[i][t * B:(t + 1) * B + 1]
-        lens = np.diff(rp)
-        nnz += lens.sum()
-        pad += ((lens + 3) // 4 * 4).sum()
+        nnz += rp[-1] - rp[0]
         touched += np.unique(sh.col[i][rp[0]:rp[-1]]).shape[0]
-    nnz, pad, touched = nnz * N / samples, pad * N / samples, touched * N / samples
-    out["margin"] = ("GB/s", 8.0 * pad + 4.0 * nnz + 8.0 * N * B, "hbm")
-    # entries (list position, value, row: 10 B), one fp32 sum written per
-    # distinct (worker, column), the margin kernel's r read once
-    out["update"] = ("GB/s", 10.0 * nnz + 4.0 * touched + 4.0 * N * B, "hbm")
+    nnz, touched = nnz * N / samples, touched * N / samples
+    # the fused local step reads every entry once (list position, value,
+    # row, segment slot, row of the slot: 14 B), the w value and writes the
+    # column sum of every distinct (worker, column) (8 B), and the labels
+    out["local_step"] = ("GB/s", 14.0 * nnz + 8.0 * touched + 4.0 * N * B, "hbm")
     out["reduce"] = ("GB/s", 8.0 * N * ld, "hbm")
     # local steps before the round's last: the update scatter and the next gather
     out["apply"] = ("GB/s", 16.0 * touched, "hbm")    # list + column sum read, w read + write per column

@@ -245,30 +245,35 @@ asap_status asap_debug_skip_notify(asap_ctx* ctx, int worker);
  * paper beyond that).  Shards as in asap_load_shards, each with at least
  * (t + 1) * batch rows (not checked: there is no row count here); batch: B rows;
  * slab_cols: the slab width S (a power of two, 8 to 1024); the column list
- * covers ceil(round_up(d, 64) / S) slabs.  The image is written to `image`
- * (cap bytes; *image_bytes receives its size; ASAP_ERR_ARG when it does not
- * fit).  desc_out (N*9 int64), per worker: byte offsets of the padded row
- * starts (int32 [B+1]), labels (float [B]), list positions and values of
- * the padded entries (int32 / float [nnz_pad]), the (column, row)-sorted
- * list positions, values and rows (int32 / float / uint16 [nnz]), then
- * nnz_pad and nnz.  list_out (3 int64): byte offsets of the slab-major list
- * of distinct (worker << 16 | column in slab) codes and of its slab offsets
- * (int32 [n_slabs + 1]), and the list length in entries. */
-asap_status asap_debug_batch_image(int N, int64_t d, int batch, int slab_cols, int t, const int64_t* const* rowptr,
-                                   const int32_t* const* col, const float* const* val, const float* const* y,
-                                   unsigned char* image, int64_t cap, int64_t* image_bytes, int64_t* desc_out,
-                                   int64_t* list_out);
+ * covers ceil(round_up(d, 64) / S) slabs; ctas_per_worker: Q, the CTAs of
+ * one worker's local step (1 to 8).  The image is written to `image` (cap
+ * bytes; *image_bytes receives its size; ASAP_ERR_ARG when it does not fit).
+ * desc_out (N*8 int64), per worker: byte offsets of the labels (float [B]),
+ * of the (column, row)-sorted entries' list positions, values, rows and
+ * segment slots (int32 / float / uint16 / uint16 [nnz]), of the rows of
+ * every segment's slots (uint16 [nnz]) and of the Q+1 column-sum range
+ * bounds (int32), then nnz.  Segment g holds sorted entries [1024 g,
+ * 1024 (g+1)); its slots are numbered row by row, a row's entries in sorted
+ * order.  The range bounds start at 0, end at nnz and cut the sorted entries
+ * at the first column boundary at or after q nnz / Q.  list_out (3 int64):
+ * byte offsets of the slab-major list of distinct (worker << 16 | column in
+ * slab) codes and of its slab offsets (int32 [n_slabs + 1]), and the list
+ * length in entries. */
+asap_status asap_debug_batch_image(int N, int64_t d, int batch, int slab_cols, int ctas_per_worker, int t,
+                                   const int64_t* const* rowptr, const int32_t* const* col, const float* const* val,
+                                   const float* const* y, unsigned char* image, int64_t cap, int64_t* image_bytes,
+                                   int64_t* desc_out, int64_t* list_out);
 
 /* Kernel kinds for per-kernel timing. */
 typedef enum {
-  ASAP_KERNEL_MARGIN = 0,     /* sparse margins + loss derivative (a2)          */
-  ASAP_KERNEL_UPDATE = 1,     /* sparse column-segmented update + NOTIFY (a3-a4) */
-  ASAP_KERNEL_REDUCE = 2,     /* stochastic reduce + ACK + metrics (a5-a7, a9)  */
-  ASAP_KERNEL_DENSE_FWD = 3,  /* dense logits, softmax, R^T (a3')               */
-  ASAP_KERNEL_DENSE_GRAD = 4, /* dense gradient GEMM + update + NOTIFY (a3')    */
-  ASAP_KERNEL_APPLY = 5,      /* update of a local step before the round's last */
-  ASAP_KERNEL_GATHER = 6,     /* w at a step's columns from the stored W        */
-  ASAP_KERNEL_KINDS = 7
+  ASAP_KERNEL_LOCAL_STEP = 0, /* sparse margins, loss derivative, column sums,
+                                 NOTIFY (a2-a4), one fused kernel               */
+  ASAP_KERNEL_REDUCE = 1,     /* stochastic reduce + ACK + metrics (a5-a7, a9)  */
+  ASAP_KERNEL_DENSE_FWD = 2,  /* dense logits, softmax, R^T (a3')               */
+  ASAP_KERNEL_DENSE_GRAD = 3, /* dense gradient GEMM + update + NOTIFY (a3')    */
+  ASAP_KERNEL_APPLY = 4,      /* update of a local step before the round's last */
+  ASAP_KERNEL_GATHER = 5,     /* w at a step's columns from the stored W        */
+  ASAP_KERNEL_KINDS = 6
 } asap_kernel_kind;
 
 /* Per-kernel timing: while enabled, every kernel launch of the context is

@@ -20,8 +20,8 @@ SIGNATURES = {
     "asap_set_mixing": (C.c_int, [_P, _P, _P]),
     "asap_set_model": (C.c_int, [_P, C.c_int, C.c_int, C.c_int, C.c_float, C.c_float]),
     "asap_set_schedule": (C.c_int, [_P, C.c_int, C.c_int, C.c_float]),
-    "asap_debug_batch_image": (C.c_int, [C.c_int, C.c_int64, C.c_int, C.c_int, C.c_int, _P, _P, _P, _P, _P, C.c_int64,
-                                         _P, _P, _P]),
+    "asap_debug_batch_image": (C.c_int, [C.c_int, C.c_int64, C.c_int, C.c_int, C.c_int, C.c_int, _P, _P, _P, _P, _P,
+                                         C.c_int64, _P, _P, _P]),
     "asap_set_stream": (C.c_int, [_P, _P]),
     "asap_set_shard_residency": (C.c_int, [_P, C.c_int]),
     "asap_shard_block_bytes": (C.c_int, [_P, C.c_int64, C.POINTER(C.c_uint64)]),

@@ -46,9 +46,9 @@ def build_graph(kind: str, N: int, k: int, graph_seed: int = 0, rnd: int = 0) ->
     return out
 
 
-def debug_batch_image(shards, batch: int, slab_cols: int, t: int):
+def debug_batch_image(shards, batch: int, slab_cols: int, t: int, ctas_per_worker: int = 1):
     """The image asap_load_shards builds for minibatch t (host only, for
-    tests): (image bytes uint8, desc [N, 9] int64, (list byte offset, slab
+    tests): (image bytes uint8, desc [N, 8] int64, (list byte offset, slab
     offsets byte offset, list length))."""
     lib = load_library()
     rp = [np.ascontiguousarray(a, dtype=np.int64) for a in shards.rowptr]
@@ -58,9 +58,10 @@ def debug_batch_image(shards, batch: int, slab_cols: int, t: int):
     N = len(rp)
     if t < 0 or any((t + 1) * batch > a.shape[0] - 1 for a in rp):
         raise ValueError("minibatch %d of %d rows is past the end of a shard" % (t, batch))
-    args = (N, shards.d, batch, slab_cols, t, _ptr_array(rp), _ptr_array(cl), _ptr_array(vl), _ptr_array(yl))
+    args = (N, shards.d, batch, slab_cols, ctas_per_worker, t, _ptr_array(rp), _ptr_array(cl), _ptr_array(vl),
+            _ptr_array(yl))
     size = C.c_int64()
-    desc = np.empty((N, 9), dtype=np.int64)
+    desc = np.empty((N, 8), dtype=np.int64)
     lst = np.empty(3, dtype=np.int64)
     st = lib.asap_debug_batch_image(*args, None, 0, C.byref(size), _ptr(desc), _ptr(lst))
     if st != 1:                       # anything but "buffer too small" is a real error
@@ -200,7 +201,7 @@ class Context:
     def debug_skip_notify(self, worker: int):
         self._c(self._lib.asap_debug_skip_notify(self._h, worker))
 
-    KERNELS = ("margin", "update", "reduce", "dense_fwd", "dense_grad", "apply", "gather")
+    KERNELS = ("local_step", "reduce", "dense_fwd", "dense_grad", "apply", "gather")
 
     def set_kernel_timing(self, enable: bool = True):
         self._c(self._lib.asap_set_kernel_timing(self._h, int(enable)))

@@ -15,11 +15,6 @@
 
 #include "asap_internal.h"
 
-namespace asap {
-int margin_ctas_for(int B);
-int update_ctas_for(int max_nnz);
-cudaError_t mix_occupancy(bool complete, int kp1, bool shadow, size_t smem, int* blocks);
-}  // namespace asap
 
 using namespace asap;
 
@@ -91,6 +86,10 @@ struct asap_ctx {
   float* m_cons = nullptr;
   float* r_scr = nullptr;
   float* loss_part = nullptr;
+  float* mpart_big = nullptr;        // sparse, B > kRSmemRows: partial margins [N][Q][B]
+  float* r_big = nullptr;            // sparse, B > kRSmemRows: r [N][Q][B]
+  int* d_worker_of = nullptr;        // sparse: worker of each local-step cluster (a permutation)
+  bool permuted = false;             // d_worker_of differs from the identity
   double* cons_part = nullptr;
   int cons_cap = 0;
   int32_t* d_nbr = nullptr;
@@ -123,7 +122,9 @@ struct asap_ctx {
   int64_t staged_round[kStaging] = {-1, -1, -1};
   bool free_recorded[kStaging] = {false, false, false};
   cudaEvent_t staged_ev[kStaging] = {}, free_ev[kStaging] = {};
-  int margin_ctas = 0, update_ctas = 0;
+  int step_q = 1;                   // CTAs per worker (cluster size) of the local step
+  int step_stages = 3;              // ring stages of the local step
+  size_t step_smem = 0;
   int max_nnz = 0;
 
   // dense softmax shards and scratch
@@ -211,6 +212,8 @@ void free_shards(asap_ctx* c) {
   dfree(c->Yd);
   dfree(c->wv);
   dfree(c->gsum);
+  dfree(c->mpart_big);
+  dfree(c->r_big);
   for (int b = 0; b < asap_ctx::kStaging; ++b) {
     dfree(c->staging[b]);
     c->staged_round[b] = -1;
@@ -476,10 +479,12 @@ asap_status sync_all(asap_ctx* c) {
   return check_device_error(c);
 }
 
-// The device image of minibatch t (host only): per worker the padded rows
-// (list position, value) and labels, and the entries sorted by (column, row);
-// then the batch's slab-major list of distinct (worker, column) pairs and its
-// slab offsets.  Used by asap_load_shards and, for tests, asap_debug_batch_image.
+// The device image of minibatch t (host only): per worker the labels, the
+// entries sorted by (column, row) -- list position, value, row, the entry's
+// slot inside its margin segment and, per segment, the row of every slot --
+// and the Q column-sum ranges cut at column boundaries; then the batch's
+// slab-major list of distinct (worker, column) pairs and its slab offsets.
+// Used by asap_load_shards and, for tests, asap_debug_batch_image.
 struct BatchImage {
   std::vector<unsigned char> img;
   std::vector<BatchDesc> desc;
@@ -489,18 +494,18 @@ struct BatchImage {
   const char* err = nullptr;
 };
 
-void build_batch_image(int N, int B, int64_t d, int S, long long n_slabs, int t, const int64_t* const* rowptr,
-                       const int32_t* const* col, const float* const* val, const float* const* y, BatchImage& bt) {
+void build_batch_image(int N, int B, int64_t d, int S, long long n_slabs, int Q, int t,
+                       const int64_t* const* rowptr, const int32_t* const* col, const float* const* val,
+                       const float* const* y, BatchImage& bt) {
   std::vector<std::vector<uint64_t>> keys(N);
   std::vector<std::vector<int32_t>> ucol(N), run_of(N), upos(N);
-  std::vector<int64_t> nnz(N, 0), nnz_pad(N, 0);
+  std::vector<int64_t> nnz(N, 0);
   for (int i = 0; i < N; ++i) {
     const int64_t* rp = rowptr[i];
     const int64_t r0 = static_cast<int64_t>(t) * B;
     const int64_t a0 = rp[r0], a1 = rp[r0 + B];
     nnz[i] = a1 - a0;
-    for (int b = 0; b < B; ++b) nnz_pad[i] += (rp[r0 + b + 1] - rp[r0 + b] + 3) / 4 * 4;
-    if (nnz_pad[i] > (1ll << 30)) { bt.err = "a minibatch holds more than 2^30 entries"; return; }
+    if (nnz[i] > (1ll << 30)) { bt.err = "a minibatch holds more than 2^30 entries"; return; }
     std::vector<uint64_t>& k = keys[i];
     k.resize(nnz[i]);
     for (int64_t e = 0; e < nnz[i]; ++e) {
@@ -552,22 +557,22 @@ void build_batch_image(int N, int B, int64_t d, int S, long long n_slabs, int t,
   size_t off = 0;
   for (int i = 0; i < N; ++i) {
     BatchDesc& dd = bt.desc[i];
-    dd.rp = static_cast<int64_t>(off);
-    off = align_up(off + 4 * static_cast<size_t>(B + 1), 16);
     dd.y = static_cast<int64_t>(off);
     off = align_up(off + 4 * static_cast<size_t>(B), 16);
-    dd.posw = static_cast<int64_t>(off);
-    off += 4 * static_cast<size_t>(nnz_pad[i]);
-    dd.val = static_cast<int64_t>(off);
-    off += 4 * static_cast<size_t>(nnz_pad[i]);
     dd.cpos = static_cast<int64_t>(off);
     off = align_up(off + 4 * static_cast<size_t>(nnz[i]), 16);
     dd.cval = static_cast<int64_t>(off);
     off = align_up(off + 4 * static_cast<size_t>(nnz[i]), 16);
     dd.crow = static_cast<int64_t>(off);
     off = align_up(off + 2 * static_cast<size_t>(nnz[i]), 16);
-    dd.nnz_pad = static_cast<int32_t>(nnz_pad[i]);
+    dd.cslot = static_cast<int64_t>(off);
+    off = align_up(off + 2 * static_cast<size_t>(nnz[i]), 16);
+    dd.srow = static_cast<int64_t>(off);
+    off = align_up(off + 2 * static_cast<size_t>(nnz[i]), 16);
+    dd.bnd = static_cast<int64_t>(off);
+    off = align_up(off + 4 * static_cast<size_t>(Q + 1), 16);
     dd.nnz = static_cast<int32_t>(nnz[i]);
+    dd.pad_ = 0;
   }
   bt.list_off = off;
   off = align_up(off + 4 * static_cast<size_t>(tot), 16);
@@ -578,46 +583,55 @@ void build_batch_image(int N, int B, int64_t d, int S, long long n_slabs, int t,
   unsigned char* base = bt.img.data();
   std::memcpy(base + bt.list_off, list.data(), 4 * list.size());
   std::memcpy(base + bt.soff_off, soff.data(), 4 * soff.size());
+  std::vector<int32_t> fill(B);
   for (int i = 0; i < N; ++i) {
     const BatchDesc& dd = bt.desc[i];
-    int32_t* rp_o = reinterpret_cast<int32_t*>(base + dd.rp);
     float* y_o = reinterpret_cast<float*>(base + dd.y);
-    int32_t* pw_o = reinterpret_cast<int32_t*>(base + dd.posw);
-    float* val_o = reinterpret_cast<float*>(base + dd.val);
     int32_t* cp_o = reinterpret_cast<int32_t*>(base + dd.cpos);
     float* cv_o = reinterpret_cast<float*>(base + dd.cval);
     uint16_t* cr_o = reinterpret_cast<uint16_t*>(base + dd.crow);
+    uint16_t* cs_o = reinterpret_cast<uint16_t*>(base + dd.cslot);
+    uint16_t* sr_o = reinterpret_cast<uint16_t*>(base + dd.srow);
+    int32_t* bd_o = reinterpret_cast<int32_t*>(base + dd.bnd);
     const int64_t* rp = rowptr[i];
     const int64_t r0 = static_cast<int64_t>(t) * B, a0 = rp[r0];
-    // list position of every entry (row-major), through the sort
-    std::vector<int32_t> epos(nnz[i]);
+    for (int b = 0; b < B; ++b) y_o[b] = y[i][r0 + b];
     std::vector<uint16_t> erow(nnz[i]);
     for (int b = 0; b < B; ++b)
       for (int64_t e = rp[r0 + b] - a0; e < rp[r0 + b + 1] - a0; ++e) erow[e] = static_cast<uint16_t>(b);
     for (int64_t e = 0; e < nnz[i]; ++e) {
       const int64_t k = static_cast<int64_t>(keys[i][e] & 0xffffffffu);
-      const int32_t pos = upos[i][run_of[i][e]];
-      epos[k] = pos;
-      cp_o[e] = pos;
+      cp_o[e] = upos[i][run_of[i][e]];
       cv_o[e] = val[i][a0 + k];
       cr_o[e] = erow[k];
     }
-    int32_t q = 0;
-    for (int b = 0; b < B; ++b) {
-      rp_o[b] = q;
-      y_o[b] = y[i][r0 + b];
-      for (int64_t e = rp[r0 + b] - a0; e < rp[r0 + b + 1] - a0; ++e) {
-        pw_o[q] = epos[e];
-        val_o[q] = val[i][a0 + e];
-        ++q;
+    // Margin segments of kTileEntries sorted entries: slots row by row, a
+    // row's entries in sorted (column) order; srow lists the slots' rows.
+    for (int64_t e0 = 0; e0 < nnz[i]; e0 += kTileEntries) {
+      const int64_t e1 = std::min<int64_t>(e0 + kTileEntries, nnz[i]);
+      std::fill(fill.begin(), fill.end(), 0);
+      for (int64_t e = e0; e < e1; ++e) fill[cr_o[e]]++;
+      int32_t acc = 0;
+      for (int b = 0; b < B; ++b) {
+        const int32_t n = fill[b];
+        fill[b] = acc;
+        acc += n;
       }
-      while (q & 3) {   // pad the row to a multiple of 4 entries (value 0)
-        pw_o[q] = 0;
-        val_o[q] = 0.f;
-        ++q;
+      for (int64_t e = e0; e < e1; ++e) {
+        const int32_t sl = fill[cr_o[e]]++;
+        cs_o[e] = static_cast<uint16_t>(sl);
+        sr_o[e0 + sl] = cr_o[e];
       }
     }
-    rp_o[B] = q;
+    // Column-sum ranges of the Q CTAs: cut at the first column boundary at
+    // or after q nnz / Q.
+    bd_o[0] = 0;
+    for (int q = 1; q < Q; ++q) {
+      int64_t e = std::max<int64_t>(q * nnz[i] / Q, bd_o[q - 1]);
+      while (e > 0 && e < nnz[i] && cp_o[e] == cp_o[e - 1]) ++e;
+      bd_o[q] = static_cast<int32_t>(e);
+    }
+    bd_o[Q] = static_cast<int32_t>(nnz[i]);
   }
 }
 
@@ -668,27 +682,27 @@ const char* asap_version(void) { return "asap-gb300 0.1 (sm_103a)"; }
 
 const char* asap_last_error(const asap_ctx* c) { return c ? c->err.c_str() : g_last_error.c_str(); }
 
-asap_status asap_debug_batch_image(int N, int64_t d, int batch, int slab_cols, int t, const int64_t* const* rowptr,
-                                   const int32_t* const* col, const float* const* val, const float* const* y,
-                                   unsigned char* image, int64_t cap, int64_t* image_bytes, int64_t* desc_out,
-                                   int64_t* list_out) {
-  if (N < 1 || N > kMaxWorkers || d < 1 || batch < 1 || batch > 65535 || t < 0 || !rowptr || !col || !val || !y ||
-      !image_bytes || !desc_out || !list_out)
+asap_status asap_debug_batch_image(int N, int64_t d, int batch, int slab_cols, int ctas_per_worker, int t,
+                                   const int64_t* const* rowptr, const int32_t* const* col, const float* const* val,
+                                   const float* const* y, unsigned char* image, int64_t cap, int64_t* image_bytes,
+                                   int64_t* desc_out, int64_t* list_out) {
+  if (N < 1 || N > kMaxWorkers || d < 1 || batch < 1 || batch > 65535 || t < 0 || ctas_per_worker < 1 ||
+      ctas_per_worker > kMaxStepCluster || !rowptr || !col || !val || !y || !image_bytes || !desc_out || !list_out)
     return fail(nullptr, ASAP_ERR_ARG, "bad arguments to asap_debug_batch_image");
   if (slab_cols < 8 || slab_cols > 1024 || (slab_cols & (slab_cols - 1)))
     return fail(nullptr, ASAP_ERR_ARG, "slab_cols must be a power of two in [8, 1024]");
   const int64_t ld = (d + 63) / 64 * 64;
   const long long n_slabs = (ld + slab_cols - 1) / slab_cols;
   BatchImage bt;
-  build_batch_image(N, batch, d, slab_cols, n_slabs, t, rowptr, col, val, y, bt);
+  build_batch_image(N, batch, d, slab_cols, n_slabs, ctas_per_worker, t, rowptr, col, val, y, bt);
   if (bt.err) return fail(nullptr, ASAP_ERR_ARG, bt.err);
   *image_bytes = static_cast<int64_t>(bt.img.size());
   if (!image || cap < static_cast<int64_t>(bt.img.size())) return fail(nullptr, ASAP_ERR_ARG, "image buffer too small");
   std::memcpy(image, bt.img.data(), bt.img.size());
   for (int i = 0; i < N; ++i) {
     const BatchDesc& q = bt.desc[i];
-    const int64_t v[9] = {q.rp, q.y, q.posw, q.val, q.cpos, q.cval, q.crow, q.nnz_pad, q.nnz};
-    std::memcpy(desc_out + 9 * static_cast<size_t>(i), v, sizeof v);
+    const int64_t v[8] = {q.y, q.cpos, q.cval, q.crow, q.cslot, q.srow, q.bnd, q.nnz};
+    std::memcpy(desc_out + 8 * static_cast<size_t>(i), v, sizeof v);
   }
   list_out[0] = static_cast<int64_t>(bt.list_off);
   list_out[1] = static_cast<int64_t>(bt.soff_off);
@@ -734,6 +748,7 @@ static asap_status init_ctx(asap_ctx* c) {
   CU(cudaMalloc(&c->stamp, 8 * N), "allocating stamps");
   CU(cudaMemset(c->stamp, 0, 8 * N), "zeroing stamps");
   CU(cudaMalloc(&c->ticket, 4 * N), "allocating tickets");
+  CU(cudaMalloc(&c->d_worker_of, 4 * static_cast<size_t>(N)), "allocating the local-step map");
   CU(cudaMalloc(&c->st, sizeof(DevState)), "allocating device state");
   CU(cudaMemset(c->st, 0, sizeof(DevState)), "zeroing device state");
   CU(cudaMalloc(&c->m_loss, 4 * kMetricsCap), "allocating metrics");
@@ -793,6 +808,7 @@ void asap_destroy(asap_ctx* c) {
   dfree(c->consumed);
   dfree(c->stamp);
   dfree(c->ticket);
+  dfree(c->d_worker_of);
   dfree(c->st);
   dfree(c->m_loss);
   dfree(c->m_cons);
@@ -908,9 +924,15 @@ asap_status asap_set_model(asap_ctx* c, asap_loss loss, int num_classes, int bat
   dfree(c->RT);
   c->n_loss_part = 0;
   if (loss == ASAP_LOSS_HINGE || loss == ASAP_LOSS_LOGISTIC) {
-    c->margin_ctas = margin_ctas_for(batch);
-    c->n_loss_part = c->N * c->margin_ctas;
-    CU(cudaMalloc(&c->r_scr, 4 * static_cast<size_t>(c->N) * batch), "allocating step scratch");
+    c->n_loss_part = c->N;
+    // The local step: one cluster of Q CTAs per worker, Q as large as keeps
+    // all clusters resident at four CTAs per SM (at most 8, the portable size).
+    c->step_q = kMaxStepCluster;
+    while (c->step_q > 1 && static_cast<int64_t>(c->N) * c->step_q > 4LL * c->sm_count) c->step_q >>= 1;
+    c->step_stages = 2;
+    c->step_smem = local_step_smem_bytes(batch, c->step_stages);
+    CU(local_step_configure(c->step_smem), "configuring the local-step kernel");
+    c->permuted = false;
   } else if (loss == ASAP_LOSS_SOFTMAX) {
     c->Cq = (num_classes + 255) / 256;
     c->n_loss_part = c->N * (batch / 128) * c->Cq;
@@ -1021,6 +1043,7 @@ asap_status asap_load_shards(asap_ctx* c, const int64_t* const* rowptr, const in
   c->s_cap = 1024;
   s0 = setup_mix(c);
   if (s0 != ASAP_OK) return s0;
+  const int Q = c->step_q;
   // Build every minibatch's image; narrow the slabs and rebuild while a
   // slab's column list is too long for the fused reduce's shared memory.
   for (;;) {
@@ -1028,7 +1051,9 @@ asap_status asap_load_shards(asap_ctx* c, const int64_t* const* rowptr, const in
     const long long n_slabs = c->n_slabs;
 
     std::vector<BatchImage> built(nb);
-    auto build_batch = [&](int t) { build_batch_image(N, B, c->d, S, n_slabs, t, rowptr, col, val, y, built[t]); };
+    auto build_batch = [&](int t) {
+      build_batch_image(N, B, c->d, S, n_slabs, Q, t, rowptr, col, val, y, built[t]);
+    };
     {
       const unsigned nthr = std::max(1u, std::min(32u, std::thread::hardware_concurrency()));
       std::vector<std::thread> pool;
@@ -1102,12 +1127,15 @@ asap_status asap_load_shards(asap_ctx* c, const int64_t* const* rowptr, const in
     CU(cudaMalloc(&c->gsum, lb), "allocating the column-sum buffer");
     CU(cudaMemset(c->wv, 0, lb), "zeroing the list value buffer");
     CU(cudaMemset(c->gsum, 0, lb), "zeroing the column-sum buffer");
+    if (B > kRSmemRows) {
+      CU(cudaMalloc(&c->mpart_big, 4 * static_cast<size_t>(N) * Q * B), "allocating the partial margins");
+      CU(cudaMalloc(&c->r_big, 4 * static_cast<size_t>(N) * Q * B), "allocating the step scratch");
+    }
     c->nb = nb;
     c->max_nnz = max_nnz;
     c->max_region = max_region;
     c->max_list = max_list;
     c->wv_step = -1;
-    c->update_ctas = update_ctas_for(max_nnz);
     c->configured_key = -1;
     return ASAP_OK;
   }
@@ -1256,16 +1284,21 @@ asap_status asap_local_step(asap_ctx* c) {
       c->launches += 1;
       c->wv_step = k;
     }
-    SparseStepArgs a;
+    LocalStepArgs a;
     a.block = block;
     a.desc = c->d_desc + static_cast<size_t>(tk) * c->N;
     a.wv = c->wv;
     a.gsum = c->gsum;
-    a.r = c->r_scr;
+    a.mpart_big = c->mpart_big;
+    a.r_big = c->r_big;
     a.loss_part = c->loss_part;
     a.ready = c->ready;
-    a.worker_ticket = c->ticket;
+    a.st = c->st;
+    a.worker_of = c->permuted ? c->d_worker_of : nullptr;
+    a.N = c->N;
     a.B = c->B;
+    a.Q = c->step_q;
+    a.stages = c->step_stages;
     a.round = static_cast<unsigned>(r);
     a.mscale = s_scale;
     a.notify = last ? 1 : 0;
@@ -1275,13 +1308,10 @@ asap_status asap_local_step(asap_ctx* c) {
       asap_status sg = prepare_graph(c, r);   // upload a regenerated graph ahead of the reduce
       if (sg != ASAP_OK) return sg;
     }
-    time_begin(c, ASAP_KERNEL_MARGIN);
-    CU(launch_margin(a, c->N, c->loss, c->margin_ctas, c->stream), "launching the margin kernel");
+    time_begin(c, ASAP_KERNEL_LOCAL_STEP);
+    CU(launch_local_step(a, c->loss, c->step_smem, c->stream), "launching the local-step kernel");
     time_end(c);
-    time_begin(c, ASAP_KERNEL_UPDATE);
-    CU(launch_update(a, c->N, c->update_ctas, c->stream), "launching the update kernel");
-    time_end(c);
-    c->launches += 2;
+    c->launches += 1;
     const float eta = lr_at(c, k);
     const float s_next = s_scale * (1.0f - eta * c->l2);
     const float upd = eta / (static_cast<float>(c->B) * s_next);

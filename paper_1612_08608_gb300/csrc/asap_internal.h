@@ -39,37 +39,52 @@ struct DevState {
 constexpr uint32_t kListPad = 0xffffffffu;   // padding entry of a column list
 
 // Where one worker's minibatch lives inside a batch block (byte offsets from
-// the block start).  Rows are padded to multiples of 4 entries (16 B) with
-// pos = 0, val = 0 so that the margin kernel can use 128-bit loads.  `pos`
-// indexes the batch's slab-major column list (one entry per distinct
-// (worker, column) of the minibatch).
+// the block start).  The minibatch's entries are kept in one order only,
+// sorted by (column, row); `cpos` indexes the batch's slab-major column list
+// (one entry per distinct (worker, column) of the minibatch).  For the
+// margins the sorted entries are cut into segments of kTileEntries; inside
+// a segment every entry has a slot, the slots of one row contiguous (rows in
+// order, a row's entries by column), and `srow` lists the row of every slot.
+// For the column sums the entries are split among the worker's Q CTAs at
+// column boundaries (`bnd`).
 struct BatchDesc {
-  int64_t rp;     // int32 [B+1]: padded row starts, in entries
   int64_t y;      // float [B]
-  int64_t posw;   // int32 [nnz_pad]: list position of each entry's column
-  int64_t val;    // float [nnz_pad]
-  int64_t cpos;   // int32 [nnz]: entries sorted by (column, row): list position
+  int64_t cpos;   // int32 [nnz]: list position of the entry's column
   int64_t cval;   // float [nnz]
   int64_t crow;   // uint16 [nnz]: row within the batch
-  int32_t nnz_pad;
+  int64_t cslot;  // uint16 [nnz]: slot within its segment
+  int64_t srow;   // uint16 [nnz]: per segment, the row of every slot
+  int64_t bnd;    // int32 [Q+1]: column-sum ranges of the worker's CTAs
   int32_t nnz;
+  int32_t pad_;
 };
 
-// Arguments of the sparse local step (margin kernel, then column sums).
-struct SparseStepArgs {
-  const unsigned char* block;  // batch block of this round
-  const BatchDesc* desc;       // [N] descriptors of this round's batch
-  const float* wv;             // w values at the round's list positions
-  float* gsum;                 // column sums at the round's list positions
-  float* r;                    // scratch [N][B]: d loss / d margin
-  float* loss_part;            // scratch [N][margin CTAs per worker]
+// Entries per margin segment and per column-sum tile (one ring stage).
+constexpr int kTileEntries = 1024;
+// Partial margins and r stay in shared memory for minibatches of at most
+// this many rows (else in global scratch).
+constexpr int kRSmemRows = 8192;
+constexpr int kLocalStepThreads = 160;   // four consumer warps + one producer warp
+constexpr int kMaxStepCluster = 8;       // CTAs per worker (portable cluster size)
+
+// Arguments of the fused sparse local step (kernels_sparse.cu): one cluster
+// of Q CTAs per worker.
+struct LocalStepArgs {
+  const unsigned char* block;  // batch block of this step
+  const BatchDesc* desc;       // [N] descriptors of this step's batch
+  const float* wv;             // w values at the step's list positions
+  float* gsum;                 // column sums at the step's list positions
+  float* mpart_big;            // [N][Q][B] partial margins (B > kRSmemRows only)
+  float* r_big;                // [N][Q][B] r (B > kRSmemRows only)
+  float* loss_part;            // [N]: minibatch loss sum per worker
   unsigned int* ready;         // NOTIFY flags [N]
-  unsigned int* worker_ticket; // [N] finished update CTAs of this round
-  int B;
+  DevState* st;
+  const int* worker_of;        // [N] worker of each cluster (a permutation), or nullptr
+  int N, B, Q, stages;
   unsigned int round;
   int skip_worker;             // fault injection: do not NOTIFY this worker
   float mscale;                // true w = mscale * (stored values): margins are scaled by it
-  int notify;                  // the column sums publish NOTIFY (last local step of the round)
+  int notify;                  // publish NOTIFY (last local step of the round)
 };
 
 // Arguments of the stochastic reduce.
@@ -145,8 +160,9 @@ asap_status build_graph_host(asap_graph_kind kind, int N, int k, uint64_t seed, 
                              int32_t* nbr, const char** why);
 
 // Launchers (kernels_*.cu).  Each returns the cudaError_t of the launch.
-cudaError_t launch_margin(const SparseStepArgs& a, int N, int loss, int margin_ctas, cudaStream_t s);
-cudaError_t launch_update(const SparseStepArgs& a, int N, int update_ctas, cudaStream_t s);
+cudaError_t launch_local_step(const LocalStepArgs& a, int loss, size_t smem, cudaStream_t s);
+size_t local_step_smem_bytes(int B, int stages);
+cudaError_t local_step_configure(size_t smem);
 cudaError_t launch_apply_update(float* W, int64_t ld, const uint32_t* list, const int* slab_off, long long n_slabs,
                                 int S, const float* gsum, float scale, int sm_count, cudaStream_t s);
 cudaError_t launch_gather_wv(const float* W, int64_t ld, const uint32_t* list, const int* slab_off, long long n_slabs,

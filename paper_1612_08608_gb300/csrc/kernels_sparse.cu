@@ -1,28 +1,39 @@
-// Local minibatch SGD step for sparse linear models (Eq. A.1, first line).
+// Local minibatch SGD step for sparse linear models (Eq. A.1, first line),
+// one fused kernel per step:
 //
-// The step is split so that no kernel touches w at random addresses:
+//   margins        m_b = sum_e val_e * wv[pos_e]
+//                  r_b = d loss(y_b, m_b) / d m_b        (hinge or logistic)
+//   column sums    g[p] = sum_{e : pos_e = p} r_{row_e} val_e
+//                  then NOTIFY ready[i] = t+1
 //
-//   margin kernel   m_b = sum_e val_e * wv[pos_e]          (8 lanes per row)
-//                   r_b = d loss(y_b, m_b) / d m_b        (hinge or logistic)
-//   update kernel   g[p] = sum_{e : pos_e = p} r_{row_e} val_e   (column sums)
-//                   then NOTIFY ready[i] = t+1
-//
-// Each round's minibatch has, per worker, a list of the distinct columns it
+// Each step's minibatch has, per worker, a list of the distinct columns it
 // touches.  The lists of all workers are laid out slab-major (by column slab
 // of the stochastic reduce, then worker, then column) and `pos` indexes that
-// list.  `wv[pos]` holds w_i[col] for the round's columns: the previous
+// list.  `wv[pos]` holds w_i[col] for the step's columns: the previous
 // round's reduce writes it while it holds the column slab in shared memory
 // (or, after parameters were written from the host, the gather kernel
 // below).  The reduce applies w_i[col] -= eta/B * g[pos] to the slab before
 // mixing it, so w_{t+1/2} never has to be written to HBM.
 //
-// Margin kernel: 8 lanes per row (4 rows in flight per warp), 128-bit loads
-// of (pos, val), the L2-resident wv gathered, a fixed butterfly sum.
-// Update kernel: entries sorted by (column, row) are
-// cut into 32-entry chunks, one warp per chunk; a segmented warp scan sums
-// each column's run and the warp holding a run's first entry owns it,
-// finishing runs that cross into later chunks itself.  No atomics on data,
-// every sum in a fixed order: the result does not depend on the schedule.
+// One cluster of Q CTAs per worker (grid N x Q, no inter-cluster waits).
+// The minibatch's entries are stored once, sorted by (column, row), and
+// streamed twice through a ring of shared-memory stages by one producer
+// warp with bulk copies (cp.async.bulk, mbarrier completion), while eight
+// consumer warps work on the stage that has landed:
+//   pass 1 (margins): CTA q takes 2048-entry segments s = q nseg/Q ...;
+//     products val * wv[pos] go to shared memory at the entry's slot (slots
+//     ordered by row, then column), a segmented scan over the slots keyed by
+//     row sums each row's products in order, and the CTA adds them to its
+//     partial margins.  A cluster barrier; every CTA then adds the Q partials
+//     of each row in rank order (distributed shared memory), forms r and,
+//     in CTA 0, the loss sum.
+//   pass 2 (column sums): CTA q takes the entries [bnd[q], bnd[q+1]), cut
+//     at column boundaries, in 2048-entry tiles; a segmented scan keyed by
+//     list position sums each column's r_row * val, the run crossing a tile
+//     boundary carried to the next tile.
+// A last cluster barrier and CTA 0 publishes NOTIFY.  No atomics, no waits
+// on other clusters, every sum in a fixed order: the result does not depend
+// on the schedule.
 #include <cuda_runtime.h>
 
 #include <cstdint>
@@ -34,8 +45,10 @@ namespace asap {
 namespace {
 
 constexpr unsigned kFull = 0xffffffffu;
-constexpr int kMarginRowsPerCta = 32;     // 8 warps x 4 rows
-constexpr int kUpdateChunksPerCta = 32;   // 8 warps x 4 chunks of 32 entries
+constexpr int kConsumers = kLocalStepThreads - 32;          // four consumer warps
+constexpr int kPerThread = kTileEntries / kConsumers;       // consecutive entries per consumer thread
+static_assert(kPerThread == 8, "a consumer thread takes 8 consecutive entries of a tile");
+constexpr unsigned long long kCopyWaitNs = 2000000000ull;   // a bulk copy never takes this long
 
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
@@ -43,35 +56,113 @@ __device__ __forceinline__ float warp_sum(float v) {
   return v;
 }
 
-__device__ __forceinline__ int4 ld_stream_i4(const int4* p) {
-  int4 v;
-  asm volatile("ld.global.nc.L1::no_allocate.v4.s32 {%0,%1,%2,%3}, [%4];"
-               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "l"(p));
-  return v;
-}
-
-__device__ __forceinline__ float4 ld_stream_f4(const float4* p) {
-  float4 v;
-  asm volatile("ld.global.nc.L1::no_allocate.v4.f32 {%0,%1,%2,%3}, [%4];"
-               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "l"(p));
-  return v;
-}
-
-// Gather of an exported w value, keeping the line in L2 (it is re-read by
-// other rows of the minibatch).
-__device__ __forceinline__ float ld_keep(const float* p, uint64_t policy) {
-  float v;
-  asm volatile("ld.global.nc.L2::cache_hint.f32 %0, [%1], %2;" : "=f"(v) : "l"(p), "l"(policy));
-  return v;
-}
-
-// Programmatic dependent launch: the next kernel in the stream may start its
-// CTAs now; this kernel waits here for the previous kernel's results.
-__device__ __forceinline__ void allow_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
-__device__ __forceinline__ void wait_previous() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
-
 __device__ __forceinline__ void st_release_u32(unsigned int* p, unsigned int v) {
   asm volatile("st.release.gpu.global.u32 [%0], %1;" :: "l"(p), "r"(v) : "memory");
+}
+
+__device__ __forceinline__ unsigned long long globaltimer_ns() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" :: "r"(smem_u32(bar)), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" :: "r"(smem_u32(bar)), "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" :: "r"(smem_u32(bar)) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
+      : "=r"(ok) : "r"(smem_u32(bar)), "r"(parity) : "memory");
+  return ok != 0;
+}
+
+// Time-limited wait on an mbarrier phase; false if the limit ran out.
+__device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const unsigned long long t0 = globaltimer_ns();
+  for (unsigned n = 1;; ++n) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((n & 255u) == 0 && globaltimer_ns() - t0 > kCopyWaitNs) return false;
+  }
+}
+
+// 4-byte asynchronous copy global -> shared (a gather), and an arrival on an
+// mbarrier once all of this thread's earlier such copies have landed.
+__device__ __forceinline__ void cp_async4(void* dst, const void* src) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" :: "r"(smem_u32(dst)), "l"(reinterpret_cast<uint64_t>(src))
+               : "memory");
+}
+
+__device__ __forceinline__ void cp_async_arrive(uint64_t* bar) {
+  asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];" :: "r"(smem_u32(bar)) : "memory");
+}
+
+// Untiled bulk copy global -> shared (16-byte aligned, size a multiple of 16).
+__device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+               :: "r"(smem_u32(dst)), "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(smem_u32(bar))
+               : "memory");
+}
+
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\nbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+
+__device__ __forceinline__ uint32_t cluster_id_x() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%clusterid.x;" : "=r"(r));
+  return r;
+}
+
+// Load of `local`'s offset in the shared memory of cluster CTA `rank`.
+__device__ __forceinline__ float ld_dsmem(const float* local, uint32_t rank) {
+  uint32_t remote;
+  float v;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(local)), "r"(rank));
+  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(remote) : "memory");
+  return v;
+}
+
+// Barrier among the consumer warps only (the producer warp keeps streaming).
+__device__ __forceinline__ void consumer_bar() {
+  asm volatile("bar.sync 1, %0;" :: "n"(kConsumers) : "memory");
+}
+
+// Consumer barrier that also returns the AND of `v` over the consumer threads.
+__device__ __forceinline__ bool consumer_bar_and(bool v) {
+  uint32_t r;
+  asm volatile(
+      "{\n .reg .pred p, q;\n setp.ne.u32 p, %1, 0;\n bar.red.and.pred q, 1, %2, p;\n selp.u32 %0, 1, 0, q;\n}"
+      : "=r"(r) : "r"(static_cast<uint32_t>(v)), "n"(kConsumers) : "memory");
+  return r != 0;
+}
+
+__device__ __forceinline__ void record_error(DevState* st, unsigned code, unsigned worker, unsigned round) {
+  if (atomicCAS(&st->err_code, 0u, code) == 0u) {
+    st->err_worker = worker;
+    st->err_round = round;
+  }
 }
 
 // loss(y, m) and r = d loss / d m.
@@ -88,184 +179,370 @@ __device__ __forceinline__ void loss_and_r(float y, float m, float& l, float& r)
   }
 }
 
-template <int LOSS>
-__global__ void __launch_bounds__(kThreads) k_margin_loss(SparseStepArgs a) {
-  // 8 lanes per row, so that each warp keeps the loads of 4 rows in flight.
-  constexpr int kLanesPerRow = 8;
-  const int i = blockIdx.y;
-  const BatchDesc dsc = a.desc[i];
-  const int* rp = reinterpret_cast<const int*>(a.block + dsc.rp);
-  const float* y = reinterpret_cast<const float*>(a.block + dsc.y);
-  const int4* pos4 = reinterpret_cast<const int4*>(a.block + dsc.posw);
-  const float4* val4 = reinterpret_cast<const float4*>(a.block + dsc.val);
-  allow_dependents();
-  const float* wv = a.wv;
-  uint64_t keep;
-  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(keep));
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int sub = lane / kLanesPerRow, sl = lane % kLanesPerRow;
-  const int b = blockIdx.x * kMarginRowsPerCta + warp * (32 / kLanesPerRow) + sub;   // 8 warps x 4 rows
-  float lsum = 0.f;
-  float acc = 0.f;
-  if (b < a.B) {
-    const int q0 = rp[b] >> 2, q1 = rp[b + 1] >> 2;
-    // Four quads per lane per pass, all loads issued before the sums; the
-    // summation order is the sequential one (quad after quad).
-    constexpr int kU = 4;
-    for (int q = q0 + sl; q < q1; q += kU * kLanesPerRow) {
-      int4 p[kU];
-      float4 v[kU];
-#pragma unroll
-      for (int u = 0; u < kU; ++u) {
-        const int qq = q + u * kLanesPerRow;
-        if (qq < q1) {
-          p[u] = ld_stream_i4(pos4 + qq);
-          v[u] = ld_stream_f4(val4 + qq);
-        } else {
-          p[u] = make_int4(0, 0, 0, 0);
-          v[u] = make_float4(0.f, 0.f, 0.f, 0.f);
-        }
-      }
-      float g[4 * kU];
-#pragma unroll
-      for (int u = 0; u < kU; ++u) {
-        g[4 * u + 0] = ld_keep(wv + p[u].x, keep);
-        g[4 * u + 1] = ld_keep(wv + p[u].y, keep);
-        g[4 * u + 2] = ld_keep(wv + p[u].z, keep);
-        g[4 * u + 3] = ld_keep(wv + p[u].w, keep);
-      }
-#pragma unroll
-      for (int u = 0; u < kU; ++u) {
-        if (q + u * kLanesPerRow < q1) {
-          acc = fmaf(v[u].x, g[4 * u + 0], acc);
-          acc = fmaf(v[u].y, g[4 * u + 1], acc);
-          acc = fmaf(v[u].z, g[4 * u + 2], acc);
-          acc = fmaf(v[u].w, g[4 * u + 3], acc);
-        }
-      }
-    }
-  }
-#pragma unroll
-  for (int o = kLanesPerRow / 2; o > 0; o >>= 1) acc += __shfl_xor_sync(kFull, acc, o);
-  if (b < a.B && sl == 0) {
-    float l, r;
-    loss_and_r<LOSS>(y[b], acc * a.mscale, l, r);
-    a.r[static_cast<int64_t>(i) * a.B + b] = r;
-    lsum = l;
-  }
-  // fixed-order sum of the CTA's 32 row losses
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) lsum += __shfl_xor_sync(kFull, lsum, o);
-  __shared__ float part[kThreads / 32];
-  if (lane == 0) part[warp] = lsum;
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    float s = 0.f;
-#pragma unroll
-    for (int k = 0; k < kThreads / 32; ++k) s += part[k];
-    a.loss_part[static_cast<int64_t>(i) * gridDim.x + blockIdx.x] = s;
-  }
+// Shared-memory layout of the local-step kernel (mirrored by
+// local_step_smem_bytes): the ring of stages, each holding one tile's list
+// positions, values and two uint16 arrays (pass 1: slots and the rows in
+// slot order; pass 2: rows); the products of a segment by slot; the
+// partial margins and r of the worker's B rows; scan and control scratch.
+struct StepSmem {
+  unsigned char* stage0;
+  uint64_t* full;
+  uint64_t* empty;
+  uint64_t* gath;       // [stages]: the w values of a margin tile are in the stage
+  float* prod;          // [kTileEntries]: products by slot (pass 1), run sums (pass 2)
+  int* okey;            // [kTileEntries]: list position of a run ending at the pair, else -1
+  float* mpart;         // [B]
+  float* r;             // [B]
+  int* keys;            // [kConsumers]: first key of each thread's pairs
+  int* keys_last;       // [kConsumers]: last key of each thread's pairs
+  float* wval;          // [kConsumers / 32]: warp aggregates of the scan
+  int* wflag;           // [kConsumers / 32]
+  float* red;           // [kConsumers / 32]
+  int* ctl;             // [0]: carry key, [1]: a copy timed out
+  float* carry;         // [1]: carried run sum
+};
+
+// pos, val, two uint16 arrays, and (pass 1) the gathered w values
+constexpr size_t kStageBytes = static_cast<size_t>(kTileEntries) * 16;
+
+__device__ __forceinline__ StepSmem carve_step(unsigned char* raw, int B, int stages) {
+  StepSmem m;
+  uintptr_t p = (reinterpret_cast<uintptr_t>(raw) + 127) & ~static_cast<uintptr_t>(127);
+  m.stage0 = reinterpret_cast<unsigned char*>(p);
+  p += kStageBytes * stages;
+  m.full = reinterpret_cast<uint64_t*>(p);
+  p += 8 * stages;
+  m.empty = reinterpret_cast<uint64_t*>(p);
+  p += 8 * stages;
+  m.gath = reinterpret_cast<uint64_t*>(p);
+  p += 8 * stages;
+  p = (p + 15) & ~static_cast<uintptr_t>(15);   // prod is read as float4
+  m.prod = reinterpret_cast<float*>(p);
+  p += 4 * kTileEntries;
+  m.okey = reinterpret_cast<int*>(p);
+  p += 4 * kTileEntries;
+  m.mpart = reinterpret_cast<float*>(p);
+  p += 4 * static_cast<size_t>(B);
+  m.r = reinterpret_cast<float*>(p);
+  p += 4 * static_cast<size_t>(B);
+  m.keys = reinterpret_cast<int*>(p);
+  p += 4 * kConsumers;
+  m.keys_last = reinterpret_cast<int*>(p);
+  p += 4 * kConsumers;
+  m.wval = reinterpret_cast<float*>(p);
+  p += 4 * (kConsumers / 32);
+  m.wflag = reinterpret_cast<int*>(p);
+  p += 4 * (kConsumers / 32);
+  m.red = reinterpret_cast<float*>(p);
+  p += 4 * (kConsumers / 32);
+  m.ctl = reinterpret_cast<int*>(p);
+  p += 8;
+  m.carry = reinterpret_cast<float*>(p);
+  return m;
 }
 
-__global__ void __launch_bounds__(kThreads) k_column_sums(SparseStepArgs a) {
-  allow_dependents();
-  const int i = blockIdx.y;
-  const BatchDesc dsc = a.desc[i];
-  const int nnz = dsc.nnz;
-  const int* cpos = reinterpret_cast<const int*>(a.block + dsc.cpos);
-  const float* cval = reinterpret_cast<const float*>(a.block + dsc.cval);
-  const uint16_t* crow = reinterpret_cast<const uint16_t*>(a.block + dsc.crow);
-  const float* r = a.r + static_cast<int64_t>(i) * a.B;
-  float* g = a.gsum;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const unsigned le_mask = (lane == 31) ? kFull : ((2u << lane) - 1u);
-
-  const int n_chunks = (nnz + 31) >> 5;
-  constexpr int kPerWarp = kUpdateChunksPerCta / (kThreads / 32);   // 4 chunks per warp per pass
-  for (int first = blockIdx.x * kUpdateChunksPerCta; first < n_chunks; first += gridDim.x * kUpdateChunksPerCta) {
-    // Load the warp's chunks first (independent), then scan them one by one.
-    int cv[kPerWarp], cpv[kPerWarp], cnx[kPerWarp], rw[kPerWarp];
-    float pv[kPerWarp];
+// Segmented inclusive scan over the pairs of a tile: consumer thread t holds
+// the eight consecutive pairs 8t .. 8t+7 (key, value); a run is a maximal
+// stretch of equal keys.  `in_key` / `in_val` is a run carried in from
+// before the tile.  On return val[u] is the sum of its run's values up to
+// and including pair u, and next_key the key of the pair after this
+// thread's last (that of thread t+1's first pair; `tail_key` for the last
+// thread).  Fixed order of additions: within a thread left to right, then a
+// fixed shuffle tree, then the warps in order.
+__device__ __forceinline__ void seg_scan8(const int (&key)[kPerThread], float (&val)[kPerThread], int in_key,
+                                          float in_val, int tail_key, int& next_key, const StepSmem& sm) {
+  const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+  sm.keys[t] = key[0];
+  sm.keys_last[t] = key[kPerThread - 1];
+  consumer_bar();
+  const int prev_key = t == 0 ? in_key : sm.keys_last[t - 1];
+  next_key = t + 1 < kConsumers ? sm.keys[t + 1] : tail_key;
+  bool any_head = false;
+  int pk = prev_key;
 #pragma unroll
-    for (int u = 0; u < kPerWarp; ++u) {
-      const int chunk = first + warp + u * (kThreads / 32);
-      const int e = chunk * 32 + lane;
-      const bool valid = chunk < n_chunks && e < nnz;
-      cv[u] = valid ? cpos[e] : -1;
-      cpv[u] = (lane == 0 && chunk < n_chunks && e > 0) ? cpos[e - 1] : -2;
-      // the entry after the chunk: does lane 31's run continue past it?
-      cnx[u] = (lane == 31 && chunk < n_chunks && e + 1 < nnz) ? cpos[e + 1] : -3;
-      pv[u] = valid ? cval[e] : 0.f;
-      rw[u] = valid ? crow[e] : -1;
-    }
-    wait_previous();   // r comes from the margin kernel
+  for (int u = 0; u < kPerThread; ++u) {
+    const bool head = key[u] != pk;
+    if (u > 0 && !head) val[u] += val[u - 1];
+    any_head = any_head || head;
+    pk = key[u];
+  }
+  // inclusive scan over the warp of (a head seen, running value of the last run)
+  float v = val[kPerThread - 1];
+  int f = any_head ? 1 : 0;
 #pragma unroll
-    for (int u = 0; u < kPerWarp; ++u)
-      if (rw[u] >= 0) pv[u] *= r[rw[u]];
-#pragma unroll
-    for (int u = 0; u < kPerWarp; ++u) {
-    const int chunk = first + warp + u * (kThreads / 32);
-    if (chunk >= n_chunks) break;                  // warp-uniform
-    const int e = chunk * 32 + lane;
-    const bool valid = e < nnz;
-    const int c = cv[u];
-    int cprev = __shfl_up_sync(kFull, c, 1);
-    if (lane == 0) cprev = cpv[u];
-    const bool head = valid && (c != cprev);
-    float p = pv[u];
-    const unsigned heads = __ballot_sync(kFull, head);
-    const unsigned hl = heads & le_mask;
-    const int start = hl ? (31 - __clz(hl)) : -1;   // first lane of this lane's run, -1: began earlier
-    const int s_eff = start < 0 ? 0 : start;
-#pragma unroll
-    for (int off = 1; off < 32; off <<= 1) {
-      const float v = __shfl_up_sync(kFull, p, off);
-      if (lane - off >= s_eff) p += v;
-    }
-    const bool next_head = __shfl_down_sync(kFull, head, 1);
-    const bool next_valid = __shfl_down_sync(kFull, valid, 1);
-    // Runs that end inside the chunk: the tail lane writes if the run began here.
-    if (valid && lane < 31 && (next_head || !next_valid) && start >= 0) g[c] = p;
-    // The run through lane 31.
-    const int c31 = __shfl_sync(kFull, c, 31);
-    const int start31 = __shfl_sync(kFull, start, 31);
-    const float p31 = __shfl_sync(kFull, p, 31);
-    if (c31 >= 0 && start31 >= 0) {
-      const int e31 = chunk * 32 + 31;
-      bool cont = (e31 + 1 < nnz) && (__shfl_sync(kFull, cnx[u], 31) == c31);
-      float acc = p31;
-      int base = e31 + 1;
-      while (cont) {
-        const int e2 = base + lane;
-        const bool in_run = (e2 < nnz) && (cpos[e2] == c31);
-        const float q = in_run ? r[crow[e2]] * cval[e2] : 0.f;
-        acc += warp_sum(q);
-        const unsigned run = __ballot_sync(kFull, in_run);
-        cont = (run == kFull) && (base + 32 < nnz) && (cpos[base + 32] == c31);
-        base += 32;
-      }
-      if (lane == 0) g[c31] = acc;
-    }
+  for (int off = 1; off < 32; off <<= 1) {
+    const float vo = __shfl_up_sync(kFull, v, off);
+    const int fo = __shfl_up_sync(kFull, f, off);
+    if (lane >= off) {
+      if (!f) v += vo;
+      f |= fo;
     }
   }
+  if (lane == 31) {
+    sm.wval[warp] = v;
+    sm.wflag[warp] = f;
+  }
+  float ev = __shfl_up_sync(kFull, v, 1);      // exclusive: the lanes before this one
+  const int ef = __shfl_up_sync(kFull, f, 1);
+  consumer_bar();
+  float pv = in_val;                           // the carried run, then the earlier warps
+  for (int w = 0; w < warp; ++w) pv = sm.wflag[w] ? sm.wval[w] : pv + sm.wval[w];
+  if (lane == 0)
+    ev = pv;
+  else if (!ef)
+    ev += pv;
+  pk = prev_key;
+#pragma unroll
+  for (int u = 0; u < kPerThread; ++u) {       // pairs before this thread's first head
+    if (key[u] != pk) break;
+    val[u] += ev;
+    pk = key[u];
+  }
+  consumer_bar();   // sm.keys / wval are reused by the next scan
+}
 
-  // A CTA without chunks has not waited for the margin kernel yet.  Were no
-  // CTA to wait (an all-empty minibatch), this grid could complete before the
-  // margin kernel, and the reduce would read its loss partials too early.
-  wait_previous();
+template <int LOSS>
+__global__ void __launch_bounds__(kLocalStepThreads, 1) k_local_step(const LocalStepArgs a) {
+  extern __shared__ unsigned char step_smem_raw[];
+  const bool big = a.B > kRSmemRows;           // partial margins and r in global memory
+  const StepSmem sm = carve_step(step_smem_raw, big ? 0 : a.B, a.stages);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int q = static_cast<int>(cluster_rank());
+  const int Q = a.Q;
+  const int cl = static_cast<int>(cluster_id_x());
+  const int i = a.worker_of ? a.worker_of[cl] : cl;
+  const BatchDesc dsc = a.desc[i];
+  const int nnz = dsc.nnz;
+  const int nseg = (nnz + kTileEntries - 1) / kTileEntries;
+  const int s0 = static_cast<int>(static_cast<long long>(q) * nseg / Q);
+  const int s1 = static_cast<int>(static_cast<long long>(q + 1) * nseg / Q);
+  const int n1 = s1 - s0;
+  const int* bnd = reinterpret_cast<const int*>(a.block + dsc.bnd);
+  const int lo = bnd[q], hi = bnd[q + 1];
+  const int T0 = lo & ~7;                      // 16-byte aligned start of the first column tile
+  const int n2 = hi > lo ? (hi - T0 + kTileEntries - 1) / kTileEntries : 0;
+  float* mpart = big ? a.mpart_big + (static_cast<size_t>(i) * Q + q) * a.B : sm.mpart;
+  float* rr = big ? a.r_big + (static_cast<size_t>(i) * Q + q) * a.B : sm.r;
 
-  // NOTIFY: the last CTA of worker i publishes ready[i] = round + 1 once all
-  // of worker i's column sums are visible device-wide.  The CTA barrier
-  // orders this CTA's writes before thread 0's fence, which is cumulative.
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    __threadfence();
-    const unsigned int done = atomicAdd(&a.worker_ticket[i], 1u);
-    if (done == gridDim.x - 1) {
-      a.worker_ticket[i] = 0u;
-      __threadfence();
-      if (a.notify && i != a.skip_worker) st_release_u32(&a.ready[i], a.round + 1u);
+  if (tid == 0) {
+    for (int st = 0; st < a.stages; ++st) {
+      mbar_init(sm.full + st, 1);
+      mbar_init(sm.empty + st, kConsumers / 32);
+      mbar_init(sm.gath + st, 32);
     }
+    sm.ctl[0] = -1;
+    sm.ctl[1] = 0;
+    sm.carry[0] = 0.f;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  for (int b = tid; b < a.B; b += kLocalStepThreads) mpart[b] = 0.f;
+  __syncthreads();
+  // The stochastic reduce that follows is a programmatic dependent: its CTAs
+  // may take SMs as this grid drains; it waits for this grid's results.
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+
+  bool ok = true;
+  if (warp == kConsumers / 32) {
+    // ================= producer warp =================
+    // Issues every tile of both passes in order; it arrives on the cluster
+    // barrier between the passes as soon as pass 1 is issued, so that it
+    // never holds up the consumers there.
+    auto issue = [&](int it) -> bool {
+      const int st = it % a.stages;
+      if (it >= a.stages && !mbar_wait_bounded(sm.empty + st, ((it / a.stages) - 1) & 1)) return false;
+      unsigned char* base = sm.stage0 + kStageBytes * st;
+      const bool pass1 = it < n1;
+      const int e0 = pass1 ? (s0 + it) * kTileEntries : T0 + (it - n1) * kTileEntries;
+      const int len = min(kTileEntries, (pass1 ? nnz : hi) - e0);
+      const uint32_t n8 = static_cast<uint32_t>((len + 7) & ~7);   // whole 16-byte rows of uint16
+      mbar_expect_tx(sm.full + st, n8 * (pass1 ? 12u : 10u));
+      bulk_load(base, a.block + dsc.cpos + 4 * static_cast<int64_t>(e0), 4 * n8, sm.full + st);
+      bulk_load(base + 4 * kTileEntries, a.block + dsc.cval + 4 * static_cast<int64_t>(e0), 4 * n8, sm.full + st);
+      if (pass1) {
+        bulk_load(base + 8 * kTileEntries, a.block + dsc.cslot + 2 * static_cast<int64_t>(e0), 2 * n8, sm.full + st);
+        bulk_load(base + 10 * kTileEntries, a.block + dsc.srow + 2 * static_cast<int64_t>(e0), 2 * n8, sm.full + st);
+      } else {
+        bulk_load(base + 8 * kTileEntries, a.block + dsc.crow + 2 * static_cast<int64_t>(e0), 2 * n8, sm.full + st);
+      }
+      return true;
+    };
+    // The w values of margin tile k: once its list positions have landed,
+    // every lane gathers 32 of them with 4-byte asynchronous copies and
+    // arrives on gath[k] when they are in.
+    auto gather = [&](int k) -> bool {
+      const int st = k % a.stages;
+      if (!mbar_wait_bounded(sm.full + st, (k / a.stages) & 1)) return false;
+      unsigned char* base = sm.stage0 + kStageBytes * st;
+      const int* spos = reinterpret_cast<const int*>(base);
+      float* wvs = reinterpret_cast<float*>(base + 12 * kTileEntries);
+      const int len = min(kTileEntries, nnz - (s0 + k) * kTileEntries);
+      for (int j = lane; j < len; j += 32) cp_async4(wvs + j, a.wv + spos[j]);
+      cp_async_arrive(sm.gath + st);
+      return true;
+    };
+    bool pok = true;
+    for (int it = 0; it < n1 && pok; ++it) {
+      if (lane == 0) pok = issue(it);
+      pok = __shfl_sync(kFull, pok, 0) != 0;
+      if (pok && it > 0) pok = __all_sync(kFull, gather(it - 1));
+    }
+    if (pok && n1 > 0) pok = __all_sync(kFull, gather(n1 - 1));
+    __syncwarp();
+    asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+    if (lane == 0) {
+      for (int it = n1; it < n1 + n2 && pok; ++it) pok = issue(it);
+      if (!pok) sm.ctl[1] = 1;
+    }
+    __syncwarp();
+    asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+  } else {
+    // ================= consumer warps =================
+    const int j0 = tid * kPerThread;           // this thread's pairs within a tile
+    // ---- pass 1: products by slot; each row's sum by a scan over the slots ----
+    for (int it = 0; it < n1 && ok; ++it) {
+      const int st = it % a.stages;
+      ok = consumer_bar_and(mbar_wait_bounded(sm.gath + st, (it / a.stages) & 1));
+      if (!ok) break;
+      const unsigned char* base = sm.stage0 + kStageBytes * st;
+      const float* sval = reinterpret_cast<const float*>(base + 4 * kTileEntries);
+      const uint16_t* sslot = reinterpret_cast<const uint16_t*>(base + 8 * kTileEntries);
+      const uint16_t* srow = reinterpret_cast<const uint16_t*>(base + 10 * kTileEntries);
+      const float* wvs = reinterpret_cast<const float*>(base + 12 * kTileEntries);
+      const int len = min(kTileEntries, nnz - (s0 + it) * kTileEntries);
+#pragma unroll
+      for (int u = 0; u < kPerThread; ++u) {   // entry u * 128 + t: consecutive threads, consecutive entries
+        const int j = u * kConsumers + tid;
+        if (j < len) sm.prod[sslot[j]] = sval[j] * wvs[j];
+      }
+      consumer_bar();
+      int key[kPerThread];
+      float val[kPerThread];
+      {
+        // slots j0 .. j0+7 (a row's slots are adjacent): vector loads
+        const float4 q0 = *reinterpret_cast<const float4*>(sm.prod + j0);
+        const float4 q1 = *reinterpret_cast<const float4*>(sm.prod + j0 + 4);
+        const uint4 rw = *reinterpret_cast<const uint4*>(srow + j0);
+        const float pv[8] = {q0.x, q0.y, q0.z, q0.w, q1.x, q1.y, q1.z, q1.w};
+        const unsigned rws[4] = {rw.x, rw.y, rw.z, rw.w};
+#pragma unroll
+        for (int u = 0; u < kPerThread; ++u) {
+          const bool in = j0 + u < len;
+          key[u] = in ? static_cast<int>((rws[u >> 1] >> (16 * (u & 1))) & 0xffffu) : -1;
+          val[u] = in ? pv[u] : 0.f;
+        }
+      }
+      int next_key;
+      seg_scan8(key, val, -2, 0.f, -1, next_key, sm);
+#pragma unroll
+      for (int u = 0; u < kPerThread; ++u) {
+        const int nk = u + 1 < kPerThread ? key[u + 1] : next_key;
+        if (key[u] >= 0 && nk != key[u]) mpart[key[u]] += val[u];   // a row's run ends: its partial
+      }
+      consumer_bar();
+      if (lane == 0) mbar_arrive(sm.empty + st);
+    }
+    // ---- the worker's margins: the Q partials of every row in rank order ----
+    if (big) __threadfence();
+    asm volatile("barrier.cluster.arrive.release.aligned;\nbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+    const float* y = reinterpret_cast<const float*>(a.block + dsc.y);
+    float lsum = 0.f;
+    for (int b = tid; b < a.B; b += kConsumers) {
+      float m = 0.f;
+      for (int qq = 0; qq < Q; ++qq)
+        m += big ? __ldcg(a.mpart_big + (static_cast<size_t>(i) * Q + qq) * a.B + b) : ld_dsmem(sm.mpart + b, qq);
+      float l, r;
+      loss_and_r<LOSS>(y[b], m * a.mscale, l, r);
+      rr[b] = r;
+      lsum += l;
+    }
+    if (q == 0) {
+      lsum = warp_sum(lsum);
+      if (lane == 0) sm.red[warp] = lsum;
+    }
+    consumer_bar();
+    if (q == 0 && tid == 0) {
+      float tot = 0.f;
+      for (int w2 = 0; w2 < kConsumers / 32; ++w2) tot += sm.red[w2];
+      a.loss_part[i] = tot;
+    }
+    ok = ok && !sm.ctl[1];
+    // ---- pass 2: column sums over [lo, hi), a run carried across tiles ----
+    float* g = a.gsum;
+    for (int k = 0; k < n2 && ok; ++k) {
+      const int it = n1 + k;
+      const int st = it % a.stages;
+      ok = consumer_bar_and(mbar_wait_bounded(sm.full + st, (it / a.stages) & 1));
+      if (!ok) break;
+      const unsigned char* base = sm.stage0 + kStageBytes * st;
+      const int* spos = reinterpret_cast<const int*>(base);
+      const float* sval = reinterpret_cast<const float*>(base + 4 * kTileEntries);
+      const uint16_t* srw = reinterpret_cast<const uint16_t*>(base + 8 * kTileEntries);
+      const int e_base = T0 + k * kTileEntries;
+      int key[kPerThread];
+      float val[kPerThread];
+      const int4 p0 = *reinterpret_cast<const int4*>(spos + j0);
+      const int4 p1 = *reinterpret_cast<const int4*>(spos + j0 + 4);
+      const float4 v0 = *reinterpret_cast<const float4*>(sval + j0);
+      const float4 v1 = *reinterpret_cast<const float4*>(sval + j0 + 4);
+      const uint4 rw = *reinterpret_cast<const uint4*>(srw + j0);
+      const int pk[8] = {p0.x, p0.y, p0.z, p0.w, p1.x, p1.y, p1.z, p1.w};
+      const float pv[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
+      const unsigned rws[4] = {rw.x, rw.y, rw.z, rw.w};
+#pragma unroll
+      for (int u = 0; u < kPerThread; ++u) {
+        const int e = e_base + j0 + u;
+        const bool valid = e >= lo && e < hi;
+        const int row = static_cast<int>((rws[u >> 1] >> (16 * (u & 1))) & 0xffffu);
+        key[u] = valid ? pk[u] : -1;
+        val[u] = valid ? (big ? __ldcg(rr + row) : sm.r[row]) * pv[u] : 0.f;
+      }
+      const int in_key = sm.ctl[0];
+      const float in_val = sm.carry[0];
+      const bool last_tile = k == n2 - 1;
+      int next_key;
+      // after the last tile the range ends at a column boundary; otherwise the
+      // run through the tile's last pair may go on in the next tile
+      seg_scan8(key, val, in_key, in_val, last_tile ? -1 : -3, next_key, sm);
+      if (tid == 0 && in_key >= 0 && key[0] != in_key) g[in_key] = in_val;   // the carried run ended before this tile
+      // Every run that ends in the tile leaves (position, sum) at its last
+      // pair; the sums are then written with consecutive threads on
+      // consecutive pairs, so that the stores coalesce.
+      {
+        int ok8[kPerThread];
+#pragma unroll
+        for (int u = 0; u < kPerThread; ++u) {
+          const int nk = u + 1 < kPerThread ? key[u + 1] : next_key;
+          ok8[u] = (key[u] >= 0 && nk != key[u] && nk != -3) ? key[u] : -1;
+        }
+        *reinterpret_cast<int4*>(sm.okey + j0) = make_int4(ok8[0], ok8[1], ok8[2], ok8[3]);
+        *reinterpret_cast<int4*>(sm.okey + j0 + 4) = make_int4(ok8[4], ok8[5], ok8[6], ok8[7]);
+        *reinterpret_cast<float4*>(sm.prod + j0) = make_float4(val[0], val[1], val[2], val[3]);
+        *reinterpret_cast<float4*>(sm.prod + j0 + 4) = make_float4(val[4], val[5], val[6], val[7]);
+      }
+      consumer_bar();
+#pragma unroll
+      for (int u = 0; u < kPerThread; ++u) {
+        const int j = u * kConsumers + tid;
+        const int k = sm.okey[j];
+        if (k >= 0) g[k] = sm.prod[j];
+      }
+      if (tid == kConsumers - 1) {             // carry the tile's last run
+        const bool open = !last_tile && key[kPerThread - 1] >= 0;
+        sm.ctl[0] = open ? key[kPerThread - 1] : -1;
+        sm.carry[0] = open ? val[kPerThread - 1] : 0.f;
+      }
+      consumer_bar();
+      if (lane == 0) mbar_arrive(sm.empty + st);
+    }
+    if (!ok && tid == 0) record_error(a.st, ASAP_ERR_CUDA, static_cast<unsigned>(i), a.round);
+  }
+  // ---- NOTIFY: every CTA's column sums are visible, then CTA 0 publishes ----
+  __threadfence();
+  const int all_ok = __syncthreads_or(!ok || sm.ctl[1]) == 0;
+  asm volatile("barrier.cluster.arrive.release.aligned;\nbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+  if (q == 0 && tid == 0 && a.notify && i != a.skip_worker) {
+    __threadfence();
+    if (all_ok) st_release_u32(&a.ready[i], a.round + 1u);
   }
 }
 
@@ -352,40 +629,41 @@ cudaError_t launch_apply_update(float* W, int64_t ld, const uint32_t* list, cons
   return cudaGetLastError();
 }
 
-cudaError_t launch_margin(const SparseStepArgs& a, int N, int loss, int margin_ctas, cudaStream_t s) {
-  const dim3 g1(margin_ctas, N);
-  if (loss == ASAP_LOSS_HINGE)
-    k_margin_loss<ASAP_LOSS_HINGE><<<g1, kThreads, 0, s>>>(a);
-  else
-    k_margin_loss<ASAP_LOSS_LOGISTIC><<<g1, kThreads, 0, s>>>(a);
-  return cudaGetLastError();
+size_t local_step_smem_bytes(int B, int stages) {
+  const size_t b_smem = B > kRSmemRows ? 0 : static_cast<size_t>(B);
+  return 128 + kStageBytes * stages + 24 * static_cast<size_t>(stages) + 16 + 8 * kTileEntries + 8 * b_smem +
+         8 * kConsumers + 12 * (kConsumers / 32) + 12;
 }
 
-cudaError_t launch_update(const SparseStepArgs& a, int N, int update_ctas, cudaStream_t s) {
-  // Launched as a programmatic dependent of the margin kernel.
+cudaError_t local_step_configure(size_t smem) {
+  cudaError_t e = cudaFuncSetAttribute(k_local_step<ASAP_LOSS_HINGE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(smem));
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(k_local_step<ASAP_LOSS_LOGISTIC>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              static_cast<int>(smem));
+}
+
+cudaError_t launch_local_step(const LocalStepArgs& a, int loss, size_t smem, cudaStream_t s) {
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(update_ctas, N);
-  cfg.blockDim = dim3(kThreads);
+  cfg.gridDim = dim3(a.N * a.Q);
+  cfg.blockDim = dim3(kLocalStepThreads);
+  cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = a.Q;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, k_column_sums, a);
+  if (loss == ASAP_LOSS_HINGE) return cudaLaunchKernelEx(&cfg, k_local_step<ASAP_LOSS_HINGE>, a);
+  return cudaLaunchKernelEx(&cfg, k_local_step<ASAP_LOSS_LOGISTIC>, a);
 }
 
 cudaError_t launch_gather_wv(const float* W, int64_t ld, const uint32_t* list, const int* slab_off, long long n_slabs,
                              int S, float* wv, int sm_count, cudaStream_t s) {
   k_gather_wv<<<slab_warp_grid(n_slabs, sm_count), kThreads, 0, s>>>(W, ld, list, slab_off, n_slabs, S, wv);
   return cudaGetLastError();
-}
-
-int margin_ctas_for(int B) { return (B + kMarginRowsPerCta - 1) / kMarginRowsPerCta; }
-int update_ctas_for(int max_nnz) {
-  const int chunks = (max_nnz + 31) / 32;
-  const int c = (chunks + kUpdateChunksPerCta - 1) / kUpdateChunksPerCta;
-  return c < 1 ? 1 : c;
 }
 
 }  // namespace asap

@@ -214,14 +214,6 @@ extern "C" asap_status asap_mix_noalloc(const float* W_in, float* W_out, int N, 
   if (kp1 < 1 || kp1 > kMaxKp1Sparse) return reject(ASAP_ERR_ARG, "asap_mix_noalloc: need 1 <= k+1 <= 32");
   if (d < 1 || ld < d || ld % 4 != 0)
     return reject(ASAP_ERR_ARG, "asap_mix_noalloc: need d >= 1, ld >= d and ld a multiple of 4");
-  {
-    // Every CTA reads rows of W_in that other CTAs may already have written
-    // to W_out: the two ranges must not overlap at all.
-    const uintptr_t a0 = reinterpret_cast<uintptr_t>(W_in), b0 = reinterpret_cast<uintptr_t>(W_out);
-    const uintptr_t bytes = static_cast<uintptr_t>(N) * static_cast<uintptr_t>(ld) * sizeof(float);
-    if (a0 < b0 + bytes && b0 < a0 + bytes)
-      return reject(ASAP_ERR_ARG, "asap_mix_noalloc: W_in and W_out must not overlap");
-  }
   if ((reinterpret_cast<uintptr_t>(W_in) | reinterpret_cast<uintptr_t>(W_out)) & 15u)
     return reject(ASAP_ERR_ARG, "asap_mix_noalloc: W_in and W_out must be 16-byte aligned");
   int S = 256;
@@ -230,6 +222,14 @@ extern "C" asap_status asap_mix_noalloc(const float* W_in, float* W_out, int N, 
   if (n_slabs > kNoAllocMaxSlabs)
     return reject(ASAP_ERR_ARG, "asap_mix_noalloc: ld too large for the built-in scratch "
                                 "(at most 32768 slabs of 256 columns for N <= 16, 16 columns for N = 256)");
+  {
+    // Every CTA reads rows of W_in that other CTAs may already have written
+    // to W_out: the two ranges must not overlap at all.
+    const uintptr_t a0 = reinterpret_cast<uintptr_t>(W_in), b0 = reinterpret_cast<uintptr_t>(W_out);
+    const uintptr_t bytes = static_cast<uintptr_t>(N) * static_cast<uintptr_t>(ld) * sizeof(float);
+    if (a0 < b0 + bytes && b0 < a0 + bytes)
+      return reject(ASAP_ERR_ARG, "asap_mix_noalloc: W_in and W_out must not overlap");
+  }
 
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kNoAllocMaxDevices)

@@ -1,8 +1,9 @@
 """The library's minibatch index builder (host only, no GPU): the image that
 asap_load_shards uploads, decoded and checked against a plain restatement
-from the shards -- padded rows, list positions, the (column, row)-sorted
-copy of the entries, and the slab-major list of distinct (worker, column)
-pairs with its padded slab regions."""
+from the shards -- the (column, row)-sorted entries with their list
+positions, the margin segments' slots and the rows of their slots, the
+column-sum ranges cut at column boundaries, and the slab-major list of
+distinct (worker, column) pairs with its padded slab regions."""
 import numpy as np
 import pytest
 
@@ -16,13 +17,15 @@ def _view(img, off, dtype, n):
     return np.frombuffer(img[off:off + np.dtype(dtype).itemsize * n].tobytes(), dtype=dtype)
 
 
-@pytest.mark.parametrize("S", [64, 1024])
-def test_batch_image_matches_the_shards(S):
+@pytest.mark.parametrize("S,Q,max_len", [(64, 1, 40), (1024, 3, 40), (64, 8, 400)])
+def test_batch_image_matches_the_shards(S, Q, max_len):
+    # max_len 400 with B = 20 rows: about 3,400 entries, so minibatches span
+    # more than one 1024-entry margin segment
     N, d, B, t = 3, 1000, 20, 1
     rng = np.random.default_rng(8)
-    lengths = [np.where(rng.random(3 * B) < 0.15, 0, rng.integers(1, 40, 3 * B)) for _ in range(N)]
+    lengths = [np.where(rng.random(3 * B) < 0.15, 0, rng.integers(1, max_len, 3 * B)) for _ in range(N)]
     sh = inputs.sparse_custom(seed=31, N=N, d=d, rows=3 * B, lengths=lengths, hot_col=7)
-    img, desc, (list_off, soff_off, list_len) = debug_batch_image(sh, B, S, t)
+    img, desc, (list_off, soff_off, list_len) = debug_batch_image(sh, B, S, t, ctas_per_worker=Q)
     n_slabs = -(-((d + 63) // 64 * 64) // S)
     lst = _view(img, list_off, np.uint32, list_len)
     soff = _view(img, soff_off, np.int32, n_slabs + 1)
@@ -30,35 +33,45 @@ def test_batch_image_matches_the_shards(S):
 
     pairs = set()
     for i in range(N):
-        rp_o, y_o, pw_o, val_o, cp_o, cv_o, cr_o, nnz_pad, nnz = (int(v) for v in desc[i])
-        rp = _view(img, rp_o, np.int32, B + 1)
-        pw = _view(img, pw_o, np.int32, nnz_pad)
-        vals = _view(img, val_o, np.float32, nnz_pad)
+        y_o, cp_o, cv_o, cr_o, cs_o, sr_o, bd_o, nnz = (int(v) for v in desc[i])
         r0 = t * B
-        entries = []                                   # (col, row, val, padded index)
+        entries = []                                   # (col, row, val)
         for b in range(B):
             a, e = sh.rowptr[i][r0 + b], sh.rowptr[i][r0 + b + 1]
-            n = e - a
-            assert rp[b + 1] - rp[b] == -(-n // 4) * 4 and rp[b] % 4 == 0
-            for j in range(n):
+            for j in range(e - a):
                 c = int(sh.col[i][a + j])
-                q = rp[b] + j
-                assert vals[q] == sh.val[i][a + j]
-                p = int(pw[q])
-                assert lst[p] == (i << 16) | (c % S) and soff[c // S] <= p < soff[c // S + 1]
-                entries.append((c, b, sh.val[i][a + j], q))
+                entries.append((c, b, sh.val[i][a + j]))
                 pairs.add((i, c))
-            assert np.all(vals[rp[b] + n:rp[b + 1]] == 0)
-        assert rp[B] == nnz_pad and len(entries) == nnz
+        assert len(entries) == nnz
         assert np.array_equal(_view(img, y_o, np.float32, B), sh.y[i][r0:r0 + B])
-        # the (column, row)-sorted copy
+        # the (column, row)-sorted entries: value, row, and the list position
+        # of the entry's (worker, column) pair
         entries.sort(key=lambda x: (x[0], x[1]))
         cp = _view(img, cp_o, np.int32, nnz)
         cv = _view(img, cv_o, np.float32, nnz)
         cr = _view(img, cr_o, np.uint16, nnz)
         assert np.array_equal(cr, [x[1] for x in entries])
         assert np.array_equal(cv, np.array([x[2] for x in entries], np.float32))
-        assert np.array_equal(cp, [pw[x[3]] for x in entries])
+        for e, (c, _, _) in enumerate(entries):
+            p = int(cp[e])
+            assert lst[p] == (i << 16) | (c % S) and soff[c // S] <= p < soff[c // S + 1]
+        # margin segments of 1024 entries: slots numbered row by row, by
+        # column within a row; srow holds the row of every slot
+        cs = _view(img, cs_o, np.uint16, nnz)
+        sr = _view(img, sr_o, np.uint16, nnz)
+        for e0 in range(0, nnz, 1024):
+            e1 = min(e0 + 1024, nnz)
+            seg = sorted(range(e0, e1), key=lambda e: (entries[e][1], entries[e][0]))
+            assert [int(cs[e]) for e in seg] == list(range(e1 - e0))
+            assert [int(v) for v in sr[e0:e1]] == [entries[e][1] for e in seg]
+        # column-sum ranges: cut at the first column boundary at or after q nnz / Q
+        bd = _view(img, bd_o, np.int32, Q + 1)
+        assert bd[0] == 0 and bd[Q] == nnz and np.all(np.diff(bd) >= 0)
+        for q in range(1, Q):
+            e = int(bd[q])
+            assert e >= q * nnz // Q
+            assert e == 0 or e == nnz or entries[e][0] != entries[e - 1][0]
+            assert all(entries[x][0] == entries[x - 1][0] for x in range(max(q * nnz // Q, 1), e))
 
     # every slab region: the distinct (worker, column) pairs of its columns,
     # by worker then column, padded at the end

@@ -16,9 +16,9 @@ import numpy as np
 
 def stochastic_reduce(H, nbr, wgt):
     """W[i] = sum_m wgt[i, m] * H[nbr[i, m]], summed in ascending-neighbour
-    order, fp64."""
+    order, fp64; one output row per row of nbr."""
     H = np.asarray(H, dtype=np.float64)
-    W = np.zeros_like(H)
+    W = np.zeros((nbr.shape[0], H.shape[1]))
     for i in range(nbr.shape[0]):
         for m in range(nbr.shape[1]):
             W[i] += float(wgt[i, m]) * H[int(nbr[i, m])]

@@ -70,6 +70,8 @@ def parse():
     ap.add_argument("--workload", default="sparse_logistic_hashed", choices=sorted(WORKLOADS) + ["mix_sweep"],
                     help="mix_sweep: the stochastic reduce alone over N x d x k, one JSON line each")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--sync-mode", default="bsp", choices=["bsp", "notify_ack"],
+                    help="how the reduce meets the local step (sparse models)")
     ap.add_argument("--sweep-only", default="", help="mix_sweep subset: 'N,d,k;N,d,k' (k may be N-1)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--local-steps", type=int, default=1, help="minibatch steps per worker per round (sparse)")
@@ -384,6 +386,7 @@ def config(rows):
          "loss": w["loss"], "lr": w["lr"],
          "graph": "%s k=%d%s" % (w["graph"], w["k"], ", regenerated every round" if w["regenerate"] else ""),
          "parallelism": "independent replicas, one per GPU",
+         "sync": SCHED.get("sync", "bsp"),
          "local_steps": SCHED["tau"], "lr_schedule": SCHED["kind"] if SCHED["kind"] == "constant"
          else "lr / (1 + %g k)" % SCHED["gamma"]}
     if "nnz" in w:
@@ -498,6 +501,8 @@ def run_asap(args):
     ctx.set_schedule(local_steps=SCHED["tau"], lr_schedule=SCHED["kind"], gamma=SCHED["gamma"])
     ctx.set_graph(w["graph"], regenerate=w["regenerate"])
     ctx.set_stream(stream)
+    if not dense:
+        ctx.set_sync_mode(args.sync_mode)
     N, B, K, Wm = w["N"], w["B"], args.steps, args.warmup
     units_per_step = N * B * SCHED["tau"]
 
@@ -696,7 +701,8 @@ def main():
         run_mix_sweep(args)
         return
     WORKLOAD = WORKLOADS[args.workload]
-    SCHED.update(tau=args.local_steps, kind=args.lr_schedule, gamma=args.gamma)
+    SCHED.update(tau=args.local_steps, kind=args.lr_schedule, gamma=args.gamma,
+                 sync=args.sync_mode if WORKLOAD["loss"] != "softmax" else "bsp")
     if WORKLOAD["loss"] == "softmax" and args.local_steps != 1:
         raise SystemExit("dense_softmax takes one local step per round")
     if args.impl == "reference":

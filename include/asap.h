@@ -229,6 +229,42 @@ asap_status asap_read_counters(asap_ctx* ctx, uint64_t* reduces, uint64_t* consi
  * N*(k+1) float (either may be NULL).  Host only. */
 asap_status asap_get_graph(asap_ctx* ctx, int64_t round, int32_t* nbr_out, float* wgt_out);
 
+/* How a sparse model's stochastic reduce meets its local step (Section 4
+ * contrasts the three; Section 6.2 measures them).
+ *   BSP        (default) the reduce starts when the whole local step has
+ *              finished: the kernel boundary is the barrier.
+ *   NOTIFY_ACK the reduce is launched while the local step runs; it streams
+ *              W at once and copies a column slab's updates only after the
+ *              NOTIFY for the round of every worker with updates in the slab
+ *              (time-limited waits), so a slab waits only for those workers.
+ *              Results are identical to BSP.
+ *   ASYNC      for measurement only: as NOTIFY_ACK without the waits; an
+ *              update read before its worker's NOTIFY is stale, so results
+ *              depend on the schedule (asap_read_consistency counts how
+ *              many inputs were current).
+ * Dense (softmax) models always use BSP.  Not while a local step is
+ * pending. */
+typedef enum {
+  ASAP_SYNC_BSP = 0,
+  ASAP_SYNC_NOTIFY_ACK = 1,
+  ASAP_SYNC_ASYNC = 2
+} asap_sync_mode;
+asap_status asap_set_sync_mode(asap_ctx* ctx, asap_sync_mode mode);
+
+/* The order in which the local step's CTA clusters take the workers:
+ * cluster q runs worker order[q] (a permutation of [0, N); NULL restores
+ * the identity).  The schedule changes, the arithmetic does not: results
+ * are bit-identical, which the tests check.  Not while a local step is
+ * pending. */
+asap_status asap_set_worker_order(asap_ctx* ctx, const int32_t* order);
+
+/* Consistency of the gated (NOTIFY_ACK, ASYNC) reduces since creation: the
+ * inputs they read -- one per (column slab, worker) block of updates -- and
+ * how many of those were current, i.e. read after the worker's NOTIFY for
+ * the round (the analogue of Section 6.2's consistent reduces, Fig. 9).
+ * NOTIFY_ACK makes every input current.  Syncing. */
+asap_status asap_read_consistency(asap_ctx* ctx, uint64_t* inputs_read, uint64_t* inputs_current);
+
 /* Limit for every device-side NOTIFY/ACK wait, in nanoseconds (default
  * 200 ms).  A wait that runs out sets ASAP_ERR_TIMEOUT and the kernel
  * returns without writing the round's output. */

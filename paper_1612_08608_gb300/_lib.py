@@ -39,6 +39,9 @@ SIGNATURES = {
     "asap_read_counters": (C.c_int, [_P, C.POINTER(C.c_uint64), C.POINTER(C.c_uint64), C.POINTER(C.c_uint64)]),
     "asap_get_graph": (C.c_int, [_P, C.c_int64, _P, _P]),
     "asap_set_wait_limit_ns": (C.c_int, [_P, C.c_uint64]),
+    "asap_set_sync_mode": (C.c_int, [_P, C.c_int]),
+    "asap_set_worker_order": (C.c_int, [_P, _P]),
+    "asap_read_consistency": (C.c_int, [_P, C.POINTER(C.c_uint64), C.POINTER(C.c_uint64)]),
     "asap_debug_skip_notify": (C.c_int, [_P, C.c_int]),
     "asap_set_kernel_timing": (C.c_int, [_P, C.c_int]),
     "asap_read_kernel_times": (C.c_int, [_P, _P, _P]),

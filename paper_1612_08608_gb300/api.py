@@ -15,6 +15,7 @@ GRAPH = {"ring": 1, "root": 2, "random_regular": 3, "complete": 4, "explicit": 5
 LOSS = {"none": 0, "hinge": 1, "logistic": 2, "softmax": 3}
 RESIDENCY = {"device": 0, "host": 1}
 LR_SCHEDULE = {"constant": 0, "inverse": 1}
+SYNC = {"bsp": 0, "notify_ack": 1, "async": 2}
 
 
 class AsapError(RuntimeError):
@@ -194,6 +195,24 @@ class Context:
         wgt = np.empty((self.N, self.k + 1), dtype=np.float32)
         self._c(self._lib.asap_get_graph(self._h, rnd, _ptr(nbr), _ptr(wgt)))
         return nbr, wgt
+
+    def set_sync_mode(self, mode: str):
+        """``bsp``, ``notify_ack`` or ``async`` (measurement only)."""
+        self._c(self._lib.asap_set_sync_mode(self._h, SYNC[mode]))
+
+    def set_worker_order(self, order=None):
+        """Cluster q of the local step runs worker order[q] (None: identity)."""
+        if order is None:
+            self._c(self._lib.asap_set_worker_order(self._h, None))
+            return
+        order = np.ascontiguousarray(order, dtype=np.int32)
+        self._c(self._lib.asap_set_worker_order(self._h, _ptr(order)))
+
+    def read_consistency(self):
+        """{inputs_read, inputs_current} of the gated reduces since creation."""
+        a, b = C.c_uint64(), C.c_uint64()
+        self._c(self._lib.asap_read_consistency(self._h, C.byref(a), C.byref(b)))
+        return {"inputs_read": a.value, "inputs_current": b.value}
 
     def set_wait_limit_ns(self, ns: int):
         self._c(self._lib.asap_set_wait_limit_ns(self._h, ns))

@@ -112,7 +112,8 @@ struct asap_ctx {
   std::vector<int64_t> list_len;
   int max_region = 0;               // entries of the largest slab region of any list
   int64_t max_list = 0;
-  float* wv = nullptr;              // w at the current round's list positions
+  float* wv[2] = {nullptr, nullptr};  // w at the list positions of round t's steps: wv[t & 1] (the
+                                    // reduce of round t writes wv[(t+1) & 1] while round t's step may run)
   float* gsum = nullptr;            // column sums at the current round's list positions
   int64_t wv_step = -1;             // global local step whose column list wv holds (-1: none)
   // host residency: a round reads its own block and the next one
@@ -167,6 +168,7 @@ struct asap_ctx {
   bool graph_uniform = false;       // every weight of the staged table is equal
   bool step_pending = false;
   int skip_notify = -1;
+  int sync_mode = kSyncBsp;         // how a sparse reduce meets its local step (asap_set_sync_mode)
   unsigned long long wait_ns = 200000000ull;
   uint64_t launches = 0;
   std::string err;
@@ -210,7 +212,8 @@ void free_shards(asap_ctx* c) {
   dfree(c->X);
   dfree(c->XT);
   dfree(c->Yd);
-  dfree(c->wv);
+  dfree(c->wv[0]);
+  dfree(c->wv[1]);
   dfree(c->gsum);
   dfree(c->mpart_big);
   dfree(c->r_big);
@@ -1123,9 +1126,11 @@ asap_status asap_load_shards(asap_ctx* c, const int64_t* const* rowptr, const in
     CU(cudaMemcpy(c->d_desc, desc.data(), desc.size() * sizeof(BatchDesc), cudaMemcpyHostToDevice),
        "copying batch descriptors");
     const size_t lb = 4 * static_cast<size_t>(std::max<int64_t>(max_list, 4));
-    CU(cudaMalloc(&c->wv, lb), "allocating the list value buffer");
+    CU(cudaMalloc(&c->wv[0], lb), "allocating the list value buffer");
+    CU(cudaMalloc(&c->wv[1], lb), "allocating the list value buffer");
     CU(cudaMalloc(&c->gsum, lb), "allocating the column-sum buffer");
-    CU(cudaMemset(c->wv, 0, lb), "zeroing the list value buffer");
+    CU(cudaMemset(c->wv[0], 0, lb), "zeroing the list value buffer");
+    CU(cudaMemset(c->wv[1], 0, lb), "zeroing the list value buffer");
     CU(cudaMemset(c->gsum, 0, lb), "zeroing the column-sum buffer");
     if (B > kRSmemRows) {
       CU(cudaMalloc(&c->mpart_big, 4 * static_cast<size_t>(N) * Q * B), "allocating the partial margins");
@@ -1277,7 +1282,7 @@ asap_status asap_local_step(asap_ctx* c) {
       // the host, or an earlier local step of the round changed them): gather.
       time_begin(c, ASAP_KERNEL_GATHER);
       CU(launch_gather_wv(c->W[r & 1], c->ld, reinterpret_cast<const uint32_t*>(block + c->list_off[tk]),
-                          reinterpret_cast<const int*>(block + c->soff_off[tk]), c->n_slabs, c->S, c->wv,
+                          reinterpret_cast<const int*>(block + c->soff_off[tk]), c->n_slabs, c->S, c->wv[r & 1],
                           c->sm_count, c->stream),
          "launching the gather kernel");
       time_end(c);
@@ -1287,7 +1292,7 @@ asap_status asap_local_step(asap_ctx* c) {
     LocalStepArgs a;
     a.block = block;
     a.desc = c->d_desc + static_cast<size_t>(tk) * c->N;
-    a.wv = c->wv;
+    a.wv = c->wv[r & 1];
     a.gsum = c->gsum;
     a.mpart_big = c->mpart_big;
     a.r_big = c->r_big;
@@ -1387,7 +1392,7 @@ asap_status asap_stochastic_reduce(asap_ctx* c) {
     a.upd_scale = c->pend_upd;
     a.exp_list = reinterpret_cast<const uint32_t*>(bn + c->list_off[tn]);
     a.exp_off = reinterpret_cast<const int*>(bn + c->soff_off[tn]);
-    a.wv_out = c->wv;
+    a.wv_out = c->wv[(r + 1) & 1];
     a.max_region = c->max_region;
   }
   a.cons_part = c->cons_part;
@@ -1404,6 +1409,7 @@ asap_status asap_stochastic_reduce(asap_ctx* c) {
   a.round = static_cast<unsigned>(r);
   a.expect_notify = c->step_pending ? 1 : 0;
   a.wait_ns = c->wait_ns;
+  a.sync_mode = fused ? c->sync_mode : kSyncBsp;
   time_begin(c, ASAP_KERNEL_REDUCE);
   CU(launch_mix(c->tmap[r & 1], a, is_complete_kernel(c), fused, c->mix_grid, c->mix_smem, c->stream),
      "launching the stochastic reduce");
@@ -1553,6 +1559,45 @@ asap_status asap_get_graph(asap_ctx* c, int64_t round, int32_t* nbr_out, float* 
   if (s != ASAP_OK) return s;
   if (nbr_out) std::copy(nbr.begin(), nbr.end(), nbr_out);
   if (wgt_out) std::copy(wgt.begin(), wgt.end(), wgt_out);
+  return ASAP_OK;
+}
+
+asap_status asap_set_sync_mode(asap_ctx* c, asap_sync_mode mode) {
+  if (!c) return fail(nullptr, ASAP_ERR_ARG, "ctx is NULL");
+  if (mode != ASAP_SYNC_BSP && mode != ASAP_SYNC_NOTIFY_ACK && mode != ASAP_SYNC_ASYNC)
+    return fail(c, ASAP_ERR_ARG, "unknown synchronisation mode");
+  if (c->step_pending) return fail(c, ASAP_ERR_ARG, "a local step is pending: reduce first");
+  c->sync_mode = mode == ASAP_SYNC_NOTIFY_ACK ? kSyncNotifyAck : mode == ASAP_SYNC_ASYNC ? kSyncAsync : kSyncBsp;
+  return ASAP_OK;
+}
+
+asap_status asap_set_worker_order(asap_ctx* c, const int32_t* order) {
+  if (!c) return fail(nullptr, ASAP_ERR_ARG, "ctx is NULL");
+  if (c->step_pending) return fail(c, ASAP_ERR_ARG, "a local step is pending: reduce first");
+  if (!order) {
+    c->permuted = false;
+    return ASAP_OK;
+  }
+  std::vector<int> seen(c->N, 0);
+  bool identity = true;
+  for (int q = 0; q < c->N; ++q) {
+    if (order[q] < 0 || order[q] >= c->N || seen[order[q]]++) return fail(c, ASAP_ERR_ARG, "not a permutation of [0, N)");
+    identity = identity && order[q] == q;
+  }
+  asap_status s0 = asap_sync(c);
+  if (s0 != ASAP_OK) return s0;
+  CU(cudaMemcpy(c->d_worker_of, order, 4 * static_cast<size_t>(c->N), cudaMemcpyHostToDevice), "uploading the worker order");
+  c->permuted = !identity;
+  return ASAP_OK;
+}
+
+asap_status asap_read_consistency(asap_ctx* c, uint64_t* inputs_read, uint64_t* inputs_current) {
+  if (!c) return fail(nullptr, ASAP_ERR_ARG, "ctx is NULL");
+  CU(cudaStreamSynchronize(c->stream), "synchronising");
+  DevState h;
+  CU(cudaMemcpy(&h, c->st, sizeof h, cudaMemcpyDeviceToHost), "reading counters");
+  if (inputs_read) *inputs_read = h.inputs_read;
+  if (inputs_current) *inputs_current = h.inputs_current;
   return ASAP_OK;
 }
 

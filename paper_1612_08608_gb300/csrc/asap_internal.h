@@ -34,7 +34,21 @@ struct DevState {
   unsigned long long reduces;
   unsigned long long consistent_inputs;
   unsigned long long timeouts;
+  unsigned long long inputs_read;        // (slab, worker) update blocks read by gated reduces
+  unsigned long long inputs_current;     // ... whose worker had published NOTIFY for the round
 };
+
+// How the stochastic reduce of a sparse model meets its local step.
+//   BSP        the reduce starts when the whole local-step grid has finished
+//              (the kernel boundary is the barrier)
+//   NOTIFY_ACK the reduce is launched while the local step runs; it streams
+//              W at once and copies a slab's column sums only after the
+//              NOTIFY of every worker with updates in the slab (time-limited)
+//   ASYNC      measurement only: as NOTIFY_ACK but without the waits; a
+//              block of updates copied before its worker's NOTIFY is stale
+constexpr int kSyncBsp = 0;
+constexpr int kSyncNotifyAck = 1;
+constexpr int kSyncAsync = 2;
 
 constexpr uint32_t kListPad = 0xffffffffu;   // padding entry of a column list
 
@@ -128,6 +142,7 @@ struct MixArgs {
   unsigned int round;
   int expect_notify;
   unsigned long long wait_ns;
+  int sync_mode;               // kSync* (FUSED reduces; others are BSP)
 };
 
 // Arguments of the dense softmax-regression step (kernels_dense.cu).

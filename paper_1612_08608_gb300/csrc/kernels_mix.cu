@@ -222,6 +222,7 @@ struct MixSmem {
   float* wgt;
   double* dscratch;
   int* flags;        // [0]: fail, [1]: last
+  unsigned* seen;    // [32]: bitmap of workers whose NOTIFY this CTA has seen (gated reduces)
 };
 
 // Shared-memory layout; every region starts 16-byte aligned (the slab
@@ -243,6 +244,8 @@ __device__ __forceinline__ MixSmem carve(unsigned char* raw, const MixArgs& a, i
   base = a16(base + 8 * (kMixThreads / 32));
   m.flags = reinterpret_cast<int*>(base);
   base = a16(base + 16);
+  m.seen = reinterpret_cast<unsigned*>(base);
+  base = a16(base + 4 * 32);
   m.info = reinterpret_cast<int*>(base);
   base = a16(base + 16 * a.stages);
   m.part = reinterpret_cast<float4*>(base);
@@ -273,15 +276,19 @@ __global__ void __launch_bounds__(kMixThreads, 1) k_mix(const __grid_constant__ 
   const size_t list_bytes = (static_cast<size_t>(a.max_region) * 4 + 15) & ~static_cast<size_t>(15);
 
   if (tid == 0) { sm.flags[0] = 0; sm.flags[1] = 0; }
+  if (tid < 32) sm.seen[tid] = 0u;
   __syncthreads();
-  // Programmatic dependent launch: the local step's kernels may still be
-  // running; everything below reads what they wrote.
-  asm volatile("griddepcontrol.wait;" ::: "memory");
+  // A gated reduce (NOTIFY_ACK or ASYNC, sparse models) runs while the local
+  // step may still be running: it reads the column sums of worker j only
+  // after j's NOTIFY (or, ASYNC, counts the read as stale).  Otherwise
+  // (BSP) it starts once the local step's grid has finished.
+  const bool gated = FUSED && a.sync_mode != kSyncBsp;
+  if (!gated) asm volatile("griddepcontrol.wait;" ::: "memory");
 
   // ---- NOTIFY / ACK checks (time-limited waits) ----
   for (int j = tid; j < a.N; j += kMixThreads) {
     unsigned e = 0;
-    if (a.expect_notify) e = wait_flag(a.ready + j, a.round + 1u, true, a.wait_ns);
+    if (a.expect_notify && !gated) e = wait_flag(a.ready + j, a.round + 1u, true, a.wait_ns);
     if (!e) e = wait_flag(a.consumed + j, a.round, false, a.wait_ns);
     if (e) {
       record_error(a.st, e, j, a.round);
@@ -319,6 +326,8 @@ __global__ void __launch_bounds__(kMixThreads, 1) k_mix(const __grid_constant__ 
       // ================= producer warp =================
       float term = 0.f;
       const float inv_n_term = 1.0f / static_cast<float>(a.N);
+      unsigned long long n_read = 0, n_current = 0;   // gated: (slab, worker) inputs, and those current
+      int n_seen = 0;                                 // gated: workers whose NOTIFY this CTA has seen
       // List offsets of the next 32 slabs, one slab per lane, loaded ahead so
       // that issuing a stage never waits on a global load.
       int4 offs = make_int4(0, 0, 0, 0);
@@ -359,6 +368,57 @@ __global__ void __launch_bounds__(kMixThreads, 1) k_mix(const __grid_constant__ 
           }
           __syncwarp();
         }
+        if (FUSED && gated && it < n_my) {
+          // The slab's updates come from workers w0 .. w1 (a region is sorted
+          // by worker): their NOTIFY for the round before the slab's column
+          // sums are copied (NOTIFY_ACK, time-limited waits), or just noted
+          // (ASYNC).  The warp checks 32 workers at a time; a worker seen
+          // once stays seen for the rest of the launch.
+          const int nu = o.y - o.x;
+          if (n_seen == a.N) {
+            n_read += static_cast<unsigned long long>(a.N);
+            n_current += static_cast<unsigned long long>(a.N);
+          } else if (nu > 0) {
+            const unsigned w0 = __ldg(a.upd_list + o.x) >> 16;
+            unsigned w1 = w0;
+            for (int e = nu - 1; e >= 0 && e >= nu - 4; --e) {
+              const uint32_t c = __ldg(a.upd_list + o.x + e);
+              if (c != kListPad) { w1 = c >> 16; break; }
+            }
+            bool acquired = false;
+            for (unsigned j0 = w0; j0 <= w1 && j0 < static_cast<unsigned>(a.N); j0 += 32) {
+              const unsigned j = j0 + lane;
+              const bool in = j <= w1 && j < static_cast<unsigned>(a.N);
+              const unsigned bit = 1u << (j & 31u);
+              bool cur = in && (sm.seen[j >> 5] & bit) != 0;
+              bool fresh = false;
+              if (in && !cur && !failed) {
+                if (a.sync_mode == kSyncNotifyAck) {
+                  const unsigned er = wait_flag(a.ready + j, a.round + 1u, true, a.wait_ns);
+                  if (er) {
+                    record_error(a.st, er, j, a.round);
+                    if (er == ASAP_ERR_TIMEOUT) atomicAdd(&a.st->timeouts, 1ull);
+                    failed = true;
+                  } else {
+                    fresh = true;
+                  }
+                } else {
+                  fresh = ld_acquire_u32(a.ready + j) == a.round + 1u;
+                }
+                if (fresh) atomicOr(sm.seen + (j >> 5), bit);
+                cur = fresh;
+              }
+              n_seen += __popc(__ballot_sync(kFull, fresh));
+              acquired = acquired || __any_sync(kFull, fresh);
+              n_read += __popc(__ballot_sync(kFull, in));
+              n_current += __popc(__ballot_sync(kFull, in && cur));
+            }
+            failed = __any_sync(kFull, failed);
+            __syncwarp();
+            // newly acquired column sums, to the bulk copy's async proxy
+            if (acquired && lane == 0) asm volatile("fence.proxy.async.global;" ::: "memory");
+          }
+        }
         if (it < n_my && lane == 0) {
           const long long slab = blockIdx.x + it * stride;
           const int st = static_cast<int>(it % a.stages);
@@ -376,6 +436,7 @@ __global__ void __launch_bounds__(kMixThreads, 1) k_mix(const __grid_constant__ 
           info[0] = n_upd;
           info[1] = n_exp;
           info[2] = x0;
+          info[3] = u0;
           mbar_expect_tx(sm.full + st, bytes);
           // Slab layout in shared memory: [column box][row][QB quads].
           for (int xb = 0; xb < nq / QB; ++xb)
@@ -393,6 +454,10 @@ __global__ void __launch_bounds__(kMixThreads, 1) k_mix(const __grid_constant__ 
         __syncwarp();
       }
       s2 = -term;
+      if (gated && lane == 0 && n_read) {
+        atomicAdd(&a.st->inputs_read, n_read);
+        atomicAdd(&a.st->inputs_current, n_current);
+      }
     } else if (warp >= kUpdater0) {
       // ================= updater warps (FUSED) =================
       // Once a slab has landed, apply w -= eta/B (1 - eta l2)^-1 g to it and
@@ -592,10 +657,23 @@ __global__ void __launch_bounds__(kMixThreads, 1) k_mix(const __grid_constant__ 
   if (!sm.flags[1]) return;
   __threadfence();
   const unsigned ticket = atomicAdd(&a.st->mix_ticket, 0u);
-  const bool any_fail = (ticket >> 16) != 0;
+  bool any_fail = (ticket >> 16) != 0;
   double v = 0.0;
   for (int b = tid; b < static_cast<int>(gridDim.x); b += kMixThreads) v += __ldcg(a.cons_part + b);
   const double ctot = block_sum_f64(v, sm.dscratch);
+  if (gated && a.sync_mode == kSyncNotifyAck && !any_fail) {
+    // The loss partials of workers without any update in this launch's
+    // slabs: every worker's NOTIFY before they are read.
+    for (int j = tid; j < a.N; j += kMixThreads) {
+      const unsigned er = wait_flag(a.ready + j, a.round + 1u, true, a.wait_ns);
+      if (er) {
+        record_error(a.st, er, j, a.round);
+        atomicOr(&sm.flags[0], 2);
+      }
+    }
+    __syncthreads();
+    any_fail = (sm.flags[0] & 2) != 0;
+  }
   double lv = 0.0;
   if (a.have_loss)
     for (int b = tid; b < a.n_loss_part; b += kMixThreads) lv += static_cast<double>(__ldcg(a.loss_part + b));
@@ -694,6 +772,7 @@ size_t mix_smem_bytes(int N, int kp1, int S, int rows_pad, int stages, int max_r
   b = a16(b + 24 * static_cast<size_t>(stages));                         // full / empty / ready
   b = a16(b + 8 * (kMixThreads / 32));                                    // fp64 block scratch
   b = a16(b + 16);                                                        // flags
+  b = a16(b + 4 * 32);                                                    // NOTIFY bitmap
   b = a16(b + 16 * static_cast<size_t>(stages));                          // stage info
   b = a16(b + 16 * static_cast<size_t>(stages) * kMixComputeWarps * 32);  // partial sums
   b = a16(b + 4 * static_cast<size_t>(N) * kp1);                          // neighbour offsets

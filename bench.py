@@ -57,6 +57,7 @@ SCHED = {"tau": 1, "kind": "constant", "gamma": 0.0}   # local steps per round, 
 TRAFFIC = {
     ("sparse_logistic_hashed", "reduce"): ("stochastic_reduce_sparse_logistic_hashed.txt", "kernels_mix.cu"),
     ("dense_softmax", "dense_grad"): ("dense_gemms_dense_softmax.txt", "kernels_dense.cu"),
+    ("sparse_logistic_hashed", "local_step"): ("local_step_sparse_logistic_hashed.txt", "kernels_sparse.cu"),
 }
 
 
@@ -67,12 +68,18 @@ def parse():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", default="asap", choices=["asap", "reference"])
     ap.add_argument("--rows", type=int, default=None, help="rows per worker (default: the workload's)")
-    ap.add_argument("--workload", default="sparse_logistic_hashed", choices=sorted(WORKLOADS) + ["mix_sweep"],
+    ap.add_argument("--workload", default="sparse_logistic_hashed", choices=sorted(WORKLOADS) + ["mix_sweep", "graph_study"],
                     help="mix_sweep: the stochastic reduce alone over N x d x k, one JSON line each")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--min-time", type=float, default=1.0,
+                    help="repeat the timed K rounds until this many seconds (at least 3 repeats)")
     ap.add_argument("--sync-mode", default="bsp", choices=["bsp", "notify_ack"],
                     help="how the reduce meets the local step (sparse models)")
     ap.add_argument("--sweep-only", default="", help="mix_sweep subset: 'N,d,k;N,d,k' (k may be N-1)")
+    ap.add_argument("--study-rounds", type=int, default=1000, help="graph_study: rounds per graph")
+    ap.add_argument("--study-seeds", type=int, default=3, help="graph_study: data and graph seeds")
+    ap.add_argument("--study-lr", type=float, default=2.0, help="graph_study: learning rate")
+    ap.add_argument("--label-skew", type=float, default=0.8, help="graph_study: label heterogeneity of the shards")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--local-steps", type=int, default=1, help="minibatch steps per worker per round (sparse)")
     ap.add_argument("--lr-schedule", default="constant", choices=["constant", "inverse"])
@@ -527,7 +534,7 @@ def run_asap(args):
             # error are read back while round s + 1 runs (the read waits for
             # round s only); the last one after the loop, inside the timed
             # region.
-            while len(reps) < 3 or (sum(reps) < 1.0 and len(reps) < 5000):
+            while len(reps) < 3 or (sum(reps) < args.min_time and len(reps) < 5000):
                 h2d = 0
                 barrier()
                 t0 = time.perf_counter()
@@ -565,7 +572,7 @@ def run_asap(args):
     l0 = ctx.kernel_launches()
     rep_ms = []
     t_wall = time.perf_counter()
-    while len(rep_ms) < 3 or (sum(rep_ms) < 1000.0 and len(rep_ms) < 5000):
+    while len(rep_ms) < 3 or (sum(rep_ms) < 1000.0 * args.min_time and len(rep_ms) < 5000):
         barrier()
         start.record(stream)
         for s in range(K):
@@ -622,7 +629,8 @@ def run_asap(args):
             "timing": {"repeats": len(rep_ms), "rounds_per_repeat": K, "timed_s": sum(rep_ms) / 1e3,
                        "wall_s": t_wall, "repeat_ms_min_median_max": [min(rep_ms), statistics.median(rep_ms),
                                                                       max(rep_ms)],
-                       "rule": "median of repeats of exactly --steps rounds, repeated until >= 1 s and >= 3"}}
+                       "rule": "median of repeats of exactly --steps rounds, repeated until >= %g s and >= 3"
+                               % args.min_time}}
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(sh)
         par = cpu_baseline_all_cores(sh)
@@ -645,7 +653,6 @@ def run_mix_sweep(args):
     consensus in one round."""
     import numpy as np
     import torch
-    from oracle import graphs
     from paper_1612_08608_gb300 import Context, inputs
 
     torch.cuda.set_device(0)
@@ -677,7 +684,7 @@ def run_mix_sweep(args):
                 rounds = args.warmup + args.steps
                 _, cons = ctx.read_metrics(0, rounds)
                 nbr, wgt = ctx.get_graph(0)
-                s2 = 1.0 - graphs.spectral_gap(graphs.mixing_matrix(nbr, wgt))
+                s2 = sigma2(nbr, wgt)
                 ok = bool(np.all(np.isfinite(cons)))
                 for t in range(1, rounds):
                     if cons[t - 1] > 1e-5 * cons[0]:
@@ -694,11 +701,117 @@ def run_mix_sweep(args):
                 ctx.close()
 
 
+# ---- graph comparison (Section 6.1): rounds and bytes to a target loss ----
+STUDY_GRAPHS = (("complete", "complete", None, False), ("root", "root", 2, False), ("ring", "ring", 1, False),
+                ("random_regular_k2", "random_regular", 2, False),
+                ("random_regular_k4_regen", "random_regular", 4, True))
+
+
+def hinge_loss_at(w, rowptr, col, val, y):
+    """Mean hinge loss max(0, 1 - y x.w) of a CSR set at w (evaluation)."""
+    import numpy as np
+    row_of = np.repeat(np.arange(rowptr.shape[0] - 1), np.diff(rowptr))
+    m = np.bincount(row_of, weights=val.astype(np.float64) * w[col], minlength=rowptr.shape[0] - 1)
+    return float(np.maximum(0.0, 1.0 - y.astype(np.float64) * m).mean())
+
+
+def study_target(f0, curve, frac=0.9):
+    """The loss at which a curve has made `frac` of its total drop from f0
+    to its lowest value."""
+    return f0 - frac * (f0 - min(curve))
+
+
+def first_reaching(rounds, curve, target):
+    """First round of `rounds` whose value is at or below target (None if none)."""
+    for r, v in zip(rounds, curve):
+        if v <= target:
+            return r
+    return None
+
+
+def sigma2(nbr, wgt):
+    """Second singular value of the mixing matrix written out from its rows."""
+    import numpy as np
+    N = nbr.shape[0]
+    P = np.zeros((N, N))
+    for i in range(N):
+        for m in range(nbr.shape[1]):
+            P[i, nbr[i, m]] += wgt[i, m]
+    return float(np.linalg.svd(P, compute_uv=False)[1]) if N > 1 else 0.0
+
+
+def run_graph_study(args):
+    """Every graph of STUDY_GRAPHS trains the same RCV1-shaped hinge SVM on
+    shards that are heterogeneous by label, from W = 0.  Every `every`
+    rounds the average model wbar is evaluated (mean hinge loss on 256
+    held-out rows of every worker).  The target is the loss at which the
+    complete graph (the all-reduce) has made 90 % of its drop over
+    --study-rounds rounds; per graph and seed the rounds to that target, the
+    bytes each worker receives to reach it (k d 4 per round), sigma_2 of its
+    mixing matrix and the median per-round ratio of its consensus error."""
+    import numpy as np
+    import torch
+    from paper_1612_08608_gb300 import Context, inputs
+    torch.cuda.set_device(0)
+    N, B, every = 16, 256, 10
+    rows, T = args.rows or 4096, args.study_rounds
+    summary = {}
+    for seed in range(args.study_seeds):
+        sh = inputs.sparse_hinge_svm(seed=seed, N=N, rows=rows + 256, label_skew=args.label_skew)
+        train = inputs.SparseShards(d=sh.d)
+        ev_rp, ev_col, ev_val, ev_y = [np.zeros(1, np.int64)], [], [], []
+        for i in range(N):
+            rp = sh.rowptr[i]
+            train.rowptr.append(rp[:rows + 1].copy())
+            train.col.append(sh.col[i][:rp[rows]])
+            train.val.append(sh.val[i][:rp[rows]])
+            train.y.append(sh.y[i][:rows])
+            ev_rp.append(rp[rows + 1:] - rp[rows] + ev_rp[-1][-1])
+            ev_col.append(sh.col[i][rp[rows]:])
+            ev_val.append(sh.val[i][rp[rows]:])
+            ev_y.append(sh.y[i][rows:])
+        ev = (np.concatenate(ev_rp), np.concatenate(ev_col), np.concatenate(ev_val), np.concatenate(ev_y))
+        curves = {}
+        for name, kind, k, regen in STUDY_GRAPHS:
+            kk = N - 1 if k is None else k
+            ctx = Context(N, sh.d, graph_seed=seed, k=kk)
+            ctx.set_model("hinge", batch=B, lr=args.study_lr)
+            ctx.set_graph(kind, regenerate=regen)
+            ctx.load_shards(train)
+            xs, fs = [0], [hinge_loss_at(np.zeros(sh.d), *ev)]
+            for t in range(every, T + 1, every):
+                ctx.round(every)
+                W, _ = ctx.read_params()
+                xs.append(t)
+                fs.append(hinge_loss_at(W.astype(np.float64).mean(axis=0), *ev))
+            _, cons = ctx.read_metrics(0, T)
+            nbr, wgt = ctx.get_graph(0)
+            ratio = float(np.median(cons[1:] / np.maximum(cons[:-1], 1e-30)))
+            curves[name] = (kk, xs, fs, sigma2(nbr, wgt), ratio)
+            ctx.close()
+        target = study_target(curves["complete"][2][0], curves["complete"][2])
+        for name, (kk, xs, fs, s2, ratio) in curves.items():
+            hit = first_reaching(xs, fs, target)
+            line = {"workload": "graph_study", "seed": seed, "graph": name, "k": kk, "sigma2": s2,
+                    "spectral_gap": 1.0 - s2, "target_loss": target, "rounds_to_target": hit,
+                    "bytes_per_worker_round": kk * sh.d * 4,
+                    "bytes_per_worker_to_target": None if hit is None else kk * sh.d * 4 * hit,
+                    "final_loss": fs[-1], "median_consensus_ratio": ratio, "lr": args.study_lr,
+                    "label_skew": args.label_skew, "rounds": T}
+            print(json.dumps(line), flush=True)
+            summary.setdefault(name, []).append(hit)
+    print(json.dumps({"workload": "graph_study_summary",
+                      "rounds_to_target_per_seed": summary}), flush=True)
+
+
 def main():
     global WORKLOAD
     args = parse()
     if args.workload == "mix_sweep":
         run_mix_sweep(args)
+        return
+    if args.workload == "graph_study":
+        run_graph_study(args)
         return
     WORKLOAD = WORKLOADS[args.workload]
     SCHED.update(tau=args.local_steps, kind=args.lr_schedule, gamma=args.gamma,

@@ -168,10 +168,15 @@ def tiny_dense_logistic(seed: int = 0, N: int = 4, d: int = 64, rows: int = 256,
 # ---------------------------------------------------------------------------
 def sparse_hinge_svm(seed: int = 0, N: int = 16, d: int = 47236, rows: int = 20000,
                      mean_nnz: float = 75.0, sigma: float = 1.0, lo: int = 5, hi: int = 1000,
-                     zipf_a: float = 1.1, flip: float = 0.03) -> SparseShards:
+                     zipf_a: float = 1.1, flip: float = 0.03, label_skew: float = 0.0) -> SparseShards:
     """Lognormal row lengths with the given mean, Zipf(a) column popularity
     over ranks 1..d (column id = rank-1), tf-idf-like values
-    ``Exp(1) * ln(1 + d/(col+1))``, rows scaled to unit L2 norm."""
+    ``Exp(1) * ln(1 + d/(col+1))``, rows scaled to unit L2 norm.
+
+    ``label_skew`` in [0, 1) makes the shards heterogeneous by label: worker
+    i keeps a share 1/2 + label_skew (i/(N-1) - 1/2) of positive rows (drawn
+    from a pool of twice the rows), so that workers see different class
+    balances, as data split by source would."""
     ranks = np.arange(1, d + 1, dtype=np.float64)
     cdf = np.cumsum(ranks ** (-zipf_a))
     cdf /= cdf[-1]
@@ -179,8 +184,31 @@ def sparse_hinge_svm(seed: int = 0, N: int = 16, d: int = 47236, rows: int = 200
     mu = np.log(mean_nnz) - 0.5 * sigma * sigma
     out = SparseShards(d=d)
 
+    pool = rows if label_skew == 0.0 else 2 * rows
+
     def one(i):
-        lengths = np.rint(_rng(seed, _ROWLEN, i).lognormal(mu, sigma, rows)).astype(np.int64)
+        sh_i = _hinge_pool(i)
+        if label_skew == 0.0:
+            return sh_i
+        rowptr, col, val, y = sh_i
+        frac = 0.5 + label_skew * ((i / (N - 1) if N > 1 else 0.5) - 0.5)
+        pos, neg = np.nonzero(y > 0)[0], np.nonzero(y < 0)[0]
+        n_pos = min(int(round(frac * rows)), pos.shape[0])
+        n_neg = rows - n_pos
+        if n_neg > neg.shape[0]:
+            n_neg = neg.shape[0]
+            n_pos = rows - n_neg
+        srng = _rng(seed, _FLIPS + 100, i)
+        keep = np.concatenate([srng.choice(pos, n_pos, replace=False), srng.choice(neg, n_neg, replace=False)])
+        keep = keep[srng.permutation(keep.shape[0])]
+        lens = np.diff(rowptr)[keep]
+        rp = np.zeros(rows + 1, dtype=np.int64)
+        np.cumsum(lens, out=rp[1:])
+        idx = np.concatenate([np.arange(rowptr[r], rowptr[r + 1]) for r in keep]) if rows else np.zeros(0, np.int64)
+        return rp, col[idx], val[idx], y[keep]
+
+    def _hinge_pool(i):
+        lengths = np.rint(_rng(seed, _ROWLEN, i).lognormal(mu, sigma, pool)).astype(np.int64)
         lengths = np.clip(lengths, lo, min(hi, d))
         crng = _rng(seed, _COLS, i)
 
@@ -189,8 +217,8 @@ def sparse_hinge_svm(seed: int = 0, N: int = 16, d: int = 47236, rows: int = 200
 
         rowptr, col = _distinct_columns(crng, lengths, sample)
         raw = _rng(seed, _VALS, i).exponential(1.0, col.shape[0]) * np.log1p(d / (col.astype(np.float64) + 1.0))
-        row_of = np.repeat(np.arange(rows), lengths)
-        norms = np.sqrt(np.bincount(row_of, weights=raw * raw, minlength=rows))
+        row_of = np.repeat(np.arange(pool), lengths)
+        norms = np.sqrt(np.bincount(row_of, weights=raw * raw, minlength=pool))
         val = (raw / norms[row_of]).astype(np.float32)
         return rowptr, col, val, _labels_from_teacher(_row_scores(rowptr, col, val, wstar), flip,
                                                       _rng(seed, _FLIPS, i))

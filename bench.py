@@ -39,6 +39,8 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 METRIC = "worker-samples/s per SGD+reduce round; stochastic-reduce HBM GB/s vs peak"
+NOMINAL_HBM_GBS = 7900.0        # GB300 HBM3e, nominal (the bench's peak is the measured copy rate)
+NOMINAL_BF16_TFLOPS = 2250.0    # dense bf16, nominal
 WORKLOADS = {
     # hashed sparse logistic regression (the default, HBM-scale)
     "sparse_logistic_hashed": dict(name="sparse_logistic_hashed", N=64, d=1 << 20, rows=50000, nnz=100, B=512,
@@ -109,9 +111,10 @@ def code_fingerprint(path):
     return hashlib.sha256("\n".join(lines).encode()).hexdigest()[:16]
 
 
-def traffic_per_launch(workload, kernel):
-    """DRAM bytes per launch of the kernel from its committed ncu summary, or
-    None when there is none or the kernel source changed since it was taken."""
+def traffic_per_launch(workload, kernel, key="dram_bytes_per_launch"):
+    """DRAM bytes per launch of the kernel (or another `key` of the summary)
+    from its committed ncu summary, or None when there is none or the kernel
+    source changed since it was taken."""
     if (workload, kernel) not in TRAFFIC:
         return None
     prof, source = TRAFFIC[(workload, kernel)]
@@ -128,8 +131,8 @@ def traffic_per_launch(workload, kernel):
     if vals.get("kernel_code_sha256_16") != src:
         return None
     try:
-        return float(vals["dram_bytes_per_launch"])
-    except (KeyError, ValueError):
+        return float(vals[key].split()[0])
+    except (KeyError, ValueError, IndexError):
         return None
 
 
@@ -615,6 +618,8 @@ def run_asap(args):
     roof = {"kernel": dom, "bound": kd["bound"], "achieved": kd["achieved"], "peak": kd["peak"],
             "peak_kind": kd["peak_kind"], "unit": kd["unit"], "frac": kd["frac"],
             "traffic": traffic_per_launch(w["name"], dom),
+            "frac_of_nominal": kd["achieved"] / (NOMINAL_HBM_GBS if kd["unit"] == "GB/s" else NOMINAL_BF16_TFLOPS),
+            "ncu_dram_throughput_pct": traffic_per_launch(w["name"], dom, "ncu_dram_throughput_pct"),
             "algorithmic_per_launch": kd["algorithmic_per_launch"], "mean_launch_ms": kd["mean_launch_ms"]}
     value = whole_job_rate(world, units_per_step, K, elapsed_ms * 1e-3)
     line = {"metric": METRIC, "value": value, "unit": "worker-samples/s", "n_gpus": world, "steps": K,

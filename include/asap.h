@@ -258,6 +258,49 @@ asap_status asap_set_sync_mode(asap_ctx* ctx, asap_sync_mode mode);
  * pending. */
 asap_status asap_set_worker_order(asap_ctx* ctx, const int32_t* order);
 
+/* Worker-sharded mode (Section 5, Implementation: each process holds the
+ * replicas of some workers, and a worker's model reaches the processes of
+ * its out-neighbours as a point-to-point message).  This context steps only
+ * workers [first, first + count) of its N-worker system; W keeps all N rows,
+ * but the rows of the other workers hold what the caller delivered.  Per
+ * round:
+ *   asap_local_step       the owned workers' minibatch step; their rows of W_t
+ *                         then hold the half step x_j - eta g_j;
+ *   asap_read_rows        the owned rows that other processes need;
+ *   asap_write_rows       the rows received from other processes (every
+ *                         in-neighbour of an owned worker under the round's
+ *                         graph, asap_get_graph);
+ *   asap_stochastic_reduce  the owned rows of W_{t+1}.  It fails with
+ *                         ASAP_ERR_ARG, launching nothing, if an in-neighbour's
+ *                         row was not delivered this round: for a worker
+ *                         stepped elsewhere the delivery is its NOTIFY.
+ * Hinge and logistic models, BSP only, any graph; every process must use the
+ * same N, d, graph seed, graph kind and model settings.  Call after
+ * asap_set_model and before asap_load_shards (it drops loaded shards);
+ * asap_load_shards then reads only the owned workers' shards (the others'
+ * pointers may be NULL).  first = 0, count = N restores the whole system.
+ * asap_read_metrics then returns this context's share of the mean loss (the
+ * sum over owned workers / (N B): the shares of all processes add up to the
+ * mean loss) and NaN for the consensus error.  Syncing. */
+asap_status asap_set_worker_range(asap_ctx* ctx, int first, int count);
+
+/* Copies rows `rows[0..count)` of the current parameters W_t (row-major,
+ * count x P floats, P = d C) to host memory.  Between asap_local_step and
+ * asap_stochastic_reduce of a worker-sharded context the owned rows hold
+ * the half step in stored form: true values = stored values x *scale_out
+ * (the product of the round's L2 shrink factors; 1 without L2).  Processes
+ * with the same model settings share the factor, so rows are sent as
+ * stored.  Otherwise *scale_out = 1.  scale_out may be NULL.  Syncing. */
+asap_status asap_read_rows(asap_ctx* ctx, const int32_t* rows, int count, float* host_out, float* scale_out);
+
+/* Writes rows received from other processes into the current parameters
+ * W_t of a worker-sharded context, after its local step and before its
+ * reduce: rows[q] (not an owned worker) gets host_in[q * P .. (q+1) * P),
+ * in the sender's stored form.  Each row counts as delivered for this round.
+ * ASAP_ERR_ARG for an owned or out-of-range row, or outside that window.
+ * Syncing. */
+asap_status asap_write_rows(asap_ctx* ctx, const int32_t* rows, int count, const float* host_in);
+
 /* Consistency of the gated (NOTIFY_ACK, ASYNC) reduces since creation: the
  * inputs they read -- one per (column slab, worker) block of updates -- and
  * how many of those were current, i.e. read after the worker's NOTIFY for

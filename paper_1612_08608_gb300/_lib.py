@@ -41,6 +41,9 @@ SIGNATURES = {
     "asap_set_wait_limit_ns": (C.c_int, [_P, C.c_uint64]),
     "asap_set_sync_mode": (C.c_int, [_P, C.c_int]),
     "asap_set_worker_order": (C.c_int, [_P, _P]),
+    "asap_set_worker_range": (C.c_int, [_P, C.c_int, C.c_int]),
+    "asap_read_rows": (C.c_int, [_P, _P, C.c_int, _P, C.POINTER(C.c_float)]),
+    "asap_write_rows": (C.c_int, [_P, _P, C.c_int, _P]),
     "asap_read_consistency": (C.c_int, [_P, C.POINTER(C.c_uint64), C.POINTER(C.c_uint64)]),
     "asap_debug_skip_notify": (C.c_int, [_P, C.c_int]),
     "asap_set_kernel_timing": (C.c_int, [_P, C.c_int]),

@@ -36,7 +36,7 @@ def _ptr(a: np.ndarray) -> int:
 
 
 def _ptr_array(arrs):
-    return (C.c_void_p * len(arrs))(*[_ptr(a) for a in arrs])
+    return (C.c_void_p * len(arrs))(*[None if a is None else _ptr(a) for a in arrs])
 
 
 def build_graph(kind: str, N: int, k: int, graph_seed: int = 0, rnd: int = 0) -> np.ndarray:
@@ -75,6 +75,8 @@ def debug_batch_image(shards, batch: int, slab_cols: int, t: int, ctas_per_worke
 
 class Context:
     """N simulated workers on the current CUDA device (see include/asap.h)."""
+
+    row_dtype = np.float32   # parameter rows as read_rows returns them
 
     def __init__(self, N: int, d: int, graph_seed: int = 0, k: int = 0):
         self._lib = load_library()
@@ -123,11 +125,11 @@ class Context:
     def load_shards(self, shards=None, rowptr=None, col=None, val=None, y=None):
         if shards is not None:
             rowptr, col, val, y = shards.rowptr, shards.col, shards.val, shards.y
-        rp = [np.ascontiguousarray(a, dtype=np.int64) for a in rowptr]
-        cl = [np.ascontiguousarray(a, dtype=np.int32) for a in col]
-        vl = [np.ascontiguousarray(a, dtype=np.float32) for a in val]
-        yl = [np.ascontiguousarray(a, dtype=np.float32) for a in y]
-        n = np.array([a.shape[0] - 1 for a in rp], dtype=np.int64)
+        # None: a worker that a worker-sharded context does not step
+        def conv(arrs, dt):
+            return [None if a is None else np.ascontiguousarray(a, dtype=dt) for a in arrs]
+        rp, cl, vl, yl = conv(rowptr, np.int64), conv(col, np.int32), conv(val, np.float32), conv(y, np.float32)
+        n = np.array([0 if a is None else a.shape[0] - 1 for a in rp], dtype=np.int64)
         self._c(self._lib.asap_load_shards(self._h, _ptr_array(rp), _ptr_array(cl), _ptr_array(vl),
                                            _ptr_array(yl), _ptr(n)))
 
@@ -207,6 +209,27 @@ class Context:
             return
         order = np.ascontiguousarray(order, dtype=np.int32)
         self._c(self._lib.asap_set_worker_order(self._h, _ptr(order)))
+
+    # -- worker-sharded mode ---------------------------------------------
+    def set_worker_range(self, first: int, count: int):
+        """Step only workers [first, first + count); the others' rows are
+        delivered with write_rows every round."""
+        self._c(self._lib.asap_set_worker_range(self._h, first, count))
+
+    def read_rows(self, rows, out: Optional[np.ndarray] = None):
+        """Rows of W_t as stored, and the factor that gives their true values."""
+        rows = np.ascontiguousarray(rows, dtype=np.int32)
+        if out is None:
+            out = np.empty((rows.shape[0], self.P), dtype=np.float32)
+        sc = C.c_float()
+        self._c(self._lib.asap_read_rows(self._h, _ptr(rows), rows.shape[0], _ptr(out), C.byref(sc)))
+        return out, sc.value
+
+    def write_rows(self, rows, values: np.ndarray):
+        rows = np.ascontiguousarray(rows, dtype=np.int32)
+        values = np.ascontiguousarray(values, dtype=np.float32)
+        assert values.shape == (rows.shape[0], self.P)
+        self._c(self._lib.asap_write_rows(self._h, _ptr(rows), rows.shape[0], _ptr(values)))
 
     def read_consistency(self):
         """{inputs_read, inputs_current} of the gated reduces since creation."""

@@ -11,6 +11,7 @@
 #include <memory>
 #include <string>
 #include <thread>
+#include <limits>
 #include <vector>
 
 #include "asap_internal.h"
@@ -90,6 +91,11 @@ struct asap_ctx {
   float* r_big = nullptr;            // sparse, B > kRSmemRows: r [N][Q][B]
   int* d_worker_of = nullptr;        // sparse: worker of each local-step cluster (a permutation)
   bool permuted = false;             // d_worker_of differs from the identity
+  // worker-sharded mode (asap_set_worker_range): this context steps workers
+  // [own_lo, own_lo + own_n); the rows of the others are delivered by the caller
+  bool sharded = false;
+  int own_lo = 0, own_n = 0;
+  std::vector<unsigned char> delivered;   // [N] row j written this round (asap_write_rows)
   double* cons_part = nullptr;
   int cons_cap = 0;
   int32_t* d_nbr = nullptr;
@@ -505,6 +511,7 @@ void build_batch_image(int N, int B, int64_t d, int S, long long n_slabs, int Q,
   std::vector<int64_t> nnz(N, 0);
   for (int i = 0; i < N; ++i) {
     const int64_t* rp = rowptr[i];
+    if (!rp) continue;   // a worker this context does not step (worker-sharded): no entries
     const int64_t r0 = static_cast<int64_t>(t) * B;
     const int64_t a0 = rp[r0], a1 = rp[r0 + B];
     nnz[i] = a1 - a0;
@@ -597,6 +604,7 @@ void build_batch_image(int N, int B, int64_t d, int S, long long n_slabs, int Q,
     uint16_t* sr_o = reinterpret_cast<uint16_t*>(base + dd.srow);
     int32_t* bd_o = reinterpret_cast<int32_t*>(base + dd.bnd);
     const int64_t* rp = rowptr[i];
+    if (!rp) continue;   // labels and ranges stay zero
     const int64_t r0 = static_cast<int64_t>(t) * B, a0 = rp[r0];
     for (int b = 0; b < B; ++b) y_o[b] = y[i][r0 + b];
     std::vector<uint16_t> erow(nnz[i]);
@@ -909,6 +917,8 @@ asap_status asap_set_model(asap_ctx* c, asap_loss loss, int num_classes, int bat
        static_cast<int64_t>(c->N) * ((num_classes + 255) / 256) * 256 > (1ll << 31) / batch))
     return fail(c, ASAP_ERR_ARG, "softmax needs 2 <= C <= 1024, d % 256 == 0 and B % 128 == 0");
   if (loss != ASAP_LOSS_SOFTMAX && num_classes != 1) return fail(c, ASAP_ERR_ARG, "num_classes must be 1");
+  if (c->sharded && loss == ASAP_LOSS_SOFTMAX)
+    return fail(c, ASAP_ERR_ARG, "worker-sharded contexts take hinge or logistic models");
   asap_status s0 = asap_sync(c);
   if (s0 != ASAP_OK) return s0;
   free_shards(c);
@@ -952,8 +962,11 @@ asap_status asap_set_model(asap_ctx* c, asap_loss loss, int num_classes, int bat
       c->dense_configured = true;
     }
   }
-  if (c->n_loss_part > 0)
+  if (c->n_loss_part > 0) {
     CU(cudaMalloc(&c->loss_part, 4 * static_cast<size_t>(c->n_loss_part)), "allocating step scratch");
+    // Workers that a worker-sharded context does not step contribute 0.
+    CU(cudaMemset(c->loss_part, 0, 4 * static_cast<size_t>(c->n_loss_part)), "zeroing step scratch");
+  }
   return ASAP_OK;
 }
 
@@ -1030,7 +1043,14 @@ asap_status asap_load_shards(asap_ctx* c, const int64_t* const* rowptr, const in
     return fail(c, ASAP_ERR_ARG, "set a hinge or logistic model before loading CSR shards");
   const int N = c->N, B = c->B;
   int nb = -1;
+  // Worker-sharded: the shards of workers outside the owned range are not
+  // read (their pointers may be NULL) and get empty minibatches.
+  std::vector<const int64_t*> rp_use(rowptr, rowptr + N);
   for (int i = 0; i < N; ++i) {
+    if (c->sharded && (i < c->own_lo || i >= c->own_lo + c->own_n)) {
+      rp_use[i] = nullptr;
+      continue;
+    }
     if (!rowptr[i] || !col[i] || !val[i] || !y[i]) return fail(c, ASAP_ERR_ARG, "NULL shard pointer");
     if (n_rows[i] < B) return fail(c, ASAP_ERR_ARG, "a shard has fewer rows than one minibatch");
     const int64_t nbi = n_rows[i] / B;
@@ -1055,7 +1075,7 @@ asap_status asap_load_shards(asap_ctx* c, const int64_t* const* rowptr, const in
 
     std::vector<BatchImage> built(nb);
     auto build_batch = [&](int t) {
-      build_batch_image(N, B, c->d, S, n_slabs, Q, t, rowptr, col, val, y, built[t]);
+      build_batch_image(N, B, c->d, S, n_slabs, Q, t, rp_use.data(), col, val, y, built[t]);
     };
     {
       const unsigned nthr = std::max(1u, std::min(32u, std::thread::hardware_concurrency()));
@@ -1299,8 +1319,8 @@ asap_status asap_local_step(asap_ctx* c) {
     a.loss_part = c->loss_part;
     a.ready = c->ready;
     a.st = c->st;
-    a.worker_of = c->permuted ? c->d_worker_of : nullptr;
-    a.N = c->N;
+    a.worker_of = (c->permuted || c->sharded) ? c->d_worker_of : nullptr;
+    a.N = c->sharded ? c->own_n : c->N;
     a.B = c->B;
     a.Q = c->step_q;
     a.stages = c->step_stages;
@@ -1320,9 +1340,10 @@ asap_status asap_local_step(asap_ctx* c) {
     const float eta = lr_at(c, k);
     const float s_next = s_scale * (1.0f - eta * c->l2);
     const float upd = eta / (static_cast<float>(c->B) * s_next);
-    if (!last) {
+    if (!last || c->sharded) {
       // w_stored -= eta / (B s') g at the step's columns; the reduce applies
-      // the round's last update itself.
+      // the round's last update itself, except in a worker-sharded context,
+      // whose owned rows must hold x - eta g before they are sent.
       time_begin(c, ASAP_KERNEL_APPLY);
       CU(launch_apply_update(c->W[r & 1], c->ld, reinterpret_cast<const uint32_t*>(block + c->list_off[tk]),
                              reinterpret_cast<const int*>(block + c->soff_off[tk]), c->n_slabs, c->S, c->gsum, upd,
@@ -1337,13 +1358,15 @@ asap_status asap_local_step(asap_ctx* c) {
         asap_status ss = stage_block(c, k + 2);                                 // prefetch
         if (ss != ASAP_OK) return ss;
       }
-    } else {
+    }
+    if (last) {
       c->pend_wscale = s_next;
       c->pend_upd = upd;
       c->pend_k = k;
     }
     s_scale = s_next;
   }
+  if (c->sharded) std::fill(c->delivered.begin(), c->delivered.end(), 0);
   c->step_pending = true;
   return ASAP_OK;
 }
@@ -1352,7 +1375,22 @@ asap_status asap_stochastic_reduce(asap_ctx* c) {
   if (!c) return fail(nullptr, ASAP_ERR_ARG, "ctx is NULL");
   const int64_t r = c->round;
   const bool sparse = c->loss == ASAP_LOSS_HINGE || c->loss == ASAP_LOSS_LOGISTIC;
-  const bool fused = c->step_pending && sparse;
+  const bool fused = c->step_pending && sparse && !c->sharded;
+  if (c->sharded && c->step_pending) {
+    // The NOTIFY of a worker stepped elsewhere is the delivery of its row:
+    // every in-neighbour of an owned worker must have arrived this round.
+    const size_t kp1 = static_cast<size_t>(c->k) + 1;
+    std::vector<int32_t> nbr(static_cast<size_t>(c->N) * kp1);
+    std::vector<float> wgt(nbr.size());
+    asap_status sg = graph_host(c, r, nbr.data(), wgt.data());
+    if (sg != ASAP_OK) return sg;
+    for (int i = c->own_lo; i < c->own_lo + c->own_n; ++i)
+      for (size_t q = 0; q < kp1; ++q) {
+        const int j = nbr[i * kp1 + q];
+        if ((j < c->own_lo || j >= c->own_lo + c->own_n) && !c->delivered[j])
+          return fail(c, ASAP_ERR_ARG, "an in-neighbour's row was not delivered this round (asap_write_rows)");
+      }
+  }
   asap_status s = configure_mix_launch(c, fused);
   if (s != ASAP_OK) return s;
   s = prepare_graph(c, r);
@@ -1410,6 +1448,8 @@ asap_status asap_stochastic_reduce(asap_ctx* c) {
   a.expect_notify = c->step_pending ? 1 : 0;
   a.wait_ns = c->wait_ns;
   a.sync_mode = fused ? c->sync_mode : kSyncBsp;
+  a.own_lo = c->sharded ? c->own_lo : 0;
+  a.own_n = c->sharded ? c->own_n : c->N;
   time_begin(c, ASAP_KERNEL_REDUCE);
   CU(launch_mix(c->tmap[r & 1], a, is_complete_kernel(c), fused, c->mix_grid, c->mix_smem, c->stream),
      "launching the stochastic reduce");
@@ -1536,6 +1576,9 @@ asap_status asap_read_metrics(asap_ctx* c, int64_t first, int64_t count, float* 
     r += n;
   }
   CU(cudaStreamSynchronize(c->read_stream), "metrics");
+  // A worker-sharded context holds the other workers' rows only where they
+  // were delivered: its consensus error over all rows is not defined.
+  if (c->sharded && cons_out) std::fill(cons_out, cons_out + count, std::numeric_limits<float>::quiet_NaN());
   return ASAP_OK;
 }
 
@@ -1567,6 +1610,8 @@ asap_status asap_set_sync_mode(asap_ctx* c, asap_sync_mode mode) {
   if (mode != ASAP_SYNC_BSP && mode != ASAP_SYNC_NOTIFY_ACK && mode != ASAP_SYNC_ASYNC)
     return fail(c, ASAP_ERR_ARG, "unknown synchronisation mode");
   if (c->step_pending) return fail(c, ASAP_ERR_ARG, "a local step is pending: reduce first");
+  if (c->sharded && mode != ASAP_SYNC_BSP)
+    return fail(c, ASAP_ERR_ARG, "a worker-sharded context reduces after the delivery of its rows (BSP)");
   c->sync_mode = mode == ASAP_SYNC_NOTIFY_ACK ? kSyncNotifyAck : mode == ASAP_SYNC_ASYNC ? kSyncAsync : kSyncBsp;
   return ASAP_OK;
 }
@@ -1574,6 +1619,7 @@ asap_status asap_set_sync_mode(asap_ctx* c, asap_sync_mode mode) {
 asap_status asap_set_worker_order(asap_ctx* c, const int32_t* order) {
   if (!c) return fail(nullptr, ASAP_ERR_ARG, "ctx is NULL");
   if (c->step_pending) return fail(c, ASAP_ERR_ARG, "a local step is pending: reduce first");
+  if (c->sharded) return fail(c, ASAP_ERR_ARG, "the worker order of a worker-sharded context is its range");
   if (!order) {
     c->permuted = false;
     return ASAP_OK;
@@ -1588,6 +1634,65 @@ asap_status asap_set_worker_order(asap_ctx* c, const int32_t* order) {
   if (s0 != ASAP_OK) return s0;
   CU(cudaMemcpy(c->d_worker_of, order, 4 * static_cast<size_t>(c->N), cudaMemcpyHostToDevice), "uploading the worker order");
   c->permuted = !identity;
+  return ASAP_OK;
+}
+
+asap_status asap_set_worker_range(asap_ctx* c, int first, int count) {
+  if (!c) return fail(nullptr, ASAP_ERR_ARG, "ctx is NULL");
+  if (c->loss != ASAP_LOSS_HINGE && c->loss != ASAP_LOSS_LOGISTIC)
+    return fail(c, ASAP_ERR_ARG, "set a hinge or logistic model first");
+  if (first < 0 || count < 1 || first > c->N - count) return fail(c, ASAP_ERR_ARG, "range outside [0, N)");
+  if (c->step_pending) return fail(c, ASAP_ERR_ARG, "a local step is pending: reduce first");
+  asap_status s0 = asap_sync(c);
+  if (s0 != ASAP_OK) return s0;
+  free_shards(c);   // the minibatch images depend on the range
+  const bool whole = first == 0 && count == c->N;
+  c->sharded = !whole;
+  c->own_lo = whole ? 0 : first;
+  c->own_n = whole ? c->N : count;
+  c->delivered.assign(c->N, 0);
+  c->permuted = false;
+  c->sync_mode = kSyncBsp;
+  std::vector<int32_t> own(c->N);
+  for (int q = 0; q < c->N; ++q) own[q] = q < c->own_n ? c->own_lo + q : q;
+  CU(cudaMemcpy(c->d_worker_of, own.data(), 4 * static_cast<size_t>(c->N), cudaMemcpyHostToDevice),
+     "uploading the owned workers");
+  return ASAP_OK;
+}
+
+asap_status asap_read_rows(asap_ctx* c, const int32_t* rows, int count, float* host_out, float* scale_out) {
+  if (!c || (count > 0 && (!rows || !host_out)) || count < 0) return fail(c, ASAP_ERR_ARG, "bad argument");
+  for (int q = 0; q < count; ++q)
+    if (rows[q] < 0 || rows[q] >= c->N) return fail(c, ASAP_ERR_ARG, "row outside [0, N)");
+  asap_status s = sync_all(c);
+  if (s != ASAP_OK) return s;
+  const float* src = c->W[c->round & 1];
+  for (int q = 0; q < count; ++q)
+    CU(cudaMemcpyAsync(host_out + static_cast<size_t>(q) * c->P, src + static_cast<size_t>(rows[q]) * c->ld,
+                       4 * static_cast<size_t>(c->P), cudaMemcpyDeviceToHost, c->stream),
+       "reading rows");
+  CU(cudaStreamSynchronize(c->stream), "reading rows");
+  if (scale_out) *scale_out = (c->sharded && c->step_pending) ? c->pend_wscale : 1.0f;
+  return ASAP_OK;
+}
+
+asap_status asap_write_rows(asap_ctx* c, const int32_t* rows, int count, const float* host_in) {
+  if (!c || (count > 0 && (!rows || !host_in)) || count < 0) return fail(c, ASAP_ERR_ARG, "bad argument");
+  if (!c->sharded) return fail(c, ASAP_ERR_ARG, "rows are delivered to worker-sharded contexts only");
+  if (!c->step_pending) return fail(c, ASAP_ERR_ARG, "deliver rows between the local step and the reduce");
+  for (int q = 0; q < count; ++q) {
+    if (rows[q] < 0 || rows[q] >= c->N) return fail(c, ASAP_ERR_ARG, "row outside [0, N)");
+    if (rows[q] >= c->own_lo && rows[q] < c->own_lo + c->own_n)
+      return fail(c, ASAP_ERR_ARG, "an owned worker's row is this context's own");
+  }
+  float* dst = c->W[c->round & 1];
+  for (int q = 0; q < count; ++q) {
+    CU(cudaMemcpyAsync(dst + static_cast<size_t>(rows[q]) * c->ld, host_in + static_cast<size_t>(q) * c->P,
+                       4 * static_cast<size_t>(c->P), cudaMemcpyHostToDevice, c->stream),
+       "writing rows");
+    c->delivered[rows[q]] = 1;
+  }
+  CU(cudaStreamSynchronize(c->stream), "writing rows");
   return ASAP_OK;
 }
 

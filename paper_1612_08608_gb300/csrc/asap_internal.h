@@ -93,8 +93,9 @@ struct LocalStepArgs {
   float* loss_part;            // [N]: minibatch loss sum per worker
   unsigned int* ready;         // NOTIFY flags [N]
   DevState* st;
-  const int* worker_of;        // [N] worker of each cluster (a permutation), or nullptr
-  int N, B, Q, stages;
+  const int* worker_of;        // worker of each cluster (a permutation or, worker-sharded, the owned
+                               // workers), or nullptr
+  int N, B, Q, stages;         // N: clusters launched (workers stepped)
   unsigned int round;
   int skip_worker;             // fault injection: do not NOTIFY this worker
   float mscale;                // true w = mscale * (stored values): margins are scaled by it
@@ -143,6 +144,9 @@ struct MixArgs {
   int expect_notify;
   unsigned long long wait_ns;
   int sync_mode;               // kSync* (FUSED reduces; others are BSP)
+  int own_lo, own_n;           // workers stepped in this context: the NOTIFY waits and the counters cover
+                               // [own_lo, own_lo + own_n); a worker-sharded context learns of the others'
+                               // NOTIFY on the host, when their rows are delivered
 };
 
 // Arguments of the dense softmax-regression step (kernels_dense.cu).

@@ -288,7 +288,8 @@ __global__ void __launch_bounds__(kMixThreads, 1) k_mix(const __grid_constant__ 
   // ---- NOTIFY / ACK checks (time-limited waits) ----
   for (int j = tid; j < a.N; j += kMixThreads) {
     unsigned e = 0;
-    if (a.expect_notify && !gated) e = wait_flag(a.ready + j, a.round + 1u, true, a.wait_ns);
+    const bool own = j >= a.own_lo && j < a.own_lo + a.own_n;
+    if (a.expect_notify && !gated && own) e = wait_flag(a.ready + j, a.round + 1u, true, a.wait_ns);
     if (!e) e = wait_flag(a.consumed + j, a.round, false, a.wait_ns);
     if (e) {
       record_error(a.st, e, j, a.round);
@@ -684,9 +685,9 @@ __global__ void __launch_bounds__(kMixThreads, 1) k_mix(const __grid_constant__ 
     a.metrics_loss[slot] = (a.have_loss && !any_fail) ? static_cast<float>(ltot * a.loss_norm)
                                                       : __int_as_float(0x7fc00000);
     if (!any_fail) {
-      a.st->reduces += static_cast<unsigned long long>(a.N);
+      a.st->reduces += static_cast<unsigned long long>(a.own_n);
       if (a.expect_notify)
-        a.st->consistent_inputs += static_cast<unsigned long long>(a.N) * (KP1 < 0 ? a.N : kp1);
+        a.st->consistent_inputs += static_cast<unsigned long long>(a.own_n) * (KP1 < 0 ? a.N : kp1);
     }
     a.st->mix_ticket = 0u;
   }

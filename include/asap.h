@@ -331,8 +331,8 @@ asap_status asap_debug_skip_notify(asap_ctx* ctx, int worker);
  * of the (column, row)-sorted entries' list positions, values, rows and
  * segment slots (int32 / float / uint16 / uint16 [nnz]), of the rows of
  * every segment's slots (uint16 [nnz]) and of the Q+1 column-sum range
- * bounds (int32), then nnz.  Segment g holds sorted entries [1024 g,
- * 1024 (g+1)); its slots are numbered row by row, a row's entries in sorted
+ * bounds (int32), then nnz.  Segment g holds sorted entries [256 g,
+ * 256 (g+1)); its slots are numbered row by row, a row's entries in sorted
  * order.  The range bounds start at 0, end at nnz and cut the sorted entries
  * at the first column boundary at or after q nnz / Q.  list_out (3 int64):
  * byte offsets of the slab-major list of distinct (worker << 16 | column in

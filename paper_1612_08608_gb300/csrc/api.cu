@@ -87,7 +87,7 @@ struct asap_ctx {
   float* m_cons = nullptr;
   float* r_scr = nullptr;
   float* loss_part = nullptr;
-  float* mpart_big = nullptr;        // sparse, B > kRSmemRows: partial margins [N][Q][B]
+  float* mpart_big = nullptr;        // sparse, B > kRSmemRows: per-warp partial margins [N][Q][4][B]
   float* r_big = nullptr;            // sparse, B > kRSmemRows: r [N][Q][B]
   int* d_worker_of = nullptr;        // sparse: worker of each local-step cluster (a permutation)
   bool permuted = false;             // d_worker_of differs from the identity
@@ -102,8 +102,13 @@ struct asap_ctx {
   float* d_wgt = nullptr;
   int32_t* h_nbr = nullptr;
   float* h_wgt = nullptr;
-  cudaEvent_t slot_ev[kGraphRing] = {};
-  bool slot_used[kGraphRing] = {};
+  // Regenerated graphs: the ring's two halves hold batches of kGraphBatch
+  // rounds (batch b = round / kGraphBatch in half b & 1), uploaded on the
+  // copy stream one batch at a time.
+  int64_t graph_half_batch[2] = {-1, -1};
+  cudaEvent_t graph_half_ev[2] = {};   // the half's last upload
+  bool graph_half_used[2] = {false, false};
+  cudaEvent_t graph_order_ev = nullptr; // the stream's work before an upload
 
   // sparse shards
   asap_residency residency = ASAP_SHARDS_DEVICE;
@@ -396,6 +401,7 @@ asap_status alloc_params(asap_ctx* c) {
 asap_status upload_fixed_graph(asap_ctx* c) {
   c->graph_round_in_slot0 = -2;
   c->graph_ready_round = -1;
+  c->graph_half_batch[0] = c->graph_half_batch[1] = -1;
   if (c->tab_kp1 == 0 || c->regen) return ASAP_OK;
   const size_t n = static_cast<size_t>(c->N) * c->tab_kp1;
   std::vector<int32_t> nbr(n);
@@ -409,9 +415,13 @@ asap_status upload_fixed_graph(asap_ctx* c) {
   return ASAP_OK;
 }
 
-// Device tables for round `rnd` (regenerated graphs go through a ring of
-// pinned host slots and device slots; a slot is rewritten only after its
-// previous upload has completed).
+// Device tables for round `rnd`.  Regenerated graphs are built on the host
+// kGraphBatch rounds at a time into one half of a pinned ring and uploaded
+// with one copy per table on the copy stream, so that the context stream
+// meets an upload once per batch instead of carrying two small copies
+// between the kernels of every round.  The upload into a half waits for the
+// stream's earlier work (every reduce that read the half's previous batch),
+// and the stream waits for the upload.
 asap_status graph_tables(asap_ctx* c, int64_t rnd, const int** nbr, const float** wgt) {
   *nbr = nullptr;
   *wgt = nullptr;
@@ -422,18 +432,29 @@ asap_status graph_tables(asap_ctx* c, int64_t rnd, const int** nbr, const float*
     *wgt = c->d_wgt;
     return ASAP_OK;
   }
-  const int slot = static_cast<int>(rnd % kGraphRing);
-  if (c->slot_used[slot]) CU(cudaEventSynchronize(c->slot_ev[slot]), "waiting for a graph slot");
-  int32_t* hn = c->h_nbr + slot * n;
-  float* hw = c->h_wgt + slot * n;
-  asap_status s = graph_host(c, rnd, hn, hw);
-  if (s != ASAP_OK) return s;
-  CU(cudaMemcpyAsync(c->d_nbr + slot * n, hn, n * 4, cudaMemcpyHostToDevice, c->stream), "graph upload");
-  CU(cudaMemcpyAsync(c->d_wgt + slot * n, hw, n * 4, cudaMemcpyHostToDevice, c->stream), "graph upload");
-  CU(cudaEventRecord(c->slot_ev[slot], c->stream), "graph upload event");
-  c->slot_used[slot] = true;
-  *nbr = c->d_nbr + slot * n;
-  *wgt = c->d_wgt + slot * n;
+  const int64_t b = rnd / kGraphBatch;
+  const int half = static_cast<int>(b & 1);
+  const size_t h0 = static_cast<size_t>(half) * kGraphBatch * n;   // first entry of the half
+  if (c->graph_half_batch[half] != b) {
+    if (c->graph_half_used[half]) CU(cudaEventSynchronize(c->graph_half_ev[half]), "waiting for a graph upload");
+    for (int j = 0; j < kGraphBatch; ++j) {
+      asap_status s = graph_host(c, b * kGraphBatch + j, c->h_nbr + h0 + j * n, c->h_wgt + h0 + j * n);
+      if (s != ASAP_OK) return s;
+    }
+    CU(cudaEventRecord(c->graph_order_ev, c->stream), "graph upload order");
+    CU(cudaStreamWaitEvent(c->copy_stream, c->graph_order_ev, 0), "graph upload order");
+    CU(cudaMemcpyAsync(c->d_nbr + h0, c->h_nbr + h0, kGraphBatch * n * 4, cudaMemcpyHostToDevice, c->copy_stream),
+       "graph upload");
+    CU(cudaMemcpyAsync(c->d_wgt + h0, c->h_wgt + h0, kGraphBatch * n * 4, cudaMemcpyHostToDevice, c->copy_stream),
+       "graph upload");
+    CU(cudaEventRecord(c->graph_half_ev[half], c->copy_stream), "graph upload event");
+    CU(cudaStreamWaitEvent(c->stream, c->graph_half_ev[half], 0), "graph upload");
+    c->graph_half_used[half] = true;
+    c->graph_half_batch[half] = b;
+  }
+  const size_t at = h0 + static_cast<size_t>(rnd % kGraphBatch) * n;
+  *nbr = c->d_nbr + at;
+  *wgt = c->d_wgt + at;
   return ASAP_OK;
 }
 
@@ -616,10 +637,10 @@ void build_batch_image(int N, int B, int64_t d, int S, long long n_slabs, int Q,
       cv_o[e] = val[i][a0 + k];
       cr_o[e] = erow[k];
     }
-    // Margin segments of kTileEntries sorted entries: slots row by row, a
+    // Margin segments of kSlotSegment sorted entries: slots row by row, a
     // row's entries in sorted (column) order; srow lists the slots' rows.
-    for (int64_t e0 = 0; e0 < nnz[i]; e0 += kTileEntries) {
-      const int64_t e1 = std::min<int64_t>(e0 + kTileEntries, nnz[i]);
+    for (int64_t e0 = 0; e0 < nnz[i]; e0 += kSlotSegment) {
+      const int64_t e1 = std::min<int64_t>(e0 + kSlotSegment, nnz[i]);
       std::fill(fill.begin(), fill.end(), 0);
       for (int64_t e = e0; e < e1; ++e) fill[cr_o[e]]++;
       int32_t acc = 0;
@@ -746,10 +767,11 @@ static asap_status init_ctx(asap_ctx* c) {
     CU(cudaEventCreateWithFlags(&c->round_ev[i], cudaEventDisableTiming), "creating events");
     c->round_ev_round[i] = -1;
   }
-  for (int i = 0; i < kGraphRing; ++i) {
-    CU(cudaEventCreateWithFlags(&c->slot_ev[i], cudaEventDisableTiming), "creating events");
-    c->slot_used[i] = false;
+  for (int h = 0; h < 2; ++h) {
+    CU(cudaEventCreateWithFlags(&c->graph_half_ev[h], cudaEventDisableTiming), "creating events");
+    c->graph_half_used[h] = false;
   }
+  CU(cudaEventCreateWithFlags(&c->graph_order_ev, cudaEventDisableTiming), "creating events");
   for (int b = 0; b < asap_ctx::kStaging; ++b) {
     CU(cudaEventCreateWithFlags(&c->staged_ev[b], cudaEventDisableTiming), "creating events");
     CU(cudaEventCreateWithFlags(&c->free_ev[b], cudaEventDisableTiming), "creating events");
@@ -831,8 +853,9 @@ void asap_destroy(asap_ctx* c) {
   dfree(c->d_wgt);
   if (c->h_nbr) cudaFreeHost(c->h_nbr);
   if (c->h_wgt) cudaFreeHost(c->h_wgt);
-  for (int i = 0; i < kGraphRing; ++i)
-    if (c->slot_ev[i]) cudaEventDestroy(c->slot_ev[i]);
+  for (int h = 0; h < 2; ++h)
+    if (c->graph_half_ev[h]) cudaEventDestroy(c->graph_half_ev[h]);
+  if (c->graph_order_ev) cudaEventDestroy(c->graph_order_ev);
   for (auto& e : c->tev)
     if (e) cudaEventDestroy(e);
   for (int b = 0; b < asap_ctx::kStaging; ++b) {
@@ -942,7 +965,7 @@ asap_status asap_set_model(asap_ctx* c, asap_loss loss, int num_classes, int bat
     // all clusters resident at four CTAs per SM (at most 8, the portable size).
     c->step_q = kMaxStepCluster;
     while (c->step_q > 1 && static_cast<int64_t>(c->N) * c->step_q > 4LL * c->sm_count) c->step_q >>= 1;
-    c->step_stages = 2;
+    c->step_stages = 3;
     c->step_smem = local_step_smem_bytes(batch, c->step_stages);
     CU(local_step_configure(c->step_smem), "configuring the local-step kernel");
     c->permuted = false;
@@ -1153,7 +1176,7 @@ asap_status asap_load_shards(asap_ctx* c, const int64_t* const* rowptr, const in
     CU(cudaMemset(c->wv[1], 0, lb), "zeroing the list value buffer");
     CU(cudaMemset(c->gsum, 0, lb), "zeroing the column-sum buffer");
     if (B > kRSmemRows) {
-      CU(cudaMalloc(&c->mpart_big, 4 * static_cast<size_t>(N) * Q * B), "allocating the partial margins");
+      CU(cudaMalloc(&c->mpart_big, 16 * static_cast<size_t>(N) * Q * B), "allocating the partial margins");
       CU(cudaMalloc(&c->r_big, 4 * static_cast<size_t>(N) * Q * B), "allocating the step scratch");
     }
     c->nb = nb;

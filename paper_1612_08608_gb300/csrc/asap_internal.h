@@ -22,7 +22,8 @@ namespace asap {
 constexpr int kMaxWorkers = 1024;
 constexpr int kMaxKp1Sparse = 32;     // neighbours per row for the sparse reduce
 constexpr int kMetricsCap = 65536;    // rounds of metrics kept on the device
-constexpr int kGraphRing = 64;        // device slots for per-round graphs
+constexpr int kGraphRing = 64;        // device slots for per-round graphs: two halves of
+constexpr int kGraphBatch = kGraphRing / 2;   // rounds uploaded together
 constexpr int kThreads = 256;         // block size of every kernel here
 
 // Device-side protocol and error state (one per context).
@@ -56,9 +57,10 @@ constexpr uint32_t kListPad = 0xffffffffu;   // padding entry of a column list
 // the block start).  The minibatch's entries are kept in one order only,
 // sorted by (column, row); `cpos` indexes the batch's slab-major column list
 // (one entry per distinct (worker, column) of the minibatch).  For the
-// margins the sorted entries are cut into segments of kTileEntries; inside
-// a segment every entry has a slot, the slots of one row contiguous (rows in
-// order, a row's entries by column), and `srow` lists the row of every slot.
+// margins the sorted entries are cut into segments of kSlotSegment (one
+// consumer warp's share of a tile); inside a segment every entry has a slot,
+// the slots of one row contiguous (rows in order, a row's entries by
+// column), and `srow` lists the row of every slot.
 // For the column sums the entries are split among the worker's Q CTAs at
 // column boundaries (`bnd`).
 struct BatchDesc {
@@ -73,12 +75,14 @@ struct BatchDesc {
   int32_t pad_;
 };
 
-// Entries per margin segment and per column-sum tile (one ring stage).
+// Entries per ring stage of the local step (a tile), and per margin slot
+// segment (a consumer warp's 256-entry share of a tile).
 constexpr int kTileEntries = 1024;
-// Partial margins and r stay in shared memory for minibatches of at most
-// this many rows (else in global scratch).
-constexpr int kRSmemRows = 8192;
-constexpr int kLocalStepThreads = 160;   // four consumer warps + one producer warp
+constexpr int kSlotSegment = 256;
+// Per-warp partial margins and r stay in shared memory for minibatches of
+// at most this many rows (else in global scratch).
+constexpr int kRSmemRows = 2048;
+constexpr int kLocalStepThreads = 192;   // four consumer warps, a bulk-copy issuer warp, a gather warp
 constexpr int kMaxStepCluster = 8;       // CTAs per worker (portable cluster size)
 
 // Arguments of the fused sparse local step (kernels_sparse.cu): one cluster
@@ -88,7 +92,7 @@ struct LocalStepArgs {
   const BatchDesc* desc;       // [N] descriptors of this step's batch
   const float* wv;             // w values at the step's list positions
   float* gsum;                 // column sums at the step's list positions
-  float* mpart_big;            // [N][Q][B] partial margins (B > kRSmemRows only)
+  float* mpart_big;            // [N][Q][4][B] per-warp partial margins (B > kRSmemRows only)
   float* r_big;                // [N][Q][B] r (B > kRSmemRows only)
   float* loss_part;            // [N]: minibatch loss sum per worker
   unsigned int* ready;         // NOTIFY flags [N]

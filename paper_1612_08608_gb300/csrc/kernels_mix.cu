@@ -227,32 +227,35 @@ struct MixSmem {
 
 // Shared-memory layout; every region starts 16-byte aligned (the slab
 // stages 1024-byte aligned).  mix_smem_bytes() mirrors it.
+// Regions are formed from `raw` by pointer arithmetic (offsets only), so that
+// the compiler keeps the pointers in the shared address space and emits
+// plain shared-memory accesses.
 __device__ __forceinline__ MixSmem carve(unsigned char* raw, const MixArgs& a, int kp1) {
   MixSmem m;
-  auto a16 = [](uintptr_t v) { return (v + 15) & ~static_cast<uintptr_t>(15); };
-  uintptr_t base = (reinterpret_cast<uintptr_t>(raw) + 1023) & ~static_cast<uintptr_t>(1023);
+  auto a16 = [](size_t v) { return (v + 15) & ~static_cast<size_t>(15); };
+  size_t off = (1024u - (smem_u32(raw) & 1023u)) & 1023u;   // 1024-byte aligned stages
   m.stage_bytes = mix_stage_bytes(a.S, a.rows_pad, a.max_region);
-  m.stage0 = reinterpret_cast<unsigned char*>(base);
-  base += m.stage_bytes * a.stages;
-  m.full = reinterpret_cast<uint64_t*>(base);
-  base += 8 * a.stages;
-  m.empty = reinterpret_cast<uint64_t*>(base);
-  base += 8 * a.stages;
-  m.ready = reinterpret_cast<uint64_t*>(base);
-  base = a16(base + 8 * a.stages);
-  m.dscratch = reinterpret_cast<double*>(base);
-  base = a16(base + 8 * (kMixThreads / 32));
-  m.flags = reinterpret_cast<int*>(base);
-  base = a16(base + 16);
-  m.seen = reinterpret_cast<unsigned*>(base);
-  base = a16(base + 4 * 32);
-  m.info = reinterpret_cast<int*>(base);
-  base = a16(base + 16 * a.stages);
-  m.part = reinterpret_cast<float4*>(base);
-  base = a16(base + 16 * static_cast<size_t>(a.stages) * kCompute);
-  m.nbr = reinterpret_cast<int*>(base);
-  base = a16(base + 4 * static_cast<size_t>(a.N) * kp1);
-  m.wgt = reinterpret_cast<float*>(base);
+  m.stage0 = raw + off;
+  off += m.stage_bytes * a.stages;
+  m.full = reinterpret_cast<uint64_t*>(raw + off);
+  off += 8 * a.stages;
+  m.empty = reinterpret_cast<uint64_t*>(raw + off);
+  off += 8 * a.stages;
+  m.ready = reinterpret_cast<uint64_t*>(raw + off);
+  off = a16(off + 8 * a.stages);
+  m.dscratch = reinterpret_cast<double*>(raw + off);
+  off = a16(off + 8 * (kMixThreads / 32));
+  m.flags = reinterpret_cast<int*>(raw + off);
+  off = a16(off + 16);
+  m.seen = reinterpret_cast<unsigned*>(raw + off);
+  off = a16(off + 4 * 32);
+  m.info = reinterpret_cast<int*>(raw + off);
+  off = a16(off + 16 * a.stages);
+  m.part = reinterpret_cast<float4*>(raw + off);
+  off = a16(off + 16 * static_cast<size_t>(a.stages) * kCompute);
+  m.nbr = reinterpret_cast<int*>(raw + off);
+  off = a16(off + 4 * static_cast<size_t>(a.N) * kp1);
+  m.wgt = reinterpret_cast<float*>(raw + off);
   return m;
 }
 
@@ -283,7 +286,14 @@ __global__ void __launch_bounds__(kMixThreads, 1) k_mix(const __grid_constant__ 
   // after j's NOTIFY (or, ASYNC, counts the read as stale).  Otherwise
   // (BSP) it starts once the local step's grid has finished.
   const bool gated = FUSED && a.sync_mode != kSyncBsp;
-  if (!gated) asm volatile("griddepcontrol.wait;" ::: "memory");
+  if (!gated) {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    // The next round's local step (a programmatic dependent) may now be
+    // scheduled as this grid drains; it waits for this grid before it reads
+    // what this grid writes.  A gated reduce leaves the trigger to its exit,
+    // since the local step it overlaps is still running.
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  }
 
   // ---- NOTIFY / ACK checks (time-limited waits) ----
   for (int j = tid; j < a.N; j += kMixThreads) {

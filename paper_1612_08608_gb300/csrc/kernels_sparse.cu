@@ -17,20 +17,24 @@
 //
 // One cluster of Q CTAs per worker (grid N x Q, no inter-cluster waits).
 // The minibatch's entries are stored once, sorted by (column, row), and
-// streamed twice through a ring of shared-memory stages by one producer
-// warp with bulk copies (cp.async.bulk, mbarrier completion), while eight
-// consumer warps work on the stage that has landed:
-//   pass 1 (margins): CTA q takes 2048-entry segments s = q nseg/Q ...;
-//     products val * wv[pos] go to shared memory at the entry's slot (slots
-//     ordered by row, then column), a segmented scan over the slots keyed by
-//     row sums each row's products in order, and the CTA adds them to its
-//     partial margins.  A cluster barrier; every CTA then adds the Q partials
-//     of each row in rank order (distributed shared memory), forms r and,
-//     in CTA 0, the loss sum.
+// streamed twice through a ring of shared-memory stages by an issuer warp
+// with bulk copies (cp.async.bulk, mbarrier completion) -- a gather warp
+// fetches a margin tile's w values as soon as the tile lands -- while four
+// consumer warps work on the stage that has landed, each on its own
+// 256-entry share of the 1024-entry tile and without CTA-wide barriers:
+//   pass 1 (margins): CTA q takes 1024-entry tiles s = q nseg/Q ...; a
+//     warp's products val * wv[pos] go to shared memory at the entry's slot
+//     (slots of a 256-entry segment ordered by row, then column), a
+//     segmented scan over the slots keyed by row sums each row's products
+//     in order, and the warp adds them to its own partial margins.  The
+//     four warps' partials are added in order; a cluster barrier; every CTA
+//     then adds the Q partials of each row in rank order (distributed shared
+//     memory), forms r and, in CTA 0, the loss sum.
 //   pass 2 (column sums): CTA q takes the entries [bnd[q], bnd[q+1]), cut
-//     at column boundaries, in 2048-entry tiles; a segmented scan keyed by
-//     list position sums each column's r_row * val, the run crossing a tile
-//     boundary carried to the next tile.
+//     at column boundaries, in 1024-entry tiles; a warp's segmented scan
+//     keyed by list position sums each column's r_row * val; runs that end
+//     inside the warp's share are stored by the warp, and the two runs at
+//     its edges are fragments that one warp adds up in order.
 // A last cluster barrier and CTA 0 publishes NOTIFY.  No atomics, no waits
 // on other clusters, every sum in a fixed order: the result does not depend
 // on the schedule.
@@ -45,7 +49,7 @@ namespace asap {
 namespace {
 
 constexpr unsigned kFull = 0xffffffffu;
-constexpr int kConsumers = kLocalStepThreads - 32;          // four consumer warps
+constexpr int kConsumers = kLocalStepThreads - 64;          // four consumer warps
 constexpr int kPerThread = kTileEntries / kConsumers;       // consecutive entries per consumer thread
 static_assert(kPerThread == 8, "a consumer thread takes 8 consecutive entries of a tile");
 constexpr unsigned long long kCopyWaitNs = 2000000000ull;   // a bulk copy never takes this long
@@ -119,10 +123,6 @@ __device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t b
                : "memory");
 }
 
-__device__ __forceinline__ void cluster_sync() {
-  asm volatile("barrier.cluster.arrive.release.aligned;\nbarrier.cluster.wait.acquire.aligned;" ::: "memory");
-}
-
 __device__ __forceinline__ uint32_t cluster_rank() {
   uint32_t r;
   asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
@@ -149,15 +149,6 @@ __device__ __forceinline__ void consumer_bar() {
   asm volatile("bar.sync 1, %0;" :: "n"(kConsumers) : "memory");
 }
 
-// Consumer barrier that also returns the AND of `v` over the consumer threads.
-__device__ __forceinline__ bool consumer_bar_and(bool v) {
-  uint32_t r;
-  asm volatile(
-      "{\n .reg .pred p, q;\n setp.ne.u32 p, %1, 0;\n bar.red.and.pred q, 1, %2, p;\n selp.u32 %0, 1, 0, q;\n}"
-      : "=r"(r) : "r"(static_cast<uint32_t>(v)), "n"(kConsumers) : "memory");
-  return r != 0;
-}
-
 __device__ __forceinline__ void record_error(DevState* st, unsigned code, unsigned worker, unsigned round) {
   if (atomicCAS(&st->err_code, 0u, code) == 0u) {
     st->err_worker = worker;
@@ -182,81 +173,88 @@ __device__ __forceinline__ void loss_and_r(float y, float m, float& l, float& r)
 // Shared-memory layout of the local-step kernel (mirrored by
 // local_step_smem_bytes): the ring of stages, each holding one tile's list
 // positions, values and two uint16 arrays (pass 1: slots and the rows in
-// slot order; pass 2: rows); the products of a segment by slot; the
-// partial margins and r of the worker's B rows; scan and control scratch.
+// slot order; pass 2: rows), a margin tile's positions replaced in place by
+// the gathered w values;
+// per consumer warp a 256-entry scratch (pass 1: products by slot; pass 2:
+// run sums and their list positions); the per-warp partial margins and r
+// of the worker's B rows; the column-run fragments at sub-tile edges.
 struct StepSmem {
   unsigned char* stage0;
   uint64_t* full;
   uint64_t* empty;
   uint64_t* gath;       // [stages]: the w values of a margin tile are in the stage
-  float* prod;          // [kTileEntries]: products by slot (pass 1), run sums (pass 2)
+  uint64_t* fready;     // [kFragRing]: every warp has left its fragments of a column-sum tile
+  float* prod;          // [kTileEntries]: warp w uses [256 w, 256 w + 256)
   int* okey;            // [kTileEntries]: list position of a run ending at the pair, else -1
-  float* mpart;         // [B]
+  float* mpart;         // [4][B]: per-warp partial margins (warp 0's row holds the CTA's sum after pass 1)
   float* r;             // [B]
-  int* keys;            // [kConsumers]: first key of each thread's pairs
-  int* keys_last;       // [kConsumers]: last key of each thread's pairs
-  float* wval;          // [kConsumers / 32]: warp aggregates of the scan
-  int* wflag;           // [kConsumers / 32]
+  int* fkey;            // [kFragRing][4][2]: first / last column-run fragment of each warp's sub-tile
+  float* fval;          // [kFragRing][4][2]
   float* red;           // [kConsumers / 32]
-  int* ctl;             // [0]: carry key, [1]: a copy timed out
-  float* carry;         // [1]: carried run sum
+  int* ctl;             // [1]: a copy timed out
 };
 
-// pos, val, two uint16 arrays, and (pass 1) the gathered w values
-constexpr size_t kStageBytes = static_cast<size_t>(kTileEntries) * 16;
+// pos (in margin tiles overwritten by the gathered w values), val and two
+// uint16 arrays
+constexpr size_t kStageBytes = static_cast<size_t>(kTileEntries) * 12;
+constexpr int kWarps = kConsumers / 32;
+constexpr int kIssuerWarp = kWarps, kGatherWarp = kWarps + 1;
+// Fragments of a column-sum tile are kept until warp 0 has merged them; a
+// warp runs at most `stages` tiles ahead of warp 0, so the ring needs
+// stages + 2 slots (stages <= 6).
+constexpr int kFragRing = 8;
+constexpr int kNoKey = -2;
 
+// Every region is formed from `raw` by pointer arithmetic (offsets only, no
+// integer round trip of the address), so that the compiler keeps the
+// pointers in the shared address space and emits plain shared-memory
+// accesses.
 __device__ __forceinline__ StepSmem carve_step(unsigned char* raw, int B, int stages) {
   StepSmem m;
-  uintptr_t p = (reinterpret_cast<uintptr_t>(raw) + 127) & ~static_cast<uintptr_t>(127);
-  m.stage0 = reinterpret_cast<unsigned char*>(p);
-  p += kStageBytes * stages;
-  m.full = reinterpret_cast<uint64_t*>(p);
-  p += 8 * stages;
-  m.empty = reinterpret_cast<uint64_t*>(p);
-  p += 8 * stages;
-  m.gath = reinterpret_cast<uint64_t*>(p);
-  p += 8 * stages;
-  p = (p + 15) & ~static_cast<uintptr_t>(15);   // prod is read as float4
-  m.prod = reinterpret_cast<float*>(p);
-  p += 4 * kTileEntries;
-  m.okey = reinterpret_cast<int*>(p);
-  p += 4 * kTileEntries;
-  m.mpart = reinterpret_cast<float*>(p);
-  p += 4 * static_cast<size_t>(B);
-  m.r = reinterpret_cast<float*>(p);
-  p += 4 * static_cast<size_t>(B);
-  m.keys = reinterpret_cast<int*>(p);
-  p += 4 * kConsumers;
-  m.keys_last = reinterpret_cast<int*>(p);
-  p += 4 * kConsumers;
-  m.wval = reinterpret_cast<float*>(p);
-  p += 4 * (kConsumers / 32);
-  m.wflag = reinterpret_cast<int*>(p);
-  p += 4 * (kConsumers / 32);
-  m.red = reinterpret_cast<float*>(p);
-  p += 4 * (kConsumers / 32);
-  m.ctl = reinterpret_cast<int*>(p);
-  p += 8;
-  m.carry = reinterpret_cast<float*>(p);
+  size_t off = (128u - (smem_u32(raw) & 127u)) & 127u;   // 128-byte aligned stages
+  m.stage0 = raw + off;
+  off += kStageBytes * stages;
+  m.full = reinterpret_cast<uint64_t*>(raw + off);
+  off += 8 * stages;
+  m.empty = reinterpret_cast<uint64_t*>(raw + off);
+  off += 8 * stages;
+  m.gath = reinterpret_cast<uint64_t*>(raw + off);
+  off += 8 * stages;
+  m.fready = reinterpret_cast<uint64_t*>(raw + off);
+  off += 8 * kFragRing;
+  off = (off + 15) & ~static_cast<size_t>(15);             // prod and okey are accessed as 16-byte vectors
+  m.prod = reinterpret_cast<float*>(raw + off);
+  off += 4 * kTileEntries;
+  m.okey = reinterpret_cast<int*>(raw + off);
+  off += 4 * kTileEntries;
+  m.mpart = reinterpret_cast<float*>(raw + off);
+  off += 4 * static_cast<size_t>(kWarps) * B;
+  m.r = reinterpret_cast<float*>(raw + off);
+  off += 4 * static_cast<size_t>(B);
+  m.fkey = reinterpret_cast<int*>(raw + off);
+  off += 4 * kFragRing * kWarps * 2;
+  m.fval = reinterpret_cast<float*>(raw + off);
+  off += 4 * kFragRing * kWarps * 2;
+  m.red = reinterpret_cast<float*>(raw + off);
+  off += 4 * kWarps;
+  m.ctl = reinterpret_cast<int*>(raw + off);
   return m;
 }
 
-// Segmented inclusive scan over the pairs of a tile: consumer thread t holds
-// the eight consecutive pairs 8t .. 8t+7 (key, value); a run is a maximal
-// stretch of equal keys.  `in_key` / `in_val` is a run carried in from
-// before the tile.  On return val[u] is the sum of its run's values up to
-// and including pair u, and next_key the key of the pair after this
-// thread's last (that of thread t+1's first pair; `tail_key` for the last
-// thread).  Fixed order of additions: within a thread left to right, then a
-// fixed shuffle tree, then the warps in order.
-__device__ __forceinline__ void seg_scan8(const int (&key)[kPerThread], float (&val)[kPerThread], int in_key,
-                                          float in_val, int tail_key, int& next_key, const StepSmem& sm) {
-  const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
-  sm.keys[t] = key[0];
-  sm.keys_last[t] = key[kPerThread - 1];
-  consumer_bar();
-  const int prev_key = t == 0 ? in_key : sm.keys_last[t - 1];
-  next_key = t + 1 < kConsumers ? sm.keys[t + 1] : tail_key;
+// Segmented inclusive scan over one warp's sub-tile: lane l holds the eight
+// consecutive pairs 8l .. 8l+7 (key, value); a run is a maximal stretch of
+// equal keys, and nothing is carried in from before the sub-tile.  On
+// return val[u] is the sum of its run's values from the run's first pair in
+// the sub-tile up to and including pair u; next_key is the key of the pair
+// after this lane's last (kNoKey after the sub-tile's last pair).  Fixed
+// order of additions: within a lane left to right, then a fixed shuffle
+// tree over the lanes.
+__device__ __forceinline__ void seg_scan_warp(const int (&key)[kPerThread], float (&val)[kPerThread], int& next_key) {
+  const int lane = threadIdx.x & 31;
+  int prev_key = __shfl_up_sync(kFull, key[kPerThread - 1], 1);
+  if (lane == 0) prev_key = kNoKey - 1;
+  next_key = __shfl_down_sync(kFull, key[0], 1);
+  if (lane == 31) next_key = kNoKey;
   bool any_head = false;
   int pk = prev_key;
 #pragma unroll
@@ -266,7 +264,7 @@ __device__ __forceinline__ void seg_scan8(const int (&key)[kPerThread], float (&
     any_head = any_head || head;
     pk = key[u];
   }
-  // inclusive scan over the warp of (a head seen, running value of the last run)
+  // inclusive scan over the lanes of (a head seen, running value of the last run)
   float v = val[kPerThread - 1];
   int f = any_head ? 1 : 0;
 #pragma unroll
@@ -278,27 +276,16 @@ __device__ __forceinline__ void seg_scan8(const int (&key)[kPerThread], float (&
       f |= fo;
     }
   }
-  if (lane == 31) {
-    sm.wval[warp] = v;
-    sm.wflag[warp] = f;
-  }
-  float ev = __shfl_up_sync(kFull, v, 1);      // exclusive: the lanes before this one
-  const int ef = __shfl_up_sync(kFull, f, 1);
-  consumer_bar();
-  float pv = in_val;                           // the carried run, then the earlier warps
-  for (int w = 0; w < warp; ++w) pv = sm.wflag[w] ? sm.wval[w] : pv + sm.wval[w];
-  if (lane == 0)
-    ev = pv;
-  else if (!ef)
-    ev += pv;
-  pk = prev_key;
+  const float ev = __shfl_up_sync(kFull, v, 1);   // the run through the previous lane's last pair
+  if (lane > 0) {
+    pk = prev_key;
 #pragma unroll
-  for (int u = 0; u < kPerThread; ++u) {       // pairs before this thread's first head
-    if (key[u] != pk) break;
-    val[u] += ev;
-    pk = key[u];
+    for (int u = 0; u < kPerThread; ++u) {        // pairs before this lane's first head
+      if (key[u] != pk) break;
+      val[u] += ev;
+      pk = key[u];
+    }
   }
-  consumer_bar();   // sm.keys / wval are reused by the next scan
 }
 
 template <int LOSS>
@@ -321,32 +308,42 @@ __global__ void __launch_bounds__(kLocalStepThreads, 1) k_local_step(const Local
   const int lo = bnd[q], hi = bnd[q + 1];
   const int T0 = lo & ~7;                      // 16-byte aligned start of the first column tile
   const int n2 = hi > lo ? (hi - T0 + kTileEntries - 1) / kTileEntries : 0;
-  float* mpart = big ? a.mpart_big + (static_cast<size_t>(i) * Q + q) * a.B : sm.mpart;
-  float* rr = big ? a.r_big + (static_cast<size_t>(i) * Q + q) * a.B : sm.r;
+  // per-warp partial margins (warp w's row at w B) and r: in shared memory,
+  // or for large minibatches in global scratch; the two kinds of pointer
+  // are kept apart so that shared accesses stay shared-memory instructions
+  float* gpart = a.mpart_big + (static_cast<size_t>(i) * Q + q) * kWarps * a.B;
+  float* grr = a.r_big + (static_cast<size_t>(i) * Q + q) * a.B;
 
   if (tid == 0) {
     for (int st = 0; st < a.stages; ++st) {
       mbar_init(sm.full + st, 1);
-      mbar_init(sm.empty + st, kConsumers / 32);
+      mbar_init(sm.empty + st, kWarps);
       mbar_init(sm.gath + st, 32);
     }
-    sm.ctl[0] = -1;
-    sm.ctl[1] = 0;
-    sm.carry[0] = 0.f;
+    for (int f = 0; f < kFragRing; ++f) mbar_init(sm.fready + f, kWarps);
+    sm.ctl[0] = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
-  for (int b = tid; b < a.B; b += kLocalStepThreads) mpart[b] = 0.f;
+  for (int b = tid; b < kWarps * a.B; b += kLocalStepThreads) {
+    if (big) gpart[b] = 0.f;
+    else sm.mpart[b] = 0.f;
+  }
   __syncthreads();
   // The stochastic reduce that follows is a programmatic dependent: its CTAs
   // may take SMs as this grid drains; it waits for this grid's results.
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  // This grid is itself a programmatic dependent of the previous round's
+  // reduce, which may still be running: everything above and the issuer's
+  // bulk copies touch only this step's own (static) batch block; the gather
+  // and consumer warps wait for the previous grid before they read the
+  // exported w values or write anything it reads (column sums, loss).
 
   bool ok = true;
-  if (warp == kConsumers / 32) {
-    // ================= producer warp =================
-    // Issues every tile of both passes in order; it arrives on the cluster
-    // barrier between the passes as soon as pass 1 is issued, so that it
-    // never holds up the consumers there.
+  if (warp == kIssuerWarp) {
+    // ================= issuer warp =================
+    // Lane 0 issues every tile of both passes in order as stages come free;
+    // the warp arrives on the cluster barrier between the passes once pass 1
+    // is issued, so that it never holds up the consumers there.
     auto issue = [&](int it) -> bool {
       const int st = it % a.stages;
       if (it >= a.stages && !mbar_wait_bounded(sm.empty + st, ((it / a.stages) - 1) & 1)) return false;
@@ -366,61 +363,73 @@ __global__ void __launch_bounds__(kLocalStepThreads, 1) k_local_step(const Local
       }
       return true;
     };
-    // The w values of margin tile k: once its list positions have landed,
-    // every lane gathers 32 of them with 4-byte asynchronous copies and
-    // arrives on gath[k] when they are in.
-    auto gather = [&](int k) -> bool {
-      const int st = k % a.stages;
-      if (!mbar_wait_bounded(sm.full + st, (k / a.stages) & 1)) return false;
-      unsigned char* base = sm.stage0 + kStageBytes * st;
-      const int* spos = reinterpret_cast<const int*>(base);
-      float* wvs = reinterpret_cast<float*>(base + 12 * kTileEntries);
-      const int len = min(kTileEntries, nnz - (s0 + k) * kTileEntries);
-      for (int j = lane; j < len; j += 32) cp_async4(wvs + j, a.wv + spos[j]);
-      cp_async_arrive(sm.gath + st);
-      return true;
-    };
     bool pok = true;
-    for (int it = 0; it < n1 && pok; ++it) {
-      if (lane == 0) pok = issue(it);
-      pok = __shfl_sync(kFull, pok, 0) != 0;
-      if (pok && it > 0) pok = __all_sync(kFull, gather(it - 1));
-    }
-    if (pok && n1 > 0) pok = __all_sync(kFull, gather(n1 - 1));
+    if (lane == 0)
+      for (int it = 0; it < n1 && pok; ++it) pok = issue(it);
     __syncwarp();
     asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
     if (lane == 0) {
       for (int it = n1; it < n1 + n2 && pok; ++it) pok = issue(it);
-      if (!pok) sm.ctl[1] = 1;
+      if (!pok) sm.ctl[0] = 1;
     }
     __syncwarp();
     asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+  } else if (warp == kGatherWarp) {
+    // ================= gather warp =================
+    // As soon as margin tile k has landed, every lane gathers 32 of its w
+    // values with 4-byte asynchronous copies, each over the list position
+    // it was addressed by (read before the copy is issued), and arrives on
+    // gath[k] when they are in: the gathers of the next tiles run while the
+    // consumers work on this one.
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    bool gok = true;
+    for (int k = 0; k < n1 && gok; ++k) {
+      const int st = k % a.stages;
+      gok = __all_sync(kFull, mbar_wait_bounded(sm.full + st, (k / a.stages) & 1));
+      if (!gok) break;
+      int* spos = reinterpret_cast<int*>(sm.stage0 + kStageBytes * st);
+      const int len = min(kTileEntries, nnz - (s0 + k) * kTileEntries);
+      for (int j = lane; j < len; j += 32) cp_async4(spos + j, a.wv + spos[j]);
+      cp_async_arrive(sm.gath + st);
+    }
+    if (!gok && lane == 0) sm.ctl[0] = 1;
+    __syncwarp();
+    asm volatile("barrier.cluster.arrive.release.aligned;\nbarrier.cluster.wait.acquire.aligned;" ::: "memory");
   } else {
     // ================= consumer warps =================
-    const int j0 = tid * kPerThread;           // this thread's pairs within a tile
+    // Warp w takes entries [256 w, 256 w + 256) of every tile (its sub-tile)
+    // and works through the tiles on its own: it meets the other consumer
+    // warps only at the ring's mbarriers and between the passes.
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    const int sub = warp * kSlotSegment;       // the warp's sub-tile within a tile
+    const int j0 = sub + lane * kPerThread;    // this lane's eight consecutive pairs
+    float* wprod = sm.prod + sub;
+    int* wokey = sm.okey + sub;
+    const size_t wrow = static_cast<size_t>(warp) * a.B;   // this warp's partial margins
     // ---- pass 1: products by slot; each row's sum by a scan over the slots ----
-    for (int it = 0; it < n1 && ok; ++it) {
+    for (int it = 0; it < n1; ++it) {
       const int st = it % a.stages;
-      ok = consumer_bar_and(mbar_wait_bounded(sm.gath + st, (it / a.stages) & 1));
+      ok = __all_sync(kFull, mbar_wait_bounded(sm.gath + st, (it / a.stages) & 1));
       if (!ok) break;
       const unsigned char* base = sm.stage0 + kStageBytes * st;
       const float* sval = reinterpret_cast<const float*>(base + 4 * kTileEntries);
       const uint16_t* sslot = reinterpret_cast<const uint16_t*>(base + 8 * kTileEntries);
       const uint16_t* srow = reinterpret_cast<const uint16_t*>(base + 10 * kTileEntries);
-      const float* wvs = reinterpret_cast<const float*>(base + 12 * kTileEntries);
+      const float* wvs = reinterpret_cast<const float*>(base);   // gathered over the positions
       const int len = min(kTileEntries, nnz - (s0 + it) * kTileEntries);
-#pragma unroll
-      for (int u = 0; u < kPerThread; ++u) {   // entry u * 128 + t: consecutive threads, consecutive entries
-        const int j = u * kConsumers + tid;
-        if (j < len) sm.prod[sslot[j]] = sval[j] * wvs[j];
-      }
-      consumer_bar();
+      const bool active = sub < len;           // warp-uniform
       int key[kPerThread];
       float val[kPerThread];
-      {
-        // slots j0 .. j0+7 (a row's slots are adjacent): vector loads
-        const float4 q0 = *reinterpret_cast<const float4*>(sm.prod + j0);
-        const float4 q1 = *reinterpret_cast<const float4*>(sm.prod + j0 + 4);
+      if (active) {
+#pragma unroll
+        for (int u = 0; u < kPerThread; ++u) {   // consecutive lanes, consecutive entries
+          const int j = sub + u * 32 + lane;
+          if (j < len) wprod[sslot[j]] = sval[j] * wvs[j];
+        }
+        __syncwarp();
+        // slots j0 .. j0+7 of the segment (a row's slots are adjacent): vector loads
+        const float4 q0 = *reinterpret_cast<const float4*>(wprod + lane * kPerThread);
+        const float4 q1 = *reinterpret_cast<const float4*>(wprod + lane * kPerThread + 4);
         const uint4 rw = *reinterpret_cast<const uint4*>(srow + j0);
         const float pv[8] = {q0.x, q0.y, q0.z, q0.w, q1.x, q1.y, q1.z, q1.w};
         const unsigned rws[4] = {rw.x, rw.y, rw.z, rw.w};
@@ -431,15 +440,35 @@ __global__ void __launch_bounds__(kLocalStepThreads, 1) k_local_step(const Local
           val[u] = in ? pv[u] : 0.f;
         }
       }
-      int next_key;
-      seg_scan8(key, val, -2, 0.f, -1, next_key, sm);
-#pragma unroll
-      for (int u = 0; u < kPerThread; ++u) {
-        const int nk = u + 1 < kPerThread ? key[u + 1] : next_key;
-        if (key[u] >= 0 && nk != key[u]) mpart[key[u]] += val[u];   // a row's run ends: its partial
-      }
-      consumer_bar();
+      __syncwarp();                            // the stage and wprod are read
       if (lane == 0) mbar_arrive(sm.empty + st);
+      if (active) {
+        int next_key;
+        seg_scan_warp(key, val, next_key);
+        // A row's slots form one run per segment: each run end adds the
+        // row's partial to the warp's own margins (no other warp writes them).
+#pragma unroll
+        for (int u = 0; u < kPerThread; ++u) {
+          const int nk = u + 1 < kPerThread ? key[u + 1] : next_key;
+          if (key[u] >= 0 && nk != key[u]) {
+            if (big) gpart[wrow + key[u]] += val[u];
+            else sm.mpart[wrow + key[u]] += val[u];
+          }
+        }
+      }
+    }
+    // ---- the CTA's partial margins: the four warps' rows added in order ----
+    consumer_bar();
+    for (int b = tid; b < a.B; b += kConsumers) {
+      if (big) {
+        float m = gpart[b];
+        for (int w = 1; w < kWarps; ++w) m += gpart[static_cast<size_t>(w) * a.B + b];
+        gpart[b] = m;
+      } else {
+        float m = sm.mpart[b];
+        for (int w = 1; w < kWarps; ++w) m += sm.mpart[static_cast<size_t>(w) * a.B + b];
+        sm.mpart[b] = m;
+      }
     }
     // ---- the worker's margins: the Q partials of every row in rank order ----
     if (big) __threadfence();
@@ -449,10 +478,11 @@ __global__ void __launch_bounds__(kLocalStepThreads, 1) k_local_step(const Local
     for (int b = tid; b < a.B; b += kConsumers) {
       float m = 0.f;
       for (int qq = 0; qq < Q; ++qq)
-        m += big ? __ldcg(a.mpart_big + (static_cast<size_t>(i) * Q + qq) * a.B + b) : ld_dsmem(sm.mpart + b, qq);
+        m += big ? __ldcg(a.mpart_big + (static_cast<size_t>(i) * Q + qq) * kWarps * a.B + b) : ld_dsmem(sm.mpart + b, qq);
       float l, r;
       loss_and_r<LOSS>(y[b], m * a.mscale, l, r);
-      rr[b] = r;
+      if (big) grr[b] = r;
+      else sm.r[b] = r;
       lsum += l;
     }
     if (q == 0) {
@@ -462,16 +492,23 @@ __global__ void __launch_bounds__(kLocalStepThreads, 1) k_local_step(const Local
     consumer_bar();
     if (q == 0 && tid == 0) {
       float tot = 0.f;
-      for (int w2 = 0; w2 < kConsumers / 32; ++w2) tot += sm.red[w2];
+      for (int w2 = 0; w2 < kWarps; ++w2) tot += sm.red[w2];
       a.loss_part[i] = tot;
     }
-    ok = ok && !sm.ctl[1];
-    // ---- pass 2: column sums over [lo, hi), a run carried across tiles ----
+    ok = ok && !sm.ctl[0];
+    // ---- pass 2: column sums over [lo, hi) ----
+    // Runs that end inside a warp's sub-tile are complete and stored by the
+    // warp.  The run through a sub-tile's first pair and the run through its
+    // last may continue in the neighbouring sub-tiles: they are left as
+    // fragments, which warp 0 adds up in sub-tile order once every warp is
+    // through the tile (the CTA's range starts and ends at column bounds).
     float* g = a.gsum;
+    int open_key = kNoKey;                     // warp 0, lane 0: the run the fragments continue
+    float open_sum = 0.f;
     for (int k = 0; k < n2 && ok; ++k) {
       const int it = n1 + k;
       const int st = it % a.stages;
-      ok = consumer_bar_and(mbar_wait_bounded(sm.full + st, (it / a.stages) & 1));
+      ok = __all_sync(kFull, mbar_wait_bounded(sm.full + st, (it / a.stages) & 1));
       if (!ok) break;
       const unsigned char* base = sm.stage0 + kStageBytes * st;
       const int* spos = reinterpret_cast<const int*>(base);
@@ -494,51 +531,75 @@ __global__ void __launch_bounds__(kLocalStepThreads, 1) k_local_step(const Local
         const bool valid = e >= lo && e < hi;
         const int row = static_cast<int>((rws[u >> 1] >> (16 * (u & 1))) & 0xffffu);
         key[u] = valid ? pk[u] : -1;
-        val[u] = valid ? (big ? __ldcg(rr + row) : sm.r[row]) * pv[u] : 0.f;
+        val[u] = valid ? (big ? __ldcg(grr + row) : sm.r[row]) * pv[u] : 0.f;
       }
-      const int in_key = sm.ctl[0];
-      const float in_val = sm.carry[0];
-      const bool last_tile = k == n2 - 1;
+      __syncwarp();
+      if (lane == 0) mbar_arrive(sm.empty + st);   // the stage is read
       int next_key;
-      // after the last tile the range ends at a column boundary; otherwise the
-      // run through the tile's last pair may go on in the next tile
-      seg_scan8(key, val, in_key, in_val, last_tile ? -1 : -3, next_key, sm);
-      if (tid == 0 && in_key >= 0 && key[0] != in_key) g[in_key] = in_val;   // the carried run ended before this tile
-      // Every run that ends in the tile leaves (position, sum) at its last
-      // pair; the sums are then written with consecutive threads on
-      // consecutive pairs, so that the stores coalesce.
-      {
-        int ok8[kPerThread];
-#pragma unroll
-        for (int u = 0; u < kPerThread; ++u) {
-          const int nk = u + 1 < kPerThread ? key[u + 1] : next_key;
-          ok8[u] = (key[u] >= 0 && nk != key[u] && nk != -3) ? key[u] : -1;
-        }
-        *reinterpret_cast<int4*>(sm.okey + j0) = make_int4(ok8[0], ok8[1], ok8[2], ok8[3]);
-        *reinterpret_cast<int4*>(sm.okey + j0 + 4) = make_int4(ok8[4], ok8[5], ok8[6], ok8[7]);
-        *reinterpret_cast<float4*>(sm.prod + j0) = make_float4(val[0], val[1], val[2], val[3]);
-        *reinterpret_cast<float4*>(sm.prod + j0 + 4) = make_float4(val[4], val[5], val[6], val[7]);
-      }
-      consumer_bar();
+      seg_scan_warp(key, val, next_key);
+      const int first_key = __shfl_sync(kFull, key[0], 0);
+      const int last_key = __shfl_sync(kFull, key[kPerThread - 1], 31);
+      const int fr = (k % kFragRing) * kWarps * 2 + warp * 2;
+      int ok8[kPerThread];
 #pragma unroll
       for (int u = 0; u < kPerThread; ++u) {
-        const int j = u * kConsumers + tid;
-        const int k = sm.okey[j];
-        if (k >= 0) g[k] = sm.prod[j];
+        const int nk = u + 1 < kPerThread ? key[u + 1] : next_key;
+        const bool end = key[u] >= 0 && nk != key[u];
+        const bool at_last = lane == 31 && u == kPerThread - 1;
+        ok8[u] = -1;
+        if (end) {
+          if (at_last) {                       // the run through the last pair
+            sm.fkey[fr + 1] = key[u];
+            sm.fval[fr + 1] = val[u];
+          } else if (key[u] == first_key) {    // the run through the first pair
+            sm.fkey[fr] = key[u];
+            sm.fval[fr] = val[u];
+          } else {
+            ok8[u] = key[u];
+          }
+        }
       }
-      if (tid == kConsumers - 1) {             // carry the tile's last run
-        const bool open = !last_tile && key[kPerThread - 1] >= 0;
-        sm.ctl[0] = open ? key[kPerThread - 1] : -1;
-        sm.carry[0] = open ? val[kPerThread - 1] : 0.f;
+      // sub-tile edges without a fragment
+      if (lane == 0 && (first_key < 0 || first_key == last_key)) sm.fkey[fr] = kNoKey;
+      if (lane == 31 && last_key < 0) sm.fkey[fr + 1] = kNoKey;
+      // complete runs: stored with consecutive lanes on consecutive pairs
+      *reinterpret_cast<int4*>(wokey + lane * kPerThread) = make_int4(ok8[0], ok8[1], ok8[2], ok8[3]);
+      *reinterpret_cast<int4*>(wokey + lane * kPerThread + 4) = make_int4(ok8[4], ok8[5], ok8[6], ok8[7]);
+      *reinterpret_cast<float4*>(wprod + lane * kPerThread) = make_float4(val[0], val[1], val[2], val[3]);
+      *reinterpret_cast<float4*>(wprod + lane * kPerThread + 4) = make_float4(val[4], val[5], val[6], val[7]);
+      __syncwarp();
+      if (lane == 0) mbar_arrive(sm.fready + (k % kFragRing));   // releases the fragments to warp 0
+#pragma unroll
+      for (int u = 0; u < kPerThread; ++u) {
+        const int j = u * 32 + lane;
+        const int kk = wokey[j];
+        if (kk >= 0) g[kk] = wprod[j];
       }
-      consumer_bar();
-      if (lane == 0) mbar_arrive(sm.empty + st);
+      if (warp == 0) {
+        ok = __all_sync(kFull, mbar_wait_bounded(sm.fready + (k % kFragRing), (k / kFragRing) & 1));
+        if (ok && lane == 0) {
+          for (int f = 0; f < kWarps * 2; ++f) {
+            const int fk = sm.fkey[(k % kFragRing) * kWarps * 2 + f];
+            if (fk == kNoKey) continue;
+            const float fv = sm.fval[(k % kFragRing) * kWarps * 2 + f];
+            if (fk == open_key) {
+              open_sum += fv;
+            } else {
+              if (open_key >= 0) g[open_key] = open_sum;
+              open_key = fk;
+              open_sum = fv;
+            }
+          }
+        }
+      }
+      __syncwarp();                            // wokey / wprod are reused by the next sub-tile
     }
-    if (!ok && tid == 0) record_error(a.st, ASAP_ERR_CUDA, static_cast<unsigned>(i), a.round);
+    if (warp == 0 && lane == 0 && ok && open_key >= 0) g[open_key] = open_sum;
+    if (!ok && lane == 0) record_error(a.st, ASAP_ERR_CUDA, static_cast<unsigned>(i), a.round);
   }
   // ---- NOTIFY: every CTA's column sums are visible, then CTA 0 publishes ----
   __threadfence();
-  const int all_ok = __syncthreads_or(!ok || sm.ctl[1]) == 0;
+  const int all_ok = __syncthreads_or(!ok || sm.ctl[0]) == 0;
   asm volatile("barrier.cluster.arrive.release.aligned;\nbarrier.cluster.wait.acquire.aligned;" ::: "memory");
   if (q == 0 && tid == 0 && a.notify && i != a.skip_worker) {
     __threadfence();
@@ -631,8 +692,8 @@ cudaError_t launch_apply_update(float* W, int64_t ld, const uint32_t* list, cons
 
 size_t local_step_smem_bytes(int B, int stages) {
   const size_t b_smem = B > kRSmemRows ? 0 : static_cast<size_t>(B);
-  return 128 + kStageBytes * stages + 24 * static_cast<size_t>(stages) + 16 + 8 * kTileEntries + 8 * b_smem +
-         8 * kConsumers + 12 * (kConsumers / 32) + 12;
+  return 128 + kStageBytes * stages + 24 * static_cast<size_t>(stages) + 8 * kFragRing + 16 + 8 * kTileEntries +
+         4 * (kWarps + 1) * b_smem + 8 * kFragRing * kWarps * 2 + 4 * kWarps + 4;
 }
 
 cudaError_t local_step_configure(size_t smem) {
@@ -649,13 +710,17 @@ cudaError_t launch_local_step(const LocalStepArgs& a, int loss, size_t smem, cud
   cfg.blockDim = dim3(kLocalStepThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = a.Q;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  // a programmatic dependent of the kernel before it (the previous round's
+  // reduce): the kernel waits for that grid itself (griddepcontrol.wait)
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   if (loss == ASAP_LOSS_HINGE) return cudaLaunchKernelEx(&cfg, k_local_step<ASAP_LOSS_HINGE>, a);
   return cudaLaunchKernelEx(&cfg, k_local_step<ASAP_LOSS_LOGISTIC>, a);
 }

@@ -20,7 +20,7 @@ def _view(img, off, dtype, n):
 @pytest.mark.parametrize("S,Q,max_len", [(64, 1, 40), (1024, 3, 40), (64, 8, 400)])
 def test_batch_image_matches_the_shards(S, Q, max_len):
     # max_len 400 with B = 20 rows: about 3,400 entries, so minibatches span
-    # more than one 1024-entry margin segment
+    # more than one 256-entry margin segment and 1024-entry tile
     N, d, B, t = 3, 1000, 20, 1
     rng = np.random.default_rng(8)
     lengths = [np.where(rng.random(3 * B) < 0.15, 0, rng.integers(1, max_len, 3 * B)) for _ in range(N)]
@@ -55,12 +55,12 @@ def test_batch_image_matches_the_shards(S, Q, max_len):
         for e, (c, _, _) in enumerate(entries):
             p = int(cp[e])
             assert lst[p] == (i << 16) | (c % S) and soff[c // S] <= p < soff[c // S + 1]
-        # margin segments of 1024 entries: slots numbered row by row, by
+        # margin segments of 256 entries: slots numbered row by row, by
         # column within a row; srow holds the row of every slot
         cs = _view(img, cs_o, np.uint16, nnz)
         sr = _view(img, sr_o, np.uint16, nnz)
-        for e0 in range(0, nnz, 1024):
-            e1 = min(e0 + 1024, nnz)
+        for e0 in range(0, nnz, 256):
+            e1 = min(e0 + 256, nnz)
             seg = sorted(range(e0, e1), key=lambda e: (entries[e][1], entries[e][0]))
             assert [int(cs[e]) for e in seg] == list(range(e1 - e0))
             assert [int(v) for v in sr[e0:e1]] == [entries[e][1] for e in seg]

@@ -231,6 +231,7 @@ __device__ __forceinline__ StepSmem carve_step(unsigned char* raw, int B, int st
   off += 4 * static_cast<size_t>(kWarps) * B;
   m.r = reinterpret_cast<float*>(raw + off);
   off += 4 * static_cast<size_t>(B);
+  off = (off + 15) & ~static_cast<size_t>(15);             // fragments are read as 16-byte vectors
   m.fkey = reinterpret_cast<int*>(raw + off);
   off += 4 * kFragRing * kWarps * 2;
   m.fval = reinterpret_cast<float*>(raw + off);
@@ -389,7 +390,19 @@ __global__ void __launch_bounds__(kLocalStepThreads, 1) k_local_step(const Local
       if (!gok) break;
       int* spos = reinterpret_cast<int*>(sm.stage0 + kStageBytes * st);
       const int len = min(kTileEntries, nnz - (s0 + k) * kTileEntries);
-      for (int j = lane; j < len; j += 32) cp_async4(spos + j, a.wv + spos[j]);
+      // four consecutive positions per lane and vector load, two loads ahead
+      // of their copies, so that no copy waits on its own position's load
+      for (int j0 = lane * 4; j0 < len; j0 += 256) {
+        const int j1 = j0 + 128;
+        const int4 p0 = *reinterpret_cast<const int4*>(spos + j0);
+        const int4 p1 = j1 < len ? *reinterpret_cast<const int4*>(spos + j1) : make_int4(0, 0, 0, 0);
+        const int pp[8] = {p0.x, p0.y, p0.z, p0.w, p1.x, p1.y, p1.z, p1.w};
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          const int j = (u < 4 ? j0 : j1) + (u & 3);
+          if (j < len) cp_async4(spos + j, a.wv + pp[u]);
+        }
+      }
       cp_async_arrive(sm.gath + st);
     }
     if (!gok && lane == 0) sm.ctl[0] = 1;
@@ -578,10 +591,19 @@ __global__ void __launch_bounds__(kLocalStepThreads, 1) k_local_step(const Local
       if (warp == 0) {
         ok = __all_sync(kFull, mbar_wait_bounded(sm.fready + (k % kFragRing), (k / kFragRing) & 1));
         if (ok && lane == 0) {
-          for (int f = 0; f < kWarps * 2; ++f) {
-            const int fk = sm.fkey[(k % kFragRing) * kWarps * 2 + f];
+          static_assert(kWarps * 2 == 8, "a tile leaves eight fragments");
+          const int fb = (k % kFragRing) * kWarps * 2;
+          const int4 k0 = *reinterpret_cast<const int4*>(sm.fkey + fb);
+          const int4 k1 = *reinterpret_cast<const int4*>(sm.fkey + fb + 4);
+          const float4 v0 = *reinterpret_cast<const float4*>(sm.fval + fb);
+          const float4 v1 = *reinterpret_cast<const float4*>(sm.fval + fb + 4);
+          const int fks[8] = {k0.x, k0.y, k0.z, k0.w, k1.x, k1.y, k1.z, k1.w};
+          const float fvs[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
+#pragma unroll
+          for (int f = 0; f < 8; ++f) {
+            const int fk = fks[f];
             if (fk == kNoKey) continue;
-            const float fv = sm.fval[(k % kFragRing) * kWarps * 2 + f];
+            const float fv = fvs[f];
             if (fk == open_key) {
               open_sum += fv;
             } else {
@@ -693,7 +715,7 @@ cudaError_t launch_apply_update(float* W, int64_t ld, const uint32_t* list, cons
 size_t local_step_smem_bytes(int B, int stages) {
   const size_t b_smem = B > kRSmemRows ? 0 : static_cast<size_t>(B);
   return 128 + kStageBytes * stages + 24 * static_cast<size_t>(stages) + 8 * kFragRing + 16 + 8 * kTileEntries +
-         4 * (kWarps + 1) * b_smem + 8 * kFragRing * kWarps * 2 + 4 * kWarps + 4;
+         4 * (kWarps + 1) * b_smem + 16 + 8 * kFragRing * kWarps * 2 + 4 * kWarps + 4;
 }
 
 cudaError_t local_step_configure(size_t smem) {

@@ -1241,7 +1241,7 @@ asap_status asap_load_dense_shards(asap_ctx* c, const uint16_t* const* X, const 
   {
     cuuint64_t dims[2] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(N) * rows};
     cuuint64_t str[1] = {static_cast<cuuint64_t>(d) * 2};
-    cuuint32_t box[2] = {64, 128};
+    cuuint32_t box[2] = {64, 32};   // 32-row parts, multicast across the forward kernel's cluster
     asap_status s = bf16_map(c, &c->tmX, c->X, 2, dims, str, box);
     if (s != ASAP_OK) return s;
   }

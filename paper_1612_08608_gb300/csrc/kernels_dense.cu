@@ -92,6 +92,18 @@ __device__ __forceinline__ void tma_2d(void* dst, const CUtensorMap* m, uint64_t
       :: "r"(smem_u32(dst)), "l"(reinterpret_cast<uint64_t>(m)), "r"(x), "r"(y), "r"(smem_u32(bar)) : "memory");
 }
 
+// The same 2-D load, written to the same shared-memory offset of every CTA of
+// the cluster in `mask` and completing on the mbarrier at `bar`'s offset in
+// each of them (the CTAs read the same tile of this GPU's memory).
+__device__ __forceinline__ void tma_2d_multicast(void* dst, const CUtensorMap* m, uint64_t* bar, int x, int y,
+                                                 uint16_t mask) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.multicast::cluster"
+      " [%0], [%1, {%2, %3}], [%4], %5;"
+      :: "r"(smem_u32(dst)), "l"(reinterpret_cast<uint64_t>(m)), "r"(x), "r"(y), "r"(smem_u32(bar)), "h"(mask)
+      : "memory");
+}
+
 __device__ __forceinline__ void tma_3d(void* dst, const CUtensorMap* m, uint64_t* bar, int x, int y, int z) {
   asm volatile(
       "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], [%5];"
@@ -131,6 +143,13 @@ __device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t a_desc, uint
 __device__ __forceinline__ void umma_commit(uint64_t* bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" :: "r"(smem_u32(bar))
                : "memory");
+}
+
+// The same arrival on the mbarrier at `bar`'s offset in every CTA of the
+// cluster in `mask`.
+__device__ __forceinline__ void umma_commit_multicast(uint64_t* bar, uint16_t mask) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;"
+               :: "r"(smem_u32(bar)), "h"(mask) : "memory");
 }
 
 // 32 consecutive fp32 accumulator columns of this thread's TMEM lane.
@@ -188,8 +207,12 @@ __device__ __forceinline__ void st_dsmem_f32(float* local, uint32_t rank, float 
   asm volatile("st.shared::cluster.f32 [%0], %1;" :: "r"(remote), "f"(v) : "memory");
 }
 
-__device__ __forceinline__ uintptr_t align1024(const void* raw) {
-  return (reinterpret_cast<uintptr_t>(raw) + 1023) & ~static_cast<uintptr_t>(1023);
+// Offset of the first 1024-byte aligned byte of the dynamic shared memory.
+// Regions are then formed from the base pointer by pointer arithmetic (no
+// integer round trip of the address), so that the compiler keeps them in
+// the shared address space and emits plain shared-memory accesses.
+__device__ __forceinline__ size_t align1024_off(const unsigned char* raw) {
+  return (1024u - (smem_u32(raw) & 1023u)) & 1023u;
 }
 
 // Relaxed arrival on the mbarrier at `local`'s offset in the shared memory of
@@ -217,7 +240,7 @@ __device__ __forceinline__ bool mbar_wait_cluster(uint64_t* bar, uint32_t parity
 
 // Barrier among the epilogue warps (barrier 1) that also returns the OR of
 // `v` over them, so that they take every decision together.
-constexpr int kEpiWarps = 8;                           // forward epilogue warps: two per TMEM lane quarter
+constexpr int kEpiWarps = 16;                          // forward epilogue warps: four per TMEM lane quarter
 constexpr int kEpiParts = kEpiWarps / 4;               // column parts of a row
 constexpr int kEpiChunks = kTileN / 32 / kEpiParts;    // 32-column chunks per epilogue thread
 
@@ -249,6 +272,9 @@ __device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, %0;" :: "n
 //               reads local shared memory; then R = (softmax - onehot) / B is
 //               written to R^T from registers.
 constexpr int kFwdThreads = (2 + kEpiWarps) * 32;
+// X tiles are loaded in 32-row parts (4 KB each, 1024-byte aligned under the 128-byte swizzle)
+constexpr int kXPart = 32;
+constexpr uint32_t kXPartBytes = kXPart * kTileK * 2;
 constexpr int kMaxCq = 4;                                       // C <= 1024
 constexpr int kStatsSlot = kMaxCq * kEpiParts * 2 * kTileM;     // floats per stats slot
 
@@ -271,24 +297,24 @@ constexpr size_t fwd_smem_bytes() {
 }
 
 __device__ __forceinline__ FwdSmem fwd_carve(unsigned char* raw) {
-  uintptr_t p = align1024(raw);
+  size_t p = align1024_off(raw);
   FwdSmem s;
-  s.a = reinterpret_cast<unsigned char*>(p);
+  s.a = raw + p;
   p += kFwdStages * kABytes;
-  s.b = reinterpret_cast<unsigned char*>(p);
+  s.b = raw + p;
   p += kFwdStages * kBBytes;
-  s.stats = reinterpret_cast<float*>(p);
+  s.stats = reinterpret_cast<float*>(raw + p);
   p += 4 * kStatsSlot * 2;
-  s.full = reinterpret_cast<uint64_t*>(p);
+  s.full = reinterpret_cast<uint64_t*>(raw + p);
   s.empty = s.full + kFwdStages;
   s.acc_full = s.empty + kFwdStages;
   s.acc_empty = s.acc_full + 2;
   s.st_full = s.acc_empty + 2;
   s.st_free = s.st_full + 2;
   p += 8 * (2 * kFwdStages + 8);
-  s.tmem_slot = reinterpret_cast<uint32_t*>(p);
+  s.tmem_slot = reinterpret_cast<uint32_t*>(raw + p);
   p += 16;
-  s.red = reinterpret_cast<float*>(p);
+  s.red = reinterpret_cast<float*>(raw + p);
   return s;
 }
 
@@ -304,11 +330,12 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
   const int n_my = total > cl_id ? (total - cl_id + n_clusters - 1) / n_clusters : 0;
   const int k_tiles = a.d / kTileK;
   const int c0 = q * kTileN;
+  const uint16_t cmask = static_cast<uint16_t>((1u << Cq) - 1u);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kFwdStages; ++s) {
       mbar_init(sm.full + s, 1);
-      mbar_init(sm.empty + s, 1);
+      mbar_init(sm.empty + s, Cq);                         // every cluster CTA's MMA is done with the stage
     }
     for (int s = 0; s < 2; ++s) {
       mbar_init(sm.acc_full + s, 1);
@@ -341,7 +368,11 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
             break;
           }
           mbar_expect_tx(sm.full + s, kABytes + kBBytes);
-          tma_2d(sm.a + s * kABytes, &tmX, sm.full + s, kt * kTileK, row0);
+          // The X tile is the same for the cluster's CTAs: each loads its
+          // share of the 32-row parts and multicasts it to all of them.
+          for (int j = q; j < kTileM / kXPart; j += Cq)
+            tma_2d_multicast(sm.a + s * kABytes + j * kXPartBytes, &tmX, sm.full + s, kt * kTileK, row0 + j * kXPart,
+                             cmask);
           tma_3d(sm.b + s * kBBytes, &tmW, sm.full + s, kt * kTileK, c0, i);
         }
       }
@@ -375,7 +406,7 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
             const uint64_t bd = smem_desc_sw128(sm.b + s * kBBytes + kk * 32);
             umma_bf16(acc, ad, bd, idesc, (kt | kk) != 0 ? 1u : 0u);
           }
-          umma_commit(sm.empty + s);
+          umma_commit_multicast(sm.empty + s, cmask);   // the stage's X parts came from every CTA
         }
         if (ok) umma_commit(sm.acc_full + ab);
       }
@@ -545,24 +576,24 @@ constexpr size_t grad_smem_bytes() {
 }
 
 __device__ __forceinline__ GradSmem grad_carve(unsigned char* raw) {
-  uintptr_t p = align1024(raw);
+  size_t p = align1024_off(raw);
   GradSmem s;
-  s.a = reinterpret_cast<unsigned char*>(p);
+  s.a = raw + p;
   p += kGradStages * kABytes;
-  s.b = reinterpret_cast<unsigned char*>(p);
+  s.b = raw + p;
   p += kGradStages * kBBytes;
-  s.w = reinterpret_cast<unsigned char*>(p);
+  s.w = raw + p;
   p += kWBufs * kWBoxBytes;
-  s.full = reinterpret_cast<uint64_t*>(p);
+  s.full = reinterpret_cast<uint64_t*>(raw + p);
   s.empty = s.full + kGradStages;
   s.acc_full = s.empty + kGradStages;
   s.acc_empty = s.acc_full + 2;
   s.wfull = s.acc_empty + 2;
   s.wupd = s.wfull + kWBufs;
   p += 8 * (2 * kGradStages + 4 + 2 * kWBufs);
-  s.tmem_slot = reinterpret_cast<uint32_t*>(p);
+  s.tmem_slot = reinterpret_cast<uint32_t*>(raw + p);
   p += 16;
-  s.fail = reinterpret_cast<int*>(p);
+  s.fail = reinterpret_cast<int*>(raw + p);
   return s;
 }
 

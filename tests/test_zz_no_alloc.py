@@ -7,10 +7,11 @@ is checked against the context's own stochastic reduce and against the CPU
 oracle (Eq. A.1, second line, and the consensus error) on two calls in a
 row (the second call starts from the first call's output, so the shared
 scratch array holds the previous call's contents).  After a warm-up call,
-further calls leave the device's free memory and torch's allocation count
-unchanged.  Collected last on purpose: a run that stops at the first
+further calls do not lower the device's free memory and leave torch's
+allocation count unchanged.  Collected last on purpose: a run that stops at the first
 failure has already run every other test."""
 import ctypes as C
+import gc
 
 import numpy as np
 import pytest
@@ -74,13 +75,17 @@ def test_mix_noalloc_matches_stochastic_reduce_twice(N, d, k):
         assert abs(cons.item() - cw) <= 1e-4 * cw + 1e-6, (t, cons.item(), cw)
         prev = got.astype(np.float64)
 
-    # No allocation: free device memory and torch's count stay put.
+    # No allocation: free device memory does not drop and torch's count stays
+    # put.  Contexts of earlier tests are collected first; one released while
+    # the calls run could only raise the free figure, never lower it.
+    gc.collect()
+    torch.cuda.synchronize()
     free0, alloc0 = torch.cuda.mem_get_info()[0], torch.cuda.memory_allocated()
     for t in range(6):
         src, dst = (W_a, W_b) if t % 2 == 0 else (W_b, W_a)
         assert _noalloc(lib, src, dst, N, d, ld, d_nbr, d_wgt, k + 1, cons, stream) == 0
     torch.cuda.synchronize()
-    assert torch.cuda.mem_get_info()[0] == free0
+    assert torch.cuda.mem_get_info()[0] >= free0
     assert torch.cuda.memory_allocated() == alloc0
 
 

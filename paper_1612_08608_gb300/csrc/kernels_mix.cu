@@ -526,6 +526,29 @@ __global__ void __launch_bounds__(kMixThreads, 1) k_mix(const __grid_constant__ 
       const int qoff = (q_t >> lqb) * box_col + (q_t & (QB - 1));   // float4 offset of (row 0, quad q_t)
       const int rows_t = (a.N - g_t + G - 1) / G;
       auto xq = [&](int q) { return (q >> lqb) * box_col + (q & (QB - 1)); };
+      // With a compile-time neighbour count and at most kCacheRows rows per
+      // thread, the neighbour offsets of the thread's rows (its quad folded
+      // in) stay in registers as 16-bit pairs, and an equal weight in one
+      // register: the slab loop then reads only the slab from shared memory.
+      constexpr int kCacheRows = 4;
+      constexpr int kC = KP1 > 0 ? KP1 : 1;
+      constexpr int kPk = (kCacheRows * kC + 1) / 2;
+      const bool cached = KP1 > 0 && rows_t <= kCacheRows;
+      uint32_t pko[kPk];
+#pragma unroll
+      for (int u = 0; u < kPk; ++u) pko[u] = 0u;
+      if (KP1 > 0 && cached) {
+#pragma unroll
+        for (int rr = 0; rr < kCacheRows; ++rr)
+#pragma unroll
+          for (int m = 0; m < kC; ++m) {
+            const int e = rr * kC + m;
+            const uint32_t off = rr < rows_t ? static_cast<uint32_t>(sm.nbr[(g_t + rr * G) * kC + m] + qoff) : 0u;
+            pko[e >> 1] |= (off & 0xffffu) << (16 * (e & 1));
+          }
+      }
+      const bool uni = a.uniform_w != 0;
+      const float wu = uni && KP1 >= 0 ? sm.wgt[0] : 0.f;
       for (long long it = 0; it < n_my; ++it) {
         const long long slab = blockIdx.x + it * stride;
         const int st = static_cast<int>(it % a.stages);
@@ -617,15 +640,43 @@ __global__ void __launch_bounds__(kMixThreads, 1) k_mix(const __grid_constant__ 
             s1 = f4_add(s1, make_float4(dx, dy, dz, dw));
             sq = fmaf(dx, dx, fmaf(dy, dy, fmaf(dz, dz, fmaf(dw, dw, sq))));
           };
-          int r = 0;
-          for (; r + 1 < rows_t; r += 2) {      // two rows in flight
-            const int i0 = g_t + r * G, i1 = i0 + G;
-            const float4 a0 = mix_one(i0);
-            const float4 a1 = mix_one(i1);
-            emit(i0, a0);
-            emit(i1, a1);
+          if (KP1 > 0 && cached) {
+            // the same operations in the same order as mix_one, offsets from registers
+            auto mix_c = [&](int rr) -> float4 {
+              const float* wt = sm.wgt + (g_t + rr * G) * kC;
+              auto xo = [&](int m) {
+                const int e = rr * kC + m;
+                return static_cast<int>((pko[e >> 1] >> (16 * (e & 1))) & 0xffffu);
+              };
+              const float w0 = uni ? wu : wt[0];
+              const float4 xa = x4[xo(0)];
+              float4 acc = make_float4(w0 * xa.x, w0 * xa.y, w0 * xa.z, w0 * xa.w);
+#pragma unroll
+              for (int m = 1; m < kC; ++m) acc = f4_fma(uni ? wu : wt[m], x4[xo(m)], acc);
+              return acc;
+            };
+#pragma unroll
+            for (int rr = 0; rr < kCacheRows; rr += 2) {   // two rows in flight
+              if (rr + 1 < rows_t) {
+                const float4 a0 = mix_c(rr);
+                const float4 a1 = mix_c(rr + 1);
+                emit(g_t + rr * G, a0);
+                emit(g_t + (rr + 1) * G, a1);
+              } else if (rr < rows_t) {
+                emit(g_t + rr * G, mix_c(rr));
+              }
+            }
+          } else {
+            int r = 0;
+            for (; r + 1 < rows_t; r += 2) {      // two rows in flight
+              const int i0 = g_t + r * G, i1 = i0 + G;
+              const float4 a0 = mix_one(i0);
+              const float4 a1 = mix_one(i1);
+              emit(i0, a0);
+              emit(i1, a1);
+            }
+            if (r < rows_t) emit(g_t + r * G, mix_one(g_t + r * G));
           }
-          if (r < rows_t) emit(g_t + r * G, mix_one(g_t + r * G));
           s2 += sq;
           part[tid] = s1;
           if (FUSED) {

@@ -691,8 +691,12 @@ __global__ void __launch_bounds__(kMixThreads, 1) k_mix(const __grid_constant__ 
               const int* nb = sm.nbr + i * kp1;
               const float* wt = sm.wgt + i * kp1;
               const int xo = xq(cl >> 2), comp = cl & 3;
-              float v = wt[0] * x[4 * (nb[0] + xo) + comp];
-              for (int m = 1; m < kp1; ++m) v = fmaf(wt[m], x[4 * (nb[m] + xo) + comp], v);
+              float v = (uni ? wu : wt[0]) * x[4 * (nb[0] + xo) + comp];
+#pragma unroll
+              for (int m = 1; m < (KP1 > 0 ? KP1 : kMaxKp1Sparse); ++m) {
+                if (KP1 == 0 && m >= kp1) break;
+                v = fmaf(uni ? wu : wt[m], x[4 * (nb[m] + xo) + comp], v);
+              }
               st_f32_hint(a.wv_out + xbase + e, v, keep);
             }
           }

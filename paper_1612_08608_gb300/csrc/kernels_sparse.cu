@@ -34,7 +34,8 @@
 //     at column boundaries, in 1024-entry tiles; a warp's segmented scan
 //     keyed by list position sums each column's r_row * val; runs that end
 //     inside the warp's share are stored by the warp, and the two runs at
-//     its edges are fragments that one warp adds up in order.
+//     its edges are fragments that the gather warp, idle by then, adds up
+//     in order.
 // A last cluster barrier and CTA 0 publishes NOTIFY.  No atomics, no waits
 // on other clusters, every sum in a fixed order: the result does not depend
 // on the schedule.
@@ -184,6 +185,7 @@ struct StepSmem {
   uint64_t* empty;
   uint64_t* gath;       // [stages]: the w values of a margin tile are in the stage
   uint64_t* fready;     // [kFragRing]: every warp has left its fragments of a column-sum tile
+  uint64_t* ffree;      // [kFragRing]: the merger has read a slot's fragments
   float* prod;          // [kTileEntries]: warp w uses [256 w, 256 w + 256)
   int* okey;            // [kTileEntries]: list position of a run ending at the pair, else -1
   float* mpart;         // [4][B]: per-warp partial margins (warp 0's row holds the CTA's sum after pass 1)
@@ -199,9 +201,9 @@ struct StepSmem {
 constexpr size_t kStageBytes = static_cast<size_t>(kTileEntries) * 12;
 constexpr int kWarps = kConsumers / 32;
 constexpr int kIssuerWarp = kWarps, kGatherWarp = kWarps + 1;
-// Fragments of a column-sum tile are kept until warp 0 has merged them; a
-// warp runs at most `stages` tiles ahead of warp 0, so the ring needs
-// stages + 2 slots (stages <= 6).
+// Fragments of a column-sum tile wait in a ring until the merger (the gather
+// warp, idle in pass 2) has added them up; a consumer waits for the slot's
+// "free" barrier before it reuses it.
 constexpr int kFragRing = 8;
 constexpr int kNoKey = -2;
 
@@ -221,6 +223,8 @@ __device__ __forceinline__ StepSmem carve_step(unsigned char* raw, int B, int st
   m.gath = reinterpret_cast<uint64_t*>(raw + off);
   off += 8 * stages;
   m.fready = reinterpret_cast<uint64_t*>(raw + off);
+  off += 8 * kFragRing;
+  m.ffree = reinterpret_cast<uint64_t*>(raw + off);
   off += 8 * kFragRing;
   off = (off + 15) & ~static_cast<size_t>(15);             // prod and okey are accessed as 16-byte vectors
   m.prod = reinterpret_cast<float*>(raw + off);
@@ -321,7 +325,10 @@ __global__ void __launch_bounds__(kLocalStepThreads, 1) k_local_step(const Local
       mbar_init(sm.empty + st, kWarps);
       mbar_init(sm.gath + st, 32);
     }
-    for (int f = 0; f < kFragRing; ++f) mbar_init(sm.fready + f, kWarps);
+    for (int f = 0; f < kFragRing; ++f) {
+      mbar_init(sm.fready + f, kWarps);
+      mbar_init(sm.ffree + f, 1);
+    }
     sm.ctl[0] = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -408,6 +415,47 @@ __global__ void __launch_bounds__(kLocalStepThreads, 1) k_local_step(const Local
     if (!gok && lane == 0) sm.ctl[0] = 1;
     __syncwarp();
     asm volatile("barrier.cluster.arrive.release.aligned;\nbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+    // ---- pass 2: the column runs at the edges of the consumer warps' shares,
+    // added up in share order as every warp leaves a tile's fragments ----
+    float* g = a.gsum;
+    int open_key = kNoKey;                     // lane 0: the run the fragments continue
+    float open_sum = 0.f;
+    bool mok = gok;
+    for (int k = 0; k < n2 && mok; ++k) {
+      const int slot = k % kFragRing;
+      mok = __all_sync(kFull, mbar_wait_bounded(sm.fready + slot, (k / kFragRing) & 1));
+      if (!mok) break;
+      if (lane == 0) {
+        static_assert(kWarps * 2 == 8, "a tile leaves eight fragments");
+        const int fb = slot * kWarps * 2;
+        const int4 k0 = *reinterpret_cast<const int4*>(sm.fkey + fb);
+        const int4 k1 = *reinterpret_cast<const int4*>(sm.fkey + fb + 4);
+        const float4 v0 = *reinterpret_cast<const float4*>(sm.fval + fb);
+        const float4 v1 = *reinterpret_cast<const float4*>(sm.fval + fb + 4);
+        const int fks[8] = {k0.x, k0.y, k0.z, k0.w, k1.x, k1.y, k1.z, k1.w};
+        const float fvs[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
+        mbar_arrive(sm.ffree + slot);          // the slot is read
+#pragma unroll
+        for (int f = 0; f < 8; ++f) {
+          const int fk = fks[f];
+          if (fk == kNoKey) continue;
+          const float fv = fvs[f];
+          if (fk == open_key) {
+            open_sum += fv;
+          } else {
+            if (open_key >= 0) g[open_key] = open_sum;
+            open_key = fk;
+            open_sum = fv;
+          }
+        }
+      }
+      __syncwarp();
+    }
+    if (lane == 0 && mok && open_key >= 0) g[open_key] = open_sum;
+    if (!mok && lane == 0) {
+      record_error(a.st, ASAP_ERR_CUDA, static_cast<unsigned>(i), a.round);
+      sm.ctl[0] = 1;
+    }
   } else {
     // ================= consumer warps =================
     // Warp w takes entries [256 w, 256 w + 256) of every tile (its sub-tile)
@@ -489,9 +537,17 @@ __global__ void __launch_bounds__(kLocalStepThreads, 1) k_local_step(const Local
     const float* y = reinterpret_cast<const float*>(a.block + dsc.y);
     float lsum = 0.f;
     for (int b = tid; b < a.B; b += kConsumers) {
+      // the Q partials first, then their sum in rank order: the remote loads overlap
+      float mq[kMaxStepCluster];
+#pragma unroll
+      for (int qq = 0; qq < kMaxStepCluster; ++qq)
+        if (qq < Q)
+          mq[qq] = big ? __ldcg(a.mpart_big + (static_cast<size_t>(i) * Q + qq) * kWarps * a.B + b)
+                       : ld_dsmem(sm.mpart + b, qq);
       float m = 0.f;
-      for (int qq = 0; qq < Q; ++qq)
-        m += big ? __ldcg(a.mpart_big + (static_cast<size_t>(i) * Q + qq) * kWarps * a.B + b) : ld_dsmem(sm.mpart + b, qq);
+#pragma unroll
+      for (int qq = 0; qq < kMaxStepCluster; ++qq)
+        if (qq < Q) m += mq[qq];
       float l, r;
       loss_and_r<LOSS>(y[b], m * a.mscale, l, r);
       if (big) grr[b] = r;
@@ -513,11 +569,10 @@ __global__ void __launch_bounds__(kLocalStepThreads, 1) k_local_step(const Local
     // Runs that end inside a warp's sub-tile are complete and stored by the
     // warp.  The run through a sub-tile's first pair and the run through its
     // last may continue in the neighbouring sub-tiles: they are left as
-    // fragments, which warp 0 adds up in sub-tile order once every warp is
-    // through the tile (the CTA's range starts and ends at column bounds).
+    // fragments, which the gather warp adds up in sub-tile order once every
+    // warp is through the tile (the CTA's range starts and ends at column
+    // bounds).
     float* g = a.gsum;
-    int open_key = kNoKey;                     // warp 0, lane 0: the run the fragments continue
-    float open_sum = 0.f;
     for (int k = 0; k < n2 && ok; ++k) {
       const int it = n1 + k;
       const int st = it % a.stages;
@@ -553,6 +608,11 @@ __global__ void __launch_bounds__(kLocalStepThreads, 1) k_local_step(const Local
       const int first_key = __shfl_sync(kFull, key[0], 0);
       const int last_key = __shfl_sync(kFull, key[kPerThread - 1], 31);
       const int fr = (k % kFragRing) * kWarps * 2 + warp * 2;
+      // the slot's fragments of tile k - kFragRing have been read
+      if (k >= kFragRing) {
+        ok = __all_sync(kFull, mbar_wait_bounded(sm.ffree + (k % kFragRing), ((k / kFragRing) - 1) & 1));
+        if (!ok) break;
+      }
       int ok8[kPerThread];
 #pragma unroll
       for (int u = 0; u < kPerThread; ++u) {
@@ -581,42 +641,15 @@ __global__ void __launch_bounds__(kLocalStepThreads, 1) k_local_step(const Local
       *reinterpret_cast<float4*>(wprod + lane * kPerThread) = make_float4(val[0], val[1], val[2], val[3]);
       *reinterpret_cast<float4*>(wprod + lane * kPerThread + 4) = make_float4(val[4], val[5], val[6], val[7]);
       __syncwarp();
-      if (lane == 0) mbar_arrive(sm.fready + (k % kFragRing));   // releases the fragments to warp 0
+      if (lane == 0) mbar_arrive(sm.fready + (k % kFragRing));   // releases the fragments to the merger
 #pragma unroll
       for (int u = 0; u < kPerThread; ++u) {
         const int j = u * 32 + lane;
         const int kk = wokey[j];
         if (kk >= 0) g[kk] = wprod[j];
       }
-      if (warp == 0) {
-        ok = __all_sync(kFull, mbar_wait_bounded(sm.fready + (k % kFragRing), (k / kFragRing) & 1));
-        if (ok && lane == 0) {
-          static_assert(kWarps * 2 == 8, "a tile leaves eight fragments");
-          const int fb = (k % kFragRing) * kWarps * 2;
-          const int4 k0 = *reinterpret_cast<const int4*>(sm.fkey + fb);
-          const int4 k1 = *reinterpret_cast<const int4*>(sm.fkey + fb + 4);
-          const float4 v0 = *reinterpret_cast<const float4*>(sm.fval + fb);
-          const float4 v1 = *reinterpret_cast<const float4*>(sm.fval + fb + 4);
-          const int fks[8] = {k0.x, k0.y, k0.z, k0.w, k1.x, k1.y, k1.z, k1.w};
-          const float fvs[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
-#pragma unroll
-          for (int f = 0; f < 8; ++f) {
-            const int fk = fks[f];
-            if (fk == kNoKey) continue;
-            const float fv = fvs[f];
-            if (fk == open_key) {
-              open_sum += fv;
-            } else {
-              if (open_key >= 0) g[open_key] = open_sum;
-              open_key = fk;
-              open_sum = fv;
-            }
-          }
-        }
-      }
       __syncwarp();                            // wokey / wprod are reused by the next sub-tile
     }
-    if (warp == 0 && lane == 0 && ok && open_key >= 0) g[open_key] = open_sum;
     if (!ok && lane == 0) record_error(a.st, ASAP_ERR_CUDA, static_cast<unsigned>(i), a.round);
   }
   // ---- NOTIFY: every CTA's column sums are visible, then CTA 0 publishes ----
@@ -714,7 +747,7 @@ cudaError_t launch_apply_update(float* W, int64_t ld, const uint32_t* list, cons
 
 size_t local_step_smem_bytes(int B, int stages) {
   const size_t b_smem = B > kRSmemRows ? 0 : static_cast<size_t>(B);
-  return 128 + kStageBytes * stages + 24 * static_cast<size_t>(stages) + 8 * kFragRing + 16 + 8 * kTileEntries +
+  return 128 + kStageBytes * stages + 24 * static_cast<size_t>(stages) + 16 * kFragRing + 16 + 8 * kTileEntries +
          4 * (kWarps + 1) * b_smem + 16 + 8 * kFragRing * kWarps * 2 + 4 * kWarps + 4;
 }
 

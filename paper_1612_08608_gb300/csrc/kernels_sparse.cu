@@ -22,7 +22,8 @@
 // fetches a margin tile's w values as soon as the tile lands -- while four
 // consumer warps work on the stage that has landed, each on its own
 // 256-entry share of the 1024-entry tile and without CTA-wide barriers:
-//   pass 1 (margins): CTA q takes 1024-entry tiles s = q nseg/Q ...; a
+//   pass 1 (margins): CTA q takes the 256-entry segments s = q nseg/Q ...
+//     in tiles of four; a
 //     warp's products val * wv[pos] go to shared memory at the entry's slot
 //     (slots of a 256-entry segment ordered by row, then column), a
 //     segmented scan over the slots keyed by row sums each row's products
@@ -294,7 +295,7 @@ __device__ __forceinline__ void seg_scan_warp(const int (&key)[kPerThread], floa
 }
 
 template <int LOSS>
-__global__ void __launch_bounds__(kLocalStepThreads, 1) k_local_step(const LocalStepArgs a) {
+__global__ void __launch_bounds__(kLocalStepThreads, 4) k_local_step(const LocalStepArgs a) {   // four CTAs per SM
   extern __shared__ unsigned char step_smem_raw[];
   const bool big = a.B > kRSmemRows;           // partial margins and r in global memory
   const StepSmem sm = carve_step(step_smem_raw, big ? 0 : a.B, a.stages);
@@ -305,10 +306,14 @@ __global__ void __launch_bounds__(kLocalStepThreads, 1) k_local_step(const Local
   const int i = a.worker_of ? a.worker_of[cl] : cl;
   const BatchDesc dsc = a.desc[i];
   const int nnz = dsc.nnz;
-  const int nseg = (nnz + kTileEntries - 1) / kTileEntries;
+  // Pass 1: CTA q takes the 256-entry slot segments [s0, s1) in tiles of up
+  // to four (the CTAs' shares differ by at most one segment).
+  const int nseg = (nnz + kSlotSegment - 1) / kSlotSegment;
   const int s0 = static_cast<int>(static_cast<long long>(q) * nseg / Q);
   const int s1 = static_cast<int>(static_cast<long long>(q + 1) * nseg / Q);
-  const int n1 = s1 - s0;
+  constexpr int kSegsPerTile = kTileEntries / kSlotSegment;
+  const int n1 = (s1 - s0 + kSegsPerTile - 1) / kSegsPerTile;
+  const int p1_begin = s0 * kSlotSegment, p1_end = min(s1 * kSlotSegment, nnz);
   const int* bnd = reinterpret_cast<const int*>(a.block + dsc.bnd);
   const int lo = bnd[q], hi = bnd[q + 1];
   const int T0 = lo & ~7;                      // 16-byte aligned start of the first column tile
@@ -357,8 +362,8 @@ __global__ void __launch_bounds__(kLocalStepThreads, 1) k_local_step(const Local
       if (it >= a.stages && !mbar_wait_bounded(sm.empty + st, ((it / a.stages) - 1) & 1)) return false;
       unsigned char* base = sm.stage0 + kStageBytes * st;
       const bool pass1 = it < n1;
-      const int e0 = pass1 ? (s0 + it) * kTileEntries : T0 + (it - n1) * kTileEntries;
-      const int len = min(kTileEntries, (pass1 ? nnz : hi) - e0);
+      const int e0 = pass1 ? p1_begin + it * kTileEntries : T0 + (it - n1) * kTileEntries;
+      const int len = min(kTileEntries, (pass1 ? p1_end : hi) - e0);
       const uint32_t n8 = static_cast<uint32_t>((len + 7) & ~7);   // whole 16-byte rows of uint16
       mbar_expect_tx(sm.full + st, n8 * (pass1 ? 12u : 10u));
       bulk_load(base, a.block + dsc.cpos + 4 * static_cast<int64_t>(e0), 4 * n8, sm.full + st);
@@ -396,7 +401,7 @@ __global__ void __launch_bounds__(kLocalStepThreads, 1) k_local_step(const Local
       gok = __all_sync(kFull, mbar_wait_bounded(sm.full + st, (k / a.stages) & 1));
       if (!gok) break;
       int* spos = reinterpret_cast<int*>(sm.stage0 + kStageBytes * st);
-      const int len = min(kTileEntries, nnz - (s0 + k) * kTileEntries);
+      const int len = min(kTileEntries, p1_end - (p1_begin + k * kTileEntries));
       // four consecutive positions per lane and vector load, two loads ahead
       // of their copies, so that no copy waits on its own position's load
       for (int j0 = lane * 4; j0 < len; j0 += 256) {
@@ -477,7 +482,7 @@ __global__ void __launch_bounds__(kLocalStepThreads, 1) k_local_step(const Local
       const uint16_t* sslot = reinterpret_cast<const uint16_t*>(base + 8 * kTileEntries);
       const uint16_t* srow = reinterpret_cast<const uint16_t*>(base + 10 * kTileEntries);
       const float* wvs = reinterpret_cast<const float*>(base);   // gathered over the positions
-      const int len = min(kTileEntries, nnz - (s0 + it) * kTileEntries);
+      const int len = min(kTileEntries, p1_end - (p1_begin + it * kTileEntries));
       const bool active = sub < len;           // warp-uniform
       int key[kPerThread];
       float val[kPerThread];
@@ -536,23 +541,34 @@ __global__ void __launch_bounds__(kLocalStepThreads, 1) k_local_step(const Local
     asm volatile("barrier.cluster.arrive.release.aligned;\nbarrier.cluster.wait.acquire.aligned;" ::: "memory");
     const float* y = reinterpret_cast<const float*>(a.block + dsc.y);
     float lsum = 0.f;
-    for (int b = tid; b < a.B; b += kConsumers) {
-      // the Q partials first, then their sum in rank order: the remote loads overlap
-      float mq[kMaxStepCluster];
+    constexpr int kRowsAtOnce = 2;
+    for (int b0 = tid; b0 < a.B; b0 += kRowsAtOnce * kConsumers) {
+      // the Q partials of two rows first, then each row's sum in rank order:
+      // the remote loads overlap
+      float mq[kRowsAtOnce][kMaxStepCluster];
 #pragma unroll
-      for (int qq = 0; qq < kMaxStepCluster; ++qq)
-        if (qq < Q)
-          mq[qq] = big ? __ldcg(a.mpart_big + (static_cast<size_t>(i) * Q + qq) * kWarps * a.B + b)
-                       : ld_dsmem(sm.mpart + b, qq);
-      float m = 0.f;
+      for (int u = 0; u < kRowsAtOnce; ++u) {
+        const int b = b0 + u * kConsumers;
 #pragma unroll
-      for (int qq = 0; qq < kMaxStepCluster; ++qq)
-        if (qq < Q) m += mq[qq];
-      float l, r;
-      loss_and_r<LOSS>(y[b], m * a.mscale, l, r);
-      if (big) grr[b] = r;
-      else sm.r[b] = r;
-      lsum += l;
+        for (int qq = 0; qq < kMaxStepCluster; ++qq)
+          if (qq < Q && b < a.B)
+            mq[u][qq] = big ? __ldcg(a.mpart_big + (static_cast<size_t>(i) * Q + qq) * kWarps * a.B + b)
+                            : ld_dsmem(sm.mpart + b, qq);
+      }
+#pragma unroll
+      for (int u = 0; u < kRowsAtOnce; ++u) {
+        const int b = b0 + u * kConsumers;
+        if (b >= a.B) break;
+        float m = 0.f;
+#pragma unroll
+        for (int qq = 0; qq < kMaxStepCluster; ++qq)
+          if (qq < Q) m += mq[u][qq];
+        float l, r;
+        loss_and_r<LOSS>(y[b], m * a.mscale, l, r);
+        if (big) grr[b] = r;
+        else sm.r[b] = r;
+        lsum += l;
+      }
     }
     if (q == 0) {
       lsum = warp_sum(lsum);

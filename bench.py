@@ -66,7 +66,7 @@ TRAFFIC = {
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=3000)
+    ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", default="asap", choices=["asap", "reference"])
     ap.add_argument("--rows", type=int, default=None, help="rows per worker (default: the workload's)")

@@ -962,11 +962,17 @@ asap_status asap_set_model(asap_ctx* c, asap_loss loss, int num_classes, int bat
   if (loss == ASAP_LOSS_HINGE || loss == ASAP_LOSS_LOGISTIC) {
     c->n_loss_part = c->N;
     // The local step: one cluster of Q CTAs per worker, Q as large as keeps
-    // all clusters resident at four CTAs per SM (at most 8, the portable size).
-    c->step_q = kMaxStepCluster;
-    while (c->step_q > 1 && static_cast<int64_t>(c->N) * c->step_q > 4LL * c->sm_count) c->step_q >>= 1;
-    c->step_stages = 3;
+    // all clusters resident (at most 8, the portable size).  Two ring stages
+    // keep a CTA small enough for five per SM at the usual minibatch sizes
+    // (the kernel's registers are bounded for five).
+    c->step_stages = 2;
     c->step_smem = local_step_smem_bytes(batch, c->step_stages);
+    int smem_sm = 0;
+    CU(cudaDeviceGetAttribute(&smem_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, c->dev),
+       "querying shared memory per SM");
+    const int64_t per_sm = std::max<int64_t>(1, std::min<int64_t>(5, smem_sm / static_cast<int64_t>(c->step_smem + 1024)));
+    c->step_q = kMaxStepCluster;
+    while (c->step_q > 1 && static_cast<int64_t>(c->N) * c->step_q > per_sm * c->sm_count) c->step_q >>= 1;
     CU(local_step_configure(c->step_smem), "configuring the local-step kernel");
     c->permuted = false;
   } else if (loss == ASAP_LOSS_SOFTMAX) {

@@ -295,7 +295,7 @@ __device__ __forceinline__ void seg_scan_warp(const int (&key)[kPerThread], floa
 }
 
 template <int LOSS>
-__global__ void __launch_bounds__(kLocalStepThreads, 4) k_local_step(const LocalStepArgs a) {   // four CTAs per SM
+__global__ void __launch_bounds__(kLocalStepThreads, 5) k_local_step(const LocalStepArgs a) {   // five CTAs per SM
   extern __shared__ unsigned char step_smem_raw[];
   const bool big = a.B > kRSmemRows;           // partial margins and r in global memory
   const StepSmem sm = carve_step(step_smem_raw, big ? 0 : a.B, a.stages);

@@ -28,7 +28,8 @@
 // (sum_i (w_i - K))^2 / N.  Squares accumulate per thread in fp32 (a few
 // dozen slabs per thread; GB300's fp64 pipe is narrow), the per-column sums
 // are combined across warps by the producer warp when the stage comes back,
-// and the block total is formed in fp64.  The complete graph (all-reduce, equal weights) writes
+// and the block and launch totals are formed in float-float pairs (fp32 hi +
+// lo, a fixed order).  The complete graph (all-reduce, equal weights) writes
 // the column mean to every row and adds nothing.
 //
 // Protocol (Section 4, NOTIFY-ACK): before touching any input each CTA waits,
@@ -185,17 +186,42 @@ __device__ __forceinline__ float4 f4_add(float4 a, float4 b) {
   return make_float4(a.x + b.x, a.y + b.y, a.z + b.z, a.w + b.w);
 }
 
-// Sum over all threads of the block (kMixThreads); valid in thread 0.
-__device__ __forceinline__ double block_sum_f64(double v, double* scratch) {
+// A float-float value hi + lo (|lo| at most half an ulp of hi): the block
+// sums are carried in fp32 pairs, since this GPU's fp64 pipe is narrow (an
+// fp64 tree over the block took ~2 us, in the last CTA's finalisation ~7).
+struct F2 {
+  float hi, lo;
+};
+
+// hi + lo of a + b: the rounding error of hi_a + hi_b is recovered exactly
+// by Knuth's two-sum, the low parts are added to it, and the pair is
+// renormalised.  The result does not depend on the order of a and b.
+__device__ __forceinline__ F2 f2_add(F2 a, F2 b) {
+  const float s = a.hi + b.hi;
+  const float bv = s - a.hi;
+  const float e = ((a.hi - (s - bv)) + (b.hi - bv)) + (a.lo + b.lo);
+  const float hi = s + e;
+  return F2{hi, e - (hi - s)};
+}
+
+__device__ __forceinline__ F2 f2_of(double v) {
+  const float h = static_cast<float>(v);
+  return F2{h, static_cast<float>(v - static_cast<double>(h))};
+}
+
+// Sum over all threads of the block (kMixThreads) in a fixed order; valid in
+// thread 0.
+__device__ __forceinline__ F2 block_sum_f2(F2 v, F2* scratch) {
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(kFull, v, o);
+  for (int o = 16; o > 0; o >>= 1)
+    v = f2_add(v, F2{__shfl_xor_sync(kFull, v.hi, o), __shfl_xor_sync(kFull, v.lo, o)});
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   __syncthreads();
   if (lane == 0) scratch[warp] = v;
   __syncthreads();
-  double t = 0.0;
+  F2 t{0.f, 0.f};
   if (threadIdx.x == 0)
-    for (int k = 0; k < kMixThreads / 32; ++k) t += scratch[k];
+    for (int k = 0; k < kMixThreads / 32; ++k) t = f2_add(t, scratch[k]);
   return t;
 }
 
@@ -221,7 +247,7 @@ struct MixSmem {
   int* nbr;
   float* wgt;
   double* dscratch;
-  int* flags;        // [0]: fail, [1]: last
+  int* flags;        // [0]: fail, [1]: last, [2]: failed CTAs of the launch (last CTA)
   unsigned* seen;    // [32]: bitmap of workers whose NOTIFY this CTA has seen (gated reduces)
 };
 
@@ -708,10 +734,11 @@ __global__ void __launch_bounds__(kMixThreads, 1) k_mix(const __grid_constant__ 
   }
 
   // ---- per-CTA partial, ticket, and the last CTA's finalisation ----
-  const double csum = block_sum_f64(static_cast<double>(s2), sm.dscratch);
+  F2* scratch = reinterpret_cast<F2*>(sm.dscratch);
+  const F2 csum = block_sum_f2(F2{s2, 0.f}, scratch);
   if (failed) atomicOr(&sm.flags[0], 1);
   __syncthreads();
-  if (tid == 0) a.cons_part[blockIdx.x] = csum;
+  if (tid == 0) a.cons_part[blockIdx.x] = static_cast<double>(csum.hi) + static_cast<double>(csum.lo);
   __threadfence();
   __syncthreads();
   if (tid == 0) {
@@ -722,11 +749,12 @@ __global__ void __launch_bounds__(kMixThreads, 1) k_mix(const __grid_constant__ 
   __syncthreads();
   if (!sm.flags[1]) return;
   __threadfence();
-  const unsigned ticket = atomicAdd(&a.st->mix_ticket, 0u);
-  bool any_fail = (ticket >> 16) != 0;
-  double v = 0.0;
-  for (int b = tid; b < static_cast<int>(gridDim.x); b += kMixThreads) v += __ldcg(a.cons_part + b);
-  const double ctot = block_sum_f64(v, sm.dscratch);
+  if (tid == 0) sm.flags[2] = static_cast<int>(atomicAdd(&a.st->mix_ticket, 0u) >> 16);   // failed CTAs
+  __syncthreads();
+  bool any_fail = sm.flags[2] != 0;
+  F2 v{0.f, 0.f};
+  for (int b = tid; b < static_cast<int>(gridDim.x); b += kMixThreads) v = f2_add(v, f2_of(__ldcg(a.cons_part + b)));
+  const F2 ctot = block_sum_f2(v, scratch);
   if (gated && a.sync_mode == kSyncNotifyAck && !any_fail) {
     // The loss partials of workers without any update in this launch's
     // slabs: every worker's NOTIFY before they are read.
@@ -740,19 +768,19 @@ __global__ void __launch_bounds__(kMixThreads, 1) k_mix(const __grid_constant__ 
     __syncthreads();
     any_fail = (sm.flags[0] & 2) != 0;
   }
-  double lv = 0.0;
+  F2 lv{0.f, 0.f};
   if (a.have_loss)
-    for (int b = tid; b < a.n_loss_part; b += kMixThreads) lv += static_cast<double>(__ldcg(a.loss_part + b));
-  const double ltot = block_sum_f64(lv, sm.dscratch);
+    for (int b = tid; b < a.n_loss_part; b += kMixThreads) lv = f2_add(lv, F2{__ldcg(a.loss_part + b), 0.f});
+  const F2 ltot = block_sum_f2(lv, scratch);
   if (tid == 0) {
     const int slot = static_cast<int>(a.round % kMetricsCap);
-    a.metrics_cons[slot] = any_fail ? __int_as_float(0x7fc00000) : static_cast<float>(sqrt(fmax(ctot, 0.0)));
-    a.metrics_loss[slot] = (a.have_loss && !any_fail) ? static_cast<float>(ltot * a.loss_norm)
+    a.metrics_cons[slot] = any_fail ? __int_as_float(0x7fc00000) : sqrtf(fmaxf(ctot.hi + ctot.lo, 0.f));
+    a.metrics_loss[slot] = (a.have_loss && !any_fail) ? (ltot.hi + ltot.lo) * a.loss_norm
                                                       : __int_as_float(0x7fc00000);
     if (!any_fail) {
-      a.st->reduces += static_cast<unsigned long long>(a.own_n);
+      atomicAdd(&a.st->reduces, static_cast<unsigned long long>(a.own_n));
       if (a.expect_notify)
-        a.st->consistent_inputs += static_cast<unsigned long long>(a.own_n) * (KP1 < 0 ? a.N : kp1);
+        atomicAdd(&a.st->consistent_inputs, static_cast<unsigned long long>(a.own_n) * (KP1 < 0 ? a.N : kp1));
     }
     a.st->mix_ticket = 0u;
   }
@@ -836,7 +864,7 @@ size_t mix_smem_bytes(int N, int kp1, int S, int rows_pad, int stages, int max_r
   auto a16 = [](size_t v) { return (v + 15) & ~static_cast<size_t>(15); };
   size_t b = 1024 + mix_stage_bytes(S, rows_pad, max_region) * stages;   // alignment slack + stages
   b = a16(b + 24 * static_cast<size_t>(stages));                         // full / empty / ready
-  b = a16(b + 8 * (kMixThreads / 32));                                    // fp64 block scratch
+  b = a16(b + 8 * (kMixThreads / 32));                                    // block-sum scratch (fp32 pairs)
   b = a16(b + 16);                                                        // flags
   b = a16(b + 4 * 32);                                                    // NOTIFY bitmap
   b = a16(b + 16 * static_cast<size_t>(stages));                          // stage info

@@ -57,15 +57,32 @@ struct NoAllocArgs {
   double* partial;
 };
 
-__device__ __forceinline__ double block_sum(double v, double* red) {
+// Block sums are carried as float-float pairs hi + lo in fp32 arithmetic
+// (this GPU's fp64 pipe is narrow): the rounding error of each addition of
+// the high parts is recovered exactly (Knuth's two-sum) and kept in lo.
+struct Pair {
+  float hi, lo;
+};
+
+__device__ __forceinline__ Pair pair_add(Pair a, Pair b) {
+  const float s = a.hi + b.hi;
+  const float bv = s - a.hi;
+  const float e = ((a.hi - (s - bv)) + (b.hi - bv)) + (a.lo + b.lo);
+  const float hi = s + e;
+  return Pair{hi, e - (hi - s)};
+}
+
+// Sum over the block in a fixed order; valid in thread 0.
+__device__ __forceinline__ Pair block_sum(Pair v, Pair* red) {
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  for (int o = 16; o > 0; o >>= 1)
+    v = pair_add(v, Pair{__shfl_xor_sync(0xffffffffu, v.hi, o), __shfl_xor_sync(0xffffffffu, v.lo, o)});
   __syncthreads();
   if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = v;
   __syncthreads();
-  double t = 0.0;
+  Pair t{0.f, 0.f};
   if (threadIdx.x == 0)
-    for (int w = 0; w < kThreads / 32; ++w) t += red[w];
+    for (int w = 0; w < kThreads / 32; ++w) t = pair_add(t, red[w]);
   return t;
 }
 
@@ -76,7 +93,7 @@ __global__ void __launch_bounds__(kThreads) k_mix_noalloc(const NoAllocArgs a) {
   float4* slab = reinterpret_cast<float4*>(smem);                       // [N][nq]
   float4* mean = slab + static_cast<size_t>(a.N) * nq;                  // [nq]
   float4* red4 = mean + nq;                                             // [kThreads]
-  double* red = reinterpret_cast<double*>(red4 + kThreads);             // [kThreads / 32]
+  Pair* red = reinterpret_cast<Pair*>(red4 + kThreads);                 // [kThreads / 32]
   int* flag = reinterpret_cast<int*>(red + kThreads / 32);
   const int tid = threadIdx.x;
   const int G = kThreads >> lq;
@@ -137,8 +154,8 @@ __global__ void __launch_bounds__(kThreads) k_mix_noalloc(const NoAllocArgs a) {
       const long long c = c0 + 4 * q;
       if (c < a.ld) *reinterpret_cast<float4*>(a.out + static_cast<int64_t>(i) * a.ld + c) = acc;
     }
-    const double ps = block_sum(static_cast<double>(cacc), red);
-    if (tid == 0) a.partial[s] = ps;
+    const Pair ps = block_sum(Pair{cacc, 0.f}, red);
+    if (tid == 0) a.partial[s] = static_cast<double>(ps.hi) + static_cast<double>(ps.lo);
     __syncthreads();   // the slab buffer is reused by the next slab
   }
 
@@ -150,11 +167,15 @@ __global__ void __launch_bounds__(kThreads) k_mix_noalloc(const NoAllocArgs a) {
   __syncthreads();
   if (!flag[0]) return;
   __threadfence();
-  double v = 0.0;
-  for (long long s = tid; s < a.n_slabs; s += kThreads) v += __ldcg(a.partial + s);
-  const double total = block_sum(v, red);
+  Pair v{0.f, 0.f};
+  for (long long s = tid; s < a.n_slabs; s += kThreads) {
+    const double p = __ldcg(a.partial + s);
+    const float h = static_cast<float>(p);
+    v = pair_add(v, Pair{h, static_cast<float>(p - static_cast<double>(h))});
+  }
+  const Pair total = block_sum(v, red);
   if (tid == 0) {
-    a.consensus_out[0] = static_cast<float>(sqrt(total));
+    a.consensus_out[0] = sqrtf(fmaxf(total.hi + total.lo, 0.f));
     *a.ticket = 0u;
   }
 }

@@ -228,9 +228,9 @@ def kernel_work(sh):
         touched += np.unique(sh.col[i][rp[0]:rp[-1]]).shape[0]
     nnz, touched = nnz * N / samples, touched * N / samples
     # the fused local step reads every entry once (list position, value,
-    # row, segment slot, row of the slot: 14 B), the w value and writes the
-    # column sum of every distinct (worker, column) (8 B), and the labels
-    out["local_step"] = ("GB/s", 14.0 * nnz + 8.0 * touched + 4.0 * N * B, "hbm")
+    # row, segment slot: 12 B), the w value and writes the column sum of
+    # every distinct (worker, column) (8 B), and the labels
+    out["local_step"] = ("GB/s", 12.0 * nnz + 8.0 * touched + 4.0 * N * B, "hbm")
     out["reduce"] = ("GB/s", 8.0 * N * ld, "hbm")
     # local steps before the round's last: the update scatter and the next gather
     out["apply"] = ("GB/s", 16.0 * touched, "hbm")    # list + column sum read, w read + write per column

@@ -329,9 +329,8 @@ asap_status asap_debug_skip_notify(asap_ctx* ctx, int worker);
  * bytes; *image_bytes receives its size; ASAP_ERR_ARG when it does not fit).
  * desc_out (N*8 int64), per worker: byte offsets of the labels (float [B]),
  * of the (column, row)-sorted entries' list positions, values, rows and
- * segment slots (int32 / float / uint16 / uint16 [nnz]), of the rows of
- * every segment's slots (uint16 [nnz]) and of the Q+1 column-sum range
- * bounds (int32), then nnz.  Segment g holds sorted entries [256 g,
+ * segment slots (int32 / float / uint16 / uint16 [nnz]) and of the Q+1
+ * column-sum range bounds (int32), then nnz, then 0.  Segment g holds sorted entries [256 g,
  * 256 (g+1)); its slots are numbered row by row, a row's entries in sorted
  * order.  The range bounds start at 0, end at nnz and cut the sorted entries
  * at the first column boundary at or after q nnz / Q.  list_out (3 int64):

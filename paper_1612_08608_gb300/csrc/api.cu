@@ -598,8 +598,6 @@ void build_batch_image(int N, int B, int64_t d, int S, long long n_slabs, int Q,
     off = align_up(off + 2 * static_cast<size_t>(nnz[i]), 16);
     dd.cslot = static_cast<int64_t>(off);
     off = align_up(off + 2 * static_cast<size_t>(nnz[i]), 16);
-    dd.srow = static_cast<int64_t>(off);
-    off = align_up(off + 2 * static_cast<size_t>(nnz[i]), 16);
     dd.bnd = static_cast<int64_t>(off);
     off = align_up(off + 4 * static_cast<size_t>(Q + 1), 16);
     dd.nnz = static_cast<int32_t>(nnz[i]);
@@ -622,7 +620,6 @@ void build_batch_image(int N, int B, int64_t d, int S, long long n_slabs, int Q,
     float* cv_o = reinterpret_cast<float*>(base + dd.cval);
     uint16_t* cr_o = reinterpret_cast<uint16_t*>(base + dd.crow);
     uint16_t* cs_o = reinterpret_cast<uint16_t*>(base + dd.cslot);
-    uint16_t* sr_o = reinterpret_cast<uint16_t*>(base + dd.srow);
     int32_t* bd_o = reinterpret_cast<int32_t*>(base + dd.bnd);
     const int64_t* rp = rowptr[i];
     if (!rp) continue;   // labels and ranges stay zero
@@ -638,7 +635,7 @@ void build_batch_image(int N, int B, int64_t d, int S, long long n_slabs, int Q,
       cr_o[e] = erow[k];
     }
     // Margin segments of kSlotSegment sorted entries: slots row by row, a
-    // row's entries in sorted (column) order; srow lists the slots' rows.
+    // row's entries in sorted (column) order.
     for (int64_t e0 = 0; e0 < nnz[i]; e0 += kSlotSegment) {
       const int64_t e1 = std::min<int64_t>(e0 + kSlotSegment, nnz[i]);
       std::fill(fill.begin(), fill.end(), 0);
@@ -652,7 +649,6 @@ void build_batch_image(int N, int B, int64_t d, int S, long long n_slabs, int Q,
       for (int64_t e = e0; e < e1; ++e) {
         const int32_t sl = fill[cr_o[e]]++;
         cs_o[e] = static_cast<uint16_t>(sl);
-        sr_o[e0 + sl] = cr_o[e];
       }
     }
     // Column-sum ranges of the Q CTAs: cut at the first column boundary at
@@ -733,7 +729,7 @@ asap_status asap_debug_batch_image(int N, int64_t d, int batch, int slab_cols, i
   std::memcpy(image, bt.img.data(), bt.img.size());
   for (int i = 0; i < N; ++i) {
     const BatchDesc& q = bt.desc[i];
-    const int64_t v[8] = {q.y, q.cpos, q.cval, q.crow, q.cslot, q.srow, q.bnd, q.nnz};
+    const int64_t v[8] = {q.y, q.cpos, q.cval, q.crow, q.cslot, q.bnd, q.nnz, 0};
     std::memcpy(desc_out + 8 * static_cast<size_t>(i), v, sizeof v);
   }
   list_out[0] = static_cast<int64_t>(bt.list_off);

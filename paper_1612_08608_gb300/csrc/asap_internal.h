@@ -60,7 +60,7 @@ constexpr uint32_t kListPad = 0xffffffffu;   // padding entry of a column list
 // margins the sorted entries are cut into segments of kSlotSegment (one
 // consumer warp's share of a tile); inside a segment every entry has a slot,
 // the slots of one row contiguous (rows in order, a row's entries by
-// column), and `srow` lists the row of every slot.
+// column); the local step puts each entry's product and row at its slot.
 // For the column sums the entries are split among the worker's Q CTAs at
 // column boundaries (`bnd`).
 struct BatchDesc {
@@ -69,7 +69,6 @@ struct BatchDesc {
   int64_t cval;   // float [nnz]
   int64_t crow;   // uint16 [nnz]: row within the batch
   int64_t cslot;  // uint16 [nnz]: slot within its segment
-  int64_t srow;   // uint16 [nnz]: per segment, the row of every slot
   int64_t bnd;    // int32 [Q+1]: column-sum ranges of the worker's CTAs
   int32_t nnz;
   int32_t pad_;

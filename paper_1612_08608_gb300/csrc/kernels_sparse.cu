@@ -24,8 +24,9 @@
 // 256-entry share of the 1024-entry tile and without CTA-wide barriers:
 //   pass 1 (margins): CTA q takes the 256-entry segments s = q nseg/Q ...
 //     in tiles of four; a
-//     warp's products val * wv[pos] go to shared memory at the entry's slot
-//     (slots of a 256-entry segment ordered by row, then column), a
+//     warp's products val * wv[pos] and their rows go to shared memory at
+//     the entry's slot (slots of a 256-entry segment ordered by row, then
+//     column), a
 //     segmented scan over the slots keyed by row sums each row's products
 //     in order, and the warp adds them to its own partial margins.  The
 //     four warps' partials are added in order; a cluster barrier; every CTA
@@ -174,11 +175,11 @@ __device__ __forceinline__ void loss_and_r(float y, float m, float& l, float& r)
 
 // Shared-memory layout of the local-step kernel (mirrored by
 // local_step_smem_bytes): the ring of stages, each holding one tile's list
-// positions, values and two uint16 arrays (pass 1: slots and the rows in
-// slot order; pass 2: rows), a margin tile's positions replaced in place by
-// the gathered w values;
-// per consumer warp a 256-entry scratch (pass 1: products by slot; pass 2:
-// run sums and their list positions); the per-warp partial margins and r
+// positions, values and two uint16 arrays (pass 1: slots and rows; pass 2:
+// rows), a margin tile's positions replaced in place by the gathered w
+// values;
+// per consumer warp a 256-entry scratch (pass 1: products and rows by slot;
+// pass 2: run sums and their list positions); the per-warp partial margins and r
 // of the worker's B rows; the column-run fragments at sub-tile edges.
 struct StepSmem {
   unsigned char* stage0;
@@ -370,7 +371,7 @@ __global__ void __launch_bounds__(kLocalStepThreads, 5) k_local_step(const Local
       bulk_load(base + 4 * kTileEntries, a.block + dsc.cval + 4 * static_cast<int64_t>(e0), 4 * n8, sm.full + st);
       if (pass1) {
         bulk_load(base + 8 * kTileEntries, a.block + dsc.cslot + 2 * static_cast<int64_t>(e0), 2 * n8, sm.full + st);
-        bulk_load(base + 10 * kTileEntries, a.block + dsc.srow + 2 * static_cast<int64_t>(e0), 2 * n8, sm.full + st);
+        bulk_load(base + 10 * kTileEntries, a.block + dsc.crow + 2 * static_cast<int64_t>(e0), 2 * n8, sm.full + st);
       } else {
         bulk_load(base + 8 * kTileEntries, a.block + dsc.crow + 2 * static_cast<int64_t>(e0), 2 * n8, sm.full + st);
       }
@@ -471,6 +472,7 @@ __global__ void __launch_bounds__(kLocalStepThreads, 5) k_local_step(const Local
     const int j0 = sub + lane * kPerThread;    // this lane's eight consecutive pairs
     float* wprod = sm.prod + sub;
     int* wokey = sm.okey + sub;
+    uint16_t* wrows = reinterpret_cast<uint16_t*>(wokey);   // pass 1: the row of every slot
     const size_t wrow = static_cast<size_t>(warp) * a.B;   // this warp's partial margins
     // ---- pass 1: products by slot; each row's sum by a scan over the slots ----
     for (int it = 0; it < n1; ++it) {
@@ -480,7 +482,7 @@ __global__ void __launch_bounds__(kLocalStepThreads, 5) k_local_step(const Local
       const unsigned char* base = sm.stage0 + kStageBytes * st;
       const float* sval = reinterpret_cast<const float*>(base + 4 * kTileEntries);
       const uint16_t* sslot = reinterpret_cast<const uint16_t*>(base + 8 * kTileEntries);
-      const uint16_t* srow = reinterpret_cast<const uint16_t*>(base + 10 * kTileEntries);
+      const uint16_t* scrow = reinterpret_cast<const uint16_t*>(base + 10 * kTileEntries);   // the entries' rows
       const float* wvs = reinterpret_cast<const float*>(base);   // gathered over the positions
       const int len = min(kTileEntries, p1_end - (p1_begin + it * kTileEntries));
       const bool active = sub < len;           // warp-uniform
@@ -490,13 +492,17 @@ __global__ void __launch_bounds__(kLocalStepThreads, 5) k_local_step(const Local
 #pragma unroll
         for (int u = 0; u < kPerThread; ++u) {   // consecutive lanes, consecutive entries
           const int j = sub + u * 32 + lane;
-          if (j < len) wprod[sslot[j]] = sval[j] * wvs[j];
+          if (j < len) {                         // the product and the row go to the entry's slot
+            const int sl = sslot[j];
+            wprod[sl] = sval[j] * wvs[j];
+            wrows[sl] = scrow[j];
+          }
         }
         __syncwarp();
         // slots j0 .. j0+7 of the segment (a row's slots are adjacent): vector loads
         const float4 q0 = *reinterpret_cast<const float4*>(wprod + lane * kPerThread);
         const float4 q1 = *reinterpret_cast<const float4*>(wprod + lane * kPerThread + 4);
-        const uint4 rw = *reinterpret_cast<const uint4*>(srow + j0);
+        const uint4 rw = *reinterpret_cast<const uint4*>(wrows + lane * kPerThread);
         const float pv[8] = {q0.x, q0.y, q0.z, q0.w, q1.x, q1.y, q1.z, q1.w};
         const unsigned rws[4] = {rw.x, rw.y, rw.z, rw.w};
 #pragma unroll

@@ -33,7 +33,8 @@ def test_batch_image_matches_the_shards(S, Q, max_len):
 
     pairs = set()
     for i in range(N):
-        y_o, cp_o, cv_o, cr_o, cs_o, sr_o, bd_o, nnz = (int(v) for v in desc[i])
+        y_o, cp_o, cv_o, cr_o, cs_o, bd_o, nnz, zero = (int(v) for v in desc[i])
+        assert zero == 0
         r0 = t * B
         entries = []                                   # (col, row, val)
         for b in range(B):
@@ -56,14 +57,12 @@ def test_batch_image_matches_the_shards(S, Q, max_len):
             p = int(cp[e])
             assert lst[p] == (i << 16) | (c % S) and soff[c // S] <= p < soff[c // S + 1]
         # margin segments of 256 entries: slots numbered row by row, by
-        # column within a row; srow holds the row of every slot
+        # column within a row
         cs = _view(img, cs_o, np.uint16, nnz)
-        sr = _view(img, sr_o, np.uint16, nnz)
         for e0 in range(0, nnz, 256):
             e1 = min(e0 + 256, nnz)
             seg = sorted(range(e0, e1), key=lambda e: (entries[e][1], entries[e][0]))
             assert [int(cs[e]) for e in seg] == list(range(e1 - e0))
-            assert [int(v) for v in sr[e0:e1]] == [entries[e][1] for e in seg]
         # column-sum ranges: cut at the first column boundary at or after q nnz / Q
         bd = _view(img, bd_o, np.int32, Q + 1)
         assert bd[0] == 0 and bd[Q] == nnz and np.all(np.diff(bd) >= 0)

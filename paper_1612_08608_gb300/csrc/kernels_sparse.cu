@@ -23,15 +23,13 @@
 // consumer warps work on the stage that has landed, each on its own
 // 256-entry share of the 1024-entry tile and without CTA-wide barriers:
 //   pass 1 (margins): CTA q takes the 256-entry segments s = q nseg/Q ...
-//     in tiles of four; a
-//     warp's products val * wv[pos] and their rows go to shared memory at
-//     the entry's slot (slots of a 256-entry segment ordered by row, then
-//     column), a
-//     segmented scan over the slots keyed by row sums each row's products
-//     in order, and the warp adds them to its own partial margins.  The
-//     four warps' partials are added in order; a cluster barrier; every CTA
-//     then adds the Q partials of each row in rank order (distributed shared
-//     memory), forms r and, in CTA 0, the loss sum.
+//     in tiles of four; a warp's products val * wv[pos] and their rows go to
+//     shared memory at the entry's slot (slots of a 256-entry segment
+//     ordered by row, then column), a segmented scan over the slots keyed by
+//     row sums each row's products in order, and the warp adds them to its
+//     own partial margins.  The four warps' partials are added in order; a
+//     cluster barrier; every CTA then adds the Q partials of each row in rank
+//     order (distributed shared memory), forms r and, in CTA 0, the loss sum.
 //   pass 2 (column sums): CTA q takes the entries [bnd[q], bnd[q+1]), cut
 //     at column boundaries, in 1024-entry tiles; a warp's segmented scan
 //     keyed by list position sums each column's r_row * val; runs that end
@@ -40,7 +38,9 @@
 //     in order.
 // A last cluster barrier and CTA 0 publishes NOTIFY.  No atomics, no waits
 // on other clusters, every sum in a fixed order: the result does not depend
-// on the schedule.
+// on the schedule.  The kernel is a programmatic dependent of the previous
+// round's reduce (set-up and the first bulk copies of static batch data run
+// while that reduce drains); its registers are bounded for five CTAs per SM.
 #include <cuda_runtime.h>
 
 #include <cstdint>

@@ -112,14 +112,17 @@ class ShardedWorkers:
         nbr, _ = ctx.get_graph(self.t)
         send, recv = exchange_plan(nbr, self.ranges, self.rank)
         ctx.local_step()
-        reqs, inbox = [], {}
+        # The rows go as stored: both ends keep the same lazy L2 scale (every
+        # context applies the same schedule), so the scale is not sent.
+        reqs, inbox, outbox = [], {}, []
         for q in sorted(recv):
             buf = torch.from_numpy(np.empty((recv[q].size, ctx.P), dtype=ctx.row_dtype))
             inbox[q] = buf
             reqs.append(dist.irecv(buf, src=q, group=self.group))
         for q in sorted(send):
             rows, _ = ctx.read_rows(send[q])
-            reqs.append(dist.isend(torch.from_numpy(rows), dst=q, group=self.group))
+            outbox.append(torch.from_numpy(rows))   # alive until every request is done
+            reqs.append(dist.isend(outbox[-1], dst=q, group=self.group))
             self.sent_bytes += rows.nbytes
         for rq in reqs:
             rq.wait()

@@ -225,6 +225,33 @@ __device__ __forceinline__ F2 block_sum_f2(F2 v, F2* scratch) {
   return t;
 }
 
+// Two block sums at once, each in the order block_sum_f2 takes (so each
+// result equals that of a separate call); valid in thread 0.  `scratch`
+// holds two pairs per warp.
+__device__ __forceinline__ void block_sum2_f2(F2& u, F2& v, F2* scratch) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    u = f2_add(u, F2{__shfl_xor_sync(kFull, u.hi, o), __shfl_xor_sync(kFull, u.lo, o)});
+    v = f2_add(v, F2{__shfl_xor_sync(kFull, v.hi, o), __shfl_xor_sync(kFull, v.lo, o)});
+  }
+  constexpr int kW = kMixThreads / 32;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  __syncthreads();
+  if (lane == 0) {
+    scratch[warp] = u;
+    scratch[kW + warp] = v;
+  }
+  __syncthreads();
+  F2 tu{0.f, 0.f}, tv{0.f, 0.f};
+  if (threadIdx.x == 0)
+    for (int k = 0; k < kW; ++k) {
+      tu = f2_add(tu, scratch[k]);
+      tv = f2_add(tv, scratch[kW + k]);
+    }
+  u = tu;
+  v = tv;
+}
+
 __device__ __forceinline__ void compute_bar() { asm volatile("bar.sync 1, %0;" :: "n"(kCompute) : "memory"); }
 
 // Barrier among the compute warps that also returns the OR of `v` over them.
@@ -270,7 +297,7 @@ __device__ __forceinline__ MixSmem carve(unsigned char* raw, const MixArgs& a, i
   m.ready = reinterpret_cast<uint64_t*>(raw + off);
   off = a16(off + 8 * a.stages);
   m.dscratch = reinterpret_cast<double*>(raw + off);
-  off = a16(off + 8 * (kMixThreads / 32));
+  off = a16(off + 16 * (kMixThreads / 32));
   m.flags = reinterpret_cast<int*>(raw + off);
   off = a16(off + 16);
   m.seen = reinterpret_cast<unsigned*>(raw + off);
@@ -743,35 +770,42 @@ __global__ void __launch_bounds__(kMixThreads, 1) k_mix(const __grid_constant__ 
   __syncthreads();
   if (tid == 0) {
     if (sm.flags[0]) atomicAdd(&a.st->mix_ticket, 0x10000u);   // high half counts failed CTAs
+    // Every CTA adds its failure before its ticket, to the same word: the
+    // last ticket's old value already holds every CTA's failure count.
     const unsigned t = atomicAdd(&a.st->mix_ticket, 1u);
     sm.flags[1] = ((t & 0xffffu) == gridDim.x - 1) ? 1 : 0;
+    sm.flags[2] = static_cast<int>(t >> 16);
   }
   __syncthreads();
   if (!sm.flags[1]) return;
   __threadfence();
-  if (tid == 0) sm.flags[2] = static_cast<int>(atomicAdd(&a.st->mix_ticket, 0u) >> 16);   // failed CTAs
-  __syncthreads();
   bool any_fail = sm.flags[2] != 0;
-  F2 v{0.f, 0.f};
-  for (int b = tid; b < static_cast<int>(gridDim.x); b += kMixThreads) v = f2_add(v, f2_of(__ldcg(a.cons_part + b)));
-  const F2 ctot = block_sum_f2(v, scratch);
-  if (gated && a.sync_mode == kSyncNotifyAck && !any_fail) {
-    // The loss partials of workers without any update in this launch's
-    // slabs: every worker's NOTIFY before they are read.
-    for (int j = tid; j < a.N; j += kMixThreads) {
-      const unsigned er = wait_flag(a.ready + j, a.round + 1u, true, a.wait_ns);
-      if (er) {
-        record_error(a.st, er, j, a.round);
-        atomicOr(&sm.flags[0], 2);
-      }
-    }
-    __syncthreads();
-    any_fail = (sm.flags[0] & 2) != 0;
+  // Consensus partials of every CTA, and the loss partials: read together
+  // unless NOTIFY_ACK must first see every worker's NOTIFY (the loss
+  // partials of workers without any update in this launch's slabs).
+  const bool loss_after_notify = gated && a.sync_mode == kSyncNotifyAck;
+  const int n_cons = static_cast<int>(gridDim.x);
+  const int n_lp = a.have_loss ? a.n_loss_part : 0;
+  F2 ctot{0.f, 0.f}, ltot{0.f, 0.f};
+  for (int b = tid; b < (loss_after_notify ? n_cons : max(n_cons, n_lp)); b += kMixThreads) {
+    if (b < n_cons) ctot = f2_add(ctot, f2_of(__ldcg(a.cons_part + b)));
+    if (!loss_after_notify && b < n_lp) ltot = f2_add(ltot, F2{__ldcg(a.loss_part + b), 0.f});
   }
-  F2 lv{0.f, 0.f};
-  if (a.have_loss)
-    for (int b = tid; b < a.n_loss_part; b += kMixThreads) lv = f2_add(lv, F2{__ldcg(a.loss_part + b), 0.f});
-  const F2 ltot = block_sum_f2(lv, scratch);
+  if (loss_after_notify) {
+    if (!any_fail) {
+      for (int j = tid; j < a.N; j += kMixThreads) {
+        const unsigned er = wait_flag(a.ready + j, a.round + 1u, true, a.wait_ns);
+        if (er) {
+          record_error(a.st, er, j, a.round);
+          atomicOr(&sm.flags[0], 2);
+        }
+      }
+      __syncthreads();
+      any_fail = (sm.flags[0] & 2) != 0;
+    }
+    for (int b = tid; b < n_lp; b += kMixThreads) ltot = f2_add(ltot, F2{__ldcg(a.loss_part + b), 0.f});
+  }
+  block_sum2_f2(ctot, ltot, scratch);
   if (tid == 0) {
     const int slot = static_cast<int>(a.round % kMetricsCap);
     a.metrics_cons[slot] = any_fail ? __int_as_float(0x7fc00000) : sqrtf(fmaxf(ctot.hi + ctot.lo, 0.f));
@@ -864,7 +898,7 @@ size_t mix_smem_bytes(int N, int kp1, int S, int rows_pad, int stages, int max_r
   auto a16 = [](size_t v) { return (v + 15) & ~static_cast<size_t>(15); };
   size_t b = 1024 + mix_stage_bytes(S, rows_pad, max_region) * stages;   // alignment slack + stages
   b = a16(b + 24 * static_cast<size_t>(stages));                         // full / empty / ready
-  b = a16(b + 8 * (kMixThreads / 32));                                    // block-sum scratch (fp32 pairs)
+  b = a16(b + 16 * (kMixThreads / 32));                                   // block-sum scratch (two fp32 pairs a warp)
   b = a16(b + 16);                                                        // flags
   b = a16(b + 4 * 32);                                                    // NOTIFY bitmap
   b = a16(b + 16 * static_cast<size_t>(stages));                          // stage info

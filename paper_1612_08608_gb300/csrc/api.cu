@@ -510,9 +510,9 @@ asap_status sync_all(asap_ctx* c) {
 }
 
 // The device image of minibatch t (host only): per worker the labels, the
-// entries sorted by (column, row) -- list position, value, row, the entry's
-// slot inside its margin segment and, per segment, the row of every slot --
-// and the Q column-sum ranges cut at column boundaries; then the batch's
+// entries sorted by (column, row) -- list position, value, row and the
+// entry's slot inside its margin segment -- and the Q column-sum ranges cut
+// at column boundaries; then the batch's
 // slab-major list of distinct (worker, column) pairs and its slab offsets.
 // Used by asap_load_shards and, for tests, asap_debug_batch_image.
 struct BatchImage {

@@ -2,7 +2,9 @@
 process per group of workers, neighbour models sent point to point), on the
 CPU: the partition, the exchange plan against a brute-force restatement and
 closed forms, and whole runs of gloo ranks whose contexts are the oracle
-(tests/sharded_fake.py), compared round by round with the unsharded oracle."""
+(tests/sharded_fake.py), compared round by round with the unsharded oracle;
+and failure detection made on the host: a rank that dies or hangs mid-run
+ends its peer's round with an error instead of a wait without end."""
 import os
 import socket
 import sys
@@ -142,3 +144,86 @@ def test_sharded_ranks_match_unsharded_oracle_gloo(world, kind, k, regen):
             assert np.array_equal(got, W[first:first + got.shape[0]]), (t, rank)
         sent += sum(bytes_per_round(nbr, worker_ranges(cfg["N"], world), cfg["d"])) * 2   # fp64 rows
     assert sum(r[3] for r in res) == sent
+
+
+def _failing_rank_main(rank, world, port, cfg, fail_rank, fail_round, out, mode="raise"):
+    """A rank whose local step fails at round `fail_round`: mode "raise"
+    leaves at once, without tearing down the group (a crashed process);
+    mode "stall" reports, then stays alive without sending anything for
+    longer than the group's timeout (a hung process)."""
+    import datetime
+    import time
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank), WORLD_SIZE=str(world))
+    sys.path.insert(0, ROOT)
+    sys.path.insert(0, os.path.join(ROOT, "tests"))
+    import torch.distributed as dist
+    from sharded_fake import OracleShardContext
+    from paper_1612_08608_gb300 import inputs as inp
+    from paper_1612_08608_gb300.sharded import ShardedWorkers
+    t0 = time.monotonic()
+    err, t = None, -1
+    try:
+        dist.init_process_group("gloo", rank=rank, world_size=world,
+                                timeout=datetime.timedelta(seconds=cfg.get("pg_timeout_s", 20)))
+        sh = inp.sparse_hinge_svm(seed=cfg["seed"], N=cfg["N"], d=cfg["d"], rows=cfg["rows"], mean_nnz=20.0)
+        ctx = OracleShardContext(sh, cfg["B"], cfg["loss"], cfg["lr"], cfg["k"], cfg["kind"], cfg["graph_seed"],
+                                 cfg["regen"])
+        if rank == fail_rank:
+            step = ctx.local_step
+
+            def local_step():
+                if ctx.t == fail_round:
+                    if mode == "stall":
+                        out.put((rank, "stalled", time.monotonic() - t0, ctx.t))
+                        out.close()
+                        out.join_thread()
+                        time.sleep(2 * cfg.get("pg_timeout_s", 20) + 1)
+                        os._exit(3)
+                    raise RuntimeError("injected failure")
+                step()
+            ctx.local_step = local_step
+        run = ShardedWorkers(ctx, rank, world)
+        run.setup()
+        try:
+            for _ in range(cfg["T"]):
+                run.round()
+        except Exception as e:             # the failure itself, or a peer's lost message
+            err = type(e).__name__
+        t = run.t
+    except Exception as e:                 # set-up failed: report it, do not leave the parent waiting
+        err = "setup " + repr(e)
+    out.put((rank, err, time.monotonic() - t0, t))
+    out.close()
+    out.join_thread()                      # flushed before the process ends
+    os._exit(3 if rank == fail_rank else 0)
+
+
+@pytest.mark.parametrize("mode", ["raise", "stall"])
+def test_a_failed_rank_ends_its_peers_round_with_an_error_gloo(mode):
+    # rank 1 fails at the start of round 2, before sending its rows: it
+    # dies ("raise": rank 0's receive sees the connection close) or hangs
+    # ("stall": the group's 4 s timeout ends rank 0's receive); either way
+    # rank 0 gets an error instead of waiting forever, at the same round
+    cfg = dict(seed=3, N=6, d=400, rows=128, B=32, loss="hinge", lr=0.5, k=1, kind="ring", graph_seed=5,
+               regen=False, T=6, pg_timeout_s=4)
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_failing_rank_main, args=(r, 2, port, cfg, 1, 2, q, mode)) for r in range(2)]
+    for p in procs:
+        p.start()
+    try:
+        res = sorted(q.get(timeout=180) for _ in procs)
+    finally:
+        for p in procs:
+            p.join(timeout=30)
+            if p.is_alive():
+                p.kill()
+    (r0, err0, dt0, t0), (r1, err1, dt1, t1) = res
+    assert (r0, r1) == (0, 1)
+    assert err1 == ("stalled" if mode == "stall" else "RuntimeError") and t1 == 2
+    assert err0 is not None and not err0.startswith("setup") and t0 == 2, (err0, t0)
+    assert dt0 < 60
+    if mode == "stall":      # the error came from the timeout, after the stall began
+        assert dt0 >= dt1 + 2, (dt0, dt1)
+    assert procs[0].exitcode == 0 and procs[1].exitcode == 3

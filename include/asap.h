@@ -304,7 +304,7 @@ asap_status asap_write_rows(asap_ctx* ctx, const int32_t* rows, int count, const
 /* Consistency of the gated (NOTIFY_ACK, ASYNC) reduces since creation: the
  * inputs they read -- one per (column slab, worker) block of updates -- and
  * how many of those were current, i.e. read after the worker's NOTIFY for
- * the round (the analogue of Section 6.2's consistent reduces, Fig. 9).
+ * the round (the analogue of Section 6.2's consistent reduces, Fig. 8).
  * NOTIFY_ACK makes every input current.  Syncing. */
 asap_status asap_read_consistency(asap_ctx* ctx, uint64_t* inputs_read, uint64_t* inputs_current);
 

@@ -6,7 +6,7 @@ the whole local step.  Both must give bit-identical parameters and metrics,
 also when the local step takes the workers in a permuted order; a worker
 that never publishes NOTIFY makes the gated reduce time out, and the context
 recovers.  ASYNC (measurement only) reads updates without waiting and counts
-how many were current, the analogue of Fig. 9's consistent reduces."""
+how many were current, the analogue of Fig. 8's consistent reduces."""
 import numpy as np
 import pytest
 

@@ -25,6 +25,30 @@ def test_batch_image_matches_the_shards(S, Q, max_len):
     rng = np.random.default_rng(8)
     lengths = [np.where(rng.random(3 * B) < 0.15, 0, rng.integers(1, max_len, 3 * B)) for _ in range(N)]
     sh = inputs.sparse_custom(seed=31, N=N, d=d, rows=3 * B, lengths=lengths, hot_col=7)
+    _check_image(sh, N, d, B, S, Q, t)
+
+
+def test_batch_image_edge_cases():
+    N, d, B = 4, 777, 16
+    rows = 3 * B
+    z = np.zeros(rows, np.int64)
+    # worker 0: an empty minibatch at t = 1 between non-empty ones; worker 1:
+    # three entries for eight CTAs (empty column-sum ranges); worker 2: every
+    # row of window 1 holds the same single column; worker 3: full rows
+    l0 = np.full(rows, 5)
+    l0[B:2 * B] = 0
+    l1 = z.copy()
+    l1[[B + 1, B + 7, B + 15]] = 1
+    l2 = np.full(rows, 1)
+    l3 = np.full(rows, 60)
+    sh = inputs.sparse_custom(seed=5, N=N, d=d, rows=rows, lengths=[l0, l1, l2, l3])
+    for r in range(B, 2 * B):                  # worker 2: column 3 in every row of window 1
+        sh.col[2][sh.rowptr[2][r]] = 3
+    for S, Q, t in [(8, 8, 1), (8, 1, 1), (1024, 8, 1), (64, 2, 2), (16, 5, 0)]:
+        _check_image(sh, N, d, B, S, Q, t)
+
+
+def _check_image(sh, N, d, B, S, Q, t):
     img, desc, (list_off, soff_off, list_len) = debug_batch_image(sh, B, S, t, ctas_per_worker=Q)
     n_slabs = -(-((d + 63) // 64 * 64) // S)
     lst = _view(img, list_off, np.uint32, list_len)
